@@ -1,0 +1,288 @@
+"""fp64 CPU oracle of the capped-residency MoE decode step.
+
+TEST INFRASTRUCTURE ONLY. Only ``tests/``, ``__graft_entry__.smoke()`` and
+``bench.py``'s CPU-baseline / reference leg may import this package. The CUDA
+library never calls it and shares no code with it.
+
+What it computes, per layer-step (paper, Section "Rotary GPU Concept", Fig. 1:
+host tier, slot group, lookup table sub-module id -> slot, routing result
+driving selective load and evict; the undisclosed rotary policy is replaced by
+a deterministic LRU with lower-id ties):
+
+1. routing: z = W_r h, p = softmax(z), top-k by z (ties -> lower id),
+   renormalised gates g_r = p_{e_r} / sum_j p_{e_j};
+2. residency: the distinct global ids needed this layer-step go through one
+   LRU step (``orc_lru_step``), which yields one hit/miss record per id;
+   every miss copies the expert's stored weights from the host tier into
+   its slot (the oracle keeps those slot copies and computes from them);
+3. expert FFN from the slot copy: u = silu(W_g x) * (W_u x), y_r = W_d u;
+4. combine: out = sum_r g_r y_r in rank order.
+
+All arithmetic is fp64 on exactly widened inputs (bf16/fp32 values, int4
+dequantised to q * scale). Every function here is pinned by ``tests/test_oracle_*``
+against brute force, closed forms, invariants and a hand-simulated LRU trace.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+from dataclasses import dataclass
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "moe_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "liboracle.so")
+_lib = None
+_lock = threading.Lock()
+
+DTYPE_CODES = {"fp32": 0, "bf16": 1, "int4": 2}
+
+
+class OrcRec(ctypes.Structure):
+    _fields_ = [("step", ctypes.c_int32), ("layer", ctypes.c_int32), ("expert", ctypes.c_int32),
+                ("kind", ctypes.c_int32), ("slot", ctypes.c_int32), ("evicted", ctypes.c_int32)]
+
+
+REC_DTYPE = np.dtype([("step", np.int32), ("layer", np.int32), ("expert", np.int32), ("kind", np.int32),
+                      ("slot", np.int32), ("evicted", np.int32)])
+
+
+def build(force: bool = False) -> str:
+    """Compile liboracle.so in-tree (plain C, fp64, OpenMP over matrix rows)."""
+    if not force and os.path.exists(_LIB_PATH) and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-fPIC", "-shared", "-o", tmp, _SRC,
+           "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            build()
+            L = ctypes.CDLL(_LIB_PATH)
+            vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+            L.orc_widen.argtypes = [ctypes.c_int, vp, vp, i64, i64, vp]
+            L.orc_widen.restype = ctypes.c_int
+            L.orc_matvec.argtypes = [vp, vp, i64, i64, vp]
+            L.orc_softmax.argtypes = [vp, i64, vp]
+            L.orc_topk.argtypes = [vp, i64, i32, vp, vp]
+            L.orc_router.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp]
+            L.orc_expert_ffn.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp]
+            L.orc_combine.argtypes = [vp, vp, i32, i32, vp]
+            L.orc_lru_step.argtypes = [i64, vp, vp, vp, i64, vp, i32, i32, i32, vp]
+            L.orc_lru_step.restype = i32
+            _lib = L
+    return _lib
+
+
+def _p(a):
+    if a is None:
+        return None
+    assert a.flags["C_CONTIGUOUS"], "oracle inputs must be C-contiguous"
+    return ctypes.c_void_p(a.ctypes.data)
+
+
+# ----------------------------------------------------------------------------------------------
+# single-function entry points
+
+
+def widen(dtype: str, raw: np.ndarray, rows: int, cols: int, scales: np.ndarray | None = None) -> np.ndarray:
+    out = np.empty((rows, cols), dtype=np.float64)
+    raw = np.ascontiguousarray(raw)
+    sc = None if scales is None else np.ascontiguousarray(scales, dtype=np.uint16)
+    rc = lib().orc_widen(DTYPE_CODES[dtype], _p(raw), _p(sc), rows, cols, _p(out))
+    if rc != 0:
+        raise ValueError("widen: bad dtype or shape")
+    return out
+
+
+def matvec(W: np.ndarray, x: np.ndarray) -> np.ndarray:
+    W = np.ascontiguousarray(W, dtype=np.float64)
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.empty(W.shape[0], dtype=np.float64)
+    lib().orc_matvec(_p(W), _p(x), W.shape[0], W.shape[1], _p(y))
+    return y
+
+
+def softmax(z: np.ndarray) -> np.ndarray:
+    z = np.ascontiguousarray(z, dtype=np.float64)
+    p = np.empty_like(z)
+    lib().orc_softmax(_p(z), z.size, _p(p))
+    return p
+
+
+def router(Wr: np.ndarray, h: np.ndarray, k: int, renorm: bool = True, forced_idx=None):
+    """Routing of one hidden vector -> (idx int32[k], gate f64[k], z f64[E], p f64[E])."""
+    Wr = np.ascontiguousarray(Wr, dtype=np.float64)
+    h = np.ascontiguousarray(h, dtype=np.float64)
+    E, d = Wr.shape
+    idx = np.empty(k, dtype=np.int32)
+    gate = np.empty(k, dtype=np.float64)
+    z = np.empty(E, dtype=np.float64)
+    p = np.empty(E, dtype=np.float64)
+    scratch = np.empty(2 * E + (E + 7) // 8 + 1, dtype=np.float64)
+    fi = None if forced_idx is None else np.ascontiguousarray(forced_idx, dtype=np.int32)
+    lib().orc_router(_p(Wr), _p(h), E, d, k, 1 if renorm else 0, _p(fi), _p(idx), _p(gate), _p(z), _p(p),
+                     _p(scratch))
+    return idx, gate, z, p
+
+
+def expert_ffn(Wg: np.ndarray, Wu: np.ndarray, Wd: np.ndarray, x: np.ndarray):
+    """SwiGLU expert FFN in fp64 -> (y [d], u [I])."""
+    Wg, Wu, Wd = (np.ascontiguousarray(a, dtype=np.float64) for a in (Wg, Wu, Wd))
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    I, d = Wg.shape
+    y = np.empty(d, dtype=np.float64)
+    u = np.empty(I, dtype=np.float64)
+    scratch = np.empty(3 * I, dtype=np.float64)
+    lib().orc_expert_ffn(_p(Wg), _p(Wu), _p(Wd), _p(x), d, I, _p(y), _p(u), _p(scratch))
+    return y, u
+
+
+def combine(y: np.ndarray, gate: np.ndarray) -> np.ndarray:
+    y = np.ascontiguousarray(y, dtype=np.float64)
+    gate = np.ascontiguousarray(gate, dtype=np.float64)
+    k, d = y.shape
+    out = np.empty(d, dtype=np.float64)
+    lib().orc_combine(_p(y), _p(gate), k, d, _p(out))
+    return out
+
+
+class LRUTable:
+    """Residency state (slot group + lookup table) driven one layer-step at a time."""
+
+    def __init__(self, n_gid: int, cap: int, n_experts: int):
+        self.n_gid, self.cap, self.n_experts = n_gid, cap, n_experts
+        self.slot_of = np.full(n_gid, -1, dtype=np.int32)
+        self.gid_of = np.full(cap, -1, dtype=np.int32)
+        self.last_use = np.full(n_gid, -1, dtype=np.int64)
+
+    def step(self, clock: int, needed, step: int) -> np.ndarray:
+        needed = np.ascontiguousarray(sorted(set(int(g) for g in needed)), dtype=np.int32)
+        out = np.zeros(len(needed), dtype=REC_DTYPE)
+        n = lib().orc_lru_step(self.cap, _p(self.slot_of), _p(self.gid_of), _p(self.last_use), clock, _p(needed),
+                               len(needed), self.n_experts, step, _p(out))
+        if n < 0:
+            raise RuntimeError("LRU step: capacity below the number of distinct experts in one layer-step")
+        return out
+
+
+# ----------------------------------------------------------------------------------------------
+# the full decode step
+
+
+@dataclass
+class StepResult:
+    out: np.ndarray | None  # f64 [L x B x d] (None when outputs were not requested)
+    records: np.ndarray  # REC_DTYPE, all layer-steps of this decode step in layer order
+    idx: np.ndarray  # int32 [L x B x k]
+    gate: np.ndarray  # f64 [L x B x k]
+    z: np.ndarray  # f64 [L x B x E] router logits
+
+
+class Oracle:
+    """Decode-step oracle over a stack of MoE layers with a capped slot pool.
+
+    experts(layer, expert) -> synth.ExpertWeights (raw storage) is the host tier.
+    routers[l]: raw router storage [E x d]. With keep_slot_copies the oracle copies
+    an expert's stored bytes into its slot on a miss and computes from that copy.
+    """
+
+    def __init__(self, d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots, routers, experts,
+                 renorm=True, keep_slot_copies=True):
+        self.d, self.E, self.k, self.I, self.L = d, n_experts, top_k, d_ff, n_layers
+        self.wdtype, self.adtype, self.renorm = wdtype, adtype, renorm
+        self.router_dtype = "fp32" if wdtype == "fp32" else "bf16"
+        self.routers = [widen(self.router_dtype, routers[l], n_experts, d) for l in range(n_layers)]
+        self.experts = experts
+        self.keep = keep_slot_copies
+        self.table = LRUTable(n_layers * n_experts, cap_slots, n_experts)
+        self.slots: dict[int, object] = {}
+        self.token_step = 0
+
+    @classmethod
+    def for_workload(cls, wl, cap_slots=None, keep_slot_copies=True, routers=None, experts=None):
+        import synth
+
+        routers = routers if routers is not None else [synth.router_weights(wl, l) for l in range(wl.n_layers)]
+        experts = experts if experts is not None else (lambda l, e: synth.expert_weights(wl, l, e))
+        return cls(wl.d, wl.n_experts, wl.top_k, wl.d_ff, wl.n_layers, wl.wdtype, wl.adtype,
+                   wl.cap_slots if cap_slots is None else cap_slots, routers, experts,
+                   keep_slot_copies=keep_slot_copies)
+
+    def reset(self):
+        self.table = LRUTable(self.table.n_gid, self.table.cap, self.E)
+        self.slots = {}
+        self.token_step = 0
+
+    def _widen_expert(self, w):
+        d, I, dt = self.d, self.I, self.wdtype
+        Wg = widen(dt, w.gate, I, d, w.s_gate)
+        Wu = widen(dt, w.up, I, d, w.s_up)
+        Wd = widen(dt, w.down, d, I, w.s_down)
+        return Wg, Wu, Wd
+
+    def decode_step(self, hidden_raw: np.ndarray, compute_out: bool = True, forced_idx=None) -> StepResult:
+        """One decode step over all layers. hidden_raw: raw activation storage [L x B x d]."""
+        import synth
+
+        L, B = hidden_raw.shape[0], hidden_raw.shape[1]
+        assert L == self.L and hidden_raw.shape[2] == self.d
+        h = synth.act_to_f64(hidden_raw, self.adtype)
+        idx = np.empty((L, B, self.k), dtype=np.int32)
+        gate = np.empty((L, B, self.k), dtype=np.float64)
+        z = np.empty((L, B, self.E), dtype=np.float64)
+        out = np.zeros((L, B, self.d), dtype=np.float64) if compute_out else None
+        recs = []
+        for l in range(L):
+            clock = self.token_step * L + l
+            for b in range(B):
+                fi = None if forced_idx is None else forced_idx[l, b]
+                idx[l, b], gate[l, b], z[l, b], _ = router(self.routers[l], h[l, b], self.k, self.renorm, fi)
+            needed = sorted(set(int(l * self.E + e) for e in idx[l].ravel()))
+            r = self.table.step(clock, needed, self.token_step)
+            recs.append(r)
+            for rec in r:
+                if rec["kind"] == 1:
+                    gid = int(l * self.E + rec["expert"])
+                    if self.keep:
+                        w = self.experts(l, int(rec["expert"]))
+                        self.slots[int(rec["slot"])] = (gid, _copy_expert(w))
+            if compute_out:
+                cache = {}
+                for b in range(B):
+                    ys = np.empty((self.k, self.d), dtype=np.float64)
+                    for rk in range(self.k):
+                        e = int(idx[l, b, rk])
+                        gid = l * self.E + e
+                        if gid not in cache:
+                            if self.keep:
+                                slot = int(self.table.slot_of[gid])
+                                held_gid, w = self.slots[slot]
+                                assert held_gid == gid, "slot holds another expert"
+                            else:
+                                w = self.experts(l, e)
+                            cache[gid] = self._widen_expert(w)
+                        Wg, Wu, Wd = cache[gid]
+                        ys[rk], _ = expert_ffn(Wg, Wu, Wd, h[l, b])
+                    out[l, b] = combine(ys, gate[l, b])
+        self.token_step += 1
+        return StepResult(out, np.concatenate(recs), idx, gate, z)
+
+
+def _copy_expert(w):
+    import copy
+
+    c = copy.copy(w)
+    for f in ("gate", "up", "down", "s_gate", "s_up", "s_down"):
+        v = getattr(w, f)
+        setattr(c, f, None if v is None else v.copy())
+    return c

@@ -1,0 +1,77 @@
+"""Pure-Python brute force for tiny inputs (test infrastructure only).
+
+Independent restatements used to pin the C oracle, written differently on
+purpose: routing sorts the full softmax explicitly; residency keeps a recency
+list instead of timestamps; the expert FFN is explicit Python loops.
+"""
+from __future__ import annotations
+
+import math
+
+
+def router_brute(Wr, h, k, renorm=True):
+    """Full softmax over all experts, explicit sort by (-logit, id), first k, renormalise."""
+    E = len(Wr)
+    z = [sum(Wr[e][j] * h[j] for j in range(len(h))) for e in range(E)]
+    m = max(z)
+    ex = [math.exp(v - m) for v in z]
+    tot = sum(ex)
+    p = [v / tot for v in ex]
+    order = sorted(range(E), key=lambda e: (-z[e], e))
+    sel = order[:k]
+    if renorm:
+        s = sum(p[e] for e in sel)
+        g = [p[e] / s for e in sel]
+    else:
+        g = [p[e] for e in sel]
+    return sel, g, z, p
+
+
+def expert_brute(Wg, Wu, Wd, x):
+    """y = W_d (silu(W_g x) * (W_u x)) with explicit loops."""
+    I, d = len(Wg), len(x)
+    u = []
+    for i in range(I):
+        a = sum(Wg[i][j] * x[j] for j in range(d))
+        b = sum(Wu[i][j] * x[j] for j in range(d))
+        u.append(a / (1.0 + math.exp(-a)) * b)
+    return [sum(Wd[o][i] * u[i] for i in range(I)) for o in range(len(Wd))]
+
+
+class RecencyListLRU:
+    """LRU over a fixed slot group kept as a recency list (oldest first).
+
+    Residents are ordered by (time of last use, id). Each step: needed ids are
+    pinned; misses (ascending id) take the lowest free slot, else the oldest
+    unpinned resident's slot; then every needed id moves to the back of the
+    list, in ascending id order (they share the newest use time).
+    """
+
+    def __init__(self, cap):
+        self.cap = cap
+        self.order = []  # resident ids, least recent first
+        self.slot = {}  # id -> slot
+        self.free = list(range(cap))
+
+    def step(self, needed):
+        needed = sorted(set(needed))
+        pinned = set(needed)
+        recs = []
+        for g in needed:
+            if g in self.slot:
+                recs.append((g, 0, self.slot[g], -1))
+                continue
+            if self.free:
+                s = min(self.free)
+                self.free.remove(s)
+                victim = -1
+            else:
+                victim = next((v for v in self.order if v not in pinned), None)
+                if victim is None:
+                    raise RuntimeError("capacity below the step's working set")
+                self.order.remove(victim)
+                s = self.slot.pop(victim)
+            self.slot[g] = s
+            recs.append((g, 1, s, victim))
+        self.order = [v for v in self.order if v not in pinned] + needed
+        return recs
