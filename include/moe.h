@@ -1,0 +1,182 @@
+/*
+ * moe.h -- C ABI of the GB300 capped-residency MoE decode library (libmoe.so).
+ *
+ * One decode step of a stack of Mixture-of-Experts layers whose experts do not
+ * all fit in GPU memory. This is the residency problem of the paper (Section
+ * "Rotary GPU Concept", Fig. 1): full expert weights stay in a host memory
+ * tier; a fixed-capacity group of accelerator slots holds a subset of the
+ * experts; a lookup table maps expert id -> slot; the routing result (hidden
+ * state h, routing vector r) drives selective loads into slots and evictions
+ * from them. The paper does not disclose its replacement policy; this library
+ * uses a deterministic LRU with ties broken toward the lower global expert id.
+ *
+ * Per layer, in order (layers are processed strictly one after another and a
+ * layer never looks at a later layer's input):
+ *   1. router: z = W_r h (fp32 accumulation), top-k by z (ties -> lower id),
+ *      gates g_r = softmax over the k selected logits (= p_{e_r} / sum_j p_{e_j});
+ *   2. slot lookup + LRU: hit -> slot; miss -> lowest free slot, else evict the
+ *      unpinned resident with the smallest (last use, global id);
+ *   3. misses are copied from the pinned host arena into their slots on an
+ *      internal copy stream, overlapped with the hit experts' compute;
+ *   4. SwiGLU expert FFN from the slots: u = silu(W_g x) * (W_u x), y_r = W_d u
+ *      (fp32 u and y; int4 weights dequantised in registers);
+ *   5. out = sum_r g_r y_r in rank order (deterministic).
+ *
+ * Conventions
+ *   - Every call returns a moe_status; nothing is thrown across the ABI.
+ *     moe_last_error() gives a message for the last failure on a handle.
+ *   - Pointers are host pointers unless a parameter says "device".
+ *   - Ownership: the library owns everything it allocates; register/set calls
+ *     copy the caller's buffers, which may be freed afterwards.
+ *   - Threading: one handle is used by one host thread at a time, except that
+ *     moe_register_host_experts may be called concurrently for distinct
+ *     (layer, expert) pairs.
+ *   - Device: the handle is bound to cfg.device; calls set that device.
+ */
+#ifndef MOE_H_
+#define MOE_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct moe_handle moe_handle;
+
+typedef enum {
+  MOE_OK = 0,
+  MOE_ERR_INVALID = -1,        /* bad argument or configuration */
+  MOE_ERR_OOM = -2,            /* device or pinned host allocation failed */
+  MOE_ERR_CUDA = -3,           /* a CUDA runtime call failed */
+  MOE_ERR_CAPACITY = -4,       /* slot cap below one layer-step's working set */
+  MOE_ERR_NOT_REGISTERED = -5, /* a router or expert needed by the step was never registered */
+  MOE_ERR_TIMEOUT = -6,        /* a bounded wait for the device ran out */
+  MOE_ERR_TRACE_OVERFLOW = -7  /* residency records were dropped (trace buffer full) */
+} moe_status;
+
+/* Storage types (wdtype: expert weights; adtype: activations hidden/out). */
+enum {
+  MOE_DTYPE_FP32 = 0,
+  MOE_DTYPE_BF16 = 1,
+  MOE_DTYPE_INT4_G128 = 2 /* symmetric int4, groups of 128 along the input dim, bf16 scales */
+};
+
+typedef struct {
+  int32_t d;          /* hidden size */
+  int32_t n_experts;  /* experts per layer, E (<= 256) */
+  int32_t top_k;      /* experts per token, k (<= 16, <= E) */
+  int32_t d_ff;       /* SwiGLU intermediate size, I */
+  int32_t n_layers;   /* L */
+  int32_t max_batch;  /* sequences per decode step (this version: 1) */
+  int32_t wdtype;     /* MOE_DTYPE_FP32 (needs adtype FP32), BF16 or INT4_G128 (need adtype BF16) */
+  int32_t adtype;     /* MOE_DTYPE_FP32 or MOE_DTYPE_BF16 */
+  int64_t cap_slots;  /* expert slots on the device; 0 => floor(cap_bytes / expert bytes) */
+  int64_t cap_bytes;  /* device expert-pool budget in bytes (used when cap_slots == 0) */
+  int32_t renorm;     /* 1: gates renormalised over the top k (default); 0: raw softmax probabilities */
+  int32_t device;     /* CUDA device ordinal */
+  void* device_pool;  /* optional caller-owned device buffer of >= moe_pool_bytes(cfg) bytes, 256-B aligned;
+                         NULL => the library allocates the pool */
+  int64_t trace_capacity; /* residency records kept on the host; 0 disables the trace */
+} moe_config;
+
+/* One residency record: a requested expert's outcome in one layer-step. */
+typedef struct {
+  int32_t step;    /* decode step index since create/reset */
+  int32_t layer;
+  int32_t expert;  /* expert id within the layer */
+  int32_t kind;    /* 0 hit, 1 miss */
+  int32_t slot;    /* slot holding the expert after the step */
+  int32_t evicted; /* global id (layer * E + expert) of the evicted expert; -1 if none */
+} moe_trace_rec;
+
+typedef struct {
+  int64_t steps;       /* decode steps run */
+  int64_t layer_steps; /* layer-steps run */
+  int64_t hits;
+  int64_t misses;
+  int64_t evictions;
+  int64_t miss_bytes;  /* bytes copied host -> device for misses */
+} moe_stats;
+
+/* Per-kernel-class timing gathered with CUDA events on the launching streams while
+ * profiling is on (see moe_profile_enable). */
+typedef struct {
+  char name[32];
+  int64_t launches;
+  double total_ms;
+  int64_t bytes;       /* algorithmic bytes moved by all launches (weights read + vectors read/written) */
+} moe_kernel_time;
+
+/* Bytes of one expert's weights as stored in a slot (scales included for int4). */
+int64_t moe_expert_bytes(const moe_config* cfg);
+/* Bytes the device expert pool needs for cfg (slots * 256-B aligned slot stride), or < 0 if cfg is invalid. */
+int64_t moe_pool_bytes(const moe_config* cfg);
+
+/* Validate cfg, allocate the device pool (unless cfg->device_pool is given), the pinned host
+ * arena for all n_layers * n_experts experts, router storage and work buffers.
+ * MOE_ERR_CAPACITY if the slot count is below min(E, k * max_batch), the most distinct experts
+ * one layer-step can need (a clean failure instead of a start-up that cannot run).
+ * On failure *out is NULL and nothing stays allocated. */
+moe_status moe_create(const moe_config* cfg, moe_handle** out);
+
+/* Router weights of one layer: W_r [E x d] row-major, host memory, fp32 when wdtype is FP32,
+ * else bf16. Copied to device memory (routers are always resident, outside the slot cap). */
+moe_status moe_set_router(moe_handle* h, int32_t layer, const void* w_r);
+
+/* One expert's weights into the pinned host tier (the paper's host memory tier). Row-major,
+ * out x in: w_gate [I x d], w_up [I x d], w_down [d x I].
+ *   FP32/BF16: elements of that type.
+ *   INT4_G128: packed nibbles, byte j of a row = element 2j (low nibble) and 2j+1 (high),
+ *              two's complement; `scales` = bf16 [I x d/128] (gate) ++ [I x d/128] (up)
+ *              ++ [d x I/128] (down). NULL otherwise.
+ * The weights are repacked into the slot layout. If the expert is resident its slot copy is
+ * NOT refreshed; call moe_reset_residency after re-registering resident experts. */
+moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t expert, const void* w_gate,
+                                     const void* w_up, const void* w_down, const void* scales);
+
+/* One decode step over all layers. hidden: device [n_layers x batch x d] (adtype), the input
+ * of every layer; out: device [n_layers x batch x d] (adtype). Work is ordered on `stream`
+ * (a cudaStream_t; NULL = legacy default stream). Host-driven: the call blocks once per layer
+ * until that layer's routing result has reached the host (bounded wait, MOE_ERR_TIMEOUT), and
+ * returns once the last layer's work is enqueued. hidden must stay valid and out must not be
+ * read until `stream` reaches the end of the step. Calls on one handle must use one stream or
+ * be serialised by the caller. If a CUDA call fails mid-step the residency state is reset
+ * (empty pool) and MOE_ERR_CUDA is returned. */
+moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t batch, void* stream);
+
+/* moe_decode_step on host buffers (pinned or pageable): copies hidden to the device, runs the
+ * step on an internal stream, copies out back and waits for completion. */
+moe_status moe_decode_step_host(moe_handle* h, const void* hidden_host, void* out_host, int32_t batch);
+
+/* Copy residency records [start, start + cap) of the trace into buf. *n_copied = records copied,
+ * *n_total = records kept. MOE_ERR_TRACE_OVERFLOW (after copying) if records were dropped. */
+moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* buf, int64_t cap,
+                                   int64_t* n_copied, int64_t* n_total);
+
+/* Routing of the last decode step: idx int32 [n_layers x batch x k], gate fp32 [same]. */
+moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_t n);
+
+moe_status moe_get_stats(moe_handle* h, moe_stats* out);
+
+/* Empty the slot pool (all experts non-resident), step clock 0, trace and stats cleared. */
+moe_status moe_reset_residency(moe_handle* h);
+
+/* Profiling: with on = 1, every kernel launch and miss copy of later steps is bracketed by
+ * CUDA events on its stream. moe_profile_read waits for the recorded work, then reports one
+ * entry per kernel class (router, gateup, down_combine, miss_copy) accumulated since the last
+ * read, and clears the accumulators. */
+moe_status moe_profile_enable(moe_handle* h, int32_t on);
+moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, int32_t* n_out);
+
+/* Message of the last failure on h (or of the last failed moe_create if h is NULL). */
+const char* moe_last_error(const moe_handle* h);
+
+/* Wait for outstanding work, free everything. NULL is a no-op. */
+void moe_destroy(moe_handle* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOE_H_ */

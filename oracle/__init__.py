@@ -230,6 +230,23 @@ class Oracle:
         Wd = widen(dt, w.down, d, I, w.s_down)
         return Wg, Wu, Wd
 
+    def moe_layer(self, layer: int, h_raw: np.ndarray, forced_idx=None):
+        """One layer's output for one hidden vector, reading the host tier directly.
+
+        Same definition as decode_step without the slot group; the cap invariant (outputs do
+        not depend on residency) is what lets sampled outputs of large runs be checked this way.
+        Returns (out f64 [d], idx, gate).
+        """
+        import synth
+
+        h = synth.act_to_f64(np.asarray(h_raw), self.adtype)
+        idx, gate, _, _ = router(self.routers[layer], h, self.k, self.renorm, forced_idx)
+        ys = np.empty((self.k, self.d), dtype=np.float64)
+        for rk in range(self.k):
+            Wg, Wu, Wd = self._widen_expert(self.experts(layer, int(idx[rk])))
+            ys[rk], _ = expert_ffn(Wg, Wu, Wd, h)
+        return combine(ys, gate), idx, gate
+
     def decode_step(self, hidden_raw: np.ndarray, compute_out: bool = True, forced_idx=None) -> StepResult:
         """One decode step over all layers. hidden_raw: raw activation storage [L x B x d]."""
         import synth

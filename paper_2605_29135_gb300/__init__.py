@@ -1,0 +1,161 @@
+"""GB300-native capped-residency MoE decode step (Python binding of libmoe.so).
+
+The paper's residency problem (Section "Rotary GPU Concept", Fig. 1): expert weights live in a
+pinned host tier, a fixed group of GPU slots holds a subset of them, a lookup table maps
+expert id -> slot, and the routing result drives selective loads and evictions. One decode step
+runs the router / top-k, the slot lookup with deterministic LRU eviction (lower id on ties), the
+miss copies on a side stream, the SwiGLU expert GEMVs and the rank-ordered combine, all inside
+libmoe.so. This module only marshals arguments; the method names follow the C ABI
+(include/moe.h) without the ``moe_`` prefix.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import numpy as np
+
+from . import _lib
+from ._lib import DTYPE, STATUS, KernelTime, MoeConfig, Stats, TraceRec
+
+TRACE_DTYPE = np.dtype([("step", np.int32), ("layer", np.int32), ("expert", np.int32), ("kind", np.int32),
+                        ("slot", np.int32), ("evicted", np.int32)])
+
+
+class MoEError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+def make_config(d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots=0, cap_bytes=0, renorm=True,
+                device=0, max_batch=1, trace_capacity=1 << 22, device_pool=None) -> MoeConfig:
+    return MoeConfig(d=d, n_experts=n_experts, top_k=top_k, d_ff=d_ff, n_layers=n_layers, max_batch=max_batch,
+                     wdtype=DTYPE[wdtype], adtype=DTYPE[adtype], cap_slots=cap_slots, cap_bytes=cap_bytes,
+                     renorm=1 if renorm else 0, device=device, device_pool=device_pool,
+                     trace_capacity=trace_capacity)
+
+
+def expert_bytes(cfg: MoeConfig) -> int:
+    return int(_lib.load().moe_expert_bytes(ctypes.byref(cfg)))
+
+
+def pool_bytes(cfg: MoeConfig) -> int:
+    return int(_lib.load().moe_pool_bytes(ctypes.byref(cfg)))
+
+
+def _ptr(a) -> ctypes.c_void_p:
+    if a is None:
+        return None
+    if isinstance(a, np.ndarray):
+        assert a.flags["C_CONTIGUOUS"], "arrays passed to libmoe must be C-contiguous"
+        return ctypes.c_void_p(a.ctypes.data)
+    # torch tensor
+    assert a.is_contiguous(), "tensors passed to libmoe must be contiguous"
+    return ctypes.c_void_p(a.data_ptr())
+
+
+class MoE:
+    """One library handle (moe_create ... moe_destroy)."""
+
+    def __init__(self, cfg: MoeConfig):
+        self.lib = _lib.load()
+        self.cfg = cfg
+        h = ctypes.c_void_p()
+        st = self.lib.moe_create(ctypes.byref(cfg), ctypes.byref(h))
+        if st != 0:
+            raise MoEError(st, self.lib.moe_last_error(None).decode())
+        self.h = h
+
+    # -- helpers
+    def _check(self, st):
+        if st != 0:
+            raise MoEError(st, self.lib.moe_last_error(self.h).decode())
+
+    def last_error(self) -> str:
+        return self.lib.moe_last_error(self.h).decode()
+
+    # -- ABI
+    def set_router(self, layer: int, w_r: np.ndarray):
+        self._check(self.lib.moe_set_router(self.h, layer, _ptr(np.ascontiguousarray(w_r))))
+
+    def register_host_experts(self, layer: int, expert: int, gate, up, down, scales=None):
+        g, u, dn = (np.ascontiguousarray(a) for a in (gate, up, down))
+        sc = None if scales is None else np.ascontiguousarray(scales, dtype=np.uint16)
+        self._check(self.lib.moe_register_host_experts(self.h, layer, expert, _ptr(g), _ptr(u), _ptr(dn), _ptr(sc)))
+
+    def decode_step(self, hidden, out, batch: int = 1, stream=None):
+        """hidden, out: contiguous device tensors [n_layers x batch x d]; stream: torch.cuda.Stream or None
+        (torch's current stream)."""
+        import torch
+
+        if stream is None:
+            stream = torch.cuda.current_stream(hidden.device)
+        self._check(self.lib.moe_decode_step(self.h, _ptr(hidden), _ptr(out), batch,
+                                             ctypes.c_void_p(stream.cuda_stream)))
+
+    def decode_step_host(self, hidden, out, batch: int = 1):
+        """hidden, out: host buffers (numpy arrays or CPU tensors, ideally pinned)."""
+        self._check(self.lib.moe_decode_step_host(self.h, _ptr(hidden), _ptr(out), batch))
+
+    def get_residency_trace(self) -> np.ndarray:
+        n_copied, n_total = ctypes.c_int64(), ctypes.c_int64()
+        self.lib.moe_get_residency_trace(self.h, 0, None, 0, ctypes.byref(n_copied), ctypes.byref(n_total))
+        out = np.zeros(n_total.value, dtype=TRACE_DTYPE)
+        st = self.lib.moe_get_residency_trace(self.h, 0, _ptr(out), n_total.value, ctypes.byref(n_copied),
+                                              ctypes.byref(n_total))
+        self._check(st)
+        return out[:n_copied.value]
+
+    def get_last_routing(self):
+        n = self.cfg.n_layers * self.cfg.max_batch * self.cfg.top_k
+        idx = np.empty(n, dtype=np.int32)
+        gate = np.empty(n, dtype=np.float32)
+        self._check(self.lib.moe_get_last_routing(self.h, _ptr(idx), _ptr(gate), n))
+        shape = (self.cfg.n_layers, self.cfg.max_batch, self.cfg.top_k)
+        return idx.reshape(shape), gate.reshape(shape)
+
+    def get_stats(self) -> dict:
+        s = Stats()
+        self._check(self.lib.moe_get_stats(self.h, ctypes.byref(s)))
+        return {f: getattr(s, f) for f, _ in Stats._fields_}
+
+    def reset_residency(self):
+        self._check(self.lib.moe_reset_residency(self.h))
+
+    def profile_enable(self, on: bool = True):
+        self._check(self.lib.moe_profile_enable(self.h, 1 if on else 0))
+
+    def profile_read(self) -> dict:
+        arr = (KernelTime * 8)()
+        n = ctypes.c_int32()
+        self._check(self.lib.moe_profile_read(self.h, arr, 8, ctypes.byref(n)))
+        return {arr[i].name.decode(): {"launches": arr[i].launches, "total_ms": arr[i].total_ms,
+                                       "bytes": arr[i].bytes} for i in range(n.value)}
+
+    def destroy(self):
+        if getattr(self, "h", None):
+            self.lib.moe_destroy(self.h)
+            self.h = None
+
+    close = destroy
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.destroy()
+
+
+def build(force: bool = False) -> str:
+    from .build import build as _b
+
+    return _b(force=force)
+
+
+__all__ = ["MoE", "MoEError", "make_config", "expert_bytes", "pool_bytes", "TRACE_DTYPE", "build", "TraceRec"]

@@ -1,0 +1,712 @@
+// C ABI of the capped-residency MoE decode library: handle, pinned host tier, slot pool,
+// residency table (LRU with lower-id ties), miss-copy pipeline and the per-layer schedule.
+//
+// Host-driven schedule of one layer (the routing result reaches the host through mapped
+// pinned memory; the host owns the lookup table and issues the selective loads):
+//   compute stream:  router(l) ............................ gateup(hits) [wait copy m] gateup(m) ... down+combine(l) router(l+1)
+//   host:                      wait routing(l) -> LRU -> issue miss copies -> enqueue kernels
+//   copy stream:                                 copy(m0) copy(m1) ...
+// A slot is overwritten only by a copy issued after the host saw router(l) finish; router(l)
+// runs after every kernel of layers < l on the compute stream, so no earlier reader of a
+// victim slot can still be running, and experts needed by layer l are pinned for the step.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <chrono>
+#include <cstdio>
+#include <cstring>
+#include <set>
+#include <string>
+#include <utility>
+#include <vector>
+
+#include "kernels.cuh"
+#include "moe.h"
+
+namespace {
+
+constexpr double kWaitTimeoutS = 20.0;
+
+thread_local std::string g_create_error;
+
+enum { PC_ROUTER = 0, PC_GATEUP = 1, PC_DOWN = 2, PC_COPY = 3, PC_N = 4 };
+const char* kPcName[PC_N] = {"router", "gateup", "down_combine", "miss_copy"};
+
+struct PendingTime {
+  int cls;
+  cudaEvent_t a, b;
+  int64_t bytes;
+};
+
+}  // namespace
+
+struct moe_handle {
+  moe_config cfg{};
+  moe::BlobLayout lay{};
+  int64_t slot_stride = 0;
+  int64_t n_gid = 0;
+  int64_t cap = 0;
+  int64_t asize = 0;         // activation element bytes
+  int64_t router_eb = 0;     // router element bytes
+  uint8_t* pool = nullptr;   // device slot pool
+  bool own_pool = false;
+  uint8_t* arena = nullptr;  // pinned host tier, one slot image per global expert id
+  std::vector<uint8_t> registered;
+  std::vector<uint8_t> router_set;
+  bool all_registered = false;
+  uint8_t* routers = nullptr;  // device [L][E][d]
+  moe::RouteOut* route = nullptr;      // mapped pinned (host view)
+  moe::RouteOut* route_dev = nullptr;  // device view of the same memory
+  float* z = nullptr;
+  unsigned* counter = nullptr;
+  float* u = nullptr;  // device [k][I]
+  cudaStream_t copy_stream = nullptr;
+  cudaStream_t host_stream = nullptr;
+  std::vector<cudaEvent_t> copy_ev;
+  void* hid_dev = nullptr;
+  void* out_dev = nullptr;
+  // residency state
+  std::vector<int32_t> slot_of, gid_of;
+  std::vector<int64_t> last_use;
+  std::vector<uint8_t> in_step;
+  std::set<std::pair<int64_t, int32_t>> lru;  // resident (last_use, gid)
+  std::set<int32_t> free_slots;
+  int64_t token_step = 0;
+  int64_t route_seq = 0;
+  std::vector<moe_trace_rec> trace;
+  int64_t trace_dropped = 0;
+  moe_stats stats{};
+  std::vector<int32_t> last_idx;
+  std::vector<float> last_gate;
+  // profiling
+  bool prof = false;
+  std::vector<PendingTime> pending;
+  std::vector<cudaEvent_t> ev_pool;
+  double pc_ms[PC_N] = {0, 0, 0, 0};
+  int64_t pc_launches[PC_N] = {0, 0, 0, 0};
+  int64_t pc_bytes[PC_N] = {0, 0, 0, 0};
+  std::string err;
+};
+
+namespace {
+
+moe_status fail(moe_handle* h, moe_status st, const std::string& msg) {
+  if (h)
+    h->err = msg;
+  else
+    g_create_error = msg;
+  return st;
+}
+
+moe_status cuda_fail(moe_handle* h, cudaError_t e, const char* what) {
+  return fail(h, MOE_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+#define MOE_CK(h, call)                                          \
+  do {                                                           \
+    cudaError_t e_ = (call);                                     \
+    if (e_ != cudaSuccess) return cuda_fail((h), e_, #call);     \
+  } while (0)
+
+int64_t align_up(int64_t v, int64_t a) { return (v + a - 1) / a * a; }
+
+// Returns an error message for an invalid configuration, or "" if cfg is usable.
+std::string check_config(const moe_config* c) {
+  if (!c) return "cfg is NULL";
+  if (c->d <= 0 || c->n_experts <= 0 || c->top_k <= 0 || c->d_ff <= 0 || c->n_layers <= 0)
+    return "d, n_experts, top_k, d_ff and n_layers must be positive";
+  if (c->n_experts > 256) return "n_experts must be <= 256";
+  if (c->top_k > moe::kMaxRanks || c->top_k > c->n_experts) return "top_k must be <= 16 and <= n_experts";
+  if (c->max_batch != 1) return "max_batch must be 1 in this version";
+  if ((int64_t)c->n_layers * c->n_experts > 0x7fffffffLL) return "too many experts";
+  if (c->wdtype == MOE_DTYPE_FP32) {
+    if (c->adtype != MOE_DTYPE_FP32) return "fp32 weights need fp32 activations";
+    if (c->d % 4 || c->d_ff % 4) return "fp32 needs d and d_ff multiples of 4";
+    if (c->d > 2048) return "fp32 needs d <= 2048";
+  } else if (c->wdtype == MOE_DTYPE_BF16) {
+    if (c->adtype != MOE_DTYPE_BF16) return "bf16 weights need bf16 activations";
+    if (c->d % 8 || c->d_ff % 8) return "bf16 needs d and d_ff multiples of 8";
+    if (c->d > 4096) return "bf16 needs d <= 4096";
+  } else if (c->wdtype == MOE_DTYPE_INT4_G128) {
+    if (c->adtype != MOE_DTYPE_BF16) return "int4 weights need bf16 activations";
+    if (c->d % 128 || c->d_ff % 128) return "int4 g128 needs d and d_ff multiples of 128";
+    if (c->d > 16384) return "int4 needs d <= 16384";
+  } else {
+    return "unknown wdtype";
+  }
+  // down-projection chunks per lane (<= 8) and the u staging in shared memory
+  const int64_t eb2 = c->wdtype == MOE_DTYPE_FP32 ? 8 : c->wdtype == MOE_DTYPE_BF16 ? 4 : 1;  // 2x bytes/elem
+  if ((int64_t)c->d_ff * eb2 / 2 > 8 * 32 * 16) return "d_ff too large for the down-projection kernel";
+  const int64_t ipad = align_up(c->d_ff, 32) + 4 * (align_up(c->d_ff, 32) / 32);
+  if ((int64_t)c->top_k * ipad * 4 > 200 * 1024) return "top_k * d_ff too large for shared-memory staging";
+  if (c->renorm != 0 && c->renorm != 1) return "renorm must be 0 or 1";
+  if (c->trace_capacity < 0) return "trace_capacity must be >= 0";
+  return "";
+}
+
+int64_t slots_for(const moe_config* c, int64_t stride) {
+  int64_t cap = c->cap_slots > 0 ? c->cap_slots : (c->cap_bytes > 0 ? c->cap_bytes / stride : 0);
+  const int64_t n_gid = (int64_t)c->n_layers * c->n_experts;
+  return std::min(cap, n_gid);
+}
+
+void reset_state(moe_handle* h) {
+  std::fill(h->slot_of.begin(), h->slot_of.end(), -1);
+  std::fill(h->gid_of.begin(), h->gid_of.end(), -1);
+  std::fill(h->last_use.begin(), h->last_use.end(), -1);
+  std::fill(h->in_step.begin(), h->in_step.end(), 0);
+  h->lru.clear();
+  h->free_slots.clear();
+  for (int64_t s = 0; s < h->cap; s++) h->free_slots.insert((int32_t)s);
+  h->token_step = 0;
+  h->trace.clear();
+  h->trace_dropped = 0;
+  h->stats = moe_stats{};
+}
+
+cudaEvent_t get_event(moe_handle* h) {
+  if (!h->ev_pool.empty()) {
+    cudaEvent_t e = h->ev_pool.back();
+    h->ev_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+// Accumulate finished timing pairs (all pairs when `all`, else only those whose end event has
+// completed) and recycle their events.
+void harvest(moe_handle* h, bool all) {
+  size_t keep = 0;
+  for (size_t i = 0; i < h->pending.size(); i++) {
+    PendingTime& p = h->pending[i];
+    bool done = all ? (cudaEventSynchronize(p.b) == cudaSuccess) : (cudaEventQuery(p.b) == cudaSuccess);
+    if (!done && !all) {
+      h->pending[keep++] = p;
+      continue;
+    }
+    float ms = 0.f;
+    if (done && cudaEventElapsedTime(&ms, p.a, p.b) == cudaSuccess) {
+      h->pc_ms[p.cls] += ms;
+      h->pc_launches[p.cls] += 1;
+      h->pc_bytes[p.cls] += p.bytes;
+    }
+    h->ev_pool.push_back(p.a);
+    h->ev_pool.push_back(p.b);
+  }
+  h->pending.resize(keep);
+  cudaGetLastError();
+}
+
+struct ProfScope {
+  moe_handle* h;
+  cudaStream_t s;
+  int cls;
+  int64_t bytes;
+  cudaEvent_t a = nullptr;
+  ProfScope(moe_handle* h_, cudaStream_t s_, int cls_, int64_t bytes_) : h(h_), s(s_), cls(cls_), bytes(bytes_) {
+    if (h->prof) {
+      a = get_event(h);
+      if (a) cudaEventRecord(a, s);
+    }
+  }
+  void done() {
+    if (!a) return;
+    cudaEvent_t b = get_event(h);
+    if (!b) return;
+    cudaEventRecord(b, s);
+    h->pending.push_back(PendingTime{cls, a, b, bytes});
+    a = nullptr;
+  }
+};
+
+moe_status wait_route(moe_handle* h, int64_t seq, cudaStream_t s) {
+  const auto t0 = std::chrono::steady_clock::now();
+  uint64_t spins = 0;
+  const volatile int64_t* p = &h->route->seq;
+  for (;;) {
+    if (__atomic_load_n((const int64_t*)p, __ATOMIC_ACQUIRE) == seq) return MOE_OK;
+    if ((++spins & 4095) == 0) {
+      cudaError_t e = cudaStreamQuery(s);
+      if (e != cudaSuccess && e != cudaErrorNotReady) return cuda_fail(h, e, "device fault while waiting for routing");
+      const double dt = std::chrono::duration<double>(std::chrono::steady_clock::now() - t0).count();
+      if (dt > kWaitTimeoutS) return fail(h, MOE_ERR_TIMEOUT, "timed out waiting for the routing result");
+    }
+  }
+}
+
+moe_status launch_router(moe_handle* h, int32_t layer, const void* hidden_l, cudaStream_t s) {
+  moe::RouterArgs a{};
+  a.w = h->routers + (int64_t)layer * h->cfg.n_experts * h->cfg.d * h->router_eb;
+  a.h = hidden_l;
+  a.E = h->cfg.n_experts;
+  a.d = h->cfg.d;
+  a.k = h->cfg.top_k;
+  a.renorm = h->cfg.renorm;
+  a.wdtype = h->cfg.wdtype == MOE_DTYPE_FP32 ? moe::WD_FP32 : moe::WD_BF16;
+  a.adtype = h->cfg.adtype;
+  a.z = h->z;
+  a.counter = h->counter;
+  a.out = h->route_dev;
+  a.seq = ++h->route_seq;
+  ProfScope ps(h, s, PC_ROUTER, (int64_t)a.E * a.d * h->router_eb + (int64_t)a.d * h->asize);
+  cudaError_t e = moe::launch_router(a, s);
+  ps.done();
+  if (e != cudaSuccess) return cuda_fail(h, e, "router launch");
+  return MOE_OK;
+}
+
+struct Need {
+  int32_t gid;
+  int32_t slot;
+  bool miss;
+};
+
+// One layer-step of the lookup table: same rules as the reference definition (misses in
+// ascending gid; lowest free slot first, else the unpinned resident with the smallest
+// (last_use, gid); all needed experts pinned; last_use = clock afterwards), kept in an ordered
+// set so each decision is O(log cap).
+moe_status residency_step(moe_handle* h, int32_t layer, std::vector<Need>& needs, int64_t clock) {
+  const int32_t E = h->cfg.n_experts;
+  for (auto& n : needs) h->in_step[n.gid] = 1;
+  moe_status st = MOE_OK;
+  for (auto& n : needs) {
+    moe_trace_rec rec{(int32_t)h->token_step, layer, n.gid - layer * E, 0, 0, -1};
+    if (h->slot_of[n.gid] >= 0) {
+      n.slot = h->slot_of[n.gid];
+      n.miss = false;
+      rec.kind = 0;
+      rec.slot = n.slot;
+      h->stats.hits++;
+    } else {
+      int32_t slot = -1, victim = -1;
+      if (!h->free_slots.empty()) {
+        slot = *h->free_slots.begin();
+        h->free_slots.erase(h->free_slots.begin());
+      } else {
+        for (auto it = h->lru.begin(); it != h->lru.end(); ++it) {
+          if (!h->in_step[it->second]) {
+            victim = it->second;
+            h->lru.erase(it);
+            break;
+          }
+        }
+        if (victim < 0) {
+          st = fail(h, MOE_ERR_CAPACITY, "no evictable slot (cap below the step's working set)");
+          break;
+        }
+        slot = h->slot_of[victim];
+        h->slot_of[victim] = -1;
+        h->stats.evictions++;
+      }
+      h->gid_of[slot] = n.gid;
+      h->slot_of[n.gid] = slot;
+      n.slot = slot;
+      n.miss = true;
+      rec.kind = 1;
+      rec.slot = slot;
+      rec.evicted = victim;
+      h->stats.misses++;
+      h->stats.miss_bytes += h->lay.total;
+    }
+    if (h->cfg.trace_capacity > 0) {
+      if ((int64_t)h->trace.size() < h->cfg.trace_capacity)
+        h->trace.push_back(rec);
+      else
+        h->trace_dropped++;
+    }
+  }
+  for (auto& n : needs) {
+    h->in_step[n.gid] = 0;
+    if (st != MOE_OK) continue;
+    if (h->last_use[n.gid] >= 0 && !n.miss) h->lru.erase({h->last_use[n.gid], n.gid});
+    h->last_use[n.gid] = clock;
+    h->lru.insert({clock, n.gid});
+  }
+  return st;
+}
+
+moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_t s) {
+  const moe_config& c = h->cfg;
+  const int32_t L = c.n_layers, E = c.n_experts, k = c.top_k;
+  const int64_t act_row = (int64_t)c.d * h->asize;
+  const int64_t gu_bytes = h->lay.d_off;              // GU rows + GU scales
+  const int64_t dn_bytes = h->lay.total - h->lay.d_off;  // D rows + D scales
+  if (h->prof) harvest(h, false);
+  h->last_idx.assign((size_t)L * k, -1);
+  h->last_gate.assign((size_t)L * k, 0.f);
+  moe_status st = launch_router(h, 0, hidden, s);
+  if (st != MOE_OK) return st;
+  std::vector<Need> needs;
+  std::vector<int32_t> rank_gid(k);
+  for (int32_t l = 0; l < L; l++) {
+    const void* hid_l = (const uint8_t*)hidden + (int64_t)l * act_row;
+    st = wait_route(h, h->route_seq, s);
+    if (st != MOE_OK) return st;
+    if (h->prof) harvest(h, false);
+    // routing result of layer l
+    needs.clear();
+    const volatile int32_t* ridx = h->route->idx;
+    const volatile float* rgate = h->route->gate;
+    for (int32_t r = 0; r < k; r++) {
+      const int32_t e = ridx[r];
+      if (e < 0 || e >= E) return fail(h, MOE_ERR_INVALID, "router produced an invalid expert id (non-finite logits?)");
+      h->last_idx[(size_t)l * k + r] = e;
+      h->last_gate[(size_t)l * k + r] = rgate[r];
+      rank_gid[r] = l * E + e;
+      needs.push_back(Need{l * E + e, -1, false});
+    }
+    std::sort(needs.begin(), needs.end(), [](const Need& a, const Need& b) { return a.gid < b.gid; });
+    for (size_t i = 1; i < needs.size(); i++)
+      if (needs[i].gid == needs[i - 1].gid) return fail(h, MOE_ERR_INVALID, "router produced duplicate expert ids");
+    const int64_t clock = h->token_step * L + l;
+    st = residency_step(h, l, needs, clock);
+    if (st != MOE_OK) return st;
+    h->stats.layer_steps++;
+    // selective loads: misses in ascending gid on the copy stream
+    int n_miss = 0;
+    for (auto& n : needs) {
+      if (!n.miss) continue;
+      ProfScope ps(h, h->copy_stream, PC_COPY, h->lay.total);
+      MOE_CK(h, cudaMemcpyAsync(h->pool + (int64_t)n.slot * h->slot_stride, h->arena + (int64_t)n.gid * h->slot_stride,
+                                h->lay.total, cudaMemcpyHostToDevice, h->copy_stream));
+      ps.done();
+      MOE_CK(h, cudaEventRecord(h->copy_ev[n_miss], h->copy_stream));
+      n_miss++;
+    }
+    auto slot_ptr = [&](int32_t gid) { return h->pool + (int64_t)h->slot_of[gid] * h->slot_stride; };
+    // gate-up on the hits
+    moe::GateUpArgs ga{};
+    ga.d = c.d;
+    ga.I = c.d_ff;
+    ga.adtype = c.adtype;
+    ga.lay = h->lay;
+    ga.n_tasks = 0;
+    for (int32_t r = 0; r < k; r++) {
+      const Need* n = nullptr;
+      for (auto& x : needs)
+        if (x.gid == rank_gid[r]) n = &x;
+      if (n->miss) continue;
+      ga.t[ga.n_tasks++] = moe::GateUpTask{slot_ptr(rank_gid[r]), hid_l, h->u + (int64_t)r * c.d_ff};
+    }
+    if (ga.n_tasks > 0) {
+      ProfScope ps(h, s, PC_GATEUP, (int64_t)ga.n_tasks * gu_bytes);
+      cudaError_t e = moe::launch_gateup(ga, c.wdtype, s);
+      ps.done();
+      if (e != cudaSuccess) return cuda_fail(h, e, "gate-up launch");
+    }
+    // gate-up on each miss once its copy has landed
+    int m = 0;
+    for (auto& n : needs) {
+      if (!n.miss) continue;
+      MOE_CK(h, cudaStreamWaitEvent(s, h->copy_ev[m], 0));
+      m++;
+      ga.n_tasks = 0;
+      for (int32_t r = 0; r < k; r++)
+        if (rank_gid[r] == n.gid) ga.t[ga.n_tasks++] = moe::GateUpTask{slot_ptr(n.gid), hid_l, h->u + (int64_t)r * c.d_ff};
+      ProfScope ps(h, s, PC_GATEUP, (int64_t)ga.n_tasks * gu_bytes);
+      cudaError_t e = moe::launch_gateup(ga, c.wdtype, s);
+      ps.done();
+      if (e != cudaSuccess) return cuda_fail(h, e, "gate-up launch");
+    }
+    // down projection + rank-ordered combine
+    moe::DownArgs da{};
+    da.k = k;
+    da.d = c.d;
+    da.I = c.d_ff;
+    da.adtype = c.adtype;
+    da.lay = h->lay;
+    for (int32_t r = 0; r < k; r++) {
+      da.blob[r] = slot_ptr(rank_gid[r]);
+      da.gate[r] = h->last_gate[(size_t)l * k + r];
+    }
+    da.u = h->u;
+    da.out = (uint8_t*)out + (int64_t)l * act_row;
+    {
+      ProfScope ps(h, s, PC_DOWN, (int64_t)k * dn_bytes);
+      cudaError_t e = moe::launch_down_combine(da, c.wdtype, s);
+      ps.done();
+      if (e != cudaSuccess) return cuda_fail(h, e, "down/combine launch");
+    }
+    if (l + 1 < L) {
+      st = launch_router(h, l + 1, (const uint8_t*)hidden + (int64_t)(l + 1) * act_row, s);
+      if (st != MOE_OK) return st;
+    }
+  }
+  h->token_step++;
+  h->stats.steps++;
+  return MOE_OK;
+}
+
+void free_all(moe_handle* h) {
+  if (!h) return;
+  cudaDeviceSynchronize();
+  harvest(h, true);
+  for (auto e : h->ev_pool) cudaEventDestroy(e);
+  for (auto e : h->copy_ev) cudaEventDestroy(e);
+  if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
+  if (h->host_stream) cudaStreamDestroy(h->host_stream);
+  if (h->own_pool && h->pool) cudaFree(h->pool);
+  if (h->arena) cudaFreeHost(h->arena);
+  if (h->routers) cudaFree(h->routers);
+  if (h->route) cudaFreeHost(h->route);
+  if (h->z) cudaFree(h->z);
+  if (h->counter) cudaFree(h->counter);
+  if (h->u) cudaFree(h->u);
+  if (h->hid_dev) cudaFree(h->hid_dev);
+  if (h->out_dev) cudaFree(h->out_dev);
+  cudaGetLastError();
+  delete h;
+}
+
+}  // namespace
+
+extern "C" {
+
+int64_t moe_expert_bytes(const moe_config* cfg) {
+  if (!check_config(cfg).empty()) return -1;
+  return moe::make_layout(cfg->wdtype, cfg->d, cfg->d_ff).total;
+}
+
+int64_t moe_pool_bytes(const moe_config* cfg) {
+  if (!check_config(cfg).empty()) return -1;
+  const int64_t stride = align_up(moe::make_layout(cfg->wdtype, cfg->d, cfg->d_ff).total, 256);
+  return slots_for(cfg, stride) * stride;
+}
+
+moe_status moe_create(const moe_config* cfg, moe_handle** out) {
+  if (!out) return fail(nullptr, MOE_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  std::string why = check_config(cfg);
+  if (!why.empty()) return fail(nullptr, MOE_ERR_INVALID, why);
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || cfg->device < 0 || cfg->device >= ndev) {
+    cudaGetLastError();
+    return fail(nullptr, MOE_ERR_CUDA, "no such CUDA device");
+  }
+  if (cudaSetDevice(cfg->device) != cudaSuccess) return fail(nullptr, MOE_ERR_CUDA, "cudaSetDevice failed");
+  moe_handle* h = new moe_handle();
+  h->cfg = *cfg;
+  h->lay = moe::make_layout(cfg->wdtype, cfg->d, cfg->d_ff);
+  h->slot_stride = align_up(h->lay.total, 256);
+  h->n_gid = (int64_t)cfg->n_layers * cfg->n_experts;
+  h->cap = slots_for(cfg, h->slot_stride);
+  h->asize = cfg->adtype == MOE_DTYPE_FP32 ? 4 : 2;
+  h->router_eb = cfg->wdtype == MOE_DTYPE_FP32 ? 4 : 2;
+  const int64_t need = std::min<int64_t>(cfg->n_experts, (int64_t)cfg->top_k * cfg->max_batch);
+  if (h->cap < need) {
+    char buf[160];
+    snprintf(buf, sizeof buf, "cap of %lld slots is below one layer-step's working set of %lld experts",
+             (long long)h->cap, (long long)need);
+    delete h;
+    return fail(nullptr, MOE_ERR_CAPACITY, buf);
+  }
+  auto bail = [&](moe_status st, const std::string& msg) {
+    free_all(h);
+    return fail(nullptr, st, msg);
+  };
+  if (cfg->device_pool) {
+    if ((uintptr_t)cfg->device_pool % 256) return bail(MOE_ERR_INVALID, "device_pool must be 256-byte aligned");
+    h->pool = (uint8_t*)cfg->device_pool;
+  } else {
+    if (cudaMalloc(&h->pool, h->cap * h->slot_stride) != cudaSuccess) {
+      h->pool = nullptr;
+      return bail(MOE_ERR_OOM, "device slot pool allocation failed");
+    }
+    h->own_pool = true;
+  }
+  if (cudaHostAlloc(&h->arena, h->n_gid * h->slot_stride, cudaHostAllocDefault) != cudaSuccess) {
+    h->arena = nullptr;
+    return bail(MOE_ERR_OOM, "pinned host arena allocation failed");
+  }
+  const int64_t rbytes = (int64_t)cfg->n_layers * cfg->n_experts * cfg->d * h->router_eb;
+  if (cudaMalloc(&h->routers, rbytes) != cudaSuccess) return bail(MOE_ERR_OOM, "router allocation failed");
+  if (cudaHostAlloc(&h->route, sizeof(moe::RouteOut), cudaHostAllocMapped) != cudaSuccess)
+    return bail(MOE_ERR_OOM, "mapped routing buffer allocation failed");
+  memset((void*)h->route, 0, sizeof(moe::RouteOut));
+  h->route->seq = 0;
+  if (cudaHostGetDevicePointer((void**)&h->route_dev, (void*)h->route, 0) != cudaSuccess)
+    return bail(MOE_ERR_CUDA, "mapped routing buffer has no device address");
+  if (cudaMalloc(&h->z, sizeof(float) * 256) != cudaSuccess) return bail(MOE_ERR_OOM, "z allocation failed");
+  if (cudaMalloc(&h->counter, sizeof(unsigned)) != cudaSuccess) return bail(MOE_ERR_OOM, "counter allocation failed");
+  if (cudaMemset(h->counter, 0, sizeof(unsigned)) != cudaSuccess) return bail(MOE_ERR_CUDA, "memset failed");
+  if (cudaMalloc(&h->u, sizeof(float) * cfg->top_k * cfg->d_ff) != cudaSuccess) return bail(MOE_ERR_OOM, "u allocation failed");
+  const int64_t act = (int64_t)cfg->n_layers * cfg->max_batch * cfg->d * h->asize;
+  if (cudaMalloc(&h->hid_dev, act) != cudaSuccess || cudaMalloc(&h->out_dev, act) != cudaSuccess)
+    return bail(MOE_ERR_OOM, "staging allocation failed");
+  if (cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&h->host_stream, cudaStreamNonBlocking) != cudaSuccess)
+    return bail(MOE_ERR_CUDA, "stream creation failed");
+  h->copy_ev.resize((size_t)cfg->top_k * cfg->max_batch, nullptr);
+  for (auto& e : h->copy_ev)
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
+  h->registered.assign(h->n_gid, 0);
+  h->router_set.assign(cfg->n_layers, 0);
+  h->slot_of.assign(h->n_gid, -1);
+  h->gid_of.assign(h->cap, -1);
+  h->last_use.assign(h->n_gid, -1);
+  h->in_step.assign(h->n_gid, 0);
+  if (cfg->trace_capacity > 0) h->trace.reserve((size_t)std::min<int64_t>(cfg->trace_capacity, 1 << 22));
+  reset_state(h);
+  *out = h;
+  return MOE_OK;
+}
+
+moe_status moe_set_router(moe_handle* h, int32_t layer, const void* w_r) {
+  if (!h) return MOE_ERR_INVALID;
+  if (layer < 0 || layer >= h->cfg.n_layers || !w_r) return fail(h, MOE_ERR_INVALID, "bad layer or NULL weights");
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  const int64_t bytes = (int64_t)h->cfg.n_experts * h->cfg.d * h->router_eb;
+  MOE_CK(h, cudaMemcpy(h->routers + layer * bytes, w_r, bytes, cudaMemcpyHostToDevice));
+  h->router_set[layer] = 1;
+  h->all_registered = false;
+  return MOE_OK;
+}
+
+moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t expert, const void* w_gate,
+                                     const void* w_up, const void* w_down, const void* scales) {
+  if (!h) return MOE_ERR_INVALID;
+  const moe_config& c = h->cfg;
+  if (layer < 0 || layer >= c.n_layers || expert < 0 || expert >= c.n_experts)
+    return fail(h, MOE_ERR_INVALID, "bad layer or expert id");
+  if (!w_gate || !w_up || !w_down) return fail(h, MOE_ERR_INVALID, "NULL weight pointer");
+  const bool q4 = c.wdtype == MOE_DTYPE_INT4_G128;
+  if (q4 != (scales != nullptr)) return fail(h, MOE_ERR_INVALID, "scales must be given exactly for int4 weights");
+  const int64_t gid = (int64_t)layer * c.n_experts + expert;
+  uint8_t* dst = h->arena + gid * h->slot_stride;
+  const moe::BlobLayout& L = h->lay;
+  const int64_t rb = L.row_bytes_gu;
+  const uint8_t* g = (const uint8_t*)w_gate;
+  const uint8_t* u = (const uint8_t*)w_up;
+  for (int64_t i = 0; i < c.d_ff; i++) {
+    memcpy(dst + i * 2 * rb, g + i * rb, rb);
+    memcpy(dst + i * 2 * rb + rb, u + i * rb, rb);
+  }
+  memcpy(dst + L.d_off, w_down, (size_t)(c.d * L.row_bytes_d));
+  if (q4) {
+    const int64_t G = c.d / 128;
+    const uint16_t* s = (const uint16_t*)scales;
+    uint16_t* gs = (uint16_t*)(dst + L.gu_scale_off);
+    for (int64_t i = 0; i < c.d_ff; i++) {
+      memcpy(gs + i * 2 * G, s + i * G, G * 2);
+      memcpy(gs + i * 2 * G + G, s + c.d_ff * G + i * G, G * 2);
+    }
+    memcpy(dst + L.d_scale_off, s + 2 * c.d_ff * G, (size_t)(c.d * (c.d_ff / 128) * 2));
+  }
+  if (h->slot_stride > L.total) memset(dst + L.total, 0, h->slot_stride - L.total);
+  h->registered[gid] = 1;
+  return MOE_OK;
+}
+
+moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t batch, void* stream) {
+  if (!h) return MOE_ERR_INVALID;
+  if (!hidden || !out) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
+  if (batch != 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be 1 in this version");
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  if (!h->all_registered) {
+    for (int32_t l = 0; l < h->cfg.n_layers; l++)
+      if (!h->router_set[l]) return fail(h, MOE_ERR_NOT_REGISTERED, "router of layer " + std::to_string(l) + " not set");
+    for (int64_t g = 0; g < h->n_gid; g++)
+      if (!h->registered[g])
+        return fail(h, MOE_ERR_NOT_REGISTERED, "expert " + std::to_string(g % h->cfg.n_experts) + " of layer " +
+                                                   std::to_string(g / h->cfg.n_experts) + " not registered");
+    h->all_registered = true;
+  }
+  moe_status st = decode_impl(h, hidden, out, (cudaStream_t)stream);
+  if (st != MOE_OK) {
+    // The pool contents are unknown after a failed step: wait for the streams, empty the pool.
+    std::string keep = h->err;
+    cudaStreamSynchronize((cudaStream_t)stream);
+    cudaStreamSynchronize(h->copy_stream);
+    cudaMemset(h->counter, 0, sizeof(unsigned));
+    cudaGetLastError();
+    reset_state(h);
+    h->err = keep;
+  }
+  return st;
+}
+
+moe_status moe_decode_step_host(moe_handle* h, const void* hidden_host, void* out_host, int32_t batch) {
+  if (!h) return MOE_ERR_INVALID;
+  if (!hidden_host || !out_host) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
+  if (batch != 1) return fail(h, MOE_ERR_INVALID, "batch must be 1 in this version");
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  const int64_t bytes = (int64_t)h->cfg.n_layers * batch * h->cfg.d * h->asize;
+  MOE_CK(h, cudaMemcpyAsync(h->hid_dev, hidden_host, bytes, cudaMemcpyHostToDevice, h->host_stream));
+  moe_status st = moe_decode_step(h, h->hid_dev, h->out_dev, batch, h->host_stream);
+  if (st != MOE_OK) return st;
+  MOE_CK(h, cudaMemcpyAsync(out_host, h->out_dev, bytes, cudaMemcpyDeviceToHost, h->host_stream));
+  MOE_CK(h, cudaStreamSynchronize(h->host_stream));
+  return MOE_OK;
+}
+
+moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* buf, int64_t cap, int64_t* n_copied,
+                                   int64_t* n_total) {
+  if (!h) return MOE_ERR_INVALID;
+  if (start < 0 || cap < 0 || (cap > 0 && !buf)) return fail(h, MOE_ERR_INVALID, "bad trace range");
+  const int64_t tot = (int64_t)h->trace.size();
+  const int64_t n = std::max<int64_t>(0, std::min(cap, tot - start));
+  if (n > 0) memcpy(buf, h->trace.data() + start, (size_t)n * sizeof(moe_trace_rec));
+  if (n_copied) *n_copied = n;
+  if (n_total) *n_total = tot;
+  if (h->trace_dropped > 0) return fail(h, MOE_ERR_TRACE_OVERFLOW, "trace buffer full: records were dropped");
+  return MOE_OK;
+}
+
+moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_t n) {
+  if (!h) return MOE_ERR_INVALID;
+  if (n < (int64_t)h->last_idx.size()) return fail(h, MOE_ERR_INVALID, "routing buffer too small");
+  if (idx) memcpy(idx, h->last_idx.data(), h->last_idx.size() * sizeof(int32_t));
+  if (gate) memcpy(gate, h->last_gate.data(), h->last_gate.size() * sizeof(float));
+  return MOE_OK;
+}
+
+moe_status moe_get_stats(moe_handle* h, moe_stats* out) {
+  if (!h || !out) return MOE_ERR_INVALID;
+  *out = h->stats;
+  return MOE_OK;
+}
+
+moe_status moe_reset_residency(moe_handle* h) {
+  if (!h) return MOE_ERR_INVALID;
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  MOE_CK(h, cudaDeviceSynchronize());
+  reset_state(h);
+  return MOE_OK;
+}
+
+moe_status moe_profile_enable(moe_handle* h, int32_t on) {
+  if (!h) return MOE_ERR_INVALID;
+  h->prof = on != 0;
+  return MOE_OK;
+}
+
+moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, int32_t* n_out) {
+  if (!h || (cap > 0 && !out)) return MOE_ERR_INVALID;
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  harvest(h, true);
+  int32_t n = 0;
+  for (int c = 0; c < PC_N && n < cap; c++, n++) {
+    memset(&out[n], 0, sizeof(moe_kernel_time));
+    snprintf(out[n].name, sizeof out[n].name, "%s", kPcName[c]);
+    out[n].launches = h->pc_launches[c];
+    out[n].total_ms = h->pc_ms[c];
+    out[n].bytes = h->pc_bytes[c];
+    h->pc_launches[c] = 0;
+    h->pc_ms[c] = 0;
+    h->pc_bytes[c] = 0;
+  }
+  if (n_out) *n_out = n;
+  return MOE_OK;
+}
+
+const char* moe_last_error(const moe_handle* h) { return h ? h->err.c_str() : g_create_error.c_str(); }
+
+void moe_destroy(moe_handle* h) {
+  if (!h) return;
+  cudaSetDevice(h->cfg.device);
+  free_all(h);
+}
+
+}  // extern "C"

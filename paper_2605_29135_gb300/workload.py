@@ -1,0 +1,48 @@
+"""Load a seeded synthetic workload (``synth``) into a library handle.
+
+Router weights go to the device; every expert is generated and registered into the pinned
+host tier in parallel (the ctypes calls release the GIL, so generation and repacking run on
+all host cores).
+"""
+from __future__ import annotations
+
+import os
+import threading
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+from . import MoE, make_config
+
+
+def config_for(wl, cap_slots=None, device=0, trace_capacity=1 << 22, renorm=True):
+    return make_config(wl.d, wl.n_experts, wl.top_k, wl.d_ff, wl.n_layers, wl.wdtype, wl.adtype,
+                       cap_slots=wl.cap_slots if cap_slots is None else cap_slots, renorm=renorm, device=device,
+                       max_batch=wl.batch, trace_capacity=trace_capacity)
+
+
+def create_for_workload(wl, cap_slots=None, device=0, trace_capacity=1 << 22, threads=None) -> MoE:
+    import synth
+
+    m = MoE(config_for(wl, cap_slots, device, trace_capacity))
+    try:
+        for layer in range(wl.n_layers):
+            m.set_router(layer, synth.router_weights(wl, layer))
+        local = threading.local()
+
+        def one(job):
+            layer, e = job
+            tmp = getattr(local, "tmp", None)
+            if tmp is None:
+                tmp = local.tmp = np.empty(wl.d * wl.d_ff, dtype=np.float32)
+            w = synth.expert_weights(wl, layer, e, tmp)
+            m.register_host_experts(layer, e, w.gate, w.up, w.down, w.scales_flat())
+
+        jobs = [(layer, e) for layer in range(wl.n_layers) for e in range(wl.n_experts)]
+        with ThreadPoolExecutor(max_workers=threads or os.cpu_count()) as ex:
+            for _ in ex.map(one, jobs):
+                pass
+    except BaseException:
+        m.destroy()
+        raise
+    return m

@@ -1,0 +1,76 @@
+"""The C-ABI library builds, loads and exports every function include/moe.h declares (CPU only:
+no compute call is made without a GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "moe.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(moe_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2605_29135_gb300 import _lib
+    from paper_2605_29135_gb300.build import build
+
+    build()
+    return _lib.load()
+
+
+def test_header_declares_the_binding_exports():
+    from paper_2605_29135_gb300 import _lib
+
+    assert _declared() == sorted(_lib.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared():
+        assert hasattr(lib, name), name
+        assert isinstance(getattr(lib, name), ctypes._CFuncPtr)
+
+
+def test_config_struct_layout_matches_header(lib):
+    from paper_2605_29135_gb300._lib import MoeConfig, TraceRec
+
+    # int32 x6, int32 x2, int64 x2, int32 x2, pointer, int64 (natural alignment)
+    assert ctypes.sizeof(MoeConfig) == 6 * 4 + 2 * 4 + 2 * 8 + 2 * 4 + 8 + 8
+    assert ctypes.sizeof(TraceRec) == 24
+
+
+def test_expert_and_pool_bytes_without_gpu(lib):
+    import paper_2605_29135_gb300 as P
+
+    c = P.make_config(2048, 128, 8, 768, 48, "bf16", "bf16", cap_bytes=6_000_000_000)
+    assert P.expert_bytes(c) == 9_437_184
+    assert P.pool_bytes(c) == 635 * 9_437_184
+    c4 = P.make_config(2048, 128, 8, 768, 48, "int4", "bf16", cap_bytes=6_000_000_000)
+    assert P.expert_bytes(c4) == 2_433_024
+    assert P.pool_bytes(c4) == 2466 * 2_433_024
+    c1 = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4)
+    assert P.expert_bytes(c1) == 393_216
+    bad = P.make_config(250, 8, 2, 128, 1, "int4", "bf16", cap_slots=4)
+    assert P.expert_bytes(bad) == -1
+
+
+def test_invalid_config_is_rejected_before_touching_a_device(lib):
+    import paper_2605_29135_gb300 as P
+
+    bad = P.make_config(256, 8, 9, 128, 1, "fp32", "fp32", cap_slots=4)  # top_k > E
+    h = ctypes.c_void_p()
+    st = lib.moe_create(ctypes.byref(bad), ctypes.byref(h))
+    assert st == -1 and not h.value
+    assert b"top_k" in lib.moe_last_error(None)
+
+
+def test_null_handle_calls_fail_cleanly(lib):
+    assert lib.moe_decode_step(None, None, None, 1, None) == -1
+    assert lib.moe_reset_residency(None) == -1
+    lib.moe_destroy(None)
