@@ -62,6 +62,18 @@ enum {
   MOE_DTYPE_INT4_G128 = 2 /* symmetric int4, groups of 128 along the input dim, bf16 scales */
 };
 
+/* How a decode step is scheduled (both compute the same results and the same residency trace).
+ *   MOE_SCHEDULE_DEVICE: one cooperative persistent kernel per decode step runs every layer. The
+ *     lookup table lives in device memory and is updated by the kernel; a missed expert is
+ *     streamed from the page-locked host tier over the host link by the warps that use it,
+ *     stored into its freed slot and used in the same pass, concurrently with the hit experts'
+ *     compute. moe_decode_step returns right after the launch (fully asynchronous).
+ *   MOE_SCHEDULE_HOST_COPY_ENGINE: per layer, the routing result is published to mapped host
+ *     memory, the host updates the lookup table and issues one cudaMemcpyAsync per miss on an
+ *     internal copy stream; the hit experts' kernels run while the copies are in flight and
+ *     each missed expert's kernels wait for its copy. moe_decode_step blocks once per layer. */
+enum { MOE_SCHEDULE_DEVICE = 0, MOE_SCHEDULE_HOST_COPY_ENGINE = 1 };
+
 typedef struct {
   int32_t d;          /* hidden size */
   int32_t n_experts;  /* experts per layer, E (<= 256) */
@@ -77,7 +89,11 @@ typedef struct {
   int32_t device;     /* CUDA device ordinal */
   void* device_pool;  /* optional caller-owned device buffer of >= moe_pool_bytes(cfg) bytes, 256-B aligned;
                          NULL => the library allocates the pool */
-  int64_t trace_capacity; /* residency records kept on the host; 0 disables the trace */
+  int64_t trace_capacity; /* residency records kept (device buffer for MOE_SCHEDULE_DEVICE, host otherwise);
+                             0 disables the trace */
+  int32_t schedule;       /* MOE_SCHEDULE_DEVICE (default) or MOE_SCHEDULE_HOST_COPY_ENGINE */
+  int32_t miss_ctas;      /* MOE_SCHEDULE_DEVICE: CTAs that stream missed experts over the host link
+                             while the others compute the hits (0: library default) */
 } moe_config;
 
 /* One residency record: a requested expert's outcome in one layer-step. */
@@ -137,12 +153,18 @@ moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t exper
 
 /* One decode step over all layers. hidden: device [n_layers x batch x d] (adtype), the input
  * of every layer; out: device [n_layers x batch x d] (adtype). Work is ordered on `stream`
- * (a cudaStream_t; NULL = legacy default stream). Host-driven: the call blocks once per layer
- * until that layer's routing result has reached the host (bounded wait, MOE_ERR_TIMEOUT), and
- * returns once the last layer's work is enqueued. hidden must stay valid and out must not be
+ * (a cudaStream_t; NULL = legacy default stream). hidden must stay valid and out must not be
  * read until `stream` reaches the end of the step. Calls on one handle must use one stream or
- * be serialised by the caller. If a CUDA call fails mid-step the residency state is reset
- * (empty pool) and MOE_ERR_CUDA is returned. */
+ * be serialised by the caller.
+ *   MOE_SCHEDULE_DEVICE: enqueues one kernel and returns. A failure detected on the device
+ *     (a grid barrier that timed out, an invalid routing result) is reported by the next call
+ *     on the handle that synchronises (decode_step, get_stats, get_residency_trace, ...), as
+ *     MOE_ERR_TIMEOUT or MOE_ERR_CUDA, and empties the pool.
+ *   MOE_SCHEDULE_HOST_COPY_ENGINE: blocks once per layer until that layer's routing result has
+ *     reached the host (bounded wait, MOE_ERR_TIMEOUT) and returns once the last layer's work
+ *     is enqueued.
+ * If a CUDA call fails mid-step the residency state is reset (empty pool) and MOE_ERR_CUDA is
+ * returned. */
 moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t batch, void* stream);
 
 /* moe_decode_step on host buffers (pinned or pageable): copies hidden to the device, runs the

@@ -15,7 +15,7 @@ import ctypes
 import numpy as np
 
 from . import _lib
-from ._lib import DTYPE, STATUS, KernelTime, MoeConfig, Stats, TraceRec
+from ._lib import DTYPE, SCHEDULE, STATUS, KernelTime, MoeConfig, Stats, TraceRec
 
 TRACE_DTYPE = np.dtype([("step", np.int32), ("layer", np.int32), ("expert", np.int32), ("kind", np.int32),
                         ("slot", np.int32), ("evicted", np.int32)])
@@ -28,11 +28,12 @@ class MoEError(RuntimeError):
 
 
 def make_config(d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots=0, cap_bytes=0, renorm=True,
-                device=0, max_batch=1, trace_capacity=1 << 22, device_pool=None) -> MoeConfig:
+                device=0, max_batch=1, trace_capacity=1 << 22, device_pool=None, schedule="device",
+                miss_ctas=0) -> MoeConfig:
     return MoeConfig(d=d, n_experts=n_experts, top_k=top_k, d_ff=d_ff, n_layers=n_layers, max_batch=max_batch,
                      wdtype=DTYPE[wdtype], adtype=DTYPE[adtype], cap_slots=cap_slots, cap_bytes=cap_bytes,
                      renorm=1 if renorm else 0, device=device, device_pool=device_pool,
-                     trace_capacity=trace_capacity)
+                     trace_capacity=trace_capacity, schedule=SCHEDULE[schedule], miss_ctas=miss_ctas)
 
 
 def expert_bytes(cfg: MoeConfig) -> int:
@@ -126,9 +127,9 @@ class MoE:
         self._check(self.lib.moe_profile_enable(self.h, 1 if on else 0))
 
     def profile_read(self) -> dict:
-        arr = (KernelTime * 8)()
+        arr = (KernelTime * 16)()
         n = ctypes.c_int32()
-        self._check(self.lib.moe_profile_read(self.h, arr, 8, ctypes.byref(n)))
+        self._check(self.lib.moe_profile_read(self.h, arr, 16, ctypes.byref(n)))
         return {arr[i].name.decode(): {"launches": arr[i].launches, "total_ms": arr[i].total_ms,
                                        "bytes": arr[i].bytes} for i in range(n.value)}
 

@@ -1,0 +1,646 @@
+// Device-driven decode step (sm_103a): one cooperative persistent kernel per decode step.
+//
+// Per layer, four phases separated by grid barriers:
+//   R  router logits z = W_r h, one warp per expert row;
+//   S  CTA 0: top-k (ties -> lower id) and gates, then one step of the lookup table: hits keep
+//      their slot, misses (ascending global id) take the lowest free slot, else the unpinned
+//      resident with the smallest (last use, global id); records go to the trace buffer and the
+//      per-rank plan (slot, miss flag, gate) to global memory;
+//   C  gate-up rows of every rank, u_r[i] = silu(W_g[i] . h) * (W_u[i] . h). A few "miss CTAs"
+//      stream every missed expert from the page-locked host tier over NVLink-C2C: its gate/up
+//      rows are stored into the freed slot and used for u in the same pass, and its W_d region
+//      is copied into the slot; the other CTAs compute the hit experts' rows from HBM at the
+//      same time. Capping the warps that read the host tier keeps the link's outstanding
+//      requests near what saturates it (tens of warps, not thousands);
+//   D  down rows + combine from the slots, out[o] = sum_r g_r (W_d^(r)[o] . u_r) in rank order.
+//
+// All CTAs are co-resident (cooperative launch). Every barrier wait is bounded by a timeout on
+// the global timer; on expiry the kernel sets an error flag and every CTA returns.
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "dev.cuh"
+#include "fused.cuh"
+
+namespace moe {
+namespace {
+
+using namespace dev;
+
+constexpr int kFWarps = 8;
+constexpr int kFThreads = kFWarps * 32;
+
+__device__ __forceinline__ uint64_t gtimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Grid-wide barrier over co-resident CTAs with a bounded wait. Returns false once any CTA has
+// timed out (the caller then returns).
+__device__ bool grid_sync(const FusedArgs& a) {
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile unsigned* genp = a.bar_gen;
+    const unsigned g = *genp;
+    __threadfence();
+    const unsigned arrived = atomicAdd(a.bar_count, 1u) + 1u;
+    if (arrived == gridDim.x) {
+      atomicExch(a.bar_count, 0u);
+      __threadfence();
+      atomicAdd(a.bar_gen, 1u);
+    } else {
+      const uint64_t t0 = gtimer();
+      while (*genp == g) {
+        if (*(volatile int*)a.err & FERR_BARRIER_TIMEOUT) break;
+        if (gtimer() - t0 > a.barrier_timeout_ns) {
+          atomicOr(a.err, FERR_BARRIER_TIMEOUT);
+          break;
+        }
+        __nanosleep(32);
+      }
+    }
+    __threadfence();
+  }
+  __syncthreads();
+  return (*(volatile int*)a.err & FERR_BARRIER_TIMEOUT) == 0;
+}
+
+__device__ __forceinline__ unsigned long long shfl_min_u64(unsigned long long v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const unsigned long long o = __shfl_xor_sync(kFull, v, off);
+    v = o < v ? o : v;
+  }
+  return v;
+}
+
+// Phase S, run by CTA 0 (all its threads).
+__device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t step) {
+  __shared__ int s_idx[kMaxRanks];
+  __shared__ float s_gate[kMaxRanks];
+  __shared__ int s_need[kMaxRanks];   // needed global ids, ascending
+  __shared__ int s_slot[kMaxRanks];   // slot per needed id (after the step)
+  __shared__ int s_miss[kMaxRanks];
+  __shared__ int s_evict[kMaxRanks];  // evicted global id per needed id, -1 if none
+  __shared__ int s_vslot[kMaxRanks];  // victim slots in ascending (last use, id)
+  __shared__ int s_nev;
+  __shared__ unsigned long long s_red[kFWarps];
+  const int k = a.k, E = a.E;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+  if (warp == 0) {
+    constexpr int PER = 8;  // E <= 256
+    uint32_t key[PER];
+#pragma unroll
+    for (int j = 0; j < PER; j++) {
+      const int e = j * 32 + lane;
+      key[j] = e < E ? ord_key(__ldcg(a.z + e)) : 0u;
+    }
+    float my_z = 0.f;
+    int my_i = -1;
+    for (int r = 0; r < k; r++) {
+      uint32_t bk = 0u;
+      int bi = 0x7fffffff;
+#pragma unroll
+      for (int j = 0; j < PER; j++) {
+        if (key[j] > bk) {
+          bk = key[j];
+          bi = j * 32 + lane;
+        }
+      }
+      const uint32_t mk = __reduce_max_sync(kFull, bk);
+      const int win = (int)__reduce_min_sync(kFull, bk == mk ? (uint32_t)bi : 0xffffffffu);
+      if (lane == r) {
+        my_z = key_value(mk);
+        my_i = win;
+      }
+#pragma unroll
+      for (int j = 0; j < PER; j++)
+        if (win == j * 32 + lane) key[j] = 0u;
+    }
+    const float m = __shfl_sync(kFull, my_z, 0);
+    const float ex = lane < k ? expf(my_z - m) : 0.f;
+    float denom;
+    if (a.renorm) {
+      denom = warp_sum(ex);
+    } else {
+      float part = 0.f;
+      for (int e = lane; e < E; e += 32) part += expf(__ldcg(a.z + e) - m);
+      denom = warp_sum(part);
+    }
+    if (lane < k) {
+      if (my_i < 0 || my_i >= E) {
+        atomicOr(a.err, FERR_BAD_ROUTE);
+        my_i = lane;  // keep the step well-defined; the host reports the error
+      }
+      s_idx[lane] = my_i;
+      s_gate[lane] = ex / denom;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int r = 0; r < k; r++) s_need[r] = l * E + s_idx[r];
+    for (int r = 1; r < k; r++) {  // insertion sort, k <= 16
+      const int v = s_need[r];
+      int j = r - 1;
+      while (j >= 0 && s_need[j] > v) {
+        s_need[j + 1] = s_need[j];
+        j--;
+      }
+      s_need[j + 1] = v;
+    }
+    // hits keep their slot; misses in ascending id take free slots [n_used, cap) first
+    int n_used = *a.n_used;
+    int nev = 0;
+    for (int t = 0; t < k; t++) {
+      const int sl = a.slot_of[s_need[t]];
+      s_miss[t] = sl < 0;
+      s_slot[t] = sl;
+      s_evict[t] = -1;
+      if (sl < 0) {
+        if (n_used < a.cap) {
+          s_slot[t] = n_used++;
+        } else {
+          nev++;
+        }
+      }
+    }
+    *a.n_used = n_used;
+    s_nev = nev;
+  }
+  __syncthreads();
+  // Victims: the s_nev smallest slot keys (last use, id) among occupied slots that hold no
+  // expert of this step. Free slots carry ~0 and are never picked while a real key remains.
+  for (int j = 0; j < s_nev; j++) {
+    unsigned long long best = ~0ull;
+    for (int64_t sl = threadIdx.x; sl < a.cap; sl += blockDim.x) {
+      bool skip = false;
+      for (int t = 0; t < k; t++) skip |= (s_slot[t] == sl);  // hits (pinned); misses are not yet placed
+      for (int t = 0; t < j; t++) skip |= (s_vslot[t] == sl);
+      if (skip) continue;
+      const unsigned long long key = a.slot_key[sl];
+      best = key < best ? key : best;
+    }
+    best = shfl_min_u64(best);
+    if (lane == 0) s_red[warp] = best;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned long long b = s_red[0];
+      for (int w = 1; w < kFWarps; w++) b = s_red[w] < b ? s_red[w] : b;
+      if (b == ~0ull) {
+        atomicOr(a.err, FERR_NO_VICTIM);
+        s_vslot[j] = -1;
+      } else {
+        s_vslot[j] = a.slot_of[(int)(uint32_t)(b & 0xffffffffull)];
+      }
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    int j = 0;
+    unsigned long long hits = 0, misses = 0, evictions = 0;
+    for (int t = 0; t < k; t++) {
+      const int g = s_need[t];
+      if (!s_miss[t]) {
+        hits++;
+        continue;
+      }
+      misses++;
+      if (s_slot[t] < 0) {  // needs a victim
+        const int vs = s_vslot[j++];
+        if (vs >= 0) {
+          const int v = (int)(uint32_t)(a.slot_key[vs] & 0xffffffffull);
+          a.slot_of[v] = -1;
+          s_slot[t] = vs;
+          s_evict[t] = v;
+          evictions++;
+        }
+      }
+      if (s_slot[t] >= 0) a.slot_of[g] = s_slot[t];
+    }
+    for (int t = 0; t < k; t++)
+      if (s_slot[t] >= 0) a.slot_key[s_slot[t]] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)s_need[t];
+    const unsigned long long base = *a.trace_n;
+    for (int t = 0; t < k; t++) {
+      if (base + t < (unsigned long long)a.trace_cap) {
+        TraceRec rec;
+        rec.step = (int32_t)step;
+        rec.layer = l;
+        rec.expert = s_need[t] - l * E;
+        rec.kind = s_miss[t];
+        rec.slot = s_slot[t];
+        rec.evicted = s_evict[t];
+        a.trace[base + t] = rec;
+      }
+    }
+    *a.trace_n = base + k;
+    a.stats[STAT_HITS] += hits;
+    a.stats[STAT_MISSES] += misses;
+    a.stats[STAT_EVICTIONS] += evictions;
+    a.stats[STAT_LAYER_STEPS] += 1;
+    for (int r = 0; r < k; r++) {
+      const int g = l * E + s_idx[r];
+      int t = 0;
+      while (s_need[t] != g) t++;
+      a.plan_slot[r] = s_slot[t] < 0 ? 0 : s_slot[t];
+      a.plan_gid[r] = g;
+      a.plan_miss[r] = s_miss[t];
+      a.plan_gate[r] = s_gate[r];
+      a.route_idx[l * k + r] = s_idx[r];
+      a.route_gate[l * k + r] = s_gate[r];
+    }
+  }
+}
+
+// Copy n bf16 values (scales) from src to dst with 2-byte accesses, one per lane.
+__device__ __forceinline__ void copy_scales(uint16_t* dst, const uint16_t* src, int n, int lane) {
+  for (int j = lane; j < n; j += 32) dst[j] = __ldg(src + j);
+}
+
+template <int WD>
+__device__ __forceinline__ float scale_at(const uint16_t* p, bool from_host) {
+  return bf16_bits(from_host ? __ldg(p) : __ldcg(p));
+}
+
+// One gate/up row pair of rank r: reads it from `src` (the host tier for a miss, the slot for a
+// hit), stores it into `slot` when it came from the host tier, and writes
+// u_r[i] = silu(W_g[i] . x) * (W_u[i] . x) with x staged in shared memory.
+template <int WD, int CH>
+__device__ __forceinline__ void gateup_row(const FusedArgs& a, const uint8_t* src, uint8_t* slot, bool from_host,
+                                           const uint8_t* xs, int r, int i, int lane) {
+  const int64_t rb = a.lay.row_bytes_gu;
+  const int nch = (int)(rb / 16);
+  const int G = a.d / 128;
+  const int64_t goff = (int64_t)i * 2 * rb;
+  uint4 wg[CH], wu[CH];
+#pragma unroll
+  for (int j = 0; j < CH; j++) {
+    const int c = j * 32 + lane;
+    if (c < nch) {
+      if (from_host) {
+        wg[j] = ld_stream(src + goff + (int64_t)c * 16);
+        wu[j] = ld_stream(src + goff + rb + (int64_t)c * 16);
+      } else {
+        wg[j] = ld_cg(src + goff + (int64_t)c * 16);
+        wu[j] = ld_cg(src + goff + rb + (int64_t)c * 16);
+      }
+    } else {
+      wg[j] = make_uint4(0, 0, 0, 0);
+      wu[j] = make_uint4(0, 0, 0, 0);
+    }
+  }
+  float sg[CH], su[CH];
+  if (WD == WD_INT4) {
+    const uint16_t* sp = (const uint16_t*)(src + a.lay.gu_scale_off) + (int64_t)i * 2 * G;
+#pragma unroll
+    for (int j = 0; j < CH; j++) {
+      const int c = j * 32 + lane;
+      sg[j] = c < nch ? scale_at<WD>(sp + (c >> 2), from_host) : 0.f;
+      su[j] = c < nch ? scale_at<WD>(sp + G + (c >> 2), from_host) : 0.f;
+    }
+    if (from_host) copy_scales((uint16_t*)(slot + a.lay.gu_scale_off) + (int64_t)i * 2 * G, sp, 2 * G, lane);
+  }
+  if (from_host) {
+#pragma unroll
+    for (int j = 0; j < CH; j++) {
+      const int c = j * 32 + lane;
+      if (c < nch) {
+        st_v4(slot + goff + (int64_t)c * 16, wg[j]);
+        st_v4(slot + goff + rb + (int64_t)c * 16, wu[j]);
+      }
+    }
+  }
+  float ag = 0.f, au = 0.f;
+#pragma unroll
+  for (int j = 0; j < CH; j++) {
+    const int c = j * 32 + lane;
+    if (c < nch) {
+      const uint8_t* xc = xs + (int64_t)c * Tr<WD>::xbytes;
+      if (WD == WD_INT4) {
+        ag = fmaf(sg[j], dot_chunk<WD>(wg[j], xc, 0.f), ag);
+        au = fmaf(su[j], dot_chunk<WD>(wu[j], xc, 0.f), au);
+      } else {
+        ag = dot_chunk<WD>(wg[j], xc, ag);
+        au = dot_chunk<WD>(wu[j], xc, au);
+      }
+    }
+  }
+  ag = warp_sum(ag);
+  au = warp_sum(au);
+  if (lane == 0) a.u[(int64_t)r * a.I + i] = ag / (1.0f + expf(-ag)) * au;
+}
+
+// Phase D rows (all experts in their slots) for one value of the chunks-per-lane count of a W_d row.
+template <int WD, int CHD>
+__device__ void down_rows(const FusedArgs& a, const float* us, const int* pslot, const float* pgate, int l, int gw,
+                          int W) {
+  constexpr int E = Tr<WD>::epc;
+  constexpr int KR = 24 / CHD > 8 ? 8 : (24 / CHD < 1 ? 1 : 24 / CHD);
+  const int lane = threadIdx.x & 31;
+  const int64_t rb = a.lay.row_bytes_d;
+  const int nch = (int)(rb / 16);
+  const int G = a.I / 128;
+  const int ipad = ipad_of(a.I);
+  for (int o = gw; o < a.d; o += W) {
+    float acc = 0.f;
+    for (int r0 = 0; r0 < a.k; r0 += KR) {
+      uint4 w[KR][CHD];
+      float sc[KR][CHD];
+#pragma unroll
+      for (int rr = 0; rr < KR; rr++) {
+        const int r = r0 + rr;
+        const bool rok = r < a.k;  // a predicate, not a break: keeps w[][] in registers
+        const uint8_t* slot = a.pool + (int64_t)pslot[rok ? r : 0] * a.slot_stride;
+        const int64_t roff = a.lay.d_off + (int64_t)o * rb;
+#pragma unroll
+        for (int j = 0; j < CHD; j++) {
+          const int c = j * 32 + lane;
+          w[rr][j] = (rok && c < nch) ? ld_cg(slot + roff + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+        }
+        if (WD == WD_INT4) {
+          const uint16_t* sp = (const uint16_t*)(slot + a.lay.d_scale_off) + (int64_t)o * G;
+#pragma unroll
+          for (int j = 0; j < CHD; j++) {
+            const int c = j * 32 + lane;
+            sc[rr][j] = (rok && c < nch) ? scale_at<WD>(sp + (c >> 2), false) : 0.f;
+          }
+        }
+      }
+#pragma unroll
+      for (int rr = 0; rr < KR; rr++) {
+        const int r = r0 + rr;
+        if (r >= a.k) continue;
+        const float* ur = us + r * ipad;
+        float part = 0.f;
+#pragma unroll
+        for (int j = 0; j < CHD; j++) {
+          const int c = j * 32 + lane;
+          if (c < nch) {
+            if (WD == WD_INT4)
+              part = fmaf(sc[rr][j], dot_chunk_u<WD>(w[rr][j], ur + upad(c * E), 0.f), part);
+            else
+              part = dot_chunk_u<WD>(w[rr][j], ur + upad(c * E), part);
+          }
+        }
+        acc = fmaf(pgate[r], part, acc);
+      }
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) {
+      if (WD == WD_FP32)
+        reinterpret_cast<float*>(a.out)[(int64_t)l * a.d + o] = acc;
+      else
+        reinterpret_cast<__nv_bfloat16*>(a.out)[(int64_t)l * a.d + o] = __float2bfloat16_rn(acc);
+    }
+  }
+}
+
+template <int WD, int CH>
+__global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ FusedArgs a) {
+  extern __shared__ uint4 smem4[];
+  __shared__ int p_slot[kMaxRanks], p_gid[kMaxRanks], p_miss[kMaxRanks];
+  __shared__ float p_gate[kMaxRanks];
+  __shared__ int p_mr[kMaxRanks], p_hr[kMaxRanks], p_nm, p_nh;  // miss / hit ranks of this layer-step
+  const int asize = WD == WD_FP32 ? 4 : 2;
+  const int xbytes = a.d * asize;
+  uint8_t* xs = reinterpret_cast<uint8_t*>(smem4);
+  float* us = reinterpret_cast<float*>(xs + ((xbytes + 15) & ~15));
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * kFWarps + (threadIdx.x >> 5);
+  const int W = gridDim.x * kFWarps;
+  const int64_t step = *(volatile int64_t*)a.step;
+  const int nchr = xbytes / 16;  // router rows: fp32 with fp32 weights, else bf16 (same bytes as h)
+  const int ipad = ipad_of(a.I);
+  int chd_need = (int)((a.lay.row_bytes_d / 16 + 31) / 32);
+  if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[a.L * 4] = gtimer();
+
+  for (int l = 0; l < a.L; l++) {
+    const int clock = (int)(step * a.L + l);
+    // ---- phase R: router logits
+    stage16(reinterpret_cast<uint4*>(xs), (const uint8_t*)a.hidden + (int64_t)l * xbytes, xbytes, threadIdx.x,
+            blockDim.x);
+    __syncthreads();
+    for (int e = gw; e < a.E; e += W) {
+      const uint8_t* row = a.routers + ((int64_t)l * a.E + e) * xbytes;
+      float acc = 0.f;
+      for (int c = lane; c < nchr; c += 32) {
+        if (WD == WD_FP32)
+          acc = dot_chunk<WD_FP32>(ld_stream(row + (int64_t)c * 16), xs + (int64_t)c * 16, acc);
+        else
+          acc = dot_chunk<WD_BF16>(ld_stream(row + (int64_t)c * 16), xs + (int64_t)c * 16, acc);
+      }
+      acc = warp_sum(acc);
+      if (lane == 0) a.z[e] = acc;
+    }
+    if (!grid_sync(a)) return;
+    if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 0] = gtimer();
+    // ---- phase S: selection and lookup table (CTA 0)
+    if (blockIdx.x == 0) select_and_lookup(a, l, clock, step);
+    if (!grid_sync(a)) return;
+    if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 1] = gtimer();
+    if (threadIdx.x < a.k) {
+      p_slot[threadIdx.x] = __ldcg(a.plan_slot + threadIdx.x);
+      p_gid[threadIdx.x] = __ldcg(a.plan_gid + threadIdx.x);
+      p_miss[threadIdx.x] = __ldcg(a.plan_miss + threadIdx.x);
+      p_gate[threadIdx.x] = __ldcg(a.plan_gate + threadIdx.x);
+    }
+    __syncthreads();
+    // ---- phase C: gate-up rows; miss CTAs stream the missed experts into their slots
+    if (threadIdx.x == 0) {
+      int nm = 0, nh = 0;
+      for (int r = 0; r < a.k; r++) {
+        if (p_miss[r])
+          p_mr[nm++] = r;
+        else
+          p_hr[nh++] = r;
+      }
+      p_nm = nm;
+      p_nh = nh;
+    }
+    __syncthreads();
+    const int nm = p_nm, nh = p_nh;
+    // Warm the host-link address translations of every missed expert before streaming it: one
+    // L2 prefetch per page-sized stride, issued by every thread of the grid at once. Without it
+    // the streaming warps meet each page's translation miss one after another as they advance
+    // through the expert, and the link idles while the translations resolve.
+    if (nm > 0) {
+      const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
+      const int64_t gt0 = (int64_t)blockIdx.x * kFThreads + threadIdx.x;
+      const int64_t GT = (int64_t)gridDim.x * kFThreads;
+      for (int64_t q = gt0; q < (int64_t)nm * pages; q += GT) {
+        const int m = (int)(q / pages);
+        const uint8_t* pa = a.arena + (int64_t)p_gid[p_mr[m]] * a.slot_stride + ((q - (int64_t)m * pages) << a.touch_shift);
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+      }
+    }
+    const int mctas = nm > 0 ? (a.miss_ctas < (int)gridDim.x - 1 ? a.miss_ctas : (int)gridDim.x - 1) : 0;
+    const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;  // the last CTAs (CTA 0 leads phase S)
+    if (miss_cta) {
+      const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
+      const int MW = mctas * kFWarps;
+      // gate/up rows of every missed expert: host -> slot, and u from the same registers
+      for (int p = mw; p < nm * a.I; p += MW) {
+        const int r = p_mr[p / a.I];
+        const int i = p - (p / a.I) * a.I;
+        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
+        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride;
+        gateup_row<WD, CH>(a, src, slot, true, xs, r, i, lane);
+      }
+      // W_d rows (and int4 scales) of every missed expert: a plain copy host -> slot
+      const int64_t dbytes = a.lay.total - a.lay.d_off;  // multiple of 16
+      const int64_t nq = dbytes / 16;
+      const int mt = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFThreads + threadIdx.x;
+      const int MT = mctas * kFThreads;
+      for (int m = 0; m < nm; m++) {
+        const int r = p_mr[m];
+        uint8_t* dst = a.pool + (int64_t)p_slot[r] * a.slot_stride + a.lay.d_off;
+        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride + a.lay.d_off;
+        int64_t q = mt;
+        for (; q + 3 * (int64_t)MT < nq; q += 4 * (int64_t)MT) {
+          const uint4 v0 = ld_stream(src + q * 16);
+          const uint4 v1 = ld_stream(src + (q + MT) * 16);
+          const uint4 v2 = ld_stream(src + (q + 2 * (int64_t)MT) * 16);
+          const uint4 v3 = ld_stream(src + (q + 3 * (int64_t)MT) * 16);
+          st_v4(dst + q * 16, v0);
+          st_v4(dst + (q + MT) * 16, v1);
+          st_v4(dst + (q + 2 * (int64_t)MT) * 16, v2);
+          st_v4(dst + (q + 3 * (int64_t)MT) * 16, v3);
+        }
+        for (; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
+      }
+    } else {
+      const int hw = (int)blockIdx.x * kFWarps + (threadIdx.x >> 5);
+      const int HW = ((int)gridDim.x - mctas) * kFWarps;
+      for (int p = hw; p < nh * a.I; p += HW) {
+        const int r = p_hr[p / a.I];
+        const int i = p - (p / a.I) * a.I;
+        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
+        gateup_row<WD, CH>(a, slot, slot, false, xs, r, i, lane);
+      }
+    }
+    if (!grid_sync(a)) return;
+    if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 2] = gtimer();
+    // ---- phase D: down rows + combine (missed experts' W_d streamed into their slots)
+    {
+      const float4* u4 = reinterpret_cast<const float4*>(a.u);
+      const int n4 = a.k * a.I / 4;
+      for (int q = threadIdx.x; q < n4; q += blockDim.x) {
+        const float4 v = __ldcg(u4 + q);
+        const int r = (4 * q) / a.I;
+        const int i = 4 * q - r * a.I;
+        *reinterpret_cast<float4*>(us + r * ipad + upad(i)) = v;
+      }
+    }
+    __syncthreads();
+    switch (chd_need) {
+      case 1: down_rows<WD, 1>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 2: down_rows<WD, 2>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 3: down_rows<WD, 3>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 4: down_rows<WD, 4>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 5:
+      case 6: down_rows<WD, 6>(a, us, p_slot, p_gate, l, gw, W); break;
+      default: down_rows<WD, 8>(a, us, p_slot, p_gate, l, gw, W); break;
+    }
+    if (!grid_sync(a)) return;
+    if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 3] = gtimer();
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
+}
+
+size_t fused_smem(int wdtype, int d, int I, int k) {
+  const int xbytes = d * (wdtype == WD_FP32 ? 4 : 2);
+  return (size_t)((xbytes + 15) & ~15) + (size_t)k * ipad_of(I) * sizeof(float);
+}
+
+template <int WD, int CH>
+int grid_of(size_t smem) {
+  static int occ = -1;
+  static size_t occ_smem = 0;
+  if (occ < 0 || occ_smem != smem) {
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(k_fused<WD, CH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    int o = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, k_fused<WD, CH>, kFThreads, smem) != cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    occ = o;
+    occ_smem = smem;
+  }
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms * (occ < 2 ? occ : 2);
+}
+
+template <int WD, int CH>
+cudaError_t run_fused(const FusedArgs& a, int grid, cudaStream_t s) {
+  const size_t smem = fused_smem(a.wdtype, a.d, a.I, a.k);
+  void* params[] = {(void*)&a};
+  return cudaLaunchCooperativeKernel((const void*)k_fused<WD, CH>, dim3(grid), dim3(kFThreads), params, smem, s);
+}
+
+int pick_ch_f(int64_t rb) {
+  const int need = (int)((rb / 16 + 31) / 32);
+  if (need <= 1) return 1;
+  if (need <= 2) return 2;
+  if (need <= 4) return 4;
+  if (need <= 8) return 8;
+  if (need <= 16) return 16;
+  return -1;
+}
+
+}  // namespace
+
+#define MOE_F_DISPATCH(FN, WDV, CHV, ...)                          \
+  do {                                                             \
+    switch (WDV) {                                                 \
+      case WD_FP32:                                                \
+        switch (CHV) {                                             \
+          case 1: return FN<WD_FP32, 1>(__VA_ARGS__);              \
+          case 2: return FN<WD_FP32, 2>(__VA_ARGS__);              \
+          case 4: return FN<WD_FP32, 4>(__VA_ARGS__);              \
+          case 8: return FN<WD_FP32, 8>(__VA_ARGS__);              \
+        }                                                          \
+        break;                                                     \
+      case WD_BF16:                                                \
+        switch (CHV) {                                             \
+          case 1: return FN<WD_BF16, 1>(__VA_ARGS__);              \
+          case 2: return FN<WD_BF16, 2>(__VA_ARGS__);              \
+          case 4: return FN<WD_BF16, 4>(__VA_ARGS__);              \
+          case 8: return FN<WD_BF16, 8>(__VA_ARGS__);              \
+          case 16: return FN<WD_BF16, 16>(__VA_ARGS__);            \
+        }                                                          \
+        break;                                                     \
+      case WD_INT4:                                                \
+        switch (CHV) {                                             \
+          case 1: return FN<WD_INT4, 1>(__VA_ARGS__);              \
+          case 2: return FN<WD_INT4, 2>(__VA_ARGS__);              \
+          case 4: return FN<WD_INT4, 4>(__VA_ARGS__);              \
+          case 8: return FN<WD_INT4, 8>(__VA_ARGS__);              \
+        }                                                          \
+        break;                                                     \
+    }                                                              \
+  } while (0)
+
+int fused_grid(int wdtype, int d, int I, int k) {
+  const BlobLayout lay = make_layout(wdtype, d, I);
+  const int ch = pick_ch_f(lay.row_bytes_gu);
+  const size_t smem = fused_smem(wdtype, d, I, k);
+  if (smem > 200 * 1024) return 0;
+  MOE_F_DISPATCH(grid_of, wdtype, ch, smem);
+  return 0;
+}
+
+cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s) {
+  const int ch = pick_ch_f(a.lay.row_bytes_gu);
+  MOE_F_DISPATCH(run_fused, a.wdtype, ch, a, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace moe

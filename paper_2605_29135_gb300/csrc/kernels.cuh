@@ -7,7 +7,7 @@
 //   [D rows]    W_d rows o = 0..d-1 (I elements each)
 //   [D scales]  int4 only: W_d scales, row-major [d x I/128] bf16
 // Element storage: fp32, bf16, or int4 (two's-complement nibbles, element 2j in the low nibble
-// of byte j of its row).
+// of byte j of its row). Activations are fp32 with fp32 weights and bf16 otherwise.
 #pragma once
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -27,32 +27,27 @@ struct BlobLayout {
 
 BlobLayout make_layout(int wdtype, int64_t d, int64_t I);
 
-constexpr int kMaxGateUpTasks = 16;
 constexpr int kMaxRanks = 16;
 
-struct GateUpTask {
-  const uint8_t* blob;  // expert image in its slot
-  const void* x;        // input vector [d] (adtype)
-  float* u;             // output [I] fp32
-};
-
+// u_t = silu(W_g x) * (W_u x) for the experts in blob[0..n_tasks), all on the same input x.
 struct GateUpArgs {
   int n_tasks;
   int d, I;
-  int adtype;  // 0 fp32, 1 bf16
   BlobLayout lay;
-  GateUpTask t[kMaxGateUpTasks];
+  const void* x;                   // [d] activations (fp32 with fp32 weights, else bf16)
+  const uint8_t* blob[kMaxRanks];  // expert images in their slots
+  float* u[kMaxRanks];             // outputs [I] fp32
 };
 
+// out = sum_r gate[r] * (W_d^(r) u_r), ranks in order.
 struct DownArgs {
   int k;
   int d, I;
-  int adtype;
   BlobLayout lay;
   const uint8_t* blob[kMaxRanks];  // expert images in rank order
   float gate[kMaxRanks];
   const float* u;                  // [k x I] fp32, rank-major
-  void* out;                       // [d] adtype
+  void* out;                       // [d] activations
 };
 
 // Routing result as written by the router kernel into host-mapped memory.
@@ -64,12 +59,10 @@ struct RouteOut {
 
 struct RouterArgs {
   const void* w;      // W_r [E x d] device (fp32 or bf16)
-  const void* h;      // hidden [d] (adtype)
+  const void* h;      // hidden [d]
   int E, d, k, renorm;
-  int wdtype, adtype;
-  float* z;           // [E] scratch
-  unsigned* counter;  // zero-initialised; reset by the last CTA
-  RouteOut* out;      // host-mapped
+  int wdtype;         // WD_FP32 or WD_BF16
+  RouteOut* out;      // device address of host-mapped memory
   int64_t seq;
 };
 

@@ -10,27 +10,38 @@
 // runs after every kernel of layers < l on the compute stream, so no earlier reader of a
 // victim slot can still be running, and experts needed by layer l are pinned for the step.
 #include <cuda_runtime.h>
+#include <sys/mman.h>
 
 #include <algorithm>
 #include <chrono>
 #include <cstdio>
 #include <cstring>
 #include <set>
+#include <thread>
 #include <string>
 #include <utility>
 #include <vector>
 
+#include "fused.cuh"
 #include "kernels.cuh"
 #include "moe.h"
 
 namespace {
 
 constexpr double kWaitTimeoutS = 20.0;
+// CTAs of the fused kernel that stream missed experts: enough warps to keep the host link's
+// bandwidth-delay product in flight, few enough not to flood it with outstanding requests.
+constexpr int kDefaultMissCtas = 24;
 
 thread_local std::string g_create_error;
 
-enum { PC_ROUTER = 0, PC_GATEUP = 1, PC_DOWN = 2, PC_COPY = 3, PC_N = 4 };
-const char* kPcName[PC_N] = {"router", "gateup", "down_combine", "miss_copy"};
+enum {
+  PC_ROUTER = 0, PC_GATEUP = 1, PC_DOWN = 2, PC_COPY = 3, PC_FUSED = 4,
+  PC_PH_R = 5, PC_PH_S = 6, PC_PH_C = 7, PC_PH_D = 8, PC_N = 9
+};
+const char* kPcName[PC_N] = {"router", "gateup", "down_combine", "miss_copy", "fused_step",
+                             "fused_phase_router", "fused_phase_select", "fused_phase_gateup",
+                             "fused_phase_down"};
 
 struct PendingTime {
   int cls;
@@ -51,14 +62,13 @@ struct moe_handle {
   uint8_t* pool = nullptr;   // device slot pool
   bool own_pool = false;
   uint8_t* arena = nullptr;  // pinned host tier, one slot image per global expert id
+  size_t arena_bytes = 0;
   std::vector<uint8_t> registered;
   std::vector<uint8_t> router_set;
   bool all_registered = false;
   uint8_t* routers = nullptr;  // device [L][E][d]
   moe::RouteOut* route = nullptr;      // mapped pinned (host view)
   moe::RouteOut* route_dev = nullptr;  // device view of the same memory
-  float* z = nullptr;
-  unsigned* counter = nullptr;
   float* u = nullptr;  // device [k][I]
   cudaStream_t copy_stream = nullptr;
   cudaStream_t host_stream = nullptr;
@@ -82,9 +92,34 @@ struct moe_handle {
   bool prof = false;
   std::vector<PendingTime> pending;
   std::vector<cudaEvent_t> ev_pool;
-  double pc_ms[PC_N] = {0, 0, 0, 0};
-  int64_t pc_launches[PC_N] = {0, 0, 0, 0};
-  int64_t pc_bytes[PC_N] = {0, 0, 0, 0};
+  double pc_ms[PC_N] = {};
+  int64_t pc_launches[PC_N] = {};
+  int64_t pc_bytes[PC_N] = {};
+  unsigned long long* d_phase_ts = nullptr;   // [L*4+1] per-phase timestamps of the last profiled step
+  std::vector<unsigned long long> h_phase_ts;
+  // device-driven schedule: lookup table, scratch and outputs in device memory
+  bool dev_mode = false;
+  int fgrid = 0;
+  int touch_shift = 12;
+  const uint8_t* arena_dev = nullptr;
+  int32_t* d_slot_of = nullptr;
+  unsigned long long* d_slot_key = nullptr;
+  int32_t* d_n_used = nullptr;
+  int64_t* d_step = nullptr;
+  float* d_z = nullptr;
+  int32_t* d_plan = nullptr;  // slot[k], gid[k], miss[k]
+  float* d_plan_gate = nullptr;
+  moe::TraceRec* d_trace = nullptr;
+  unsigned long long* d_trace_n = nullptr;
+  int32_t* d_route_idx = nullptr;
+  float* d_route_gate = nullptr;
+  unsigned long long* d_stats = nullptr;
+  unsigned* d_bar = nullptr;  // count, generation
+  int* d_err = nullptr;
+  int* h_err = nullptr;       // pinned copy of d_err after each step
+  cudaEvent_t err_ev = nullptr;
+  bool err_pending = false;
+  int64_t steps_launched = 0;
   std::string err;
 };
 
@@ -141,6 +176,8 @@ std::string check_config(const moe_config* c) {
   if ((int64_t)c->top_k * ipad * 4 > 200 * 1024) return "top_k * d_ff too large for shared-memory staging";
   if (c->renorm != 0 && c->renorm != 1) return "renorm must be 0 or 1";
   if (c->trace_capacity < 0) return "trace_capacity must be >= 0";
+  if (c->schedule != MOE_SCHEDULE_DEVICE && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "unknown schedule";
+  if (c->miss_ctas < 0) return "miss_ctas must be >= 0";
   return "";
 }
 
@@ -150,7 +187,24 @@ int64_t slots_for(const moe_config* c, int64_t stride) {
   return std::min(cap, n_gid);
 }
 
+void reset_device_state(moe_handle* h) {
+  if (!h->dev_mode) return;
+  cudaMemset(h->d_slot_of, 0xff, sizeof(int32_t) * h->n_gid);
+  cudaMemset(h->d_slot_key, 0xff, sizeof(unsigned long long) * h->cap);
+  cudaMemset(h->d_n_used, 0, sizeof(int32_t));
+  cudaMemset(h->d_step, 0, sizeof(int64_t));
+  cudaMemset(h->d_trace_n, 0, sizeof(unsigned long long));
+  cudaMemset(h->d_stats, 0, sizeof(unsigned long long) * moe::STAT_N);
+  cudaMemset(h->d_bar, 0, sizeof(unsigned) * 2);
+  cudaMemset(h->d_err, 0, sizeof(int));
+  cudaDeviceSynchronize();
+  *h->h_err = 0;
+  h->err_pending = false;
+  h->steps_launched = 0;
+}
+
 void reset_state(moe_handle* h) {
+  reset_device_state(h);
   std::fill(h->slot_of.begin(), h->slot_of.end(), -1);
   std::fill(h->gid_of.begin(), h->gid_of.end(), -1);
   std::fill(h->last_use.begin(), h->last_use.end(), -1);
@@ -245,9 +299,6 @@ moe_status launch_router(moe_handle* h, int32_t layer, const void* hidden_l, cud
   a.k = h->cfg.top_k;
   a.renorm = h->cfg.renorm;
   a.wdtype = h->cfg.wdtype == MOE_DTYPE_FP32 ? moe::WD_FP32 : moe::WD_BF16;
-  a.adtype = h->cfg.adtype;
-  a.z = h->z;
-  a.counter = h->counter;
   a.out = h->route_dev;
   a.seq = ++h->route_seq;
   ProfScope ps(h, s, PC_ROUTER, (int64_t)a.E * a.d * h->router_eb + (int64_t)a.d * h->asize);
@@ -380,15 +431,17 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     moe::GateUpArgs ga{};
     ga.d = c.d;
     ga.I = c.d_ff;
-    ga.adtype = c.adtype;
     ga.lay = h->lay;
+    ga.x = hid_l;
     ga.n_tasks = 0;
     for (int32_t r = 0; r < k; r++) {
       const Need* n = nullptr;
       for (auto& x : needs)
         if (x.gid == rank_gid[r]) n = &x;
       if (n->miss) continue;
-      ga.t[ga.n_tasks++] = moe::GateUpTask{slot_ptr(rank_gid[r]), hid_l, h->u + (int64_t)r * c.d_ff};
+      ga.blob[ga.n_tasks] = slot_ptr(rank_gid[r]);
+      ga.u[ga.n_tasks] = h->u + (int64_t)r * c.d_ff;
+      ga.n_tasks++;
     }
     if (ga.n_tasks > 0) {
       ProfScope ps(h, s, PC_GATEUP, (int64_t)ga.n_tasks * gu_bytes);
@@ -403,8 +456,12 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       MOE_CK(h, cudaStreamWaitEvent(s, h->copy_ev[m], 0));
       m++;
       ga.n_tasks = 0;
-      for (int32_t r = 0; r < k; r++)
-        if (rank_gid[r] == n.gid) ga.t[ga.n_tasks++] = moe::GateUpTask{slot_ptr(n.gid), hid_l, h->u + (int64_t)r * c.d_ff};
+      for (int32_t r = 0; r < k; r++) {
+        if (rank_gid[r] != n.gid) continue;
+        ga.blob[ga.n_tasks] = slot_ptr(n.gid);
+        ga.u[ga.n_tasks] = h->u + (int64_t)r * c.d_ff;
+        ga.n_tasks++;
+      }
       ProfScope ps(h, s, PC_GATEUP, (int64_t)ga.n_tasks * gu_bytes);
       cudaError_t e = moe::launch_gateup(ga, c.wdtype, s);
       ps.done();
@@ -415,7 +472,6 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     da.k = k;
     da.d = c.d;
     da.I = c.d_ff;
-    da.adtype = c.adtype;
     da.lay = h->lay;
     for (int32_t r = 0; r < k; r++) {
       da.blob[r] = slot_ptr(rank_gid[r]);
@@ -439,6 +495,141 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
   return MOE_OK;
 }
 
+// The host tier: anonymous memory advised for transparent huge pages, first touched by all
+// host cores, then page-locked with cudaHostRegister. Huge pages keep the copy engine's
+// address translations few when misses hit random experts of a tens-of-GB arena.
+moe_status alloc_arena(moe_handle* h) {
+  const size_t bytes = (size_t)(h->n_gid * h->slot_stride);
+  void* p = mmap(nullptr, bytes, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS | MAP_NORESERVE, -1, 0);
+  if (p == MAP_FAILED) return fail(h, MOE_ERR_OOM, "host arena mmap failed");
+  madvise(p, bytes, MADV_HUGEPAGE);
+  unsigned nt = std::thread::hardware_concurrency();
+  if (nt < 1) nt = 1;
+  if (nt > 64) nt = 64;
+  std::vector<std::thread> th;
+  for (unsigned t = 0; t < nt; t++)
+    th.emplace_back([=] {
+      const size_t a = bytes / nt * t, b = t + 1 == nt ? bytes : bytes / nt * (t + 1);
+      memset((uint8_t*)p + a, 0, b - a);
+    });
+  for (auto& x : th) x.join();
+  cudaError_t e = cudaHostRegister(p, bytes, cudaHostRegisterMapped);
+  if (e != cudaSuccess) {
+    munmap(p, bytes);
+    cudaGetLastError();
+    return fail(h, MOE_ERR_OOM, std::string("cudaHostRegister of the host arena failed: ") + cudaGetErrorString(e));
+  }
+  h->arena = (uint8_t*)p;
+  h->arena_bytes = bytes;
+  return MOE_OK;
+}
+
+// Device-driven schedule: report a failure flagged by an earlier fused step. With sync, waits for
+// all work and reads the live flag; otherwise reads the copy taken after the last completed step.
+// A flagged failure empties the pool and clears the flag.
+moe_status check_device_error(moe_handle* h, bool sync) {
+  if (!h->dev_mode) return MOE_OK;
+  int e = 0;
+  if (sync) {
+    cudaError_t ce = cudaDeviceSynchronize();
+    if (ce != cudaSuccess) return cuda_fail(h, ce, "decode step");
+    ce = cudaMemcpy(&e, h->d_err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (ce != cudaSuccess) return cuda_fail(h, ce, "reading the device error flag");
+  } else if (h->err_pending && cudaEventQuery(h->err_ev) == cudaSuccess) {
+    e = *(volatile int*)h->h_err;
+  }
+  cudaGetLastError();
+  if (e == 0) return MOE_OK;
+  std::string msg = "decode step failed on the device:";
+  if (e & moe::FERR_BARRIER_TIMEOUT) msg += " a grid barrier timed out;";
+  if (e & moe::FERR_BAD_ROUTE) msg += " the router produced an invalid expert id (non-finite logits?);";
+  if (e & moe::FERR_NO_VICTIM) msg += " no evictable slot;";
+  msg += " the pool was emptied";
+  reset_state(h);
+  return fail(h, (e & moe::FERR_BARRIER_TIMEOUT) ? MOE_ERR_TIMEOUT : MOE_ERR_CUDA, msg);
+}
+
+moe_status decode_device(moe_handle* h, const void* hidden, void* out, cudaStream_t s) {
+  moe_status st = check_device_error(h, false);
+  if (st != MOE_OK) return st;
+  const moe_config& c = h->cfg;
+  const int k = c.top_k;
+  moe::FusedArgs a{};
+  a.L = c.n_layers;
+  a.E = c.n_experts;
+  a.k = k;
+  a.d = c.d;
+  a.I = c.d_ff;
+  a.renorm = c.renorm;
+  a.wdtype = c.wdtype;
+  a.lay = h->lay;
+  a.slot_stride = h->slot_stride;
+  a.cap = h->cap;
+  a.routers = h->routers;
+  a.hidden = hidden;
+  a.out = out;
+  a.pool = h->pool;
+  a.arena = h->arena_dev;
+  a.slot_of = h->d_slot_of;
+  a.slot_key = h->d_slot_key;
+  a.n_used = h->d_n_used;
+  a.step = h->d_step;
+  a.z = h->d_z;
+  a.plan_slot = h->d_plan;
+  a.plan_gid = h->d_plan + k;
+  a.plan_miss = h->d_plan + 2 * k;
+  a.plan_gate = h->d_plan_gate;
+  a.u = h->u;
+  a.trace = h->d_trace;
+  a.trace_cap = c.trace_capacity;
+  a.trace_n = h->d_trace_n;
+  a.route_idx = h->d_route_idx;
+  a.route_gate = h->d_route_gate;
+  a.stats = h->d_stats;
+  a.bar_count = h->d_bar;
+  a.bar_gen = h->d_bar + 1;
+  a.err = h->d_err;
+  a.barrier_timeout_ns = 2000000000ull;
+  a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
+  a.touch_shift = h->touch_shift;
+  a.phase_ts = nullptr;
+  if (h->prof) {
+    if (!h->d_phase_ts && cudaMalloc(&h->d_phase_ts, sizeof(unsigned long long) * (4 * c.n_layers + 1)) != cudaSuccess) {
+      h->d_phase_ts = nullptr;
+      cudaGetLastError();
+    }
+    a.phase_ts = h->d_phase_ts;
+  }
+  {
+    ProfScope ps(h, s, PC_FUSED,
+                 (int64_t)c.n_layers * (k * h->lay.total + (int64_t)c.n_experts * c.d * h->router_eb));
+    cudaError_t e = moe::launch_fused(a, h->fgrid, s);
+    ps.done();
+    if (e != cudaSuccess) return cuda_fail(h, e, "fused decode step launch");
+  }
+  MOE_CK(h, cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, s));
+  MOE_CK(h, cudaEventRecord(h->err_ev, s));
+  h->err_pending = true;
+  h->steps_launched++;
+  if (a.phase_ts) {
+    // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
+    const int L = c.n_layers;
+    h->h_phase_ts.resize(4 * L + 1);
+    MOE_CK(h, cudaMemcpyAsync(h->h_phase_ts.data(), a.phase_ts, sizeof(unsigned long long) * (4 * L + 1),
+                              cudaMemcpyDeviceToHost, s));
+    MOE_CK(h, cudaStreamSynchronize(s));
+    unsigned long long prev = h->h_phase_ts[4 * L];
+    for (int l = 0; l < L; l++)
+      for (int p = 0; p < 4; p++) {
+        const unsigned long long t = h->h_phase_ts[4 * l + p];
+        h->pc_ms[PC_PH_R + p] += (double)(t - prev) * 1e-6;
+        h->pc_launches[PC_PH_R + p] += 1;
+        prev = t;
+      }
+  }
+  return MOE_OK;
+}
+
 void free_all(moe_handle* h) {
   if (!h) return;
   cudaDeviceSynchronize();
@@ -448,12 +639,20 @@ void free_all(moe_handle* h) {
   if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   if (h->host_stream) cudaStreamDestroy(h->host_stream);
   if (h->own_pool && h->pool) cudaFree(h->pool);
-  if (h->arena) cudaFreeHost(h->arena);
+  if (h->arena) {
+    cudaHostUnregister(h->arena);
+    munmap(h->arena, h->arena_bytes);
+  }
   if (h->routers) cudaFree(h->routers);
   if (h->route) cudaFreeHost(h->route);
-  if (h->z) cudaFree(h->z);
-  if (h->counter) cudaFree(h->counter);
   if (h->u) cudaFree(h->u);
+  for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_n_used,
+                  (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
+                  (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
+                  (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts})
+    if (p) cudaFree(p);
+  if (h->h_err) cudaFreeHost(h->h_err);
+  if (h->err_ev) cudaEventDestroy(h->err_ev);
   if (h->hid_dev) cudaFree(h->hid_dev);
   if (h->out_dev) cudaFree(h->out_dev);
   cudaGetLastError();
@@ -516,9 +715,9 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     }
     h->own_pool = true;
   }
-  if (cudaHostAlloc(&h->arena, h->n_gid * h->slot_stride, cudaHostAllocDefault) != cudaSuccess) {
-    h->arena = nullptr;
-    return bail(MOE_ERR_OOM, "pinned host arena allocation failed");
+  {
+    moe_status ast = alloc_arena(h);
+    if (ast != MOE_OK) return bail(ast, h->err);
   }
   const int64_t rbytes = (int64_t)cfg->n_layers * cfg->n_experts * cfg->d * h->router_eb;
   if (cudaMalloc(&h->routers, rbytes) != cudaSuccess) return bail(MOE_ERR_OOM, "router allocation failed");
@@ -528,9 +727,6 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   h->route->seq = 0;
   if (cudaHostGetDevicePointer((void**)&h->route_dev, (void*)h->route, 0) != cudaSuccess)
     return bail(MOE_ERR_CUDA, "mapped routing buffer has no device address");
-  if (cudaMalloc(&h->z, sizeof(float) * 256) != cudaSuccess) return bail(MOE_ERR_OOM, "z allocation failed");
-  if (cudaMalloc(&h->counter, sizeof(unsigned)) != cudaSuccess) return bail(MOE_ERR_OOM, "counter allocation failed");
-  if (cudaMemset(h->counter, 0, sizeof(unsigned)) != cudaSuccess) return bail(MOE_ERR_CUDA, "memset failed");
   if (cudaMalloc(&h->u, sizeof(float) * cfg->top_k * cfg->d_ff) != cudaSuccess) return bail(MOE_ERR_OOM, "u allocation failed");
   const int64_t act = (int64_t)cfg->n_layers * cfg->max_batch * cfg->d * h->asize;
   if (cudaMalloc(&h->hid_dev, act) != cudaSuccess || cudaMalloc(&h->out_dev, act) != cudaSuccess)
@@ -541,6 +737,31 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   h->copy_ev.resize((size_t)cfg->top_k * cfg->max_batch, nullptr);
   for (auto& e : h->copy_ev)
     if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
+  h->dev_mode = cfg->schedule == MOE_SCHEDULE_DEVICE;
+  if (h->dev_mode) {
+    h->fgrid = moe::fused_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
+    if (h->fgrid <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the device-driven schedule");
+    if (cudaHostGetDevicePointer((void**)&h->arena_dev, h->arena, 0) != cudaSuccess)
+      return bail(MOE_ERR_CUDA, "host arena has no device address");
+    const int k = cfg->top_k;
+    bool ok = cudaMalloc(&h->d_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
+              cudaMalloc(&h->d_slot_key, sizeof(unsigned long long) * h->cap) == cudaSuccess &&
+              cudaMalloc(&h->d_n_used, sizeof(int32_t)) == cudaSuccess &&
+              cudaMalloc(&h->d_step, sizeof(int64_t)) == cudaSuccess &&
+              cudaMalloc(&h->d_z, sizeof(float) * 256) == cudaSuccess &&
+              cudaMalloc(&h->d_plan, sizeof(int32_t) * 3 * k) == cudaSuccess &&
+              cudaMalloc(&h->d_plan_gate, sizeof(float) * k) == cudaSuccess &&
+              cudaMalloc(&h->d_trace, sizeof(moe::TraceRec) * std::max<int64_t>(1, cfg->trace_capacity)) == cudaSuccess &&
+              cudaMalloc(&h->d_trace_n, sizeof(unsigned long long)) == cudaSuccess &&
+              cudaMalloc(&h->d_route_idx, sizeof(int32_t) * cfg->n_layers * k) == cudaSuccess &&
+              cudaMalloc(&h->d_route_gate, sizeof(float) * cfg->n_layers * k) == cudaSuccess &&
+              cudaMalloc(&h->d_stats, sizeof(unsigned long long) * moe::STAT_N) == cudaSuccess &&
+              cudaMalloc(&h->d_bar, sizeof(unsigned) * 2) == cudaSuccess &&
+              cudaMalloc(&h->d_err, sizeof(int)) == cudaSuccess &&
+              cudaHostAlloc(&h->h_err, sizeof(int), cudaHostAllocDefault) == cudaSuccess &&
+              cudaEventCreateWithFlags(&h->err_ev, cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) return bail(MOE_ERR_OOM, "device state allocation failed");
+  }
   h->registered.assign(h->n_gid, 0);
   h->router_set.assign(cfg->n_layers, 0);
   h->slot_of.assign(h->n_gid, -1);
@@ -613,13 +834,13 @@ moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t
                                                    std::to_string(g / h->cfg.n_experts) + " not registered");
     h->all_registered = true;
   }
-  moe_status st = decode_impl(h, hidden, out, (cudaStream_t)stream);
+  moe_status st = h->dev_mode ? decode_device(h, hidden, out, (cudaStream_t)stream)
+                              : decode_impl(h, hidden, out, (cudaStream_t)stream);
   if (st != MOE_OK) {
     // The pool contents are unknown after a failed step: wait for the streams, empty the pool.
     std::string keep = h->err;
     cudaStreamSynchronize((cudaStream_t)stream);
     cudaStreamSynchronize(h->copy_stream);
-    cudaMemset(h->counter, 0, sizeof(unsigned));
     cudaGetLastError();
     reset_state(h);
     h->err = keep;
@@ -645,6 +866,20 @@ moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* 
                                    int64_t* n_total) {
   if (!h) return MOE_ERR_INVALID;
   if (start < 0 || cap < 0 || (cap > 0 && !buf)) return fail(h, MOE_ERR_INVALID, "bad trace range");
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  if (h->dev_mode) {
+    moe_status st = check_device_error(h, true);
+    if (st != MOE_OK) return st;
+    unsigned long long produced = 0;
+    MOE_CK(h, cudaMemcpy(&produced, h->d_trace_n, sizeof produced, cudaMemcpyDeviceToHost));
+    const int64_t kept = std::min<int64_t>((int64_t)produced, h->cfg.trace_capacity);
+    const int64_t n = std::max<int64_t>(0, std::min(cap, kept - start));
+    if (n > 0) MOE_CK(h, cudaMemcpy(buf, h->d_trace + start, (size_t)n * sizeof(moe_trace_rec), cudaMemcpyDeviceToHost));
+    if (n_copied) *n_copied = n;
+    if (n_total) *n_total = kept;
+    if ((int64_t)produced > kept) return fail(h, MOE_ERR_TRACE_OVERFLOW, "trace buffer full: records were dropped");
+    return MOE_OK;
+  }
   const int64_t tot = (int64_t)h->trace.size();
   const int64_t n = std::max<int64_t>(0, std::min(cap, tot - start));
   if (n > 0) memcpy(buf, h->trace.data() + start, (size_t)n * sizeof(moe_trace_rec));
@@ -656,6 +891,16 @@ moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* 
 
 moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_t n) {
   if (!h) return MOE_ERR_INVALID;
+  if (h->dev_mode) {
+    const int64_t cnt = (int64_t)h->cfg.n_layers * h->cfg.top_k;
+    if (n < cnt) return fail(h, MOE_ERR_INVALID, "routing buffer too small");
+    MOE_CK(h, cudaSetDevice(h->cfg.device));
+    moe_status st = check_device_error(h, true);
+    if (st != MOE_OK) return st;
+    if (idx) MOE_CK(h, cudaMemcpy(idx, h->d_route_idx, cnt * sizeof(int32_t), cudaMemcpyDeviceToHost));
+    if (gate) MOE_CK(h, cudaMemcpy(gate, h->d_route_gate, cnt * sizeof(float), cudaMemcpyDeviceToHost));
+    return MOE_OK;
+  }
   if (n < (int64_t)h->last_idx.size()) return fail(h, MOE_ERR_INVALID, "routing buffer too small");
   if (idx) memcpy(idx, h->last_idx.data(), h->last_idx.size() * sizeof(int32_t));
   if (gate) memcpy(gate, h->last_gate.data(), h->last_gate.size() * sizeof(float));
@@ -664,6 +909,20 @@ moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_
 
 moe_status moe_get_stats(moe_handle* h, moe_stats* out) {
   if (!h || !out) return MOE_ERR_INVALID;
+  if (h->dev_mode) {
+    MOE_CK(h, cudaSetDevice(h->cfg.device));
+    moe_status st = check_device_error(h, true);
+    if (st != MOE_OK) return st;
+    unsigned long long v[moe::STAT_N];
+    MOE_CK(h, cudaMemcpy(v, h->d_stats, sizeof v, cudaMemcpyDeviceToHost));
+    out->steps = h->steps_launched;
+    out->layer_steps = (int64_t)v[moe::STAT_LAYER_STEPS];
+    out->hits = (int64_t)v[moe::STAT_HITS];
+    out->misses = (int64_t)v[moe::STAT_MISSES];
+    out->evictions = (int64_t)v[moe::STAT_EVICTIONS];
+    out->miss_bytes = out->misses * h->lay.total;
+    return MOE_OK;
+  }
   *out = h->stats;
   return MOE_OK;
 }
@@ -687,7 +946,7 @@ moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, in
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   harvest(h, true);
   int32_t n = 0;
-  for (int c = 0; c < PC_N && n < cap; c++, n++) {
+  for (int c = 0; c < PC_N && n < cap; c++, n++) {  // fused_phase_*: per layer-step, from the kernel's global timer
     memset(&out[n], 0, sizeof(moe_kernel_time));
     snprintf(out[n].name, sizeof out[n].name, "%s", kPcName[c]);
     out[n].launches = h->pc_launches[c];

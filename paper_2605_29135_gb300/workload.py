@@ -15,16 +15,17 @@ import numpy as np
 from . import MoE, make_config
 
 
-def config_for(wl, cap_slots=None, device=0, trace_capacity=1 << 22, renorm=True):
+def config_for(wl, cap_slots=None, device=0, trace_capacity=1 << 22, renorm=True, schedule="device", miss_ctas=0):
     return make_config(wl.d, wl.n_experts, wl.top_k, wl.d_ff, wl.n_layers, wl.wdtype, wl.adtype,
                        cap_slots=wl.cap_slots if cap_slots is None else cap_slots, renorm=renorm, device=device,
-                       max_batch=wl.batch, trace_capacity=trace_capacity)
+                       max_batch=wl.batch, trace_capacity=trace_capacity, schedule=schedule, miss_ctas=miss_ctas)
 
 
-def create_for_workload(wl, cap_slots=None, device=0, trace_capacity=1 << 22, threads=None) -> MoE:
+def create_for_workload(wl, cap_slots=None, device=0, trace_capacity=1 << 22, threads=None,
+                        schedule="device", miss_ctas=0) -> MoE:
     import synth
 
-    m = MoE(config_for(wl, cap_slots, device, trace_capacity))
+    m = MoE(config_for(wl, cap_slots, device, trace_capacity, schedule=schedule, miss_ctas=miss_ctas))
     try:
         for layer in range(wl.n_layers):
             m.set_router(layer, synth.router_weights(wl, layer))

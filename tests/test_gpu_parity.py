@@ -27,15 +27,27 @@ def P():
     return P
 
 
-def _create(wl, cap):
+SCHEDULES = ["device", "host_copy_engine"]
+_ORACLE_CACHE = {}
+
+
+def _create(wl, cap, schedule="device"):
     from paper_2605_29135_gb300.workload import create_for_workload
 
-    return create_for_workload(wl, cap_slots=cap)
+    return create_for_workload(wl, cap_slots=cap, schedule=schedule)
 
 
-def _parity(P, wl, cap, tokens, samples=None, threads=8):
+def _oracle_routing(wl, cap, tokens, hidden, routers):
+    key = (wl, cap, tokens)
+    if key not in _ORACLE_CACHE:
+        _ORACLE_CACHE.clear()
+        _ORACLE_CACHE[key] = oracle_trace(wl, hidden, cap, routers=routers)
+    return _ORACLE_CACHE[key]
+
+
+def _parity(P, wl, cap, tokens, samples=None, threads=8, schedule="device"):
     hidden = synth.hidden_all(wl, tokens)
-    m = _create(wl, cap)
+    m = _create(wl, cap, schedule)
     try:
         out, idx, gate = run_gpu(m, hidden, wl.adtype)
         tr = m.get_residency_trace()
@@ -43,7 +55,7 @@ def _parity(P, wl, cap, tokens, samples=None, threads=8):
     finally:
         m.destroy()
     routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
-    oidx, oz, otr = oracle_trace(wl, hidden, cap, routers=routers)
+    oidx, oz, otr = _oracle_routing(wl, cap, tokens, hidden, routers)
     flips = check_routing(idx, oidx, oz, wl.top_k)
     if flips:
         _, _, otr = oracle_trace(wl, hidden, cap, forced_idx=idx, routers=routers)
@@ -72,23 +84,29 @@ def _parity(P, wl, cap, tokens, samples=None, threads=8):
     return out, tr, errs, flips
 
 
-def test_tiny_fp32_full_run(P):
+@pytest.mark.parametrize("schedule", SCHEDULES)
+def test_tiny_fp32_full_run(P, schedule):
     wl = synth.WORKLOADS["tiny_fp32"]
-    out, tr, errs, _ = _parity(P, wl, wl.cap_slots, wl.tokens)
+    out, tr, errs, _ = _parity(P, wl, wl.cap_slots, wl.tokens, schedule=schedule)
     assert (tr["kind"] == 0).sum() > 0 and (tr["evicted"] >= 0).sum() > 0
 
 
-def test_tiny_fp32_cap_invariance_bit_exact(P):
-    wl = synth.WORKLOADS["tiny_fp32"]
-    hidden = synth.hidden_all(wl)
+@pytest.mark.parametrize("name", ["tiny_fp32", "layer_bf16"])
+def test_cap_invariance_bit_exact_across_schedules(P, name):
+    # outputs do not depend on the cap (residency only changes where weights are read from) nor
+    # on the schedule: the same kernels' arithmetic runs on slot or host-tier bytes
+    wl = synth.WORKLOADS[name]
+    tokens = min(wl.tokens, 96)
+    hidden = synth.hidden_all(wl, tokens)
     outs = []
-    for cap in (wl.cap_slots, wl.n_gid):
-        m = _create(wl, cap)
+    for cap, schedule in ((wl.cap_slots, "device"), (wl.n_gid, "device"), (wl.cap_slots, "host_copy_engine")):
+        m = _create(wl, cap, schedule)
         try:
             outs.append(run_gpu(m, hidden, wl.adtype)[0])
         finally:
             m.destroy()
     np.testing.assert_array_equal(outs[0], outs[1])
+    np.testing.assert_array_equal(outs[0], outs[2])
 
 
 RAGGED = {
@@ -103,21 +121,24 @@ RAGGED = {
 }
 
 
+@pytest.mark.parametrize("schedule", SCHEDULES)
 @pytest.mark.parametrize("name", list(RAGGED))
-def test_ragged_shapes(P, name):
+def test_ragged_shapes(P, name, schedule):
     wl = RAGGED[name]
-    _parity(P, wl, wl.cap_slots, wl.tokens)
+    _parity(P, wl, wl.cap_slots, wl.tokens, schedule=schedule)
 
 
-def test_layer_bf16_full_2048_tokens(P):
+@pytest.mark.parametrize("schedule", SCHEDULES)
+def test_layer_bf16_full_2048_tokens(P, schedule):
     wl = synth.WORKLOADS["layer_bf16"]
     samples = [(t, 0) for t in range(0, wl.tokens, 64)] + [(wl.tokens - 1, 0)]
-    _parity(P, wl, wl.cap_slots, wl.tokens, samples=samples)
+    _parity(P, wl, wl.cap_slots, wl.tokens, samples=samples, schedule=schedule)
 
 
+@pytest.mark.parametrize("schedule", SCHEDULES)
 @pytest.mark.parametrize("name", ["stack48_int4", "stack48_bf16"])
-def test_stack48_full_2048_tokens(P, name):
+def test_stack48_full_2048_tokens(P, name, schedule):
     wl = synth.WORKLOADS[name]
     samples = [(t, l) for t in (0, 1023, 2047) for l in range(0, 48, 6)]
-    _, tr, errs, flips = _parity(P, wl, wl.cap_slots, wl.tokens, samples=samples, threads=16)
+    _, tr, errs, flips = _parity(P, wl, wl.cap_slots, wl.tokens, samples=samples, threads=16, schedule=schedule)
     assert len(tr) == wl.tokens * wl.n_layers * wl.top_k
