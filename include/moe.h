@@ -191,6 +191,35 @@ moe_status moe_reset_residency(moe_handle* h);
 moe_status moe_profile_enable(moe_handle* h, int32_t on);
 moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, int32_t* n_out);
 
+/* ---- Allocation-free routing --------------------------------------------------------------
+ * The paper has no counterpart to this call; it exists for callers that cannot allocate device
+ * memory at the point where they route (an inference runtime that reserves all device memory at
+ * start-up and forbids later cudaMalloc, a plug-in that runs inside a host process owning the
+ * allocator, code running under a lock that allocation would need). It needs no handle.
+ *
+ * Router GEMV + top-k + gates for `rows` hidden vectors against one router matrix, with the same
+ * arithmetic as the router stage of moe_decode_step: z = W_r h (fp32 accumulation), top-k by z
+ * (ties -> lower id), gates = softmax over the k selected logits (renorm = 1) or the
+ * full-softmax probabilities (renorm = 0).
+ *   w_r     device, [n_experts x d] row-major, fp32 (wdtype MOE_DTYPE_FP32) or bf16 (MOE_DTYPE_BF16)
+ *   hidden  device, [rows x d], same element type as w_r
+ *   idx     device output, int32 [rows x top_k], expert ids in descending logit order
+ *   gate    device output, fp32 [rows x top_k]
+ *   stream  cudaStream_t the two kernels are ordered on (NULL = legacy default stream)
+ * The logits go to a fixed scratch array of MOE_NOALLOC_MAX_ROWS * MOE_NOALLOC_MAX_EXPERTS floats
+ * (64 KiB) inside the library, held on every device that loads the library until the process
+ * exits; no memory is allocated by the call. The first call on a device looks up that array's
+ * device address (cudaGetSymbolAddress), so make the first call on each device before any stream
+ * capture. Every call reuses the same array: calls whose work overlaps on the GPU (different
+ * streams or host threads) race on it and must be serialised by the caller.
+ * Returns MOE_ERR_CAPACITY if rows > MOE_NOALLOC_MAX_ROWS or n_experts > MOE_NOALLOC_MAX_EXPERTS,
+ * MOE_ERR_INVALID for other bad arguments (top_k > 16 or > n_experts, d * element bytes not a
+ * multiple of 16 or above 48 KiB, NULL pointers), MOE_ERR_CUDA if a launch fails. */
+#define MOE_NOALLOC_MAX_ROWS 64
+#define MOE_NOALLOC_MAX_EXPERTS 256
+moe_status moe_route_noalloc(const void* w_r, const void* hidden, int32_t rows, int32_t n_experts, int32_t d,
+                             int32_t top_k, int32_t renorm, int32_t wdtype, int32_t* idx, float* gate, void* stream);
+
 /* Message of the last failure on h (or of the last failed moe_create if h is NULL). */
 const char* moe_last_error(const moe_handle* h);
 

@@ -153,10 +153,36 @@ class MoE:
         self.destroy()
 
 
+def route_noalloc(w_r, hidden, top_k: int, renorm: bool = True, stream=None):
+    """Routing without any device allocation by the library (moe_route_noalloc).
+
+    For callers that cannot allocate device memory at routing time: the logits go to a fixed
+    scratch array inside the library, and the caller passes its own outputs. w_r: device tensor
+    [E x d] (float32 or bfloat16); hidden: device tensor [rows x d] of the same dtype. Returns
+    (idx int32 [rows x top_k], gate float32 [rows x top_k]) as device tensors allocated by the
+    caller side here (torch), never by the library.
+    """
+    import torch
+
+    rows, d = hidden.shape
+    E = w_r.shape[0]
+    wd = DTYPE["fp32"] if w_r.dtype == torch.float32 else DTYPE["bf16"]
+    idx = torch.empty((rows, top_k), dtype=torch.int32, device=hidden.device)
+    gate = torch.empty((rows, top_k), dtype=torch.float32, device=hidden.device)
+    if stream is None:
+        stream = torch.cuda.current_stream(hidden.device)
+    st = _lib.load().moe_route_noalloc(_ptr(w_r), _ptr(hidden), rows, E, d, top_k, 1 if renorm else 0, wd,
+                                        _ptr(idx), _ptr(gate), ctypes.c_void_p(stream.cuda_stream))
+    if st != 0:
+        raise MoEError(st, "moe_route_noalloc rejected the arguments" if st != -3 else "moe_route_noalloc launch failed")
+    return idx, gate
+
+
 def build(force: bool = False) -> str:
     from .build import build as _b
 
     return _b(force=force)
 
 
-__all__ = ["MoE", "MoEError", "make_config", "expert_bytes", "pool_bytes", "TRACE_DTYPE", "build", "TraceRec"]
+__all__ = ["MoE", "MoEError", "make_config", "expert_bytes", "pool_bytes", "TRACE_DTYPE", "build", "TraceRec",
+           "route_noalloc"]
