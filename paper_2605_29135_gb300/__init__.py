@@ -179,7 +179,7 @@ def route_noalloc(w_r, hidden, top_k: int, renorm: bool = True, stream=None):
 
 
 def build(force: bool = False) -> str:
-    from .build import build as _b
+    from .buildsys import build as _b
 
     return _b(force=force)
 

@@ -61,7 +61,7 @@ def load(path: str | None = None):
             return _lib
         p = path or LIB_PATH
         if not os.path.exists(p):
-            raise RuntimeError(f"libmoe.so is not built ({p}); run `python -m paper_2605_29135_gb300.build` "
+            raise RuntimeError(f"libmoe.so is not built ({p}); run `python -m paper_2605_29135_gb300.buildsys` "
                                "or __graft_entry__.build()")
         L = ctypes.CDLL(p)
         vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64

@@ -19,7 +19,7 @@ def _declared():
 @pytest.fixture(scope="module")
 def lib():
     from paper_2605_29135_gb300 import _lib
-    from paper_2605_29135_gb300.build import build
+    from paper_2605_29135_gb300.buildsys import build
 
     build()
     return _lib.load()

@@ -22,7 +22,7 @@ def test_noalloc_routing_matches_decode_step_on_two_calls_in_a_row():
     import torch
 
     import paper_2605_29135_gb300 as P
-    from paper_2605_29135_gb300.build import build
+    from paper_2605_29135_gb300.buildsys import build
     from paper_2605_29135_gb300.workload import create_for_workload
 
     build()
@@ -62,7 +62,7 @@ def test_noalloc_routing_matches_decode_step_on_two_calls_in_a_row():
 
 def test_noalloc_rejects_sizes_beyond_the_scratch():
     from paper_2605_29135_gb300 import _lib
-    from paper_2605_29135_gb300.build import build
+    from paper_2605_29135_gb300.buildsys import build
 
     build()
     lib = _lib.load()
