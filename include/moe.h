@@ -184,6 +184,12 @@ moe_status moe_get_stats(moe_handle* h, moe_stats* out);
 /* Empty the slot pool (all experts non-resident), step clock 0, trace and stats cleared. */
 moe_status moe_reset_residency(moe_handle* h);
 
+/* Warm start: copy experts into free slots in ascending global id order until the pool is full
+ * (with cap_slots >= n_layers * n_experts every expert becomes resident). Preloaded experts count
+ * as used before every decode step, so they are the first victims; the copies are not residency
+ * records and do not change the stats. Synchronous; *n_loaded (optional) = experts copied. */
+moe_status moe_preload(moe_handle* h, int64_t* n_loaded);
+
 /* Profiling: with on = 1, every kernel launch and miss copy of later steps is bracketed by
  * CUDA events on its stream. moe_profile_read waits for the recorded work, then reports one
  * entry per kernel class (router, gateup, down_combine, miss_copy) accumulated since the last

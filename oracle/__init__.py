@@ -165,6 +165,21 @@ class LRUTable:
         self.gid_of = np.full(cap, -1, dtype=np.int32)
         self.last_use = np.full(n_gid, -1, dtype=np.int64)
 
+    def preload(self):
+        """Warm start: free slots take experts in ascending global id order until the group is full;
+        they count as used before every layer-step (last use -1)."""
+        free = [s for s in range(self.cap) if self.gid_of[s] < 0]
+        g = 0
+        for s in free:
+            while g < self.n_gid and self.slot_of[g] >= 0:
+                g += 1
+            if g >= self.n_gid:
+                break
+            self.gid_of[s] = g
+            self.slot_of[g] = s
+            self.last_use[g] = -1
+            g += 1
+
     def step(self, clock: int, needed, step: int) -> np.ndarray:
         needed = np.ascontiguousarray(sorted(set(int(g) for g in needed)), dtype=np.int32)
         out = np.zeros(len(needed), dtype=REC_DTYPE)
@@ -222,6 +237,15 @@ class Oracle:
         self.table = LRUTable(self.table.n_gid, self.table.cap, self.E)
         self.slots = {}
         self.token_step = 0
+
+    def preload(self):
+        """Warm start (see LRUTable.preload), copying each preloaded expert into its slot."""
+        self.table.preload()
+        if self.keep:
+            for s, g in enumerate(self.table.gid_of):
+                if g >= 0 and s not in self.slots:
+                    l, e = divmod(int(g), self.E)
+                    self.slots[s] = (int(g), _copy_expert(self.experts(l, e)))
 
     def _widen_expert(self, w):
         d, I, dt = self.d, self.I, self.wdtype

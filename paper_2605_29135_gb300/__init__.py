@@ -123,6 +123,11 @@ class MoE:
     def reset_residency(self):
         self._check(self.lib.moe_reset_residency(self.h))
 
+    def preload(self) -> int:
+        n = ctypes.c_int64()
+        self._check(self.lib.moe_preload(self.h, ctypes.byref(n)))
+        return n.value
+
     def profile_enable(self, on: bool = True):
         self._check(self.lib.moe_profile_enable(self.h, 1 if on else 0))
 

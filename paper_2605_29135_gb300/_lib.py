@@ -22,7 +22,7 @@ SCHEDULE = {"device": 0, "host_copy_engine": 1}
 EXPORTS = ["moe_expert_bytes", "moe_pool_bytes", "moe_create", "moe_set_router", "moe_register_host_experts",
            "moe_decode_step", "moe_decode_step_host", "moe_get_residency_trace", "moe_get_last_routing",
            "moe_get_stats", "moe_reset_residency", "moe_profile_enable", "moe_profile_read", "moe_last_error",
-           "moe_destroy", "moe_route_noalloc"]
+           "moe_destroy", "moe_route_noalloc", "moe_preload"]
 
 
 class MoeConfig(ctypes.Structure):
@@ -98,5 +98,7 @@ def load(path: str | None = None):
         L.moe_destroy.restype = None
         L.moe_route_noalloc.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, vp, vp, vp]
         L.moe_route_noalloc.restype = ctypes.c_int
+        L.moe_preload.argtypes = [vp, ctypes.POINTER(i64)]
+        L.moe_preload.restype = ctypes.c_int
         _lib = L
         return L

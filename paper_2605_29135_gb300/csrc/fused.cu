@@ -417,7 +417,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
   if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[a.L * 4] = gtimer();
 
   for (int l = 0; l < a.L; l++) {
-    const int clock = (int)(step * a.L + l);
+    const int clock = (int)(step * a.L + l + 1);  // 0 is older than every step (preloaded experts)
     // ---- phase R: router logits
     stage16(reinterpret_cast<uint4*>(xs), (const uint8_t*)a.hidden + (int64_t)l * xbytes, xbytes, threadIdx.x,
             blockDim.x);

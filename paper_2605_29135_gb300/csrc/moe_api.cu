@@ -411,7 +411,7 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     std::sort(needs.begin(), needs.end(), [](const Need& a, const Need& b) { return a.gid < b.gid; });
     for (size_t i = 1; i < needs.size(); i++)
       if (needs[i].gid == needs[i - 1].gid) return fail(h, MOE_ERR_INVALID, "router produced duplicate expert ids");
-    const int64_t clock = h->token_step * L + l;
+    const int64_t clock = h->token_step * L + l + 1;  // 0 is older than every step (preloaded experts)
     st = residency_step(h, l, needs, clock);
     if (st != MOE_OK) return st;
     h->stats.layer_steps++;
@@ -932,6 +932,61 @@ moe_status moe_reset_residency(moe_handle* h) {
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   MOE_CK(h, cudaDeviceSynchronize());
   reset_state(h);
+  return MOE_OK;
+}
+
+moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
+  if (!h) return MOE_ERR_INVALID;
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  if (!h->all_registered) {
+    for (int64_t g = 0; g < h->n_gid; g++)
+      if (!h->registered[g]) return fail(h, MOE_ERR_NOT_REGISTERED, "preload needs every expert registered");
+  }
+  if (h->dev_mode) {
+    moe_status st = check_device_error(h, true);
+    if (st != MOE_OK) return st;
+  } else {
+    MOE_CK(h, cudaDeviceSynchronize());
+  }
+  // current lookup table
+  std::vector<int32_t> slot_of(h->n_gid);
+  int32_t n_used = 0;
+  if (h->dev_mode) {
+    MOE_CK(h, cudaMemcpy(slot_of.data(), h->d_slot_of, sizeof(int32_t) * h->n_gid, cudaMemcpyDeviceToHost));
+    MOE_CK(h, cudaMemcpy(&n_used, h->d_n_used, sizeof n_used, cudaMemcpyDeviceToHost));
+  } else {
+    slot_of = h->slot_of;
+    n_used = (int32_t)(h->cap - (int64_t)h->free_slots.size());
+  }
+  int64_t loaded = 0;
+  std::vector<unsigned long long> keys;
+  std::vector<int32_t> kslots;
+  for (int64_t g = 0; g < h->n_gid && n_used < h->cap; g++) {
+    if (slot_of[g] >= 0) continue;
+    const int32_t slot = n_used++;
+    MOE_CK(h, cudaMemcpyAsync(h->pool + (int64_t)slot * h->slot_stride, h->arena + g * h->slot_stride, h->lay.total,
+                              cudaMemcpyHostToDevice, h->copy_stream));
+    slot_of[g] = slot;
+    keys.push_back((unsigned long long)(uint32_t)g);  // last use 0: older than every decode step
+    kslots.push_back(slot);
+    if (!h->dev_mode) {
+      h->free_slots.erase(slot);
+      h->gid_of[slot] = (int32_t)g;
+      h->slot_of[g] = slot;
+      h->last_use[g] = 0;
+      h->lru.insert({0, (int32_t)g});
+    }
+    loaded++;
+  }
+  MOE_CK(h, cudaStreamSynchronize(h->copy_stream));
+  if (h->dev_mode && loaded > 0) {
+    MOE_CK(h, cudaMemcpy(h->d_slot_of, slot_of.data(), sizeof(int32_t) * h->n_gid, cudaMemcpyHostToDevice));
+    MOE_CK(h, cudaMemcpy(h->d_n_used, &n_used, sizeof n_used, cudaMemcpyHostToDevice));
+    // preloaded slots are contiguous [n_used - loaded, n_used)
+    MOE_CK(h, cudaMemcpy(h->d_slot_key + kslots.front(), keys.data(), sizeof(unsigned long long) * keys.size(),
+                         cudaMemcpyHostToDevice));
+  }
+  if (n_loaded) *n_loaded = loaded;
   return MOE_OK;
 }
 

@@ -142,3 +142,28 @@ def test_stack48_full_2048_tokens(P, name, schedule):
     samples = [(t, l) for t in (0, 1023, 2047) for l in range(0, 48, 6)]
     _, tr, errs, flips = _parity(P, wl, wl.cap_slots, wl.tokens, samples=samples, threads=16, schedule=schedule)
     assert len(tr) == wl.tokens * wl.n_layers * wl.top_k
+
+
+@pytest.mark.parametrize("schedule", SCHEDULES)
+@pytest.mark.parametrize("cap", [4, 8])
+def test_preload_then_decode_matches_oracle(P, schedule, cap):
+    wl = synth.WORKLOADS["tiny_fp32"]
+    hidden = synth.hidden_all(wl)
+    m = _create(wl, cap, schedule)
+    try:
+        assert m.preload() == min(cap, wl.n_gid)
+        out, idx, _ = run_gpu(m, hidden, wl.adtype)
+        tr = m.get_residency_trace()
+    finally:
+        m.destroy()
+    orc = oracle.Oracle.for_workload(wl, cap_slots=cap)
+    orc.preload()
+    recs, ref = [], []
+    for t in range(wl.tokens):
+        r = orc.decode_step(hidden[t], forced_idx=idx[t])
+        recs.append(r.records)
+        ref.append(r.out)
+    np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate(recs)))
+    assert rel_l2_rows(out, np.stack(ref)).max() <= TOL["fp32"]
+    if cap >= wl.n_gid:
+        assert (tr["kind"] == 0).all()

@@ -104,3 +104,24 @@ def test_cap_at_least_all_experts_never_evicts():
             assert r["evicted"] == -1
             assert r["kind"] == (0 if int(r["expert"]) in seen else 1)
         seen.update(needed)
+
+
+def test_preload_fills_free_slots_in_id_order_and_ages_them_first():
+    # 4 slots, 8 experts: preload puts experts 0..3 in slots 0..3 with last use -1; a step needing
+    # {5, 6} then misses twice and evicts 0 and 1 (oldest, lower id first); a step needing {2, 7}
+    # hits 2 and evicts 3 (still last use -1) for 7.
+    t = oracle.LRUTable(n_gid=8, cap=4, n_experts=8)
+    t.preload()
+    assert t.gid_of.tolist() == [0, 1, 2, 3]
+    got = [(int(r["expert"]), int(r["kind"]), int(r["slot"]), int(r["evicted"])) for r in t.step(0, [5, 6], 0)]
+    assert got == [(5, 1, 0, 0), (6, 1, 1, 1)]
+    got = [(int(r["expert"]), int(r["kind"]), int(r["slot"]), int(r["evicted"])) for r in t.step(1, [2, 7], 1)]
+    assert got == [(2, 0, 2, -1), (7, 1, 3, 3)]
+
+
+def test_preload_with_cap_at_least_all_experts_makes_every_request_a_hit():
+    t = oracle.LRUTable(n_gid=6, cap=8, n_experts=6)
+    t.preload()
+    assert sorted(int(g) for g in t.gid_of if g >= 0) == list(range(6))
+    for s in range(5):
+        assert all(int(r["kind"]) == 0 for r in t.step(s, [s % 6, (s + 3) % 6], s))
