@@ -84,9 +84,11 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   __shared__ int s_slot[kMaxRanks];   // slot per needed id (after the step)
   __shared__ int s_miss[kMaxRanks];
   __shared__ int s_evict[kMaxRanks];  // evicted global id per needed id, -1 if none
-  __shared__ int s_vslot[kMaxRanks];  // victim slots in ascending (last use, id)
+  __shared__ int s_vslot[kMaxRanks];  // victims in ascending (last use, id): slot and global id
+  __shared__ int s_vgid[kMaxRanks];
   __shared__ int s_nev;
-  __shared__ unsigned long long s_red[kFWarps];
+  __shared__ unsigned long long s_ckey[kFWarps][kMaxRanks];  // each warp's smallest candidate keys
+  __shared__ int s_cslot[kFWarps][kMaxRanks];
   const int k = a.k, E = a.E;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
@@ -130,70 +132,113 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
       for (int e = lane; e < E; e += 32) part += expf(__ldcg(a.z + e) - m);
       denom = warp_sum(part);
     }
+    if (lane < k && (my_i < 0 || my_i >= E)) {
+      atomicOr(a.err, FERR_BAD_ROUTE);
+      my_i = lane;  // keep the step well-defined; the host reports the error
+    }
+    // needed ids in ascending order: each id's position is the count of smaller ids (all distinct)
+    const int gid = l * E + my_i;
+    int pos = 0;
+    for (int t = 0; t < k; t++) {
+      const int o = __shfl_sync(kFull, gid, t);
+      pos += (lane < k && o < gid) ? 1 : 0;
+    }
     if (lane < k) {
-      if (my_i < 0 || my_i >= E) {
-        atomicOr(a.err, FERR_BAD_ROUTE);
-        my_i = lane;  // keep the step well-defined; the host reports the error
-      }
       s_idx[lane] = my_i;
       s_gate[lane] = ex / denom;
+      s_need[pos] = gid;
+    }
+    __syncwarp();
+    if (lane < k) {
+      const int sl = a.slot_of[s_need[lane]];
+      s_slot[lane] = sl;
+      s_miss[lane] = sl < 0;
+      s_evict[lane] = -1;
+    }
+    __syncwarp();
+    if (lane == 0) {
+      // misses in ascending id take free slots [n_used, cap) first
+      int n_used = *a.n_used;
+      int nev = 0;
+      for (int t = 0; t < k; t++) {
+        if (s_slot[t] >= 0) continue;
+        if (n_used < a.cap)
+          s_slot[t] = n_used++;
+        else
+          nev++;
+      }
+      *a.n_used = n_used;
+      s_nev = nev;
     }
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int r = 0; r < k; r++) s_need[r] = l * E + s_idx[r];
-    for (int r = 1; r < k; r++) {  // insertion sort, k <= 16
-      const int v = s_need[r];
-      int j = r - 1;
-      while (j >= 0 && s_need[j] > v) {
-        s_need[j + 1] = s_need[j];
-        j--;
-      }
-      s_need[j + 1] = v;
-    }
-    // hits keep their slot; misses in ascending id take free slots [n_used, cap) first
-    int n_used = *a.n_used;
-    int nev = 0;
-    for (int t = 0; t < k; t++) {
-      const int sl = a.slot_of[s_need[t]];
-      s_miss[t] = sl < 0;
-      s_slot[t] = sl;
-      s_evict[t] = -1;
-      if (sl < 0) {
-        if (n_used < a.cap) {
-          s_slot[t] = n_used++;
-        } else {
-          nev++;
+  const int nev = s_nev;
+  if (nev > 0) {
+    // Victims: the nev smallest slot keys (last use, id) among slots that hold no expert of this
+    // step (every slot is occupied when eviction is needed). Each warp finds the nev smallest of
+    // its slots, warp 0 takes the nev smallest of those candidates.
+    for (int j = 0; j < nev; j++) {
+      unsigned long long best = ~0ull;
+      int bslot = -1;
+      for (int64_t sl = threadIdx.x; sl < a.cap; sl += blockDim.x) {
+        bool skip = false;
+        for (int t = 0; t < k; t++) skip |= (s_slot[t] == sl);  // hits are pinned; misses not yet placed
+        for (int t = 0; t < j; t++) skip |= (s_cslot[warp][t] == sl);
+        if (skip) continue;
+        const unsigned long long key = a.slot_key[sl];
+        if (key < best) {
+          best = key;
+          bslot = (int)sl;
         }
       }
+      const unsigned long long wmin = shfl_min_u64(best);
+      const unsigned win = __ballot_sync(kFull, best == wmin);
+      const int leader = __ffs(win) - 1;
+      const int wslot = __shfl_sync(kFull, bslot, leader);
+      if (lane == 0) {
+        s_ckey[warp][j] = wmin;
+        s_cslot[warp][j] = wmin == ~0ull ? -1 : wslot;
+      }
+      __syncwarp();
     }
-    *a.n_used = n_used;
-    s_nev = nev;
-  }
-  __syncthreads();
-  // Victims: the s_nev smallest slot keys (last use, id) among occupied slots that hold no
-  // expert of this step. Free slots carry ~0 and are never picked while a real key remains.
-  for (int j = 0; j < s_nev; j++) {
-    unsigned long long best = ~0ull;
-    for (int64_t sl = threadIdx.x; sl < a.cap; sl += blockDim.x) {
-      bool skip = false;
-      for (int t = 0; t < k; t++) skip |= (s_slot[t] == sl);  // hits (pinned); misses are not yet placed
-      for (int t = 0; t < j; t++) skip |= (s_vslot[t] == sl);
-      if (skip) continue;
-      const unsigned long long key = a.slot_key[sl];
-      best = key < best ? key : best;
-    }
-    best = shfl_min_u64(best);
-    if (lane == 0) s_red[warp] = best;
     __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned long long b = s_red[0];
-      for (int w = 1; w < kFWarps; w++) b = s_red[w] < b ? s_red[w] : b;
-      if (b == ~0ull) {
-        atomicOr(a.err, FERR_NO_VICTIM);
-        s_vslot[j] = -1;
-      } else {
-        s_vslot[j] = a.slot_of[(int)(uint32_t)(b & 0xffffffffull)];
+    if (warp == 0) {
+      const int nc = kFWarps * nev;  // <= 128 candidates, 4 per lane
+      unsigned long long ck[4];
+      int cs[4];
+#pragma unroll
+      for (int q = 0; q < 4; q++) {
+        const int c = q * 32 + lane;
+        ck[q] = c < nc ? s_ckey[c / nev][c % nev] : ~0ull;
+        cs[q] = c < nc ? s_cslot[c / nev][c % nev] : -1;
+      }
+      for (int j = 0; j < nev; j++) {
+        unsigned long long best = ~0ull;
+        int bq = 0;
+#pragma unroll
+        for (int q = 0; q < 4; q++)
+          if (ck[q] < best) {
+            best = ck[q];
+            bq = q;
+          }
+        const unsigned long long wmin = shfl_min_u64(best);
+        const unsigned win = __ballot_sync(kFull, best == wmin && wmin != ~0ull);
+        const int leader = win ? __ffs(win) - 1 : 0;
+        int vslot = -1;
+#pragma unroll
+        for (int q = 0; q < 4; q++)
+          if (q == bq) vslot = cs[q];
+        vslot = __shfl_sync(kFull, vslot, leader);
+        if (lane == leader && win) {
+#pragma unroll
+          for (int q = 0; q < 4; q++)
+            if (q == bq) ck[q] = ~0ull;
+        }
+        if (lane == 0) {
+          if (!win) atomicOr(a.err, FERR_NO_VICTIM);
+          s_vslot[j] = win ? vslot : -1;
+          s_vgid[j] = win ? (int)(uint32_t)(wmin & 0xffffffffull) : -1;
+        }
       }
     }
     __syncthreads();
@@ -209,9 +254,10 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
       }
       misses++;
       if (s_slot[t] < 0) {  // needs a victim
-        const int vs = s_vslot[j++];
+        const int vs = s_vslot[j];
+        const int v = s_vgid[j];
+        j++;
         if (vs >= 0) {
-          const int v = (int)(uint32_t)(a.slot_key[vs] & 0xffffffffull);
           a.slot_of[v] = -1;
           s_slot[t] = vs;
           s_evict[t] = v;
@@ -222,36 +268,38 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     }
     for (int t = 0; t < k; t++)
       if (s_slot[t] >= 0) a.slot_key[s_slot[t]] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)s_need[t];
-    const unsigned long long base = *a.trace_n;
-    for (int t = 0; t < k; t++) {
-      if (base + t < (unsigned long long)a.trace_cap) {
-        TraceRec rec;
-        rec.step = (int32_t)step;
-        rec.layer = l;
-        rec.expert = s_need[t] - l * E;
-        rec.kind = s_miss[t];
-        rec.slot = s_slot[t];
-        rec.evicted = s_evict[t];
-        a.trace[base + t] = rec;
-      }
-    }
-    *a.trace_n = base + k;
     a.stats[STAT_HITS] += hits;
     a.stats[STAT_MISSES] += misses;
     a.stats[STAT_EVICTIONS] += evictions;
     a.stats[STAT_LAYER_STEPS] += 1;
-    for (int r = 0; r < k; r++) {
-      const int g = l * E + s_idx[r];
-      int t = 0;
-      while (s_need[t] != g) t++;
-      a.plan_slot[r] = s_slot[t] < 0 ? 0 : s_slot[t];
-      a.plan_gid[r] = g;
-      a.plan_miss[r] = s_miss[t];
-      a.plan_gate[r] = s_gate[r];
-      a.route_idx[l * k + r] = s_idx[r];
-      a.route_gate[l * k + r] = s_gate[r];
-    }
   }
+  __syncthreads();
+  if (threadIdx.x < k) {
+    const int t = threadIdx.x;
+    const unsigned long long base = *(volatile unsigned long long*)a.trace_n;
+    if (base + t < (unsigned long long)a.trace_cap) {
+      TraceRec rec;
+      rec.step = (int32_t)step;
+      rec.layer = l;
+      rec.expert = s_need[t] - l * E;
+      rec.kind = s_miss[t];
+      rec.slot = s_slot[t];
+      rec.evicted = s_evict[t];
+      a.trace[base + t] = rec;
+    }
+    // plan of rank t
+    const int g = l * E + s_idx[t];
+    int q = 0;
+    while (s_need[q] != g) q++;
+    a.plan_slot[t] = s_slot[q] < 0 ? 0 : s_slot[q];
+    a.plan_gid[t] = g;
+    a.plan_miss[t] = s_miss[q];
+    a.plan_gate[t] = s_gate[t];
+    a.route_idx[l * k + t] = s_idx[t];
+    a.route_gate[l * k + t] = s_gate[t];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) *a.trace_n = *(volatile unsigned long long*)a.trace_n + k;
 }
 
 // Copy n bf16 values (scales) from src to dst with 2-byte accesses, one per lane.
@@ -332,10 +380,26 @@ __device__ __forceinline__ void gateup_row(const FusedArgs& a, const uint8_t* sr
   if (lane == 0) a.u[(int64_t)r * a.I + i] = ag / (1.0f + expf(-ag)) * au;
 }
 
-// Phase D rows (all experts in their slots) for one value of the chunks-per-lane count of a W_d row.
+// Stage the k u vectors ([k x I] fp32, rank-major) into shared memory, padded by 4 floats per
+// 32 so the 16-byte reads of a warp spread over all banks.
+__device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad) {
+  const float4* u4 = reinterpret_cast<const float4*>(a.u);
+  const int n4 = a.k * a.I / 4;
+#pragma unroll 4
+  for (int q = threadIdx.x; q < n4; q += blockDim.x) {
+    const float4 v = __ldcg(u4 + q);
+    const int r = (4 * q) / a.I;
+    const int i = 4 * q - r * a.I;
+    *reinterpret_cast<float4*>(us + r * ipad + upad(i)) = v;
+  }
+}
+
+// Phase D (all experts in their slots) for one value of the chunks-per-lane count of a W_d row:
+// stages u, then out[o] = sum_r g_r (W_d^(r)[o] . u_r). A warp's first rows are requested before
+// the CTA stages u, so the HBM latency overlaps the staging.
 template <int WD, int CHD>
-__device__ void down_rows(const FusedArgs& a, const float* us, const int* pslot, const float* pgate, int l, int gw,
-                          int W) {
+__device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, const float* pgate, int l, int gw,
+                           int W) {
   constexpr int E = Tr<WD>::epc;
   constexpr int KR = 24 / CHD > 8 ? 8 : (24 / CHD < 1 ? 1 : 24 / CHD);
   const int lane = threadIdx.x & 31;
@@ -343,31 +407,38 @@ __device__ void down_rows(const FusedArgs& a, const float* us, const int* pslot,
   const int nch = (int)(rb / 16);
   const int G = a.I / 128;
   const int ipad = ipad_of(a.I);
-  for (int o = gw; o < a.d; o += W) {
-    float acc = 0.f;
-    for (int r0 = 0; r0 < a.k; r0 += KR) {
-      uint4 w[KR][CHD];
-      float sc[KR][CHD];
+  uint4 w[KR][CHD];
+  float sc[KR][CHD];
+  // loads of ranks [r0, r0 + KR) of row o into w / sc (predicated, no break: keeps them in registers)
+  auto issue = [&](int o, int r0) {
 #pragma unroll
-      for (int rr = 0; rr < KR; rr++) {
-        const int r = r0 + rr;
-        const bool rok = r < a.k;  // a predicate, not a break: keeps w[][] in registers
-        const uint8_t* slot = a.pool + (int64_t)pslot[rok ? r : 0] * a.slot_stride;
-        const int64_t roff = a.lay.d_off + (int64_t)o * rb;
+    for (int rr = 0; rr < KR; rr++) {
+      const int r = r0 + rr;
+      const bool rok = r < a.k && o < a.d;
+      const uint8_t* slot = a.pool + (int64_t)pslot[r < a.k ? r : 0] * a.slot_stride;
+      const int64_t roff = a.lay.d_off + (int64_t)(o < a.d ? o : 0) * rb;
+#pragma unroll
+      for (int j = 0; j < CHD; j++) {
+        const int c = j * 32 + lane;
+        w[rr][j] = (rok && c < nch) ? ld_cg(slot + roff + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+      }
+      if (WD == WD_INT4) {
+        const uint16_t* sp = (const uint16_t*)(slot + a.lay.d_scale_off) + (int64_t)(o < a.d ? o : 0) * G;
 #pragma unroll
         for (int j = 0; j < CHD; j++) {
           const int c = j * 32 + lane;
-          w[rr][j] = (rok && c < nch) ? ld_cg(slot + roff + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
-        }
-        if (WD == WD_INT4) {
-          const uint16_t* sp = (const uint16_t*)(slot + a.lay.d_scale_off) + (int64_t)o * G;
-#pragma unroll
-          for (int j = 0; j < CHD; j++) {
-            const int c = j * 32 + lane;
-            sc[rr][j] = (rok && c < nch) ? scale_at<WD>(sp + (c >> 2), false) : 0.f;
-          }
+          sc[rr][j] = (rok && c < nch) ? scale_at<WD>(sp + (c >> 2), false) : 0.f;
         }
       }
+    }
+  };
+  issue(gw, 0);
+  stage_u(a, us, ipad);
+  __syncthreads();
+  for (int o = gw; o < a.d; o += W) {
+    float acc = 0.f;
+    for (int r0 = 0; r0 < a.k; r0 += KR) {
+      if (o != gw || r0 != 0) issue(o, r0);
 #pragma unroll
       for (int rr = 0; rr < KR; rr++) {
         const int r = r0 + rr;
@@ -418,21 +489,45 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
 
   for (int l = 0; l < a.L; l++) {
     const int clock = (int)(step * a.L + l + 1);  // 0 is older than every step (preloaded experts)
-    // ---- phase R: router logits
-    stage16(reinterpret_cast<uint4*>(xs), (const uint8_t*)a.hidden + (int64_t)l * xbytes, xbytes, threadIdx.x,
-            blockDim.x);
-    __syncthreads();
-    for (int e = gw; e < a.E; e += W) {
-      const uint8_t* row = a.routers + ((int64_t)l * a.E + e) * xbytes;
-      float acc = 0.f;
-      for (int c = lane; c < nchr; c += 32) {
-        if (WD == WD_FP32)
-          acc = dot_chunk<WD_FP32>(ld_stream(row + (int64_t)c * 16), xs + (int64_t)c * 16, acc);
-        else
-          acc = dot_chunk<WD_BF16>(ld_stream(row + (int64_t)c * 16), xs + (int64_t)c * 16, acc);
+    // ---- phase R: router logits. A warp's row loads (8 chunks per lane at a time) are issued
+    // before the CTA stages h, so their latency overlaps the staging.
+    {
+      constexpr int RG = 8;
+      const bool has_row = gw < a.E;  // at most one row per warp (the grid has >= E warps)
+      const uint8_t* row = a.routers + ((int64_t)l * a.E + (has_row ? gw : 0)) * xbytes;
+      uint4 rw[RG];
+#pragma unroll
+      for (int j = 0; j < RG; j++) {
+        const int c = j * 32 + lane;
+        rw[j] = (has_row && c < nchr) ? ld_stream(row + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
       }
-      acc = warp_sum(acc);
-      if (lane == 0) a.z[e] = acc;
+      stage16(reinterpret_cast<uint4*>(xs), (const uint8_t*)a.hidden + (int64_t)l * xbytes, xbytes, threadIdx.x,
+              blockDim.x);
+      __syncthreads();
+      if (has_row) {
+        float acc = 0.f;
+        for (int c0 = 0; c0 < nchr; c0 += 32 * RG) {
+          if (c0 > 0) {
+#pragma unroll
+            for (int j = 0; j < RG; j++) {
+              const int c = c0 + j * 32 + lane;
+              rw[j] = c < nchr ? ld_stream(row + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < RG; j++) {
+            const int c = c0 + j * 32 + lane;
+            if (c < nchr) {
+              if (WD == WD_FP32)
+                acc = dot_chunk<WD_FP32>(rw[j], xs + (int64_t)c * 16, acc);
+              else
+                acc = dot_chunk<WD_BF16>(rw[j], xs + (int64_t)c * 16, acc);
+            }
+          }
+        }
+        acc = warp_sum(acc);
+        if (lane == 0) a.z[gw] = acc;
+      }
     }
     if (!grid_sync(a)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 0] = gtimer();
@@ -522,26 +617,15 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
     }
     if (!grid_sync(a)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 2] = gtimer();
-    // ---- phase D: down rows + combine (missed experts' W_d streamed into their slots)
-    {
-      const float4* u4 = reinterpret_cast<const float4*>(a.u);
-      const int n4 = a.k * a.I / 4;
-      for (int q = threadIdx.x; q < n4; q += blockDim.x) {
-        const float4 v = __ldcg(u4 + q);
-        const int r = (4 * q) / a.I;
-        const int i = 4 * q - r * a.I;
-        *reinterpret_cast<float4*>(us + r * ipad + upad(i)) = v;
-      }
-    }
-    __syncthreads();
+    // ---- phase D: down rows + combine, every expert read from its slot
     switch (chd_need) {
-      case 1: down_rows<WD, 1>(a, us, p_slot, p_gate, l, gw, W); break;
-      case 2: down_rows<WD, 2>(a, us, p_slot, p_gate, l, gw, W); break;
-      case 3: down_rows<WD, 3>(a, us, p_slot, p_gate, l, gw, W); break;
-      case 4: down_rows<WD, 4>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, gw, W); break;
       case 5:
-      case 6: down_rows<WD, 6>(a, us, p_slot, p_gate, l, gw, W); break;
-      default: down_rows<WD, 8>(a, us, p_slot, p_gate, l, gw, W); break;
+      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, gw, W); break;
+      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, gw, W); break;
     }
     if (!grid_sync(a)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 3] = gtimer();
@@ -575,7 +659,8 @@ int grid_of(size_t smem) {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  return sms * (occ < 2 ? occ : 2);
+  const int grid = sms * (occ < 2 ? occ : 2);
+  return grid * kFWarps >= 256 ? grid : 0;  // phase R gives each expert row its own warp
 }
 
 template <int WD, int CH>
