@@ -36,32 +36,34 @@ __device__ __forceinline__ uint64_t gtimer() {
   return t;
 }
 
-// Grid-wide barrier over co-resident CTAs with a bounded wait. Returns false once any CTA has
-// timed out (the caller then returns).
-__device__ bool grid_sync(const FusedArgs& a) {
-  __threadfence();
+// Grid-wide barrier over co-resident CTAs with a bounded wait. Each CTA's arrival is one
+// release-add on a counter that only grows; barrier number n of a launch completes when the
+// counter reaches bar_base + n * gridDim.x, which every CTA polls with acquire loads. Returns
+// false once any CTA has timed out (the caller then returns).
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ bool grid_sync(const FusedArgs& a, unsigned& nbar) {
   __syncthreads();
+  nbar++;
   if (threadIdx.x == 0) {
-    volatile unsigned* genp = a.bar_gen;
-    const unsigned g = *genp;
+    const unsigned target = a.bar_base + nbar * gridDim.x;
     __threadfence();
-    const unsigned arrived = atomicAdd(a.bar_count, 1u) + 1u;
-    if (arrived == gridDim.x) {
-      atomicExch(a.bar_count, 0u);
-      __threadfence();
-      atomicAdd(a.bar_gen, 1u);
-    } else {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a.bar_count), "r"(1u) : "memory");
+    if ((int)(ld_acquire_u32(a.bar_count) - target) < 0) {
       const uint64_t t0 = gtimer();
-      while (*genp == g) {
+      while ((int)(ld_acquire_u32(a.bar_count) - target) < 0) {
         if (*(volatile int*)a.err & FERR_BARRIER_TIMEOUT) break;
         if (gtimer() - t0 > a.barrier_timeout_ns) {
           atomicOr(a.err, FERR_BARRIER_TIMEOUT);
           break;
         }
-        __nanosleep(32);
+        __nanosleep(20);
       }
     }
-    __threadfence();
   }
   __syncthreads();
   return (*(volatile int*)a.err & FERR_BARRIER_TIMEOUT) == 0;
@@ -485,6 +487,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
   const int nchr = xbytes / 16;  // router rows: fp32 with fp32 weights, else bf16 (same bytes as h)
   const int ipad = ipad_of(a.I);
   int chd_need = (int)((a.lay.row_bytes_d / 16 + 31) / 32);
+  unsigned nbar = 0;  // grid barriers passed in this launch
   if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[a.L * 4] = gtimer();
 
   for (int l = 0; l < a.L; l++) {
@@ -529,11 +532,11 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
         if (lane == 0) a.z[gw] = acc;
       }
     }
-    if (!grid_sync(a)) return;
+    if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 0] = gtimer();
     // ---- phase S: selection and lookup table (CTA 0)
     if (blockIdx.x == 0) select_and_lookup(a, l, clock, step);
-    if (!grid_sync(a)) return;
+    if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 1] = gtimer();
     if (threadIdx.x < a.k) {
       p_slot[threadIdx.x] = __ldcg(a.plan_slot + threadIdx.x);
@@ -615,7 +618,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
         gateup_row<WD, CH>(a, slot, slot, false, xs, r, i, lane);
       }
     }
-    if (!grid_sync(a)) return;
+    if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 2] = gtimer();
     // ---- phase D: down rows + combine, every expert read from its slot
     switch (chd_need) {
@@ -627,7 +630,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
       case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, gw, W); break;
       default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, gw, W); break;
     }
-    if (!grid_sync(a)) return;
+    if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 3] = gtimer();
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;

@@ -45,8 +45,8 @@ struct FusedArgs {
   int32_t* route_idx;          // [L][k] routing of the last step
   float* route_gate;           // [L][k]
   unsigned long long* stats;   // [STAT_N]
-  unsigned* bar_count;
-  unsigned* bar_gen;
+  unsigned* bar_count;         // monotonic arrival counter of the grid barriers (wraps mod 2^32)
+  unsigned bar_base;           // its value when this launch starts
   int* err;                    // FERR_* flags, sticky until the host clears them
   unsigned long long barrier_timeout_ns;
   unsigned long long* phase_ts; // optional [L][4]: global-timer ns at the end of phases R, S, C, D

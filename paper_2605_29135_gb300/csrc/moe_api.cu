@@ -101,6 +101,7 @@ struct moe_handle {
   bool dev_mode = false;
   int fgrid = 0;
   int touch_shift = 12;
+  unsigned bar_epoch = 0;  // grid-barrier counter value at the start of the next fused launch
   const uint8_t* arena_dev = nullptr;
   int32_t* d_slot_of = nullptr;
   unsigned long long* d_slot_key = nullptr;
@@ -196,6 +197,7 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_trace_n, 0, sizeof(unsigned long long));
   cudaMemset(h->d_stats, 0, sizeof(unsigned long long) * moe::STAT_N);
   cudaMemset(h->d_bar, 0, sizeof(unsigned) * 2);
+  h->bar_epoch = 0;
   cudaMemset(h->d_err, 0, sizeof(int));
   cudaDeviceSynchronize();
   *h->h_err = 0;
@@ -587,7 +589,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, cudaStrea
   a.route_gate = h->d_route_gate;
   a.stats = h->d_stats;
   a.bar_count = h->d_bar;
-  a.bar_gen = h->d_bar + 1;
+  a.bar_base = h->bar_epoch;
   a.err = h->d_err;
   a.barrier_timeout_ns = 2000000000ull;
   a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
@@ -611,6 +613,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, cudaStrea
   MOE_CK(h, cudaEventRecord(h->err_ev, s));
   h->err_pending = true;
   h->steps_launched++;
+  h->bar_epoch += 4u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 4 barriers per layer
   if (a.phase_ts) {
     // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
     const int L = c.n_layers;
