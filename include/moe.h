@@ -71,7 +71,11 @@ enum {
  *   MOE_SCHEDULE_HOST_COPY_ENGINE: per layer, the routing result is published to mapped host
  *     memory, the host updates the lookup table and issues one cudaMemcpyAsync per miss on an
  *     internal copy stream; the hit experts' kernels run while the copies are in flight and
- *     each missed expert's kernels wait for its copy. moe_decode_step blocks once per layer. */
+ *     each missed expert's kernels wait for its copy. moe_decode_step blocks once per layer.
+ * Batched decoding (max_batch > 1, device schedule only; the paper describes batch-1 decoding and
+ * has no counterpart): per layer the needed experts are the union of the batch's top-k choices,
+ * one lookup-table step runs for that union (one record per distinct expert, ascending id), and
+ * each needed expert is read once and applied to every sequence routed to it. */
 enum { MOE_SCHEDULE_DEVICE = 0, MOE_SCHEDULE_HOST_COPY_ENGINE = 1 };
 
 typedef struct {
@@ -80,7 +84,8 @@ typedef struct {
   int32_t top_k;      /* experts per token, k (<= 16, <= E) */
   int32_t d_ff;       /* SwiGLU intermediate size, I */
   int32_t n_layers;   /* L */
-  int32_t max_batch;  /* sequences per decode step (this version: 1) */
+  int32_t max_batch;  /* most sequences per decode step, 1..64. Above 1 needs MOE_SCHEDULE_DEVICE, and a
+                         cap that can evict (cap < n_layers * n_experts) must be at most 4096 slots */
   int32_t wdtype;     /* MOE_DTYPE_FP32 (needs adtype FP32), BF16 or INT4_G128 (need adtype BF16) */
   int32_t adtype;     /* MOE_DTYPE_FP32 or MOE_DTYPE_BF16 */
   int64_t cap_slots;  /* expert slots on the device; 0 => floor(cap_bytes / expert bytes) */
@@ -151,8 +156,9 @@ moe_status moe_set_router(moe_handle* h, int32_t layer, const void* w_r);
 moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t expert, const void* w_gate,
                                      const void* w_up, const void* w_down, const void* scales);
 
-/* One decode step over all layers. hidden: device [n_layers x batch x d] (adtype), the input
- * of every layer; out: device [n_layers x batch x d] (adtype). Work is ordered on `stream`
+/* One decode step over all layers for `batch` sequences (1 <= batch <= max_batch; MOE_ERR_INVALID
+ * otherwise). hidden: device [n_layers x batch x d] (adtype), the input of every layer; out:
+ * device [n_layers x batch x d] (adtype). Work is ordered on `stream`
  * (a cudaStream_t; NULL = legacy default stream). hidden must stay valid and out must not be
  * read until `stream` reaches the end of the step. Calls on one handle must use one stream or
  * be serialised by the caller.
@@ -176,7 +182,9 @@ moe_status moe_decode_step_host(moe_handle* h, const void* hidden_host, void* ou
 moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* buf, int64_t cap,
                                    int64_t* n_copied, int64_t* n_total);
 
-/* Routing of the last decode step: idx int32 [n_layers x batch x k], gate fp32 [same]. */
+/* Routing of the last decode step: idx int32 [n_layers x max_batch x k], gate fp32 [same]; n is
+ * the entries buf can hold (MOE_ERR_INVALID if below n_layers * max_batch * k). Rows b >= the last
+ * step's batch are stale. */
 moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_t n);
 
 moe_status moe_get_stats(moe_handle* h, moe_stats* out);
@@ -192,8 +200,10 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded);
 
 /* Profiling: with on = 1, every kernel launch and miss copy of later steps is bracketed by
  * CUDA events on its stream. moe_profile_read waits for the recorded work, then reports one
- * entry per kernel class (router, gateup, down_combine, miss_copy) accumulated since the last
- * read, and clears the accumulators. */
+ * entry per kernel class (router, gateup, down_combine, miss_copy, fused_step) and, for the
+ * device schedule, per phase of the fused kernel (fused_phase_router, _select, _gateup, _down,
+ * and for batches _topk, _combine: per layer-step durations from the kernel's global timer),
+ * accumulated since the last read, and clears the accumulators. */
 moe_status moe_profile_enable(moe_handle* h, int32_t on);
 moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, int32_t* n_out);
 

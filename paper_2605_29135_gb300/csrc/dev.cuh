@@ -128,6 +128,13 @@ __device__ __forceinline__ void st_v4(uint8_t* p, const uint4& v) {
   asm volatile("st.global.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");
 }
 
+// An empty asm that claims to rewrite w: a loop that applies the same packed weights to several
+// activation vectors then unpacks them inside the loop instead of keeping every unpacked value
+// live across it (which would not fit in registers).
+__device__ __forceinline__ void opaque(uint4& w) {
+  asm volatile("" : "+r"(w.x), "+r"(w.y), "+r"(w.z), "+r"(w.w));
+}
+
 __host__ __device__ __forceinline__ int upad(int i) { return i + 4 * (i >> 5); }
 __host__ __device__ __forceinline__ int ipad_of(int I) { return upad((I + 31) & ~31); }
 

@@ -21,6 +21,8 @@
 
 #include "dev.cuh"
 #include "fused.cuh"
+#include "grid.cuh"
+#include "topk.cuh"
 
 namespace moe {
 namespace {
@@ -29,45 +31,6 @@ using namespace dev;
 
 constexpr int kFWarps = 8;
 constexpr int kFThreads = kFWarps * 32;
-
-__device__ __forceinline__ uint64_t gtimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-// Grid-wide barrier over co-resident CTAs with a bounded wait. Each CTA's arrival is one
-// release-add on a counter that only grows; barrier number n of a launch completes when the
-// counter reaches bar_base + n * gridDim.x, which every CTA polls with acquire loads. Returns
-// false once any CTA has timed out (the caller then returns).
-__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
-  unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
-__device__ bool grid_sync(const FusedArgs& a, unsigned& nbar) {
-  __syncthreads();
-  nbar++;
-  if (threadIdx.x == 0) {
-    const unsigned target = a.bar_base + nbar * gridDim.x;
-    __threadfence();
-    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a.bar_count), "r"(1u) : "memory");
-    if ((int)(ld_acquire_u32(a.bar_count) - target) < 0) {
-      const uint64_t t0 = gtimer();
-      while ((int)(ld_acquire_u32(a.bar_count) - target) < 0) {
-        if (*(volatile int*)a.err & FERR_BARRIER_TIMEOUT) break;
-        if (gtimer() - t0 > a.barrier_timeout_ns) {
-          atomicOr(a.err, FERR_BARRIER_TIMEOUT);
-          break;
-        }
-        __nanosleep(20);
-      }
-    }
-  }
-  __syncthreads();
-  return (*(volatile int*)a.err & FERR_BARRIER_TIMEOUT) == 0;
-}
 
 __device__ __forceinline__ unsigned long long shfl_min_u64(unsigned long long v) {
 #pragma unroll
@@ -95,45 +58,9 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (warp == 0) {
-    constexpr int PER = 8;  // E <= 256
-    uint32_t key[PER];
-#pragma unroll
-    for (int j = 0; j < PER; j++) {
-      const int e = j * 32 + lane;
-      key[j] = e < E ? ord_key(__ldcg(a.z + e)) : 0u;
-    }
-    float my_z = 0.f;
-    int my_i = -1;
-    for (int r = 0; r < k; r++) {
-      uint32_t bk = 0u;
-      int bi = 0x7fffffff;
-#pragma unroll
-      for (int j = 0; j < PER; j++) {
-        if (key[j] > bk) {
-          bk = key[j];
-          bi = j * 32 + lane;
-        }
-      }
-      const uint32_t mk = __reduce_max_sync(kFull, bk);
-      const int win = (int)__reduce_min_sync(kFull, bk == mk ? (uint32_t)bi : 0xffffffffu);
-      if (lane == r) {
-        my_z = key_value(mk);
-        my_i = win;
-      }
-#pragma unroll
-      for (int j = 0; j < PER; j++)
-        if (win == j * 32 + lane) key[j] = 0u;
-    }
-    const float m = __shfl_sync(kFull, my_z, 0);
-    const float ex = lane < k ? expf(my_z - m) : 0.f;
-    float denom;
-    if (a.renorm) {
-      denom = warp_sum(ex);
-    } else {
-      float part = 0.f;
-      for (int e = lane; e < E; e += 32) part += expf(__ldcg(a.z + e) - m);
-      denom = warp_sum(part);
-    }
+    int my_i;
+    float my_g;
+    warp_topk(a.z, E, k, a.renorm, lane, my_i, my_g);
     if (lane < k && (my_i < 0 || my_i >= E)) {
       atomicOr(a.err, FERR_BAD_ROUTE);
       my_i = lane;  // keep the step well-defined; the host reports the error
@@ -147,7 +74,7 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     }
     if (lane < k) {
       s_idx[lane] = my_i;
-      s_gate[lane] = ex / denom;
+      s_gate[lane] = my_g;
       s_need[pos] = gid;
     }
     __syncwarp();

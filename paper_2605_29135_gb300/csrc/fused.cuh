@@ -59,4 +59,62 @@ struct FusedArgs {
 int fused_grid(int wdtype, int d, int I, int k);
 cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s);
 
+// Batched decode step: B sequences per step, one cooperative kernel over all layers. Per layer
+// the needed experts are the union of every sequence's top k; each needed expert is read once
+// and applied to all the sequences routed to it (a grouped GEMV).
+constexpr int kMaxBatch = 64;
+constexpr int kBatchedEvictCap = 4096;  // slot counts this large or smaller can evict in a batched step
+constexpr int kBatchedPhases = 6;       // router, top-k, select, gate-up, down, combine
+
+struct BatchArgs {
+  int L, E, k, d, I, renorm, wdtype;
+  int B;                       // sequences this step (<= Bmax)
+  int Bmax;                    // row stride of the routing log
+  BlobLayout lay;
+  int64_t slot_stride;
+  int64_t cap;
+  int64_t n_gid;
+  const uint8_t* routers;      // device [L][E][d]
+  const void* hidden;          // device [L][B][d]
+  void* out;                   // device [L][B][d]
+  uint8_t* pool;
+  const uint8_t* arena;
+  int32_t* slot_of;
+  unsigned long long* slot_key;
+  int32_t* n_used;
+  int64_t* step;
+  // per-layer scratch
+  float* z;                    // [B][E]
+  int32_t* sel_e;              // [B*k] expert of pair p = b*k + r
+  float* sel_g;                // [B*k] its gate
+  int32_t* plan_n;             // [2] distinct experts needed this layer-step, and how many missed
+  int32_t* plan_slot;          // [E] per needed expert: the misses (ascending id), then the hits
+  int32_t* plan_gid;           // [E]
+  int32_t* plan_miss;          // [E]
+  int32_t* plan_off;           // [E] start of its pairs in plan_tok
+  int32_t* plan_cnt;           // [E] number of pairs routed to it
+  int32_t* plan_tok;           // [B*k] pair indices grouped by needed expert, ascending
+  float* u;                    // [B*k][I]
+  float* y;                    // [B*k][d]
+  TraceRec* trace;
+  int64_t trace_cap;
+  unsigned long long* trace_n;
+  int32_t* route_idx;          // [L][Bmax][k]
+  float* route_gate;           // [L][Bmax][k]
+  unsigned long long* stats;
+  unsigned* bar_count;
+  unsigned bar_base;
+  int* err;
+  unsigned long long barrier_timeout_ns;
+  unsigned long long* phase_ts; // optional [L][kBatchedPhases] + 1
+  int miss_ctas;
+  int touch_shift;
+  int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
+};
+
+// Pairs staged per group for this shape, and the co-resident grid (0: shape or cap unsupported).
+int batched_tg(int wdtype, int d, int I);
+int fused_batched_grid(int wdtype, int d, int I, int64_t cap, int64_t n_gid);
+cudaError_t launch_fused_batched(const BatchArgs& a, int grid, cudaStream_t s);
+
 }  // namespace moe

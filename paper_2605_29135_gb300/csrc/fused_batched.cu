@@ -1,0 +1,746 @@
+// Batched device-driven decode step (sm_103a): B sequences decode together, one cooperative
+// persistent kernel per step over all layers.
+//
+// Per layer, six phases separated by grid barriers:
+//   R  router logits z[b][e] = W_r[e] . h_b. A warp holds one router row in registers and applies
+//      it to a block of 8 sequences;
+//   T  per sequence b (one warp each): top k with ties to the lower id, and the gates. Pair
+//      p = b * k + r is rank r of sequence b;
+//   S  CTA 0: the needed experts are the union of all pairs' experts, ascending. One step of the
+//      lookup table for that set: hits keep their slot, misses (ascending id) take the lowest
+//      free slots, then the residents that no pair needs, smallest (last use, id) first (a bitonic
+//      sort of the slot keys in shared memory). It writes one trace record per needed expert, and
+//      the plan: the needed experts (misses first, then hits) with their slots and, per expert,
+//      the ascending list of pairs routed to it;
+//   C  grouped gate-up: a work item is (needed expert, block of rows). The CTA stages the
+//      activations of the expert's pairs in shared memory, and each warp reads a row pair once
+//      and applies it to every staged pair: u_p[i] = silu(W_g[i] . h_b) * (W_u[i] . h_b). Missed
+//      experts are worked by the last "miss CTAs": they read the rows from the page-locked host
+//      tier over NVLink-C2C, store them into the expert's slot and use them from registers, and
+//      copy the expert's W_d region into the slot; the other CTAs work the hits from HBM;
+//   D  grouped down projection: a work item is (needed expert, block of W_d rows); the CTA stages
+//      u of the expert's pairs and each warp applies its rows to all of them, y_p = W_d u_p;
+//   E  combine per sequence in rank order: out[b] = sum_r g_{b,r} y_{b*k+r}.
+//
+// Each expert is read from memory once per layer-step however many pairs it serves. All CTAs are
+// co-resident; every barrier wait is bounded and sets an error flag on expiry.
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include <algorithm>
+
+#include "dev.cuh"
+#include "fused.cuh"
+#include "grid.cuh"
+#include "topk.cuh"
+
+namespace moe {
+namespace {
+
+using namespace dev;
+
+constexpr int kBWarps = 8;
+constexpr int kBThreads = kBWarps * 32;
+constexpr int kMaxPairs = kMaxBatch * kMaxRanks;
+constexpr int kRowsGU = 64;   // gate/up row pairs per work item
+constexpr int kRowsD = 128;   // W_d rows per work item
+constexpr int kTGMax = 16;    // pairs staged per group
+
+int tg_of(int wdtype, int d, int I) {
+  const int xpad = (d * (wdtype == WD_FP32 ? 4 : 2) + 15) & ~15;
+  const int per = std::max(xpad, ipad_of(I) * 4);
+  return std::max(1, std::min(kTGMax, (96 * 1024) / per));
+}
+
+int sort_n_of(int64_t cap, int64_t n_gid) {
+  if (cap >= n_gid) return 0;  // never evicts
+  int n = 1;
+  while (n < cap) n <<= 1;
+  return n;
+}
+
+size_t batched_smem(int wdtype, int d, int I, int64_t cap, int64_t n_gid) {
+  const int xpad = (d * (wdtype == WD_FP32 ? 4 : 2) + 15) & ~15;
+  const size_t per = (size_t)std::max(xpad, ipad_of(I) * 4);
+  return std::max((size_t)tg_of(wdtype, d, I) * per, (size_t)sort_n_of(cap, n_gid) * sizeof(unsigned long long));
+}
+
+// ---- phase R: logits of one router row for up to 8 sequences
+template <int WDR>
+__device__ __forceinline__ void router_item(const BatchArgs& a, int l, int e, int b0, int lane) {
+  constexpr int RG = 8;
+  const int xbytes = a.d * (WDR == WD_FP32 ? 4 : 2);
+  const int nchr = xbytes / 16;
+  const uint8_t* row = a.routers + ((int64_t)l * a.E + e) * xbytes;
+  const int nt = a.B - b0 < 8 ? a.B - b0 : 8;
+  uint4 rw[RG];
+  if (nchr <= 32 * RG) {
+#pragma unroll
+    for (int j = 0; j < RG; j++) {
+      const int c = j * 32 + lane;
+      rw[j] = c < nchr ? ld_cg(row + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+    }
+  }
+#pragma unroll 1
+  for (int t = 0; t < nt; t++) {
+    const uint8_t* x = (const uint8_t*)a.hidden + ((int64_t)l * a.B + b0 + t) * xbytes;
+    float acc = 0.f;
+    for (int c0 = 0; c0 < nchr; c0 += 32 * RG) {
+      if (nchr > 32 * RG) {
+#pragma unroll
+        for (int j = 0; j < RG; j++) {
+          const int c = c0 + j * 32 + lane;
+          rw[j] = c < nchr ? ld_cg(row + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < RG; j++) {
+        const int c = c0 + j * 32 + lane;
+        if (c < nchr) acc = dot_chunk<WDR>(rw[j], x + (int64_t)c * 16, acc);
+      }
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) a.z[(int64_t)(b0 + t) * a.E + e] = acc;
+  }
+}
+
+// ---- phase S: union of the pairs' experts, one lookup-table step, trace and plan (CTA 0)
+__device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t step, unsigned long long* keys) {
+  __shared__ int s_sel[kMaxPairs];
+  __shared__ int s_flag[256];
+  __shared__ int s_need[256];    // needed expert ids (within the layer), ascending
+  __shared__ int s_slot[256];
+  __shared__ int s_miss[256];
+  __shared__ int s_mbefore[256]; // misses among needed[0..q)
+  __shared__ int s_evict[256];
+  __shared__ int s_pos[256];     // plan position of needed q: misses first, then hits
+  __shared__ int s_cnt[256];     // pairs per plan position
+  __shared__ int s_off[256];
+  __shared__ int s_n, s_nm, s_nused0, s_nfree, s_nev, s_nevicted;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int E = a.E, k = a.k, P = a.B * a.k;
+
+  for (int p = tid; p < P; p += blockDim.x) s_sel[p] = __ldcg(a.sel_e + p);
+  for (int e = tid; e < 256; e += blockDim.x) s_flag[e] = 0;
+  if (tid == 0) s_nevicted = 0;
+  __syncthreads();
+  for (int p = tid; p < P; p += blockDim.x) s_flag[s_sel[p]] = 1;
+  __syncthreads();
+  if (warp == 0) {
+    int base = 0;
+    for (int e0 = 0; e0 < E; e0 += 32) {
+      const int e = e0 + lane;
+      const bool f = e < E && s_flag[e];
+      const unsigned m = __ballot_sync(kFull, f);
+      if (f) s_need[base + __popc(m & ((1u << lane) - 1u))] = e;
+      base += __popc(m);
+    }
+    if (lane == 0) s_n = base;
+  }
+  __syncthreads();
+  const int n = s_n;
+  for (int q = tid; q < n; q += blockDim.x) {
+    const int sl = a.slot_of[l * E + s_need[q]];
+    s_slot[q] = sl;
+    s_miss[q] = sl < 0;
+    s_evict[q] = -1;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    int base = 0;
+    for (int q0 = 0; q0 < n; q0 += 32) {
+      const int q = q0 + lane;
+      const bool f = q < n && s_miss[q];
+      const unsigned m = __ballot_sync(kFull, f);
+      if (q < n) s_mbefore[q] = base + __popc(m & ((1u << lane) - 1u));
+      base += __popc(m);
+    }
+    if (lane == 0) {
+      const int nused = *a.n_used;
+      const int nfree = (int)(a.cap - nused);
+      const int take = base < nfree ? base : nfree;
+      *a.n_used = nused + take;
+      s_nm = base;
+      s_nused0 = nused;
+      s_nfree = nfree;
+      s_nev = base - take;
+    }
+  }
+  __syncthreads();
+  const int nm = s_nm, nfree = s_nfree, nev = s_nev;
+  if (nev > 0) {
+    // Every slot is occupied. Sort the slot keys (last use << 32 | id) ascending, with the slots
+    // of this step's hits pinned at the maximum: the first nev keys are the victims.
+    int N2 = 1;
+    while (N2 < a.cap) N2 <<= 1;
+    for (int s = tid; s < N2; s += blockDim.x) keys[s] = s < a.cap ? a.slot_key[s] : ~0ull;
+    __syncthreads();
+    for (int q = tid; q < n; q += blockDim.x)
+      if (!s_miss[q]) keys[s_slot[q]] = ~0ull;
+    __syncthreads();
+    for (int size = 2; size <= N2; size <<= 1) {
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        for (int i = tid; i < N2 / 2; i += blockDim.x) {
+          const int lo = 2 * i - (i & (stride - 1));
+          const int hi = lo + stride;
+          const unsigned long long x = keys[lo], y = keys[hi];
+          const bool up = (lo & size) == 0;
+          if ((x > y) == up) {
+            keys[lo] = y;
+            keys[hi] = x;
+          }
+        }
+        __syncthreads();
+      }
+    }
+  }
+  // place the misses: free slots first, then the victims in ascending key order
+  for (int q = tid; q < n; q += blockDim.x) {
+    if (!s_miss[q]) continue;
+    const int m = s_mbefore[q];
+    int slot = -1;
+    if (m < nfree) {
+      slot = s_nused0 + m;
+    } else {
+      const unsigned long long key = keys[m - nfree];
+      if (key == ~0ull) {
+        atomicOr(a.err, FERR_NO_VICTIM);
+      } else {
+        const int v = (int)(uint32_t)(key & 0xffffffffull);
+        slot = a.slot_of[v];
+        s_evict[q] = v;
+        atomicAdd(&s_nevicted, 1);
+      }
+    }
+    s_slot[q] = slot;
+  }
+  __syncthreads();
+  for (int q = tid; q < n; q += blockDim.x)
+    if (s_evict[q] >= 0) a.slot_of[s_evict[q]] = -1;
+  __syncthreads();
+  const unsigned long long base_rec = *(volatile unsigned long long*)a.trace_n;
+  for (int q = tid; q < n; q += blockDim.x) {
+    const int gid = l * E + s_need[q];
+    const int sl = s_slot[q];
+    if (s_miss[q] && sl >= 0) a.slot_of[gid] = sl;
+    if (sl >= 0) a.slot_key[sl] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)gid;
+    if (base_rec + q < (unsigned long long)a.trace_cap) {
+      TraceRec rec;
+      rec.step = (int32_t)step;
+      rec.layer = l;
+      rec.expert = s_need[q];
+      rec.kind = s_miss[q];
+      rec.slot = sl;
+      rec.evicted = s_evict[q];
+      a.trace[base_rec + q] = rec;
+    }
+    s_pos[q] = s_miss[q] ? s_mbefore[q] : nm + (q - s_mbefore[q]);
+  }
+  __syncthreads();
+  // pairs per needed expert, ascending pair order (one warp per expert, a ballot per 32 pairs)
+  for (int q = warp; q < n; q += kBWarps) {
+    const int e = s_need[q];
+    int cnt = 0;
+    for (int p0 = 0; p0 < P; p0 += 32) {
+      const int p = p0 + lane;
+      cnt += __popc(__ballot_sync(kFull, p < P && s_sel[p] == e));
+    }
+    if (lane == 0) s_cnt[s_pos[q]] = cnt;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    // exclusive scan of s_cnt[0..n) in plan order: 8 consecutive entries per lane
+    int v[8], sum = 0;
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+      const int q = lane * 8 + j;
+      v[j] = q < n ? s_cnt[q] : 0;
+      sum += v[j];
+    }
+    int inc = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int o = __shfl_up_sync(kFull, inc, off);
+      if (lane >= off) inc += o;
+    }
+    int run = inc - sum;
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+      const int q = lane * 8 + j;
+      if (q < n) s_off[q] = run;
+      run += v[j];
+    }
+  }
+  __syncthreads();
+  for (int q = warp; q < n; q += kBWarps) {
+    const int e = s_need[q];
+    const int pos = s_pos[q];
+    int w = s_off[pos];
+    for (int p0 = 0; p0 < P; p0 += 32) {
+      const int p = p0 + lane;
+      const bool f = p < P && s_sel[p] == e;
+      const unsigned m = __ballot_sync(kFull, f);
+      if (f) a.plan_tok[w + __popc(m & ((1u << lane) - 1u))] = p;
+      w += __popc(m);
+    }
+    if (lane == 0) {
+      const int sl = s_slot[q];
+      a.plan_slot[pos] = sl < 0 ? 0 : sl;
+      a.plan_gid[pos] = l * E + e;
+      a.plan_miss[pos] = s_miss[q];
+      a.plan_off[pos] = s_off[pos];
+      a.plan_cnt[pos] = s_cnt[pos];
+    }
+  }
+  if (tid == 0) {
+    a.plan_n[0] = n;
+    a.plan_n[1] = nm;
+    a.stats[STAT_HITS] += (unsigned long long)(n - nm);
+    a.stats[STAT_MISSES] += (unsigned long long)nm;
+    a.stats[STAT_LAYER_STEPS] += 1;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    a.stats[STAT_EVICTIONS] += (unsigned long long)s_nevicted;
+    *a.trace_n = base_rec + n;
+  }
+}
+
+template <int WD>
+__device__ __forceinline__ float scale_b(const uint16_t* p, bool from_host) {
+  return bf16_bits(from_host ? __ldg(p) : __ldcg(p));
+}
+
+// ---- phase C: one gate/up row pair of an expert applied to the tg staged pairs
+template <int WD, int CH>
+__device__ __forceinline__ void gateup_rows(const BatchArgs& a, const uint8_t* src, uint8_t* slot, bool from_host,
+                                            const uint8_t* xs, int xpad, const int* pidx, int tg, int i, int lane) {
+  const int64_t rb = a.lay.row_bytes_gu;
+  const int nch = (int)(rb / 16);
+  const int G = a.d / 128;
+  const int64_t goff = (int64_t)i * 2 * rb;
+  uint4 wg[CH], wu[CH];
+#pragma unroll
+  for (int j = 0; j < CH; j++) {
+    const int c = j * 32 + lane;
+    if (c < nch) {
+      if (from_host) {
+        wg[j] = ld_stream(src + goff + (int64_t)c * 16);
+        wu[j] = ld_stream(src + goff + rb + (int64_t)c * 16);
+      } else {
+        wg[j] = ld_cg(src + goff + (int64_t)c * 16);
+        wu[j] = ld_cg(src + goff + rb + (int64_t)c * 16);
+      }
+    } else {
+      wg[j] = make_uint4(0, 0, 0, 0);
+      wu[j] = make_uint4(0, 0, 0, 0);
+    }
+  }
+  float sg[CH], su[CH];
+  if (WD == WD_INT4) {
+    const uint16_t* sp = (const uint16_t*)(src + a.lay.gu_scale_off) + (int64_t)i * 2 * G;
+#pragma unroll
+    for (int j = 0; j < CH; j++) {
+      const int c = j * 32 + lane;
+      sg[j] = c < nch ? scale_b<WD>(sp + (c >> 2), from_host) : 0.f;
+      su[j] = c < nch ? scale_b<WD>(sp + G + (c >> 2), from_host) : 0.f;
+    }
+    if (from_host) {
+      uint16_t* dp = (uint16_t*)(slot + a.lay.gu_scale_off) + (int64_t)i * 2 * G;
+      for (int j = lane; j < 2 * G; j += 32) dp[j] = __ldg(sp + j);
+    }
+  }
+  if (from_host) {
+#pragma unroll
+    for (int j = 0; j < CH; j++) {
+      const int c = j * 32 + lane;
+      if (c < nch) {
+        st_v4(slot + goff + (int64_t)c * 16, wg[j]);
+        st_v4(slot + goff + rb + (int64_t)c * 16, wu[j]);
+      }
+    }
+  }
+#pragma unroll 1
+  for (int t = 0; t < tg; t++) {
+    const uint8_t* xt = xs + (int64_t)t * xpad;
+#pragma unroll
+    for (int j = 0; j < CH; j++) {
+      opaque(wg[j]);
+      opaque(wu[j]);
+    }
+    float ag = 0.f, au = 0.f;
+#pragma unroll
+    for (int j = 0; j < CH; j++) {
+      const int c = j * 32 + lane;
+      if (c < nch) {
+        const uint8_t* xc = xt + (int64_t)c * Tr<WD>::xbytes;
+        if (WD == WD_INT4) {
+          ag = fmaf(sg[j], dot_chunk<WD>(wg[j], xc, 0.f), ag);
+          au = fmaf(su[j], dot_chunk<WD>(wu[j], xc, 0.f), au);
+        } else {
+          ag = dot_chunk<WD>(wg[j], xc, ag);
+          au = dot_chunk<WD>(wu[j], xc, au);
+        }
+      }
+    }
+    ag = warp_sum(ag);
+    au = warp_sum(au);
+    if (lane == 0) a.u[(int64_t)pidx[t] * a.I + i] = ag / (1.0f + expf(-ag)) * au;
+  }
+}
+
+// Stage the activations of pairs plan_tok[off + g0 .. + tg) into xs (one row of xpad bytes each).
+__device__ __forceinline__ void stage_x(const BatchArgs& a, int l, int off, int g0, int tg, uint8_t* xs, int xpad,
+                                        int* pidx) {
+  const int xbytes = a.d * (a.wdtype == WD_FP32 ? 4 : 2);
+  const int nq = xbytes / 16;
+  if (threadIdx.x < tg) pidx[threadIdx.x] = __ldcg(a.plan_tok + off + g0 + threadIdx.x);
+  for (int q = threadIdx.x; q < tg * nq; q += blockDim.x) {
+    const int t = q / nq;
+    const int c = q - t * nq;
+    const int p = __ldcg(a.plan_tok + off + g0 + t);
+    const int b = p / a.k;
+    const uint4* src = reinterpret_cast<const uint4*>((const uint8_t*)a.hidden + ((int64_t)l * a.B + b) * xbytes);
+    *reinterpret_cast<uint4*>(xs + (int64_t)t * xpad + (int64_t)c * 16) = __ldg(src + c);
+  }
+}
+
+template <int WD, int CH>
+__device__ void gateup_item(const BatchArgs& a, int l, int pos, int rblk, bool host_src, uint8_t* smem, int* pidx,
+                            int tgmax) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int xpad = (a.d * (WD == WD_FP32 ? 4 : 2) + 15) & ~15;
+  const int gid = __ldcg(a.plan_gid + pos);
+  const int off = __ldcg(a.plan_off + pos);
+  const int cnt = __ldcg(a.plan_cnt + pos);
+  uint8_t* slot = a.pool + (int64_t)__ldcg(a.plan_slot + pos) * a.slot_stride;
+  const uint8_t* host = a.arena + (int64_t)gid * a.slot_stride;
+  const int i0 = rblk * kRowsGU;
+  const int i1 = i0 + kRowsGU < a.I ? i0 + kRowsGU : a.I;
+  for (int g0 = 0; g0 < cnt; g0 += tgmax) {
+    const int tg = cnt - g0 < tgmax ? cnt - g0 : tgmax;
+    __syncthreads();  // the previous group's readers are done with xs
+    stage_x(a, l, off, g0, tg, smem, xpad, pidx);
+    __syncthreads();
+    const bool from_host = host_src && g0 == 0;  // later groups reread the rows from the slot
+    for (int i = i0 + warp; i < i1; i += kBWarps)
+      gateup_rows<WD, CH>(a, from_host ? host : slot, slot, from_host, smem, xpad, pidx, tg, i, lane);
+  }
+  if (host_src) {
+    // this item's share of the expert's W_d region (and int4 scales): a plain copy host -> slot
+    const int nrb = (a.I + kRowsGU - 1) / kRowsGU;
+    const int64_t nq = (a.lay.total - a.lay.d_off) / 16;
+    const int64_t q0 = nq * rblk / nrb, q1 = nq * (rblk + 1) / nrb;
+    const uint8_t* src = host + a.lay.d_off;
+    uint8_t* dst = slot + a.lay.d_off;
+    const int T = blockDim.x;
+    int64_t q = q0 + threadIdx.x;
+    for (; q + 3 * (int64_t)T < q1; q += 4 * (int64_t)T) {
+      const uint4 v0 = ld_stream(src + q * 16);
+      const uint4 v1 = ld_stream(src + (q + T) * 16);
+      const uint4 v2 = ld_stream(src + (q + 2 * (int64_t)T) * 16);
+      const uint4 v3 = ld_stream(src + (q + 3 * (int64_t)T) * 16);
+      st_v4(dst + q * 16, v0);
+      st_v4(dst + (q + T) * 16, v1);
+      st_v4(dst + (q + 2 * (int64_t)T) * 16, v2);
+      st_v4(dst + (q + 3 * (int64_t)T) * 16, v3);
+    }
+    for (; q < q1; q += T) st_v4(dst + q * 16, ld_stream(src + q * 16));
+  }
+}
+
+// ---- phase D: KR rows of W_d (o, o + 8, ...) applied to the tg staged u vectors
+template <int WD, int CHD>
+__device__ void down_item(const BatchArgs& a, int pos, int oblk, float* us, int* pidx, int tgmax) {
+  constexpr int EPC = Tr<WD>::epc;
+  constexpr int KR = 16 / CHD > 4 ? 4 : (16 / CHD < 1 ? 1 : 16 / CHD);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t rb = a.lay.row_bytes_d;
+  const int nch = (int)(rb / 16);
+  const int G = a.I / 128;
+  const int ipad = ipad_of(a.I);
+  const int off = __ldcg(a.plan_off + pos);
+  const int cnt = __ldcg(a.plan_cnt + pos);
+  const uint8_t* slot = a.pool + (int64_t)__ldcg(a.plan_slot + pos) * a.slot_stride;
+  const int o0 = oblk * kRowsD;
+  const int o1 = o0 + kRowsD < a.d ? o0 + kRowsD : a.d;
+  for (int g0 = 0; g0 < cnt; g0 += tgmax) {
+    const int tg = cnt - g0 < tgmax ? cnt - g0 : tgmax;
+    __syncthreads();
+    if (threadIdx.x < tg) pidx[threadIdx.x] = __ldcg(a.plan_tok + off + g0 + threadIdx.x);
+    __syncthreads();
+    for (int q = threadIdx.x; q < tg * a.I; q += blockDim.x) {
+      const int t = q / a.I;
+      const int i = q - t * a.I;
+      us[t * ipad + upad(i)] = __ldcg(a.u + (int64_t)pidx[t] * a.I + i);
+    }
+    __syncthreads();
+    for (int ob = o0 + warp; ob < o1; ob += kBWarps * KR) {
+      uint4 w[KR][CHD];
+      float sc[KR][CHD];
+#pragma unroll
+      for (int rr = 0; rr < KR; rr++) {
+        const int o = ob + rr * kBWarps;
+        const bool ok = o < o1;
+        const int64_t roff = a.lay.d_off + (int64_t)(ok ? o : o0) * rb;
+#pragma unroll
+        for (int j = 0; j < CHD; j++) {
+          const int c = j * 32 + lane;
+          w[rr][j] = (ok && c < nch) ? ld_cg(slot + roff + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+        }
+        if (WD == WD_INT4) {
+          const uint16_t* sp = (const uint16_t*)(slot + a.lay.d_scale_off) + (int64_t)(ok ? o : o0) * G;
+#pragma unroll
+          for (int j = 0; j < CHD; j++) {
+            const int c = j * 32 + lane;
+            sc[rr][j] = (ok && c < nch) ? bf16_bits(__ldcg(sp + (c >> 2))) : 0.f;
+          }
+        }
+      }
+#pragma unroll 1
+      for (int t = 0; t < tg; t++) {
+        const float* ut = us + t * ipad;
+#pragma unroll
+        for (int rr = 0; rr < KR; rr++)
+#pragma unroll
+          for (int j = 0; j < CHD; j++) opaque(w[rr][j]);
+#pragma unroll
+        for (int rr = 0; rr < KR; rr++) {
+          float part = 0.f;
+#pragma unroll
+          for (int j = 0; j < CHD; j++) {
+            const int c = j * 32 + lane;
+            if (c < nch) {
+              if (WD == WD_INT4)
+                part = fmaf(sc[rr][j], dot_chunk_u<WD>(w[rr][j], ut + upad(c * EPC), 0.f), part);
+              else
+                part = dot_chunk_u<WD>(w[rr][j], ut + upad(c * EPC), part);
+            }
+          }
+          part = warp_sum(part);
+          const int o = ob + rr * kBWarps;
+          if (lane == 0 && o < o1) a.y[(int64_t)pidx[t] * a.d + o] = part;
+        }
+      }
+    }
+  }
+}
+
+template <int WD, int CH>
+__global__ void __launch_bounds__(kBThreads, 2) k_fused_batched(const __grid_constant__ BatchArgs a) {
+  extern __shared__ uint4 smem4[];
+  __shared__ int pidx[kTGMax];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(smem4);
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kBWarps + warp;
+  const int W = gridDim.x * kBWarps;
+  const int64_t step = *(volatile int64_t*)a.step;
+  const int tgmax = a.tg_max;
+  const int chd_need = (int)((a.lay.row_bytes_d / 16 + 31) / 32);
+  const int nrb = (a.I + kRowsGU - 1) / kRowsGU;
+  const int nob = (a.d + kRowsD - 1) / kRowsD;
+  unsigned nbar = 0;
+  if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[a.L * kBatchedPhases] = gtimer();
+  auto mark = [&](int l, int ph) {
+    if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * kBatchedPhases + ph] = gtimer();
+  };
+
+  for (int l = 0; l < a.L; l++) {
+    const int clock = (int)(step * a.L + l + 1);  // 0 is older than every step (preloaded experts)
+    // ---- R
+    {
+      const int nb8 = (a.B + 7) / 8;
+      for (int it = gw; it < a.E * nb8; it += W) {
+        const int e = it / nb8;
+        const int b0 = (it - e * nb8) * 8;
+        if (WD == WD_FP32)
+          router_item<WD_FP32>(a, l, e, b0, lane);
+        else
+          router_item<WD_BF16>(a, l, e, b0, lane);
+      }
+    }
+    if (!grid_sync(a, nbar)) return;
+    mark(l, 0);
+    // ---- T
+    for (int b = gw; b < a.B; b += W) {
+      int my_i;
+      float my_g;
+      warp_topk(a.z + (int64_t)b * a.E, a.E, a.k, a.renorm, lane, my_i, my_g);
+      if (lane < a.k) {
+        if (my_i < 0 || my_i >= a.E) {
+          atomicOr(a.err, FERR_BAD_ROUTE);
+          my_i = lane;  // keep the step well-defined; the host reports the error
+        }
+        a.sel_e[b * a.k + lane] = my_i;
+        a.sel_g[b * a.k + lane] = my_g;
+        a.route_idx[((int64_t)l * a.Bmax + b) * a.k + lane] = my_i;
+        a.route_gate[((int64_t)l * a.Bmax + b) * a.k + lane] = my_g;
+      }
+    }
+    if (!grid_sync(a, nbar)) return;
+    mark(l, 1);
+    // ---- S
+    if (blockIdx.x == 0) batched_select(a, l, clock, step, reinterpret_cast<unsigned long long*>(smem));
+    if (!grid_sync(a, nbar)) return;
+    mark(l, 2);
+    // ---- C
+    {
+      const int n = __ldcg(a.plan_n);
+      const int nm = __ldcg(a.plan_n + 1);
+      if (nm > 0) {
+        // warm the host-link address translations of every missed expert (one L2 prefetch per page)
+        const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
+        const int64_t gt0 = (int64_t)blockIdx.x * kBThreads + threadIdx.x;
+        const int64_t GT = (int64_t)gridDim.x * kBThreads;
+        for (int64_t q = gt0; q < (int64_t)nm * pages; q += GT) {
+          const int m = (int)(q / pages);
+          const uint8_t* pa =
+              a.arena + (int64_t)__ldcg(a.plan_gid + m) * a.slot_stride + ((q - (int64_t)m * pages) << a.touch_shift);
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+        }
+      }
+      const int mctas = nm > 0 ? (a.miss_ctas < (int)gridDim.x - 1 ? a.miss_ctas : (int)gridDim.x - 1) : 0;
+      const int hctas = (int)gridDim.x - mctas;
+      if ((int)blockIdx.x >= hctas) {
+        for (int it = (int)blockIdx.x - hctas; it < nm * nrb; it += mctas)
+          gateup_item<WD, CH>(a, l, it / nrb, it % nrb, true, smem, pidx, tgmax);
+      } else {
+        for (int it = blockIdx.x; it < (n - nm) * nrb; it += hctas)
+          gateup_item<WD, CH>(a, l, nm + it / nrb, it % nrb, false, smem, pidx, tgmax);
+      }
+    }
+    if (!grid_sync(a, nbar)) return;
+    mark(l, 3);
+    // ---- D
+    {
+      const int n = __ldcg(a.plan_n);
+      float* us = reinterpret_cast<float*>(smem);
+      for (int it = blockIdx.x; it < n * nob; it += gridDim.x) {
+        const int pos = it / nob, ob = it % nob;
+        switch (chd_need) {
+          case 1: down_item<WD, 1>(a, pos, ob, us, pidx, tgmax); break;
+          case 2: down_item<WD, 2>(a, pos, ob, us, pidx, tgmax); break;
+          case 3: down_item<WD, 3>(a, pos, ob, us, pidx, tgmax); break;
+          case 4: down_item<WD, 4>(a, pos, ob, us, pidx, tgmax); break;
+          case 5:
+          case 6: down_item<WD, 6>(a, pos, ob, us, pidx, tgmax); break;
+          default: down_item<WD, 8>(a, pos, ob, us, pidx, tgmax); break;
+        }
+      }
+    }
+    if (!grid_sync(a, nbar)) return;
+    mark(l, 4);
+    // ---- E: out[b][o] = sum_r g_{b,r} y_{b*k+r}[o], ranks in order
+    {
+      const int64_t nout = (int64_t)a.B * a.d;
+      for (int64_t q = (int64_t)blockIdx.x * kBThreads + threadIdx.x; q < nout; q += (int64_t)gridDim.x * kBThreads) {
+        const int b = (int)(q / a.d);
+        const int o = (int)(q - (int64_t)b * a.d);
+        float acc = 0.f;
+        for (int r = 0; r < a.k; r++) {
+          const int p = b * a.k + r;
+          acc = fmaf(__ldcg(a.sel_g + p), __ldcg(a.y + (int64_t)p * a.d + o), acc);
+        }
+        const int64_t oi = ((int64_t)l * a.B + b) * a.d + o;
+        if (WD == WD_FP32)
+          reinterpret_cast<float*>(a.out)[oi] = acc;
+        else
+          reinterpret_cast<__nv_bfloat16*>(a.out)[oi] = __float2bfloat16_rn(acc);
+      }
+    }
+    if (!grid_sync(a, nbar)) return;
+    mark(l, 5);
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
+}
+
+int pick_ch_b(int64_t rb) {
+  const int need = (int)((rb / 16 + 31) / 32);
+  if (need <= 1) return 1;
+  if (need <= 2) return 2;
+  if (need <= 4) return 4;
+  if (need <= 8) return 8;
+  if (need <= 16) return 16;
+  return -1;
+}
+
+template <int WD, int CH>
+int grid_of_b(size_t smem) {
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(k_fused_batched<WD, CH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  int occ = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_fused_batched<WD, CH>, kBThreads, smem) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms * (occ < 2 ? occ : 2);
+}
+
+template <int WD, int CH>
+cudaError_t run_fused_b(const BatchArgs& a, int grid, cudaStream_t s) {
+  const size_t smem = batched_smem(a.wdtype, a.d, a.I, a.cap, a.n_gid);
+  void* params[] = {(void*)&a};
+  return cudaLaunchCooperativeKernel((const void*)k_fused_batched<WD, CH>, dim3(grid), dim3(kBThreads), params, smem,
+                                     s);
+}
+
+}  // namespace
+
+#define MOE_B_DISPATCH(FN, WDV, CHV, ...)               \
+  do {                                                  \
+    switch (WDV) {                                      \
+      case WD_FP32:                                     \
+        switch (CHV) {                                  \
+          case 1: return FN<WD_FP32, 1>(__VA_ARGS__);   \
+          case 2: return FN<WD_FP32, 2>(__VA_ARGS__);   \
+          case 4: return FN<WD_FP32, 4>(__VA_ARGS__);   \
+          case 8: return FN<WD_FP32, 8>(__VA_ARGS__);   \
+        }                                               \
+        break;                                          \
+      case WD_BF16:                                     \
+        switch (CHV) {                                  \
+          case 1: return FN<WD_BF16, 1>(__VA_ARGS__);   \
+          case 2: return FN<WD_BF16, 2>(__VA_ARGS__);   \
+          case 4: return FN<WD_BF16, 4>(__VA_ARGS__);   \
+          case 8: return FN<WD_BF16, 8>(__VA_ARGS__);   \
+          case 16: return FN<WD_BF16, 16>(__VA_ARGS__); \
+        }                                               \
+        break;                                          \
+      case WD_INT4:                                     \
+        switch (CHV) {                                  \
+          case 1: return FN<WD_INT4, 1>(__VA_ARGS__);   \
+          case 2: return FN<WD_INT4, 2>(__VA_ARGS__);   \
+          case 4: return FN<WD_INT4, 4>(__VA_ARGS__);   \
+          case 8: return FN<WD_INT4, 8>(__VA_ARGS__);   \
+        }                                               \
+        break;                                          \
+    }                                                   \
+  } while (0)
+
+int batched_tg(int wdtype, int d, int I) { return tg_of(wdtype, d, I); }
+
+int fused_batched_grid(int wdtype, int d, int I, int64_t cap, int64_t n_gid) {
+  if (sort_n_of(cap, n_gid) > kBatchedEvictCap) return 0;
+  const BlobLayout lay = make_layout(wdtype, d, I);
+  const int ch = pick_ch_b(lay.row_bytes_gu);
+  const size_t smem = batched_smem(wdtype, d, I, cap, n_gid);
+  if (smem > 200 * 1024) return 0;
+  MOE_B_DISPATCH(grid_of_b, wdtype, ch, smem);
+  return 0;
+}
+
+cudaError_t launch_fused_batched(const BatchArgs& a, int grid, cudaStream_t s) {
+  const int ch = pick_ch_b(a.lay.row_bytes_gu);
+  MOE_B_DISPATCH(run_fused_b, a.wdtype, ch, a, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace moe

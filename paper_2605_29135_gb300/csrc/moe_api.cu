@@ -37,11 +37,11 @@ thread_local std::string g_create_error;
 
 enum {
   PC_ROUTER = 0, PC_GATEUP = 1, PC_DOWN = 2, PC_COPY = 3, PC_FUSED = 4,
-  PC_PH_R = 5, PC_PH_S = 6, PC_PH_C = 7, PC_PH_D = 8, PC_N = 9
+  PC_PH_R = 5, PC_PH_S = 6, PC_PH_C = 7, PC_PH_D = 8, PC_PH_T = 9, PC_PH_E = 10, PC_N = 11
 };
 const char* kPcName[PC_N] = {"router", "gateup", "down_combine", "miss_copy", "fused_step",
                              "fused_phase_router", "fused_phase_select", "fused_phase_gateup",
-                             "fused_phase_down"};
+                             "fused_phase_down", "fused_phase_topk", "fused_phase_combine"};
 
 struct PendingTime {
   int cls;
@@ -95,11 +95,13 @@ struct moe_handle {
   double pc_ms[PC_N] = {};
   int64_t pc_launches[PC_N] = {};
   int64_t pc_bytes[PC_N] = {};
-  unsigned long long* d_phase_ts = nullptr;   // [L*4+1] per-phase timestamps of the last profiled step
+  unsigned long long* d_phase_ts = nullptr;   // [L*phases+1] per-phase timestamps of the last profiled step
   std::vector<unsigned long long> h_phase_ts;
   // device-driven schedule: lookup table, scratch and outputs in device memory
   bool dev_mode = false;
+  bool batched = false;    // device schedule with max_batch > 1: the batched kernel
   int fgrid = 0;
+  int tg_max = 0;
   int touch_shift = 12;
   unsigned bar_epoch = 0;  // grid-barrier counter value at the start of the next fused launch
   const uint8_t* arena_dev = nullptr;
@@ -108,8 +110,10 @@ struct moe_handle {
   int32_t* d_n_used = nullptr;
   int64_t* d_step = nullptr;
   float* d_z = nullptr;
-  int32_t* d_plan = nullptr;  // slot[k], gid[k], miss[k]
-  float* d_plan_gate = nullptr;
+  int32_t* d_plan = nullptr;  // batch 1: slot[k], gid[k], miss[k]; batched: n, nm, 5 x [E], pairs[Bmax*k]
+  float* d_plan_gate = nullptr;  // batch 1: gate[k]; batched: gate per pair [Bmax*k]
+  int32_t* d_sel_e = nullptr;    // batched: expert per pair [Bmax*k]
+  float* d_y = nullptr;          // batched: W_d u per pair [Bmax*k][d]
   moe::TraceRec* d_trace = nullptr;
   unsigned long long* d_trace_n = nullptr;
   int32_t* d_route_idx = nullptr;
@@ -153,7 +157,8 @@ std::string check_config(const moe_config* c) {
     return "d, n_experts, top_k, d_ff and n_layers must be positive";
   if (c->n_experts > 256) return "n_experts must be <= 256";
   if (c->top_k > moe::kMaxRanks || c->top_k > c->n_experts) return "top_k must be <= 16 and <= n_experts";
-  if (c->max_batch != 1) return "max_batch must be 1 in this version";
+  if (c->max_batch < 1 || c->max_batch > moe::kMaxBatch) return "max_batch must be in [1, 64]";
+  if (c->max_batch > 1 && c->schedule != MOE_SCHEDULE_DEVICE) return "max_batch above 1 needs the device schedule";
   if ((int64_t)c->n_layers * c->n_experts > 0x7fffffffLL) return "too many experts";
   if (c->wdtype == MOE_DTYPE_FP32) {
     if (c->adtype != MOE_DTYPE_FP32) return "fp32 weights need fp32 activations";
@@ -174,7 +179,8 @@ std::string check_config(const moe_config* c) {
   const int64_t eb2 = c->wdtype == MOE_DTYPE_FP32 ? 8 : c->wdtype == MOE_DTYPE_BF16 ? 4 : 1;  // 2x bytes/elem
   if ((int64_t)c->d_ff * eb2 / 2 > 8 * 32 * 16) return "d_ff too large for the down-projection kernel";
   const int64_t ipad = align_up(c->d_ff, 32) + 4 * (align_up(c->d_ff, 32) / 32);
-  if ((int64_t)c->top_k * ipad * 4 > 200 * 1024) return "top_k * d_ff too large for shared-memory staging";
+  if (c->max_batch == 1 && (int64_t)c->top_k * ipad * 4 > 200 * 1024)
+    return "top_k * d_ff too large for shared-memory staging";
   if (c->renorm != 0 && c->renorm != 1) return "renorm must be 0 or 1";
   if (c->trace_capacity < 0) return "trace_capacity must be >= 0";
   if (c->schedule != MOE_SCHEDULE_DEVICE && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "unknown schedule";
@@ -551,9 +557,110 @@ moe_status check_device_error(moe_handle* h, bool sync) {
   return fail(h, (e & moe::FERR_BARRIER_TIMEOUT) ? MOE_ERR_TIMEOUT : MOE_ERR_CUDA, msg);
 }
 
-moe_status decode_device(moe_handle* h, const void* hidden, void* out, cudaStream_t s) {
+// Per-phase durations of the last profiled step from the kernel's global-timer stamps.
+moe_status harvest_phases(moe_handle* h, const unsigned long long* d_ts, int nph, const int* cls, cudaStream_t s) {
+  const int L = h->cfg.n_layers;
+  h->h_phase_ts.resize((size_t)nph * L + 1);
+  MOE_CK(h, cudaMemcpyAsync(h->h_phase_ts.data(), d_ts, sizeof(unsigned long long) * (nph * L + 1),
+                            cudaMemcpyDeviceToHost, s));
+  MOE_CK(h, cudaStreamSynchronize(s));
+  unsigned long long prev = h->h_phase_ts[(size_t)nph * L];
+  for (int l = 0; l < L; l++)
+    for (int p = 0; p < nph; p++) {
+      const unsigned long long t = h->h_phase_ts[(size_t)nph * l + p];
+      h->pc_ms[cls[p]] += (double)(t - prev) * 1e-6;
+      h->pc_launches[cls[p]] += 1;
+      prev = t;
+    }
+  return MOE_OK;
+}
+
+unsigned long long* phase_buffer(moe_handle* h) {
+  if (!h->prof) return nullptr;
+  if (!h->d_phase_ts &&
+      cudaMalloc(&h->d_phase_ts, sizeof(unsigned long long) * (moe::kBatchedPhases * h->cfg.n_layers + 1)) !=
+          cudaSuccess) {
+    h->d_phase_ts = nullptr;
+    cudaGetLastError();
+  }
+  return h->d_phase_ts;
+}
+
+moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
+  const moe_config& c = h->cfg;
+  const int k = c.top_k, E = c.n_experts;
+  moe::BatchArgs a{};
+  a.L = c.n_layers;
+  a.E = E;
+  a.k = k;
+  a.d = c.d;
+  a.I = c.d_ff;
+  a.renorm = c.renorm;
+  a.wdtype = c.wdtype;
+  a.B = batch;
+  a.Bmax = c.max_batch;
+  a.lay = h->lay;
+  a.slot_stride = h->slot_stride;
+  a.cap = h->cap;
+  a.n_gid = h->n_gid;
+  a.routers = h->routers;
+  a.hidden = hidden;
+  a.out = out;
+  a.pool = h->pool;
+  a.arena = h->arena_dev;
+  a.slot_of = h->d_slot_of;
+  a.slot_key = h->d_slot_key;
+  a.n_used = h->d_n_used;
+  a.step = h->d_step;
+  a.z = h->d_z;
+  a.sel_e = h->d_sel_e;
+  a.sel_g = h->d_plan_gate;
+  a.plan_n = h->d_plan;
+  a.plan_slot = h->d_plan + 2;
+  a.plan_gid = h->d_plan + 2 + E;
+  a.plan_miss = h->d_plan + 2 + 2 * E;
+  a.plan_off = h->d_plan + 2 + 3 * E;
+  a.plan_cnt = h->d_plan + 2 + 4 * E;
+  a.plan_tok = h->d_plan + 2 + 5 * E;
+  a.u = h->u;
+  a.y = h->d_y;
+  a.trace = h->d_trace;
+  a.trace_cap = c.trace_capacity;
+  a.trace_n = h->d_trace_n;
+  a.route_idx = h->d_route_idx;
+  a.route_gate = h->d_route_gate;
+  a.stats = h->d_stats;
+  a.bar_count = h->d_bar;
+  a.bar_base = h->bar_epoch;
+  a.err = h->d_err;
+  a.barrier_timeout_ns = 2000000000ull;
+  a.phase_ts = phase_buffer(h);
+  a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
+  a.touch_shift = h->touch_shift;
+  a.tg_max = h->tg_max;
+  {
+    ProfScope ps(h, s, PC_FUSED, (int64_t)c.n_layers * (int64_t)E * c.d * h->router_eb);
+    cudaError_t e = moe::launch_fused_batched(a, h->fgrid, s);
+    ps.done();
+    if (e != cudaSuccess) return cuda_fail(h, e, "batched decode step launch");
+  }
+  MOE_CK(h, cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, s));
+  MOE_CK(h, cudaEventRecord(h->err_ev, s));
+  h->err_pending = true;
+  h->steps_launched++;
+  // every CTA arrives at each phase's barrier once per layer
+  h->bar_epoch += (unsigned)moe::kBatchedPhases * (unsigned)c.n_layers * (unsigned)h->fgrid;
+  if (a.phase_ts) {
+    static const int cls[moe::kBatchedPhases] = {PC_PH_R, PC_PH_T, PC_PH_S, PC_PH_C, PC_PH_D, PC_PH_E};
+    return harvest_phases(h, a.phase_ts, moe::kBatchedPhases, cls, s);
+  }
+  return MOE_OK;
+}
+
+moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
   moe_status st = check_device_error(h, false);
   if (st != MOE_OK) return st;
+  if (h->batched) return decode_batched(h, hidden, out, batch, s);
   const moe_config& c = h->cfg;
   const int k = c.top_k;
   moe::FusedArgs a{};
@@ -594,14 +701,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, cudaStrea
   a.barrier_timeout_ns = 2000000000ull;
   a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
   a.touch_shift = h->touch_shift;
-  a.phase_ts = nullptr;
-  if (h->prof) {
-    if (!h->d_phase_ts && cudaMalloc(&h->d_phase_ts, sizeof(unsigned long long) * (4 * c.n_layers + 1)) != cudaSuccess) {
-      h->d_phase_ts = nullptr;
-      cudaGetLastError();
-    }
-    a.phase_ts = h->d_phase_ts;
-  }
+  a.phase_ts = phase_buffer(h);
   {
     ProfScope ps(h, s, PC_FUSED,
                  (int64_t)c.n_layers * (k * h->lay.total + (int64_t)c.n_experts * c.d * h->router_eb));
@@ -616,19 +716,8 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, cudaStrea
   h->bar_epoch += 4u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 4 barriers per layer
   if (a.phase_ts) {
     // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
-    const int L = c.n_layers;
-    h->h_phase_ts.resize(4 * L + 1);
-    MOE_CK(h, cudaMemcpyAsync(h->h_phase_ts.data(), a.phase_ts, sizeof(unsigned long long) * (4 * L + 1),
-                              cudaMemcpyDeviceToHost, s));
-    MOE_CK(h, cudaStreamSynchronize(s));
-    unsigned long long prev = h->h_phase_ts[4 * L];
-    for (int l = 0; l < L; l++)
-      for (int p = 0; p < 4; p++) {
-        const unsigned long long t = h->h_phase_ts[4 * l + p];
-        h->pc_ms[PC_PH_R + p] += (double)(t - prev) * 1e-6;
-        h->pc_launches[PC_PH_R + p] += 1;
-        prev = t;
-      }
+    static const int cls[4] = {PC_PH_R, PC_PH_S, PC_PH_C, PC_PH_D};
+    return harvest_phases(h, a.phase_ts, 4, cls, s);
   }
   return MOE_OK;
 }
@@ -652,7 +741,7 @@ void free_all(moe_handle* h) {
   for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_n_used,
                   (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
                   (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
-                  (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts})
+                  (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y})
     if (p) cudaFree(p);
   if (h->h_err) cudaFreeHost(h->h_err);
   if (h->err_ev) cudaEventDestroy(h->err_ev);
@@ -730,7 +819,8 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   h->route->seq = 0;
   if (cudaHostGetDevicePointer((void**)&h->route_dev, (void*)h->route, 0) != cudaSuccess)
     return bail(MOE_ERR_CUDA, "mapped routing buffer has no device address");
-  if (cudaMalloc(&h->u, sizeof(float) * cfg->top_k * cfg->d_ff) != cudaSuccess) return bail(MOE_ERR_OOM, "u allocation failed");
+  if (cudaMalloc(&h->u, sizeof(float) * cfg->max_batch * cfg->top_k * cfg->d_ff) != cudaSuccess)
+    return bail(MOE_ERR_OOM, "u allocation failed");
   const int64_t act = (int64_t)cfg->n_layers * cfg->max_batch * cfg->d * h->asize;
   if (cudaMalloc(&h->hid_dev, act) != cudaSuccess || cudaMalloc(&h->out_dev, act) != cudaSuccess)
     return bail(MOE_ERR_OOM, "staging allocation failed");
@@ -741,23 +831,36 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   for (auto& e : h->copy_ev)
     if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
   h->dev_mode = cfg->schedule == MOE_SCHEDULE_DEVICE;
-  if (h->dev_mode) {
+  h->batched = h->dev_mode && cfg->max_batch > 1;
+  if (h->batched) {
+    h->fgrid = moe::fused_batched_grid(cfg->wdtype, cfg->d, cfg->d_ff, h->cap, h->n_gid);
+    h->tg_max = moe::batched_tg(cfg->wdtype, cfg->d, cfg->d_ff);
+    if (h->fgrid <= 0)
+      return bail(MOE_ERR_INVALID, "shape or cap not supported by the batched schedule (a cap that can evict must be "
+                                   "at most 4096 slots)");
+  } else if (h->dev_mode) {
     h->fgrid = moe::fused_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
     if (h->fgrid <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the device-driven schedule");
+  }
+  if (h->dev_mode) {
     if (cudaHostGetDevicePointer((void**)&h->arena_dev, h->arena, 0) != cudaSuccess)
       return bail(MOE_ERR_CUDA, "host arena has no device address");
     const int k = cfg->top_k;
+    const int64_t pairs = (int64_t)cfg->max_batch * k;
+    const int64_t plan_ints = h->batched ? 2 + 5 * (int64_t)cfg->n_experts + pairs : 3 * (int64_t)k;
     bool ok = cudaMalloc(&h->d_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
               cudaMalloc(&h->d_slot_key, sizeof(unsigned long long) * h->cap) == cudaSuccess &&
               cudaMalloc(&h->d_n_used, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_step, sizeof(int64_t)) == cudaSuccess &&
-              cudaMalloc(&h->d_z, sizeof(float) * 256) == cudaSuccess &&
-              cudaMalloc(&h->d_plan, sizeof(int32_t) * 3 * k) == cudaSuccess &&
-              cudaMalloc(&h->d_plan_gate, sizeof(float) * k) == cudaSuccess &&
+              cudaMalloc(&h->d_z, sizeof(float) * 256 * cfg->max_batch) == cudaSuccess &&
+              cudaMalloc(&h->d_plan, sizeof(int32_t) * plan_ints) == cudaSuccess &&
+              cudaMalloc(&h->d_plan_gate, sizeof(float) * pairs) == cudaSuccess &&
+              (!h->batched || cudaMalloc(&h->d_sel_e, sizeof(int32_t) * pairs) == cudaSuccess) &&
+              (!h->batched || cudaMalloc(&h->d_y, sizeof(float) * pairs * cfg->d) == cudaSuccess) &&
               cudaMalloc(&h->d_trace, sizeof(moe::TraceRec) * std::max<int64_t>(1, cfg->trace_capacity)) == cudaSuccess &&
               cudaMalloc(&h->d_trace_n, sizeof(unsigned long long)) == cudaSuccess &&
-              cudaMalloc(&h->d_route_idx, sizeof(int32_t) * cfg->n_layers * k) == cudaSuccess &&
-              cudaMalloc(&h->d_route_gate, sizeof(float) * cfg->n_layers * k) == cudaSuccess &&
+              cudaMalloc(&h->d_route_idx, sizeof(int32_t) * cfg->n_layers * pairs) == cudaSuccess &&
+              cudaMalloc(&h->d_route_gate, sizeof(float) * cfg->n_layers * pairs) == cudaSuccess &&
               cudaMalloc(&h->d_stats, sizeof(unsigned long long) * moe::STAT_N) == cudaSuccess &&
               cudaMalloc(&h->d_bar, sizeof(unsigned) * 2) == cudaSuccess &&
               cudaMalloc(&h->d_err, sizeof(int)) == cudaSuccess &&
@@ -826,7 +929,7 @@ moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t exper
 moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t batch, void* stream) {
   if (!h) return MOE_ERR_INVALID;
   if (!hidden || !out) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
-  if (batch != 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be 1 in this version");
+  if (batch < 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be in [1, max_batch]");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   if (!h->all_registered) {
     for (int32_t l = 0; l < h->cfg.n_layers; l++)
@@ -837,7 +940,7 @@ moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t
                                                    std::to_string(g / h->cfg.n_experts) + " not registered");
     h->all_registered = true;
   }
-  moe_status st = h->dev_mode ? decode_device(h, hidden, out, (cudaStream_t)stream)
+  moe_status st = h->dev_mode ? decode_device(h, hidden, out, batch, (cudaStream_t)stream)
                               : decode_impl(h, hidden, out, (cudaStream_t)stream);
   if (st != MOE_OK) {
     // The pool contents are unknown after a failed step: wait for the streams, empty the pool.
@@ -854,7 +957,7 @@ moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t
 moe_status moe_decode_step_host(moe_handle* h, const void* hidden_host, void* out_host, int32_t batch) {
   if (!h) return MOE_ERR_INVALID;
   if (!hidden_host || !out_host) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
-  if (batch != 1) return fail(h, MOE_ERR_INVALID, "batch must be 1 in this version");
+  if (batch < 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be in [1, max_batch]");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   const int64_t bytes = (int64_t)h->cfg.n_layers * batch * h->cfg.d * h->asize;
   MOE_CK(h, cudaMemcpyAsync(h->hid_dev, hidden_host, bytes, cudaMemcpyHostToDevice, h->host_stream));
@@ -895,7 +998,7 @@ moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* 
 moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_t n) {
   if (!h) return MOE_ERR_INVALID;
   if (h->dev_mode) {
-    const int64_t cnt = (int64_t)h->cfg.n_layers * h->cfg.top_k;
+    const int64_t cnt = (int64_t)h->cfg.n_layers * h->cfg.max_batch * h->cfg.top_k;
     if (n < cnt) return fail(h, MOE_ERR_INVALID, "routing buffer too small");
     MOE_CK(h, cudaSetDevice(h->cfg.device));
     moe_status st = check_device_error(h, true);

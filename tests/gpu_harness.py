@@ -13,7 +13,8 @@ NEAR_TIE = 1e-4  # oracle logit gap under which a top-k flip is accepted
 
 
 def run_gpu(m, hidden: np.ndarray, dtype_out: str):
-    """Decode every step of `hidden` [T x L x B x d] through moe_decode_step on device buffers."""
+    """Decode every step of `hidden` [T x L x B x d] through moe_decode_step on device buffers
+    (B sequences per step)."""
     import torch
 
     T = hidden.shape[0]
@@ -26,9 +27,11 @@ def run_gpu(m, hidden: np.ndarray, dtype_out: str):
     out = torch.empty(hid.shape, dtype=tdt, device=dev)
     idx = np.empty(hidden.shape[:3] + (m.cfg.top_k,), dtype=np.int32)
     gate = np.empty(idx.shape, dtype=np.float32)
+    B = hidden.shape[2]
     for t in range(T):
-        m.decode_step(hid[t], out[t])
-        idx[t], gate[t] = m.get_last_routing()
+        m.decode_step(hid[t], out[t], batch=B)
+        i, g = m.get_last_routing()
+        idx[t], gate[t] = i[:, :B], g[:, :B]
     torch.cuda.synchronize()
     o = out.float().cpu().numpy().astype(np.float64)
     return o, idx, gate

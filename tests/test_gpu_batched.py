@@ -1,0 +1,190 @@
+"""GPU parity of the batched decode step (max_batch > 1) against the fp64 oracle.
+
+Per layer-step the needed experts are the union of all sequences' top-k choices; the oracle
+runs one lookup-table step for that union (one record per distinct expert, ascending id) and
+evaluates every sequence's experts. Checks, through the C ABI, on the same seeded inputs:
+the residency trace bit-exact; top-k ids exact except near-ties; gates to fp32 rounding;
+outputs per (token, layer, sequence) row within the dtype's relative L2 bound. Shapes span
+several work items with ragged tails (d, d_ff not multiples of the item sizes, odd batch
+sizes), a Qwen3-30B-A3B-shaped layer at batch 64, and the 48-layer stack at batch 64 with
+a 6 GB pool cap (635 slots) for a few steps.
+"""
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests.gpu_harness import TOL, check_routing, oracle_trace, rel_l2_rows, run_gpu, trace_tuples
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    import paper_2605_29135_gb300 as P
+
+    P.build()
+    return P
+
+
+def _create(wl, cap, **kw):
+    from paper_2605_29135_gb300.workload import create_for_workload
+
+    return create_for_workload(wl, cap_slots=cap, **kw)
+
+
+def _check_outputs(wl, hidden, idx, gate, out, samples, threads=8):
+    routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
+    orc = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers)
+
+    def one(tlb):
+        t, l, b = tlb
+        ref, _, g = orc.moe_layer(l, hidden[t, l, b], forced_idx=idx[t, l, b])
+        return t, l, b, ref, g
+
+    with ThreadPoolExecutor(max_workers=threads) as ex:
+        res = list(ex.map(one, samples))
+    errs = []
+    for t, l, b, ref, g in res:
+        np.testing.assert_allclose(gate[t, l, b], g, rtol=2e-5, atol=1e-6)
+        errs.append(rel_l2_rows(out[t, l, b], ref))
+    errs = np.array(errs)
+    assert errs.max() <= TOL[wl.wdtype], f"max rel L2 {errs.max():.3e} (mean {errs.mean():.3e})"
+    return errs
+
+
+def _parity(wl, cap, samples=None, threads=8, preload=False):
+    hidden = synth.hidden_all(wl)
+    m = _create(wl, cap)
+    try:
+        if preload:
+            m.preload()
+        out, idx, gate = run_gpu(m, hidden, wl.adtype)
+        tr = m.get_residency_trace()
+        stats = m.get_stats()
+    finally:
+        m.destroy()
+    routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
+    if preload:
+        orc = oracle.Oracle.for_workload(wl, cap_slots=cap, keep_slot_copies=False, routers=routers)
+        orc.preload()
+        otr = np.concatenate([orc.decode_step(hidden[t], compute_out=False, forced_idx=idx[t]).records
+                              for t in range(wl.tokens)])
+    else:
+        oidx, oz, otr = oracle_trace(wl, hidden, cap, routers=routers)
+        if check_routing(idx, oidx, oz, wl.top_k):
+            _, _, otr = oracle_trace(wl, hidden, cap, forced_idx=idx, routers=routers)
+    np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(otr))
+    assert stats["hits"] + stats["misses"] == len(tr)
+    assert stats["misses"] == int((tr["kind"] == 1).sum())
+    assert stats["evictions"] == int((tr["evicted"] >= 0).sum())
+    if samples is None:
+        samples = [(t, l, b) for t in range(wl.tokens) for l in range(wl.n_layers) for b in range(wl.batch)]
+    _check_outputs(wl, hidden, idx, gate, out, samples, threads)
+    return out, tr
+
+
+BATCHED = {
+    "fp32": synth.Workload("b_fp32", d=256, n_experts=8, top_k=2, d_ff=128, n_layers=3, wdtype="fp32",
+                           adtype="fp32", tokens=24, batch=4, rho=0.9, cap_slots=10),
+    "fp32_ragged": synth.Workload("b_fp32_ragged", d=100, n_experts=5, top_k=2, d_ff=36, n_layers=2, wdtype="fp32",
+                                  adtype="fp32", tokens=16, batch=3, rho=0.9, cap_slots=6),
+    "bf16_ragged": synth.Workload("b_bf16_ragged", d=640, n_experts=24, top_k=5, d_ff=200, n_layers=3,
+                                  wdtype="bf16", adtype="bf16", tokens=10, batch=5, rho=0.8, cap_slots=30),
+    "int4": synth.Workload("b_int4", d=384, n_experts=12, top_k=3, d_ff=256, n_layers=2, wdtype="int4",
+                           adtype="bf16", tokens=10, batch=6, rho=0.8, cap_slots=14),
+    "bf16_wide": synth.Workload("b_bf16_wide", d=4096, n_experts=64, top_k=16, d_ff=1536, n_layers=2,
+                                wdtype="bf16", adtype="bf16", tokens=3, batch=7, rho=0.8, cap_slots=80),
+}
+
+
+@pytest.mark.parametrize("name", list(BATCHED))
+def test_batched_small_shapes(P, name):
+    wl = BATCHED[name]
+    out, tr = _parity(wl, wl.cap_slots)
+    assert (tr["kind"] == 0).any() and (tr["evicted"] >= 0).any()
+
+
+def test_batched_cap_invariance_bit_exact(P):
+    # residency only changes where the weights are read from: outputs with a capped pool that
+    # evicts every step and with every expert resident are identical
+    wl = BATCHED["bf16_ragged"]
+    hidden = synth.hidden_all(wl)
+    outs = []
+    for cap in (wl.cap_slots, wl.n_gid):
+        m = _create(wl, cap)
+        try:
+            outs.append(run_gpu(m, hidden, wl.adtype)[0])
+        finally:
+            m.destroy()
+    np.testing.assert_array_equal(outs[0], outs[1])
+
+
+def test_batched_preload_all_resident_only_hits(P):
+    wl = BATCHED["int4"]
+    _, tr = _parity(wl, wl.n_gid, preload=True)
+    assert (tr["kind"] == 0).all()
+
+
+def test_batch_size_varies_between_steps(P):
+    # a handle made for up to 6 sequences decodes steps of 6, 1, 4 and 6 sequences; the oracle
+    # runs the same steps on the same rows
+    import torch
+
+    wl = BATCHED["int4"]
+    hidden = synth.hidden_all(wl)
+    sizes = [6, 1, 4, 6]
+    m = _create(wl, wl.cap_slots)
+    dev = torch.device("cuda", 0)
+    outs, idxs = [], []
+    try:
+        for t, B in enumerate(sizes):
+            h = torch.from_numpy(np.ascontiguousarray(hidden[t, :, :B]).view(np.int16)).to(dev).view(torch.bfloat16)
+            o = torch.empty_like(h)
+            m.decode_step(h, o, batch=B)
+            i, _ = m.get_last_routing()
+            idxs.append(i[:, :B].copy())
+            outs.append(o.float().cpu().numpy().astype(np.float64))
+        tr = m.get_residency_trace()
+    finally:
+        m.destroy()
+    orc = oracle.Oracle.for_workload(wl, keep_slot_copies=False)
+    recs = []
+    for t, B in enumerate(sizes):
+        r = orc.decode_step(np.ascontiguousarray(hidden[t, :, :B]), forced_idx=idxs[t])
+        recs.append(r.records)
+        assert rel_l2_rows(outs[t], r.out).max() <= TOL[wl.wdtype]
+    np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate(recs)))
+
+
+def test_batch_above_max_is_rejected(P):
+    import torch
+
+    wl = BATCHED["fp32"]
+    m = _create(wl, wl.cap_slots)
+    try:
+        h = torch.zeros((wl.n_layers, wl.batch + 1, wl.d), dtype=torch.float32, device="cuda")
+        with pytest.raises(P.MoEError) as ei:
+            m.decode_step(h, torch.empty_like(h), batch=wl.batch + 1)
+        assert ei.value.status == -1  # MOE_ERR_INVALID
+    finally:
+        m.destroy()
+
+
+def test_layer_bf16_batch64(P):
+    # Qwen3-30B-A3B-shaped layers, 64 sequences: 512 routed pairs per layer-step over ~126 experts
+    wl = synth.WORKLOADS["layer_bf16"].replace(name="layer_bf16_b64", n_layers=2, batch=64, tokens=4, cap_slots=200)
+    rng = np.random.default_rng(0)
+    samples = [(t, l, int(b)) for t in range(wl.tokens) for l in range(wl.n_layers)
+               for b in rng.choice(64, size=4, replace=False)]
+    _parity(wl, wl.cap_slots, samples=samples, threads=16)
+
+
+def test_stack48_batch64_capped_steps(P):
+    # the 48-layer bf16 stack at batch 64 under the 6 GB pool cap (635 slots): a few full steps
+    wl = synth.WORKLOADS["stack48_batch64"].replace(tokens=3)
+    samples = [(t, l, b) for t in (0, 2) for l in (0, 17, 47) for b in (0, 31, 63)]
+    _, tr = _parity(wl, wl.cap_slots, samples=samples, threads=16)
+    assert (tr["evicted"] >= 0).any()
