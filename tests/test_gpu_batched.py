@@ -88,11 +88,11 @@ def _parity(wl, cap, samples=None, threads=8, preload=False):
 
 BATCHED = {
     "fp32": synth.Workload("b_fp32", d=256, n_experts=8, top_k=2, d_ff=128, n_layers=3, wdtype="fp32",
-                           adtype="fp32", tokens=24, batch=4, rho=0.9, cap_slots=10),
+                           adtype="fp32", tokens=24, batch=4, rho=0.9, cap_slots=13),
     "fp32_ragged": synth.Workload("b_fp32_ragged", d=100, n_experts=5, top_k=2, d_ff=36, n_layers=2, wdtype="fp32",
                                   adtype="fp32", tokens=16, batch=3, rho=0.9, cap_slots=6),
     "bf16_ragged": synth.Workload("b_bf16_ragged", d=640, n_experts=24, top_k=5, d_ff=200, n_layers=3,
-                                  wdtype="bf16", adtype="bf16", tokens=10, batch=5, rho=0.8, cap_slots=30),
+                                  wdtype="bf16", adtype="bf16", tokens=10, batch=5, rho=0.8, cap_slots=40),
     "int4": synth.Workload("b_int4", d=384, n_experts=12, top_k=3, d_ff=256, n_layers=2, wdtype="int4",
                            adtype="bf16", tokens=10, batch=6, rho=0.8, cap_slots=14),
     "bf16_wide": synth.Workload("b_bf16_wide", d=4096, n_experts=64, top_k=16, d_ff=1536, n_layers=2,
