@@ -1,14 +1,16 @@
 #!/usr/bin/env python3
-"""Benchmark: batch-1 MoE decode under a 6 GB expert cap on one GB300 (tokens/s).
+"""Benchmark: MoE decode under a 6 GB expert cap on one GB300 (tokens/s).
 
 Workload (default ``stack48_bf16``): a 48-layer stack of Qwen3-30B-A3B-shaped MoE layers (d=2048,
 128 experts, top-8, SwiGLU I=768, bf16), 6144 experts (58 GB) in pinned host memory, a 6 GB
-device expert pool (635 slots) under global LRU, per-layer AR(1) hidden streams (rho=0.8).
-One step = one decode token through all 48 layers (router, residency, miss copies, expert
-FFN, combine), i.e. the whole hot path. Inputs are seeded synthetic data.
+device expert pool (635 slots) under global LRU, per-layer AR(1) hidden streams (rho=0.8),
+batch 1. One step = one decode token through all 48 layers (router, residency, miss copies,
+expert FFN, combine), i.e. the whole hot path. ``--workload stack48_batch64`` runs the batched
+configuration: 64 sequences per step (tokens/s counts all 64), same stack and cap.
+Inputs are seeded synthetic data.
 
 Prints one JSON line (rank 0). ``--impl reference`` times the fp64 CPU oracle on the same
-workload instead (the reference arm; one step = one layer of one token).
+workload instead (the reference arm; one step = one layer of one sequence's token).
 """
 from __future__ import annotations
 
@@ -128,10 +130,14 @@ def oracle_cpu_baseline(wl, hidden, budget_s: float = 15.0):
 
     The host tier of the oracle is the seeded generator; experts needed by the sampled tokens are
     generated before the clock starts, so only the oracle's own work (routing, residency, slot
-    copies, expert FFN, combine) is timed."""
+    copies, expert FFN, combine) is timed. A batch of several sequences is sampled per (layer,
+    sequence) instead (one decode step of the batch would take minutes)."""
     import oracle
     import synth
     from concurrent.futures import ThreadPoolExecutor
+
+    if wl.batch > 1:
+        return oracle_layer_sample(wl, hidden, budget_s)
 
     routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
     probe = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers)
@@ -155,6 +161,55 @@ def oracle_cpu_baseline(wl, hidden, budget_s: float = 15.0):
     return {"value": done / dt, "unit": "tok/s", "cores": os.cpu_count(), "kind": "oracle",
             "sample": f"{done} whole decode token(s) of {wl.name} ({wl.n_layers} layers, cap {wl.cap_slots}), "
                       f"cold pool, fp64, {dt:.1f} s"}
+
+
+def sample_units(wl, n_units):
+    """(token, layer, sequence) units in decode order: sequences fastest, then layers, then tokens."""
+    per_tok = wl.n_layers * wl.batch
+    return [(i // per_tok, (i % per_tok) // wl.batch, i % wl.batch) for i in range(n_units)]
+
+
+def layer_oracle(wl, hidden, units):
+    """An oracle whose host tier holds exactly the experts the given units route to (generated up
+    front, outside any timing), and a function that runs one unit's MoE layer."""
+    import oracle
+    import synth
+    from concurrent.futures import ThreadPoolExecutor
+
+    routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
+    need = set()
+    for t, l, b in units:
+        idx, _, _, _ = oracle.router(oracle.widen(wl.router_dtype, routers[l], wl.n_experts, wl.d),
+                                     synth.act_to_f64(hidden[t, l, b], wl.adtype), wl.top_k)
+        need.update((l, int(e)) for e in idx)
+    with ThreadPoolExecutor(max_workers=os.cpu_count()) as ex:
+        cache = dict(zip(sorted(need), ex.map(lambda le: synth.expert_weights(wl, *le), sorted(need))))
+    orc = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers, experts=lambda l, e: cache[(l, e)])
+
+    def run(u):
+        t, l, b = u
+        orc.moe_layer(l, hidden[t, l, b])
+
+    return run
+
+
+def oracle_layer_sample(wl, hidden, budget_s):
+    """The oracle's MoE layer for one sequence at a time (router, expert FFN, combine), in decode
+    order, until the time budget is spent; tokens/s = sequence-layers / n_layers / time."""
+    units = sample_units(wl, max(2, int(budget_s)))
+    run = layer_oracle(wl, hidden, units)
+    run(units[0])  # warm (first-touch of the widened weights' buffers)
+    t0 = time.perf_counter()
+    done = 0
+    for u in units[1:]:
+        run(u)
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": done / wl.n_layers / dt, "unit": "tok/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{done} (layer, sequence) units of {wl.name} (batch {wl.batch}, {wl.n_layers} layers): "
+                      f"router + top-k expert FFN + combine in fp64, {dt:.1f} s; tok/s = units / layers / s"}
 
 
 def kernel_source_digest() -> str:
@@ -201,14 +256,14 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
         m.preload()
         n_tok = hid_dev.shape[0]
         for i in range(3):
-            m.decode_step(hid_dev[i % n_tok], out_dev, stream=stream)
+            m.decode_step(hid_dev[i % n_tok], out_dev, batch=wl.batch, stream=stream)
         torch.cuda.synchronize()
         s0 = m.get_stats()
         m.profile_enable(True)
         m.profile_read()
         steps = max(8, min(args.steps, 100))
         for i in range(3, 3 + steps):
-            m.decode_step(hid_dev[i % n_tok], out_dev, stream=stream)
+            m.decode_step(hid_dev[i % n_tok], out_dev, batch=wl.batch, stream=stream)
         prof = m.profile_read()
         m.profile_enable(False)
         s1 = m.get_stats()
@@ -217,18 +272,24 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
     kern = {k: v for k, v in prof.items() if k in ("router", "gateup", "down_combine", "fused_step") and v["launches"]}
     dom = max(kern, key=lambda k: kern[k]["total_ms"])
     dk = kern[dom]
-    step_bytes = wl.n_layers * (wl.top_k * eb + wl.router_bytes())
+    # algorithmic bytes of one step: every distinct expert the step needs (one residency record
+    # each), read once, plus the routers
+    experts_per_step = ((s1["hits"] - s0["hits"]) + (s1["misses"] - s0["misses"])) / steps
+    step_bytes = experts_per_step * eb + wl.n_layers * wl.router_bytes()
     per_launch = step_bytes if dom == "fused_step" else dk["bytes"] / dk["launches"]
     avg_s = dk["total_ms"] * 1e-3 / dk["launches"]
     achieved = per_launch / avg_s / 1e9
     phases = {k[len("fused_phase_"):]: round(v["total_ms"] * 1e3 / v["launches"], 2)
               for k, v in prof.items() if k.startswith("fused_phase_") and v["launches"]}
-    return {"bound": "hbm", "kernel": "k_fused" if dom == "fused_step" else dom,
-            "workload": f"{wl.name} with all {wl.n_gid} experts resident (preloaded), batch 1",
+    kname = ("k_fused_batched" if wl.batch > 1 else "k_fused") if dom == "fused_step" else dom
+    traffic_file = f"{kname}_{wl.name}_resident.md".replace("k_fused_stack48_bf16", "k_fused_stack48")
+    return {"bound": "hbm", "kernel": kname,
+            "workload": f"{wl.name} with all {wl.n_gid} experts resident (preloaded), batch {wl.batch}",
             "achieved": achieved, "peak": peak_hbm, "unit": "GB/s", "frac": achieved / peak_hbm,
             "peak_source": f"{peak_src} hbm_gbs (copy; burst figure: kernel timed per launch)",
-            "traffic": stored_traffic("k_fused_stack48_resident.md") if dom == "fused_step" else None,
-            "bytes_per_launch": per_launch, "avg_launch_us": avg_s * 1e6, "launches": dk["launches"],
+            "traffic": stored_traffic(traffic_file) if dom == "fused_step" else None,
+            "bytes_per_launch": per_launch, "experts_per_step": experts_per_step,
+            "avg_launch_us": avg_s * 1e6, "launches": dk["launches"],
             "misses_in_window": s1["misses"] - s0["misses"], "phase_us_per_layer": phases}
 
 
@@ -243,39 +304,27 @@ def run_reference(args, wl):
         return 0
     L = wl.n_layers
     n_ls = args.warmup + args.steps
-    tokens = (n_ls + L - 1) // L
-    hidden = synth.hidden_all(wl, tokens)
-    routers = [synth.router_weights(wl, l) for l in range(L)]
-    probe = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers)
-    need = set()
-    for t in range(tokens):
-        r = probe.decode_step(hidden[t], compute_out=False)
-        for l in range(L):
-            need.update((l, int(e)) for e in r.idx[l, 0])
-    with ThreadPoolExecutor(max_workers=os.cpu_count()) as ex:
-        cache = dict(zip(sorted(need), ex.map(lambda le: synth.expert_weights(wl, *le), sorted(need))))
-    orc = oracle.Oracle.for_workload(wl, routers=routers, experts=lambda l, e: cache[(l, e)])
-    def layer_step(i):
-        t, l = divmod(i, L)
-        orc.moe_layer(l, hidden[t, l, 0])
-
-    for i in range(args.warmup):
-        layer_step(i)
+    units = sample_units(wl, n_ls)
+    hidden = synth.hidden_all(wl, units[-1][0] + 1)
+    run = layer_oracle(wl, hidden, units)
+    for u in units[:args.warmup]:
+        run(u)
     t0 = time.perf_counter()
-    for i in range(args.warmup, n_ls):
-        layer_step(i)
+    for u in units[args.warmup:]:
+        run(u)
     dt = time.perf_counter() - t0
     tok_s = args.steps / L / dt
-    line = {"metric": "MoE decode tok/s at batch 1 under 6 GB expert cap (fp64 CPU oracle)", "value": tok_s,
+    line = {"metric": "MoE decode tok/s at batch 1 under 6 GB expert cap; expert-path HBM GB/s vs peak", "value": tok_s,
             "unit": "tok/s", "impl": "reference", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f64", "data": "synthetic (seeded)",
             "config": {"workload": wl.name, "layers": L, "d": wl.d, "experts": wl.n_experts, "top_k": wl.top_k,
-                       "d_ff": wl.d_ff, "cap_slots": wl.cap_slots, "batch": 1, "step": "one layer of one token"},
+                       "d_ff": wl.d_ff, "cap_slots": wl.cap_slots, "batch": wl.batch,
+                       "step": "one layer of one sequence's token (router, top-k expert FFN, combine)"},
             "cpu_baseline": {"value": tok_s, "unit": "tok/s", "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": f"{args.steps} layer-steps (= {args.steps / L:.2f} tokens) of {wl.name}, "
-                                       "each layer's expert FFN read from the host tier (residency does not change "
-                                       "outputs)"},
+                             "sample": f"{args.steps} (layer, sequence) units (= {args.steps / L:.2f} tokens) of "
+                                       f"{wl.name} in decode order, each layer's expert FFN read from the host tier "
+                                       "(residency does not change outputs)"},
             "e2e": {"value": tok_s, "unit": "tok/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -295,6 +344,7 @@ def main():
     ap.add_argument("--no-resident", action="store_true", help="skip the all-resident roofline measurement")
     ap.add_argument("--layers", type=int, default=None, help="layer count override (small profiling cases)")
     ap.add_argument("--preload", action="store_true", help="fill the pool (moe_preload) before the warm-up")
+    ap.add_argument("--miss-ctas", type=int, default=0, help="CTAs streaming missed experts (0: library default)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -333,11 +383,13 @@ def main():
                                        f"{avail / 1e9:.0f} GB available"}), flush=True)
         return 1
 
-    n_tok = wl.tokens
-    hidden = synth.hidden_all(wl, n_tok)  # [T x L x 1 x d] bf16 bits / fp32
+    # distinct inputs: every step of a batch-1 run; for batches enough for the timed passes
+    # (later steps wrap around)
+    n_tok = wl.tokens if wl.batch == 1 else min(wl.tokens, args.warmup + 2 * args.steps + 64)
+    hidden = synth.hidden_all(wl, n_tok)  # [T x L x B x d] bf16 bits / fp32
     thp0 = anon_huge_kb()
     t_setup = time.perf_counter()
-    m = create_for_workload(wl, device=local, trace_capacity=0, schedule=args.schedule)
+    m = create_for_workload(wl, device=local, trace_capacity=0, schedule=args.schedule, miss_ctas=args.miss_ctas)
     t_setup = time.perf_counter() - t_setup
     thp_gb = (anon_huge_kb() - thp0) / 1e6
     eb = P.expert_bytes(m.cfg)
@@ -350,7 +402,7 @@ def main():
     stream = torch.cuda.current_stream()
 
     def step(i):
-        m.decode_step(hid_dev[i % n_tok], out_dev, stream=stream)
+        m.decode_step(hid_dev[i % n_tok], out_dev, batch=wl.batch, stream=stream)
 
     if args.preload:
         m.preload()
@@ -399,12 +451,12 @@ def main():
     hid_host = torch.from_numpy(hidden.view(np.float32) if wl.adtype == "fp32" else hidden.view(np.int16)).pin_memory()
     out_host = torch.empty_like(hid_host[0]).pin_memory()
     base = args.warmup + 2 * args.steps
-    m.decode_step_host(hid_host[base % n_tok], out_host)
+    m.decode_step_host(hid_host[base % n_tok], out_host, batch=wl.batch)
     if world > 1:
         torch.distributed.barrier()
     t0 = time.perf_counter()
     for i in range(base + 1, base + 1 + e2e_steps):
-        m.decode_step_host(hid_host[i % n_tok], out_host)
+        m.decode_step_host(hid_host[i % n_tok], out_host, batch=wl.batch)
     e2e_s = time.perf_counter() - t0
     if world > 1:
         t = torch.tensor([e2e_s], device="cuda")
@@ -417,8 +469,10 @@ def main():
     launch_classes = ("router", "gateup", "down_combine", "fused_step")
     launches = sum(v["launches"] for k, v in prof.items() if k in launch_classes)
     misses = s1["misses"] - s0["misses"]
+    hits = s1["hits"] - s0["hits"]
     miss_bytes_step = misses * eb / args.steps
-    hbm_bytes_step = wl.n_layers * (wl.top_k * eb + wl.router_bytes())
+    # every distinct expert a step needs is read once (one residency record each), plus the routers
+    hbm_bytes_step = (hits + misses) / args.steps * eb + wl.n_layers * wl.router_bytes()
     t_hbm = hbm_bytes_step / (peak_hbm * 1e9)
     t_h2d = miss_bytes_step / (h2d_gbs * 1e9)
     t_star = max(t_hbm, t_h2d)
@@ -433,14 +487,17 @@ def main():
                    "top_k": wl.top_k, "d_ff": wl.d_ff, "weights": wl.wdtype, "cap_slots": wl.cap_slots,
                    "cap_bytes": wl.cap_slots * eb, "host_tier_bytes": wl.n_gid * eb, "batch": wl.batch,
                    "parallelism": "replicas" if world > 1 else "single GPU", "schedule": args.schedule,
-                   "l2": "inputs larger than L2 (6 GB pool, 3.6 GB of expert weights read per step)"},
+                   "miss_ctas": args.miss_ctas or "default",
+                   "l2": f"inputs larger than L2 ({wl.cap_slots * eb / 1e9:.1f} GB pool, "
+                         f"{hbm_bytes_step / 1e9:.1f} GB of expert weights read per step)"},
         "step_roofline": {"bound": "h2d" if t_h2d >= t_hbm else "hbm", "t_star_ms": t_star * 1e3,
                           "frac": t_star * 1e3 / ms_step, "hbm_bytes_per_step": hbm_bytes_step,
                           "miss_bytes_per_step": miss_bytes_step, "h2d_peak_gbs": h2d_gbs,
                           "h2d_peak_source": "pinned copy-engine ceiling measured in this run (expert-sized chunks)",
                           "hbm_peak_gbs": peak_hbm,
                           "achieved_h2d_gbs": miss_bytes_step / (ms_step * 1e-3) / 1e9,
-                          "hit_rate": 1.0 - misses / max(1, (s1["hits"] - s0["hits"]) + misses)},
+                          "hit_rate": 1.0 - misses / max(1, hits + misses),
+                          "experts_per_step": (hits + misses) / args.steps},
         "profiled_pass_ms_per_step": ms_prof / args.steps,
         "roofline": None,
         "kernels": {k: {"launches": v["launches"], "total_ms": round(v["total_ms"], 3),

@@ -97,8 +97,9 @@ typedef struct {
   int64_t trace_capacity; /* residency records kept (device buffer for MOE_SCHEDULE_DEVICE, host otherwise);
                              0 disables the trace */
   int32_t schedule;       /* MOE_SCHEDULE_DEVICE (default) or MOE_SCHEDULE_HOST_COPY_ENGINE */
-  int32_t miss_ctas;      /* MOE_SCHEDULE_DEVICE: CTAs that stream missed experts over the host link
-                             while the others compute the hits (0: library default) */
+  int32_t miss_ctas;      /* MOE_SCHEDULE_DEVICE, max_batch 1: CTAs that stream missed experts over the
+                             host link while the others compute the hits (0: library default). Batched
+                             steps hand work items to all CTAs, missed experts first, and ignore it */
 } moe_config;
 
 /* One residency record: a requested expert's outcome in one layer-step. */

@@ -107,7 +107,7 @@ struct BatchArgs {
   int* err;
   unsigned long long barrier_timeout_ns;
   unsigned long long* phase_ts; // optional [L][kBatchedPhases] + 1
-  int miss_ctas;
+  unsigned* work;              // [2] work-item counters of phases C and D (reset in phase S)
   int touch_shift;
   int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
 };

@@ -14,12 +14,16 @@
 //      the ascending list of pairs routed to it;
 //   C  grouped gate-up: a work item is (needed expert, block of rows). The CTA stages the
 //      activations of the expert's pairs in shared memory, and each warp reads a row pair once
-//      and applies it to every staged pair: u_p[i] = silu(W_g[i] . h_b) * (W_u[i] . h_b). Missed
-//      experts are worked by the last "miss CTAs": they read the rows from the page-locked host
-//      tier over NVLink-C2C, store them into the expert's slot and use them from registers, and
-//      copy the expert's W_d region into the slot; the other CTAs work the hits from HBM;
+//      and applies it to every staged pair: u_p[i] = silu(W_g[i] . h_b) * (W_u[i] . h_b). A
+//      missed expert's item reads its rows from the page-locked host tier over NVLink-C2C,
+//      stores them into the expert's slot and uses them from registers, and copies its share of
+//      the expert's W_d region into the slot. CTAs take items from a global counter, the missed
+//      experts' items first: while misses remain every CTA streams the host tier (many misses per
+//      layer-step need all the requests in flight the grid can issue), and the hit items fill in
+//      behind them;
 //   D  grouped down projection: a work item is (needed expert, block of W_d rows); the CTA stages
-//      u of the expert's pairs and each warp applies its rows to all of them, y_p = W_d u_p;
+//      u of the expert's pairs and each warp applies its rows to all of them, y_p = W_d u_p.
+//      Items again come from a global counter (experts with many pairs take longer);
 //   E  combine per sequence in rank order: out[b] = sum_r g_{b,r} y_{b*k+r}.
 //
 // Each expert is read from memory once per layer-step however many pairs it serves. All CTAs are
@@ -295,6 +299,8 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   if (tid == 0) {
     a.plan_n[0] = n;
     a.plan_n[1] = nm;
+    a.work[0] = 0u;  // the previous layer's phases C and D are complete (grid barriers since)
+    a.work[1] = 0u;
     a.stats[STAT_HITS] += (unsigned long long)(n - nm);
     a.stats[STAT_MISSES] += (unsigned long long)nm;
     a.stats[STAT_LAYER_STEPS] += 1;
@@ -526,10 +532,19 @@ __device__ void down_item(const BatchArgs& a, int pos, int oblk, float* us, int*
   }
 }
 
+// Next work item of a phase for the whole CTA (thread 0 draws it from the phase's counter).
+__device__ __forceinline__ int next_item(unsigned* ctr, int* s_item) {
+  __syncthreads();  // every thread has read the previous item
+  if (threadIdx.x == 0) *s_item = (int)atomicAdd(ctr, 1u);
+  __syncthreads();
+  return *s_item;
+}
+
 template <int WD, int CH>
 __global__ void __launch_bounds__(kBThreads, 2) k_fused_batched(const __grid_constant__ BatchArgs a) {
   extern __shared__ uint4 smem4[];
   __shared__ int pidx[kTGMax];
+  __shared__ int s_item;
   uint8_t* smem = reinterpret_cast<uint8_t*>(smem4);
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -600,14 +615,10 @@ __global__ void __launch_bounds__(kBThreads, 2) k_fused_batched(const __grid_con
           asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
         }
       }
-      const int mctas = nm > 0 ? (a.miss_ctas < (int)gridDim.x - 1 ? a.miss_ctas : (int)gridDim.x - 1) : 0;
-      const int hctas = (int)gridDim.x - mctas;
-      if ((int)blockIdx.x >= hctas) {
-        for (int it = (int)blockIdx.x - hctas; it < nm * nrb; it += mctas)
-          gateup_item<WD, CH>(a, l, it / nrb, it % nrb, true, smem, pidx, tgmax);
-      } else {
-        for (int it = blockIdx.x; it < (n - nm) * nrb; it += hctas)
-          gateup_item<WD, CH>(a, l, nm + it / nrb, it % nrb, false, smem, pidx, tgmax);
+      // items: plan position (misses first) x row block
+      for (int it = next_item(a.work, &s_item); it < n * nrb; it = next_item(a.work, &s_item)) {
+        const int pos = it / nrb;
+        gateup_item<WD, CH>(a, l, pos, it - pos * nrb, pos < nm, smem, pidx, tgmax);
       }
     }
     if (!grid_sync(a, nbar)) return;
@@ -616,7 +627,7 @@ __global__ void __launch_bounds__(kBThreads, 2) k_fused_batched(const __grid_con
     {
       const int n = __ldcg(a.plan_n);
       float* us = reinterpret_cast<float*>(smem);
-      for (int it = blockIdx.x; it < n * nob; it += gridDim.x) {
+      for (int it = next_item(a.work + 1, &s_item); it < n * nob; it = next_item(a.work + 1, &s_item)) {
         const int pos = it / nob, ob = it % nob;
         switch (chd_need) {
           case 1: down_item<WD, 1>(a, pos, ob, us, pidx, tgmax); break;

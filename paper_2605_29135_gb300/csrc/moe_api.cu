@@ -119,7 +119,7 @@ struct moe_handle {
   int32_t* d_route_idx = nullptr;
   float* d_route_gate = nullptr;
   unsigned long long* d_stats = nullptr;
-  unsigned* d_bar = nullptr;  // count, generation
+  unsigned* d_bar = nullptr;  // barrier count, (unused), batched work-item counters [2]
   int* d_err = nullptr;
   int* h_err = nullptr;       // pinned copy of d_err after each step
   cudaEvent_t err_ev = nullptr;
@@ -202,7 +202,7 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_step, 0, sizeof(int64_t));
   cudaMemset(h->d_trace_n, 0, sizeof(unsigned long long));
   cudaMemset(h->d_stats, 0, sizeof(unsigned long long) * moe::STAT_N);
-  cudaMemset(h->d_bar, 0, sizeof(unsigned) * 2);
+  cudaMemset(h->d_bar, 0, sizeof(unsigned) * 4);
   h->bar_epoch = 0;
   cudaMemset(h->d_err, 0, sizeof(int));
   cudaDeviceSynchronize();
@@ -635,7 +635,7 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.err = h->d_err;
   a.barrier_timeout_ns = 2000000000ull;
   a.phase_ts = phase_buffer(h);
-  a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
+  a.work = h->d_bar + 2;
   a.touch_shift = h->touch_shift;
   a.tg_max = h->tg_max;
   {
@@ -862,7 +862,7 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
               cudaMalloc(&h->d_route_idx, sizeof(int32_t) * cfg->n_layers * pairs) == cudaSuccess &&
               cudaMalloc(&h->d_route_gate, sizeof(float) * cfg->n_layers * pairs) == cudaSuccess &&
               cudaMalloc(&h->d_stats, sizeof(unsigned long long) * moe::STAT_N) == cudaSuccess &&
-              cudaMalloc(&h->d_bar, sizeof(unsigned) * 2) == cudaSuccess &&
+              cudaMalloc(&h->d_bar, sizeof(unsigned) * 4) == cudaSuccess &&
               cudaMalloc(&h->d_err, sizeof(int)) == cudaSuccess &&
               cudaHostAlloc(&h->h_err, sizeof(int), cudaHostAllocDefault) == cudaSuccess &&
               cudaEventCreateWithFlags(&h->err_ev, cudaEventDisableTiming) == cudaSuccess;
