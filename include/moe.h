@@ -78,6 +78,17 @@ enum {
  * each needed expert is read once and applied to every sequence routed to it. */
 enum { MOE_SCHEDULE_DEVICE = 0, MOE_SCHEDULE_HOST_COPY_ENGINE = 1 };
 
+/* Expert FFN of batched steps (max_batch > 1).
+ *   MOE_BATCHED_AUTO: tensor cores when the shape allows (bf16 weights, d a multiple of 128,
+ *     d_ff of 64): per layer-step each needed expert's gate/up and down matrices are multiplied
+ *     with the stacked activations of the pairs routed to it (tcgen05 MMA, operands streamed by
+ *     TMA, fp32 accumulation; u is rounded to bf16 between the two projections). Missed experts
+ *     are first copied into their slots, so hits and misses share the arithmetic. Other shapes:
+ *     CUDA cores, as MOE_BATCHED_CUDA_CORES.
+ *   MOE_BATCHED_CUDA_CORES: grouped GEMV on CUDA cores (fp32 accumulation, fp32 u); missed
+ *     experts stream from the host tier straight into their slot and the compute. */
+enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
+
 typedef struct {
   int32_t d;          /* hidden size */
   int32_t n_experts;  /* experts per layer, E (<= 256) */
@@ -100,6 +111,7 @@ typedef struct {
   int32_t miss_ctas;      /* MOE_SCHEDULE_DEVICE, max_batch 1: CTAs that stream missed experts over the
                              host link while the others compute the hits (0: library default). Batched
                              steps hand work items to all CTAs, missed experts first, and ignore it */
+  int32_t batched_path;   /* MOE_BATCHED_AUTO (default) or MOE_BATCHED_CUDA_CORES */
 } moe_config;
 
 /* One residency record: a requested expert's outcome in one layer-step. */

@@ -1,6 +1,8 @@
 // Device-driven decode step: one cooperative persistent kernel runs every layer of a decode
 // step (router, slot lookup + LRU, miss transfer, expert FFN, combine) with no host round trip.
 #pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -14,7 +16,9 @@ struct TraceRec {
 };
 
 enum { STAT_HITS = 0, STAT_MISSES = 1, STAT_EVICTIONS = 2, STAT_LAYER_STEPS = 3, STAT_N = 4 };
-enum { FERR_BARRIER_TIMEOUT = 1, FERR_BAD_ROUTE = 2, FERR_NO_VICTIM = 4 };
+enum { FERR_BARRIER_TIMEOUT = 1, FERR_BAD_ROUTE = 2, FERR_NO_VICTIM = 4, FERR_PIPE_TIMEOUT = 8 };
+// Flags after which every CTA leaves the kernel at its next grid barrier.
+constexpr int FERR_FATAL = FERR_BARRIER_TIMEOUT | FERR_PIPE_TIMEOUT;
 
 struct FusedArgs {
   int L, E, k, d, I, renorm, wdtype;
@@ -67,6 +71,15 @@ constexpr int kBatchedEvictCap = 4096;  // slot counts this large or smaller can
 constexpr int kBatchedPhases = 6;       // router, top-k, select, gate-up, down, combine
 
 struct BatchArgs {
+  // Tensor-core variant (bf16 weights): TMA maps over the slot pool and over the pairs'
+  // activations and u vectors in plan order (pairs grouped by expert, so an expert's pairs are
+  // consecutive rows).
+  CUtensorMap map_gu;          // pool gate/up rows: dims {d, 2I, cap}, box {64, 128, 1}, 128-B swizzle
+  CUtensorMap map_d;           // pool W_d rows: dims {I, d, cap}, box {64, 128, 1}
+  CUtensorMap map_x;           // xg: dims {d, Bmax*k}, box {64, 16}
+  CUtensorMap map_u;           // ug: dims {I, Bmax*k}, box {64, 16}
+  __nv_bfloat16* xg;           // [Bmax*k][d] activation of each pair, plan order
+  __nv_bfloat16* ug;           // [Bmax*k][I] u of each pair, plan order
   int L, E, k, d, I, renorm, wdtype;
   int B;                       // sequences this step (<= Bmax)
   int Bmax;                    // row stride of the routing log
@@ -116,5 +129,12 @@ struct BatchArgs {
 int batched_tg(int wdtype, int d, int I);
 int fused_batched_grid(int wdtype, int d, int I, int64_t cap, int64_t n_gid);
 cudaError_t launch_fused_batched(const BatchArgs& a, int grid, cudaStream_t s);
+
+// Tensor-core variant: bf16 weights, d a multiple of 128 and I of 64. Seven phases per layer
+// (router, top-k, select, gather, gate-up, down, combine).
+constexpr int kBatchedTcPhases = 7;
+bool batched_tc_supported(int wdtype, int d, int I);
+int fused_batched_tc_grid(int d, int I, int64_t cap, int64_t n_gid);
+cudaError_t launch_fused_batched_tc(const BatchArgs& a, int grid, cudaStream_t s);
 
 }  // namespace moe

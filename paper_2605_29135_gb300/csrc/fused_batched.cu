@@ -36,6 +36,7 @@
 #include "dev.cuh"
 #include "fused.cuh"
 #include "grid.cuh"
+#include "tc.cuh"
 #include "topk.cuh"
 
 namespace moe {
@@ -122,7 +123,7 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   __shared__ int s_off[256];
   __shared__ int s_n, s_nm, s_nused0, s_nfree, s_nev, s_nevicted;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int E = a.E, k = a.k, P = a.B * a.k;
+  const int E = a.E, P = a.B * a.k;
 
   for (int p = tid; p < P; p += blockDim.x) s_sel[p] = __ldcg(a.sel_e + p);
   for (int e = tid; e < 256; e += blockDim.x) s_flag[e] = 0;
@@ -532,6 +533,57 @@ __device__ void down_item(const BatchArgs& a, int pos, int oblk, float* us, int*
   }
 }
 
+// ---- phase R for all CTAs: one warp per (router row, block of 8 sequences)
+__device__ __forceinline__ void phase_router(const BatchArgs& a, int l, int gw, int W, int lane) {
+  const int nb8 = (a.B + 7) / 8;
+  for (int it = gw; it < a.E * nb8; it += W) {
+    const int e = it / nb8;
+    const int b0 = (it - e * nb8) * 8;
+    if (a.wdtype == WD_FP32)
+      router_item<WD_FP32>(a, l, e, b0, lane);
+    else
+      router_item<WD_BF16>(a, l, e, b0, lane);
+  }
+}
+
+// ---- phase T: one warp per sequence
+__device__ __forceinline__ void phase_topk(const BatchArgs& a, int l, int gw, int W, int lane) {
+  for (int b = gw; b < a.B; b += W) {
+    int my_i;
+    float my_g;
+    warp_topk(a.z + (int64_t)b * a.E, a.E, a.k, a.renorm, lane, my_i, my_g);
+    if (lane < a.k) {
+      if (my_i < 0 || my_i >= a.E) {
+        atomicOr(a.err, FERR_BAD_ROUTE);
+        my_i = lane;  // keep the step well-defined; the host reports the error
+      }
+      a.sel_e[b * a.k + lane] = my_i;
+      a.sel_g[b * a.k + lane] = my_g;
+      a.route_idx[((int64_t)l * a.Bmax + b) * a.k + lane] = my_i;
+      a.route_gate[((int64_t)l * a.Bmax + b) * a.k + lane] = my_g;
+    }
+  }
+}
+
+// ---- phase E: out[b][o] = sum_r g_{b,r} y_{b*k+r}[o], ranks in order
+__device__ __forceinline__ void phase_combine(const BatchArgs& a, int l) {
+  const int64_t nout = (int64_t)a.B * a.d;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nout; q += (int64_t)gridDim.x * blockDim.x) {
+    const int b = (int)(q / a.d);
+    const int o = (int)(q - (int64_t)b * a.d);
+    float acc = 0.f;
+    for (int r = 0; r < a.k; r++) {
+      const int p = b * a.k + r;
+      acc = fmaf(__ldcg(a.sel_g + p), __ldcg(a.y + (int64_t)p * a.d + o), acc);
+    }
+    const int64_t oi = ((int64_t)l * a.B + b) * a.d + o;
+    if (a.wdtype == WD_FP32)
+      reinterpret_cast<float*>(a.out)[oi] = acc;
+    else
+      reinterpret_cast<__nv_bfloat16*>(a.out)[oi] = __float2bfloat16_rn(acc);
+  }
+}
+
 // Next work item of a phase for the whole CTA (thread 0 draws it from the phase's counter).
 __device__ __forceinline__ int next_item(unsigned* ctr, int* s_item) {
   __syncthreads();  // every thread has read the previous item
@@ -563,36 +615,10 @@ __global__ void __launch_bounds__(kBThreads, 2) k_fused_batched(const __grid_con
 
   for (int l = 0; l < a.L; l++) {
     const int clock = (int)(step * a.L + l + 1);  // 0 is older than every step (preloaded experts)
-    // ---- R
-    {
-      const int nb8 = (a.B + 7) / 8;
-      for (int it = gw; it < a.E * nb8; it += W) {
-        const int e = it / nb8;
-        const int b0 = (it - e * nb8) * 8;
-        if (WD == WD_FP32)
-          router_item<WD_FP32>(a, l, e, b0, lane);
-        else
-          router_item<WD_BF16>(a, l, e, b0, lane);
-      }
-    }
+    phase_router(a, l, gw, W, lane);
     if (!grid_sync(a, nbar)) return;
     mark(l, 0);
-    // ---- T
-    for (int b = gw; b < a.B; b += W) {
-      int my_i;
-      float my_g;
-      warp_topk(a.z + (int64_t)b * a.E, a.E, a.k, a.renorm, lane, my_i, my_g);
-      if (lane < a.k) {
-        if (my_i < 0 || my_i >= a.E) {
-          atomicOr(a.err, FERR_BAD_ROUTE);
-          my_i = lane;  // keep the step well-defined; the host reports the error
-        }
-        a.sel_e[b * a.k + lane] = my_i;
-        a.sel_g[b * a.k + lane] = my_g;
-        a.route_idx[((int64_t)l * a.Bmax + b) * a.k + lane] = my_i;
-        a.route_gate[((int64_t)l * a.Bmax + b) * a.k + lane] = my_g;
-      }
-    }
+    phase_topk(a, l, gw, W, lane);
     if (!grid_sync(a, nbar)) return;
     mark(l, 1);
     // ---- S
@@ -642,28 +668,302 @@ __global__ void __launch_bounds__(kBThreads, 2) k_fused_batched(const __grid_con
     }
     if (!grid_sync(a, nbar)) return;
     mark(l, 4);
-    // ---- E: out[b][o] = sum_r g_{b,r} y_{b*k+r}[o], ranks in order
-    {
-      const int64_t nout = (int64_t)a.B * a.d;
-      for (int64_t q = (int64_t)blockIdx.x * kBThreads + threadIdx.x; q < nout; q += (int64_t)gridDim.x * kBThreads) {
-        const int b = (int)(q / a.d);
-        const int o = (int)(q - (int64_t)b * a.d);
-        float acc = 0.f;
-        for (int r = 0; r < a.k; r++) {
-          const int p = b * a.k + r;
-          acc = fmaf(__ldcg(a.sel_g + p), __ldcg(a.y + (int64_t)p * a.d + o), acc);
-        }
-        const int64_t oi = ((int64_t)l * a.B + b) * a.d + o;
-        if (WD == WD_FP32)
-          reinterpret_cast<float*>(a.out)[oi] = acc;
-        else
-          reinterpret_cast<__nv_bfloat16*>(a.out)[oi] = __float2bfloat16_rn(acc);
-      }
-    }
+    phase_combine(a, l);
     if (!grid_sync(a, nbar)) return;
     mark(l, 5);
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
+}
+
+// =============================================================================================
+// Tensor-core variant (bf16 weights). Phases C and D become grouped GEMMs on tcgen05: a work item
+// is (needed expert, 128-row tile of its weight matrix); the A operand (weights, 128 rows x 64 K
+// per stage) and the B operand (the expert's pairs, N = pair count rounded up to 16 rows x 64 K)
+// stream from global memory into a ring of shared-memory stages by TMA; one thread issues the
+// MMAs (M = 128, N, K = 16) into a TMEM accumulator; four epilogue warps read the accumulator
+// back (TMEM lane = weight row, column = pair). Per CTA: warp 0 lane 0 produces, warp 1 lane 0
+// issues MMAs, warps 4-7 run the epilogue, two accumulators alternate so the epilogue of one
+// item overlaps the MMAs of the next. Missed experts are copied host -> slot in the phase before
+// (G), so every expert's arithmetic is the same whether it hit or missed.
+
+constexpr int kTcStages = 6;
+constexpr int kTcABytes = 128 * 64 * 2;             // one A stage: 128 rows x 64 bf16
+constexpr int kTcStageBytes = kTcABytes + 64 * 128; // + up to 64 B-operand rows of 128 B
+constexpr int kTcAccCols = 64;                      // fp32 columns per accumulator (N <= 64)
+constexpr int kTcTmemCols = 2 * kTcAccCols;
+constexpr int kTcCopyChunk = 256 * 1024;            // bytes per miss-copy work item
+constexpr unsigned long long kPipeTimeoutNs = 2000000000ull;
+
+struct TcShared {
+  uint64_t full[kTcStages];   // stage loaded (TMA transaction bytes)
+  uint64_t empty[kTcStages];  // stage consumed (tcgen05.commit)
+  uint64_t accfull[2];        // accumulator complete (tcgen05.commit)
+  uint64_t accempty[2];       // accumulator read back (4 epilogue warps)
+  uint32_t tmem;
+};
+
+// Position in the stage ring and the accumulator pair; the producer, the MMA thread and the
+// epilogue threads each keep a copy and advance it over the same item sequence.
+struct TcRing {
+  uint32_t stage = 0, sphase = 0, acc = 0, aphase = 0;
+  __device__ void next_stage() {
+    if (++stage == kTcStages) {
+      stage = 0;
+      sphase ^= 1u;
+    }
+  }
+  __device__ void next_acc() {
+    if (++acc == 2) {
+      acc = 0;
+      aphase ^= 1u;
+    }
+  }
+};
+
+struct TcGemm {
+  const CUtensorMap* map_a;  // weights in the slot pool (3D: K, row, slot)
+  const CUtensorMap* map_b;  // pairs in plan order (2D: K, row)
+  int mtiles;                // 128-row tiles per expert
+  int nkb;                   // 64-wide K blocks
+};
+
+__device__ __forceinline__ bool tc_wait(const BatchArgs& a, uint64_t* bar, uint32_t parity) {
+  if (tc::mbar_wait(bar, parity, kPipeTimeoutNs, a.err, FERR_FATAL)) return true;
+  atomicOr(a.err, FERR_PIPE_TIMEOUT);
+  return false;
+}
+
+__device__ void tc_produce(const BatchArgs& a, TcShared& st, const TcGemm& g, int nitems, uint8_t* stages,
+                           TcRing& r) {
+  tc::fence_proxy_async_global();  // the B rows (and missed experts) were written by ordinary stores
+  for (int it = blockIdx.x; it < nitems; it += gridDim.x) {
+    const int pos = it / g.mtiles, mt = it - pos * g.mtiles;
+    const int slot = __ldcg(a.plan_slot + pos), off = __ldcg(a.plan_off + pos), cnt = __ldcg(a.plan_cnt + pos);
+    const int nb16 = (cnt + 15) >> 4;
+    for (int kb = 0; kb < g.nkb; kb++) {
+      if (!tc_wait(a, &st.empty[r.stage], r.sphase ^ 1u)) return;
+      uint8_t* sa = stages + r.stage * kTcStageBytes;
+      tc::mbar_expect_tx(&st.full[r.stage], (uint32_t)(kTcABytes + nb16 * 2048));
+      tc::tma_load_3d(sa, g.map_a, &st.full[r.stage], kb * 64, mt * 128, slot);
+      for (int j = 0; j < nb16; j++)
+        tc::tma_load_2d(sa + kTcABytes + j * 2048, g.map_b, &st.full[r.stage], kb * 64, off + 16 * j);
+      r.next_stage();
+    }
+  }
+}
+
+__device__ void tc_mma(const BatchArgs& a, TcShared& st, const TcGemm& g, int nitems, uint8_t* stages, TcRing& r) {
+  for (int it = blockIdx.x; it < nitems; it += gridDim.x) {
+    const int pos = it / g.mtiles;
+    const int cnt = __ldcg(a.plan_cnt + pos);
+    const uint32_t idesc = tc::idesc_bf16(128, ((cnt + 15) >> 4) * 16);
+    if (!tc_wait(a, &st.accempty[r.acc], r.aphase ^ 1u)) return;
+    tc::fence_after_sync();
+    const uint32_t d = st.tmem + r.acc * kTcAccCols;
+    for (int kb = 0; kb < g.nkb; kb++) {
+      if (!tc_wait(a, &st.full[r.stage], r.sphase)) return;
+      tc::fence_after_sync();
+      const uint32_t sa = tc::smem_u32(stages + r.stage * kTcStageBytes);
+      const uint64_t da = tc::desc_sw128(sa), db = tc::desc_sw128(sa + kTcABytes);
+#pragma unroll
+      for (int j = 0; j < 4; j++)  // K = 16 per MMA: the next 32 B of every 128-B row
+        tc::mma_bf16(d, da + (uint64_t)(2 * j), db + (uint64_t)(2 * j), idesc, (kb | j) != 0);
+      tc::mma_commit(&st.empty[r.stage]);
+      r.next_stage();
+    }
+    tc::mma_commit(&st.accfull[r.acc]);
+    r.next_acc();
+  }
+}
+
+// Epilogue warps 4-7: warp q = warp % 4 reads TMEM lanes [32q, 32q + 32), i.e. weight rows
+// mt * 128 + 32q + lane, 16 pair columns at a time; f consumes them.
+template <typename F>
+__device__ void tc_epilogue(const BatchArgs& a, TcShared& st, const TcGemm& g, int nitems, TcRing& r, F&& f) {
+  const int q = (threadIdx.x >> 5) & 3, lane = threadIdx.x & 31;
+  for (int it = blockIdx.x; it < nitems; it += gridDim.x) {
+    const int pos = it / g.mtiles, mt = it - pos * g.mtiles;
+    const int off = __ldcg(a.plan_off + pos), cnt = __ldcg(a.plan_cnt + pos);
+    if (!tc_wait(a, &st.accfull[r.acc], r.aphase)) return;
+    tc::fence_after_sync();
+    const uint32_t t0 = st.tmem + r.acc * kTcAccCols + ((uint32_t)(q * 32) << 16);
+    const int row = mt * 128 + q * 32 + lane;
+    for (int c0 = 0; c0 < cnt; c0 += 16) {
+      float v[16];
+      tc::tmem_ld16(t0 + (uint32_t)c0, v);
+      f(off, cnt, row, c0, v, lane);
+    }
+    tc::fence_before_sync();
+    __syncwarp();
+    if (lane == 0) tc::mbar_arrive(&st.accempty[r.acc]);
+    r.next_acc();
+  }
+}
+
+// ---- phase G: the pairs' activations into plan order (xg), and every missed expert's image
+// host -> slot (chunks handed out dynamically, after a translation warm-up as in phase C of the
+// CUDA-core variant).
+__device__ void tc_gather_copy(const BatchArgs& a, int l, int gw, int W, int lane, int* s_item) {
+  const int nm = __ldcg(a.plan_n + 1);
+  const int P = a.B * a.k;
+  if (nm > 0) {
+    const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
+    const int64_t gt0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t GT = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t q = gt0; q < (int64_t)nm * pages; q += GT) {
+      const int m = (int)(q / pages);
+      const uint8_t* pa =
+          a.arena + (int64_t)__ldcg(a.plan_gid + m) * a.slot_stride + ((q - (int64_t)m * pages) << a.touch_shift);
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+    }
+  }
+  const int nq = a.d * 2 / 16;
+  for (int j = gw; j < P; j += W) {
+    const int b = __ldcg(a.plan_tok + j) / a.k;
+    const uint4* src = reinterpret_cast<const uint4*>((const uint8_t*)a.hidden + ((int64_t)l * a.B + b) * a.d * 2);
+    uint8_t* dst = reinterpret_cast<uint8_t*>(a.xg) + (int64_t)j * a.d * 2;
+    for (int c = lane; c < nq; c += 32) st_v4(dst + c * 16, __ldg(src + c));
+  }
+  const int cpe = (int)((a.lay.total + kTcCopyChunk - 1) / kTcCopyChunk);
+  for (int it = next_item(a.work, s_item); it < nm * cpe; it = next_item(a.work, s_item)) {
+    const int m = it / cpe, c = it - m * cpe;
+    const int64_t b0 = (int64_t)c * kTcCopyChunk;
+    const int64_t b1 = b0 + kTcCopyChunk < a.lay.total ? b0 + kTcCopyChunk : a.lay.total;
+    const uint8_t* src = a.arena + (int64_t)__ldcg(a.plan_gid + m) * a.slot_stride;
+    uint8_t* dst = a.pool + (int64_t)__ldcg(a.plan_slot + m) * a.slot_stride;
+    const int T = blockDim.x;
+    int64_t q = b0 / 16 + threadIdx.x;
+    const int64_t q1 = b1 / 16;
+    for (; q + 3 * (int64_t)T < q1; q += 4 * (int64_t)T) {
+      const uint4 v0 = ld_stream(src + q * 16);
+      const uint4 v1 = ld_stream(src + (q + T) * 16);
+      const uint4 v2 = ld_stream(src + (q + 2 * (int64_t)T) * 16);
+      const uint4 v3 = ld_stream(src + (q + 3 * (int64_t)T) * 16);
+      st_v4(dst + q * 16, v0);
+      st_v4(dst + (q + T) * 16, v1);
+      st_v4(dst + (q + 2 * (int64_t)T) * 16, v2);
+      st_v4(dst + (q + 3 * (int64_t)T) * 16, v3);
+    }
+    for (; q < q1; q += T) st_v4(dst + q * 16, ld_stream(src + q * 16));
+  }
+}
+
+__global__ void __launch_bounds__(kBThreads, 1) k_fused_batched_tc(const __grid_constant__ BatchArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  __shared__ TcShared st;
+  __shared__ int s_item;
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kBWarps + warp;
+  const int W = gridDim.x * kBWarps;
+  const int64_t step = *(volatile int64_t*)a.step;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kTcStages; i++) {
+      tc::mbar_init(&st.full[i], 1);
+      tc::mbar_init(&st.empty[i], 1);
+    }
+    for (int i = 0; i < 2; i++) {
+      tc::mbar_init(&st.accfull[i], 1);
+      tc::mbar_init(&st.accempty[i], 4);
+    }
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&a.map_gu);
+    tc::prefetch_tmap(&a.map_d);
+    tc::prefetch_tmap(&a.map_x);
+    tc::prefetch_tmap(&a.map_u);
+  }
+  if (warp == 2) {
+    tc::tmem_alloc(&st.tmem, kTcTmemCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[a.L * kBatchedTcPhases] = gtimer();
+  auto mark = [&](int l, int ph) {
+    if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * kBatchedTcPhases + ph] = gtimer();
+  };
+  const TcGemm gu{&a.map_gu, &a.map_x, 2 * a.I / 128, a.d / 64};
+  const TcGemm dn{&a.map_d, &a.map_u, a.d / 128, a.I / 64};
+  TcRing ring;
+  unsigned nbar = 0;
+
+  auto layers = [&]() -> bool {
+    for (int l = 0; l < a.L; l++) {
+      const int clock = (int)(step * a.L + l + 1);
+      phase_router(a, l, gw, W, lane);
+      if (!grid_sync(a, nbar)) return false;
+      mark(l, 0);
+      phase_topk(a, l, gw, W, lane);
+      if (!grid_sync(a, nbar)) return false;
+      mark(l, 1);
+      if (blockIdx.x == 0) batched_select(a, l, clock, step, reinterpret_cast<unsigned long long*>(smem));
+      if (!grid_sync(a, nbar)) return false;
+      mark(l, 2);
+      tc_gather_copy(a, l, gw, W, lane, &s_item);
+      tc::fence_proxy_async_global();
+      if (!grid_sync(a, nbar)) return false;
+      mark(l, 3);
+      // ---- C: [gate; up] rows x pairs -> u = silu(gate) * up, bf16, plan order
+      {
+        const int items = __ldcg(a.plan_n) * gu.mtiles;
+        if (warp == 0) {
+          if (lane == 0) tc_produce(a, st, gu, items, smem, ring);
+        } else if (warp == 1) {
+          if (lane == 0) tc_mma(a, st, gu, items, smem, ring);
+        } else if (warp >= 4) {
+          tc_epilogue(a, st, gu, items, ring, [&](int off, int cnt, int row, int c0, float(&v)[16], int ln) {
+            // rows alternate gate, up of one intermediate index: lanes 2j and 2j + 1 hold a pair
+            const int i = row >> 1;
+#pragma unroll
+            for (int t = 0; t < 16; t++) {
+              const float other = __shfl_xor_sync(kFull, v[t], 1);
+              if (!(ln & 1) && c0 + t < cnt) {
+                const float g = v[t];
+                a.ug[(int64_t)(off + c0 + t) * a.I + i] = __float2bfloat16_rn(g / (1.0f + expf(-g)) * other);
+              }
+            }
+          });
+        }
+      }
+      tc::fence_proxy_async_global();
+      if (!grid_sync(a, nbar)) return false;
+      mark(l, 4);
+      // ---- D: W_d rows x pairs -> y[pair][row]
+      {
+        const int items = __ldcg(a.plan_n) * dn.mtiles;
+        if (warp == 0) {
+          if (lane == 0) tc_produce(a, st, dn, items, smem, ring);
+        } else if (warp == 1) {
+          if (lane == 0) tc_mma(a, st, dn, items, smem, ring);
+        } else if (warp >= 4) {
+          tc_epilogue(a, st, dn, items, ring, [&](int off, int cnt, int row, int c0, float(&v)[16], int) {
+#pragma unroll
+            for (int t = 0; t < 16; t++)
+              if (c0 + t < cnt) a.y[(int64_t)__ldcg(a.plan_tok + off + c0 + t) * a.d + row] = v[t];
+          });
+        }
+      }
+      if (!grid_sync(a, nbar)) return false;
+      mark(l, 5);
+      phase_combine(a, l);
+      if (!grid_sync(a, nbar)) return false;
+      mark(l, 6);
+    }
+    return true;
+  };
+  const bool ok = layers();
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (warp == 2) tc::tmem_dealloc(st.tmem, kTcTmemCols);
+  if (ok && blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
+}
+
+size_t batched_tc_smem(int64_t cap, int64_t n_gid) {
+  return std::max((size_t)kTcStages * kTcStageBytes, (size_t)sort_n_of(cap, n_gid) * sizeof(unsigned long long)) +
+         1024;
 }
 
 int pick_ch_b(int64_t rb) {
@@ -752,6 +1052,35 @@ cudaError_t launch_fused_batched(const BatchArgs& a, int grid, cudaStream_t s) {
   const int ch = pick_ch_b(a.lay.row_bytes_gu);
   MOE_B_DISPATCH(run_fused_b, a.wdtype, ch, a, grid, s);
   return cudaErrorInvalidValue;
+}
+
+bool batched_tc_supported(int wdtype, int d, int I) {
+  return wdtype == WD_BF16 && d % 128 == 0 && I % 64 == 0 && d <= 16384 && I <= 16384;
+}
+
+int fused_batched_tc_grid(int d, int I, int64_t cap, int64_t n_gid) {
+  if (!batched_tc_supported(WD_BF16, d, I) || sort_n_of(cap, n_gid) > kBatchedEvictCap) return 0;
+  const size_t smem = batched_tc_smem(cap, n_gid);
+  if (cudaFuncSetAttribute(k_fused_batched_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  int occ = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_fused_batched_tc, kBThreads, smem) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return occ >= 1 ? sms : 0;  // one CTA per SM: its TMEM allocation never waits on another CTA's
+}
+
+cudaError_t launch_fused_batched_tc(const BatchArgs& a, int grid, cudaStream_t s) {
+  const size_t smem = batched_tc_smem(a.cap, a.n_gid);
+  void* params[] = {(void*)&a};
+  return cudaLaunchCooperativeKernel((const void*)k_fused_batched_tc, dim3(grid), dim3(kBThreads), params, smem, s);
 }
 
 }  // namespace moe

@@ -9,6 +9,8 @@
 // A slot is overwritten only by a copy issued after the host saw router(l) finish; router(l)
 // runs after every kernel of layers < l on the compute stream, so no earlier reader of a
 // victim slot can still be running, and experts needed by layer l are pinned for the step.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <sys/mman.h>
 
@@ -37,11 +39,12 @@ thread_local std::string g_create_error;
 
 enum {
   PC_ROUTER = 0, PC_GATEUP = 1, PC_DOWN = 2, PC_COPY = 3, PC_FUSED = 4,
-  PC_PH_R = 5, PC_PH_S = 6, PC_PH_C = 7, PC_PH_D = 8, PC_PH_T = 9, PC_PH_E = 10, PC_N = 11
+  PC_PH_R = 5, PC_PH_S = 6, PC_PH_C = 7, PC_PH_D = 8, PC_PH_T = 9, PC_PH_E = 10, PC_PH_G = 11, PC_N = 12
 };
 const char* kPcName[PC_N] = {"router", "gateup", "down_combine", "miss_copy", "fused_step",
                              "fused_phase_router", "fused_phase_select", "fused_phase_gateup",
-                             "fused_phase_down", "fused_phase_topk", "fused_phase_combine"};
+                             "fused_phase_down", "fused_phase_topk", "fused_phase_combine",
+                             "fused_phase_gather"};
 
 struct PendingTime {
   int cls;
@@ -100,6 +103,10 @@ struct moe_handle {
   // device-driven schedule: lookup table, scratch and outputs in device memory
   bool dev_mode = false;
   bool batched = false;    // device schedule with max_batch > 1: the batched kernel
+  bool batched_tc = false; // ... in its tensor-core variant
+  CUtensorMap map_gu{}, map_d{}, map_x{}, map_u{};
+  __nv_bfloat16* d_xg = nullptr;  // tensor-core variant: pairs' activations / u in plan order
+  __nv_bfloat16* d_ug = nullptr;
   int fgrid = 0;
   int tg_max = 0;
   int touch_shift = 12;
@@ -185,6 +192,7 @@ std::string check_config(const moe_config* c) {
   if (c->trace_capacity < 0) return "trace_capacity must be >= 0";
   if (c->schedule != MOE_SCHEDULE_DEVICE && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "unknown schedule";
   if (c->miss_ctas < 0) return "miss_ctas must be >= 0";
+  if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
   return "";
 }
 
@@ -578,7 +586,7 @@ moe_status harvest_phases(moe_handle* h, const unsigned long long* d_ts, int nph
 unsigned long long* phase_buffer(moe_handle* h) {
   if (!h->prof) return nullptr;
   if (!h->d_phase_ts &&
-      cudaMalloc(&h->d_phase_ts, sizeof(unsigned long long) * (moe::kBatchedPhases * h->cfg.n_layers + 1)) !=
+      cudaMalloc(&h->d_phase_ts, sizeof(unsigned long long) * (moe::kBatchedTcPhases * h->cfg.n_layers + 1)) !=
           cudaSuccess) {
     h->d_phase_ts = nullptr;
     cudaGetLastError();
@@ -638,9 +646,15 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.work = h->d_bar + 2;
   a.touch_shift = h->touch_shift;
   a.tg_max = h->tg_max;
+  a.map_gu = h->map_gu;
+  a.map_d = h->map_d;
+  a.map_x = h->map_x;
+  a.map_u = h->map_u;
+  a.xg = h->d_xg;
+  a.ug = h->d_ug;
   {
     ProfScope ps(h, s, PC_FUSED, (int64_t)c.n_layers * (int64_t)E * c.d * h->router_eb);
-    cudaError_t e = moe::launch_fused_batched(a, h->fgrid, s);
+    cudaError_t e = h->batched_tc ? moe::launch_fused_batched_tc(a, h->fgrid, s) : moe::launch_fused_batched(a, h->fgrid, s);
     ps.done();
     if (e != cudaSuccess) return cuda_fail(h, e, "batched decode step launch");
   }
@@ -649,10 +663,12 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   h->err_pending = true;
   h->steps_launched++;
   // every CTA arrives at each phase's barrier once per layer
-  h->bar_epoch += (unsigned)moe::kBatchedPhases * (unsigned)c.n_layers * (unsigned)h->fgrid;
+  const int nph = h->batched_tc ? moe::kBatchedTcPhases : moe::kBatchedPhases;
+  h->bar_epoch += (unsigned)nph * (unsigned)c.n_layers * (unsigned)h->fgrid;
   if (a.phase_ts) {
     static const int cls[moe::kBatchedPhases] = {PC_PH_R, PC_PH_T, PC_PH_S, PC_PH_C, PC_PH_D, PC_PH_E};
-    return harvest_phases(h, a.phase_ts, moe::kBatchedPhases, cls, s);
+    static const int cls_tc[moe::kBatchedTcPhases] = {PC_PH_R, PC_PH_T, PC_PH_S, PC_PH_G, PC_PH_C, PC_PH_D, PC_PH_E};
+    return harvest_phases(h, a.phase_ts, nph, h->batched_tc ? cls_tc : cls, s);
   }
   return MOE_OK;
 }
@@ -722,6 +738,58 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   return MOE_OK;
 }
 
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+    cudaGetLastError();
+  }
+  return fn;
+}
+
+// bf16 tensor map with the 128-byte swizzle; dims[0] is the contiguous (K) dimension.
+bool encode_map(CUtensorMap* m, void* base, cuuint32_t rank, const cuuint64_t* dims, const cuuint64_t* strides,
+                const cuuint32_t* box) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, base, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Buffers and TMA maps of the tensor-core batched kernel: the weights in the slot pool, and the
+// pairs' activations / u vectors in plan order (rows padded to a multiple of 16, zeroed).
+moe_status make_tc_maps(moe_handle* h) {
+  const moe_config& c = h->cfg;
+  const int64_t rows = std::max<int64_t>(16, align_up((int64_t)c.max_batch * c.top_k, 16));
+  if (cudaMalloc(&h->d_xg, rows * c.d * 2) != cudaSuccess || cudaMalloc(&h->d_ug, rows * c.d_ff * 2) != cudaSuccess)
+    return fail(h, MOE_ERR_OOM, "tensor-core staging allocation failed");
+  if (cudaMemset(h->d_xg, 0, rows * c.d * 2) != cudaSuccess || cudaMemset(h->d_ug, 0, rows * c.d_ff * 2) != cudaSuccess)
+    return fail(h, MOE_ERR_CUDA, "tensor-core staging memset failed");
+  const cuuint64_t dgu[3] = {(cuuint64_t)c.d, (cuuint64_t)(2 * c.d_ff), (cuuint64_t)h->cap};
+  const cuuint64_t sgu[2] = {(cuuint64_t)c.d * 2, (cuuint64_t)h->slot_stride};
+  const cuuint64_t dd[3] = {(cuuint64_t)c.d_ff, (cuuint64_t)c.d, (cuuint64_t)h->cap};
+  const cuuint64_t sd[2] = {(cuuint64_t)c.d_ff * 2, (cuuint64_t)h->slot_stride};
+  const cuuint32_t box_w[3] = {64, 128, 1};
+  const cuuint64_t dx[2] = {(cuuint64_t)c.d, (cuuint64_t)rows};
+  const cuuint64_t sx[1] = {(cuuint64_t)c.d * 2};
+  const cuuint64_t du[2] = {(cuuint64_t)c.d_ff, (cuuint64_t)rows};
+  const cuuint64_t su[1] = {(cuuint64_t)c.d_ff * 2};
+  const cuuint32_t box_p[2] = {64, 16};
+  if (!encode_map(&h->map_gu, h->pool, 3, dgu, sgu, box_w) ||
+      !encode_map(&h->map_d, h->pool + h->lay.d_off, 3, dd, sd, box_w) ||
+      !encode_map(&h->map_x, h->d_xg, 2, dx, sx, box_p) || !encode_map(&h->map_u, h->d_ug, 2, du, su, box_p))
+    return fail(h, MOE_ERR_CUDA, "TMA tensor map encoding failed");
+  return MOE_OK;
+}
+
 void free_all(moe_handle* h) {
   if (!h) return;
   cudaDeviceSynchronize();
@@ -741,7 +809,8 @@ void free_all(moe_handle* h) {
   for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_n_used,
                   (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
                   (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
-                  (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y})
+                  (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y,
+                  (void*)h->d_xg, (void*)h->d_ug})
     if (p) cudaFree(p);
   if (h->h_err) cudaFreeHost(h->h_err);
   if (h->err_ev) cudaEventDestroy(h->err_ev);
@@ -832,7 +901,16 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
   h->dev_mode = cfg->schedule == MOE_SCHEDULE_DEVICE;
   h->batched = h->dev_mode && cfg->max_batch > 1;
-  if (h->batched) {
+  h->batched_tc = h->batched && cfg->batched_path == MOE_BATCHED_AUTO &&
+                  moe::batched_tc_supported(cfg->wdtype, cfg->d, cfg->d_ff);
+  if (h->batched_tc) {
+    h->fgrid = moe::fused_batched_tc_grid(cfg->d, cfg->d_ff, h->cap, h->n_gid);
+    if (h->fgrid <= 0)
+      return bail(MOE_ERR_INVALID, "cap not supported by the batched schedule (a cap that can evict must be at "
+                                   "most 4096 slots)");
+    moe_status ms = make_tc_maps(h);
+    if (ms != MOE_OK) return bail(ms, h->err);
+  } else if (h->batched) {
     h->fgrid = moe::fused_batched_grid(cfg->wdtype, cfg->d, cfg->d_ff, h->cap, h->n_gid);
     h->tg_max = moe::batched_tg(cfg->wdtype, cfg->d, cfg->d_ff);
     if (h->fgrid <= 0)

@@ -7,7 +7,9 @@ the residency trace bit-exact; top-k ids exact except near-ties; gates to fp32 r
 outputs per (token, layer, sequence) row within the dtype's relative L2 bound. Shapes span
 several work items with ragged tails (d, d_ff not multiples of the item sizes, odd batch
 sizes), a Qwen3-30B-A3B-shaped layer at batch 64, and the 48-layer stack at batch 64 with
-a 6 GB pool cap (635 slots) for a few steps.
+a 6 GB pool cap (635 slots) for a few steps. bf16 shapes whose d is a multiple of 128 and d_ff
+of 64 run both expert-FFN paths: tensor cores (tcgen05 grouped GEMM, pairs per expert padded
+to 16, 32, 48 or 64 columns) and CUDA cores.
 """
 from concurrent.futures import ThreadPoolExecutor
 
@@ -55,9 +57,9 @@ def _check_outputs(wl, hidden, idx, gate, out, samples, threads=8):
     return errs
 
 
-def _parity(wl, cap, samples=None, threads=8, preload=False):
+def _parity(wl, cap, samples=None, threads=8, preload=False, path="auto"):
     hidden = synth.hidden_all(wl)
-    m = _create(wl, cap)
+    m = _create(wl, cap, batched_path=path)
     try:
         if preload:
             m.preload()
@@ -97,24 +99,44 @@ BATCHED = {
                            adtype="bf16", tokens=10, batch=6, rho=0.8, cap_slots=14),
     "bf16_wide": synth.Workload("b_bf16_wide", d=4096, n_experts=64, top_k=16, d_ff=1536, n_layers=2,
                                 wdtype="bf16", adtype="bf16", tokens=3, batch=7, rho=0.8, cap_slots=80),
+    # tensor-core shapes: 3 row tiles of W_d, 3 of [gate; up]; 66 pairs over 20 experts
+    "bf16_tc": synth.Workload("b_bf16_tc", d=384, n_experts=20, top_k=6, d_ff=192, n_layers=2, wdtype="bf16",
+                              adtype="bf16", tokens=8, batch=11, rho=0.8, cap_slots=28),
+    # 128 pairs over 3 experts: 36..46 pairs per expert (N = 48)
+    "bf16_dense": synth.Workload("b_bf16_dense", d=256, n_experts=3, top_k=2, d_ff=128, n_layers=3, wdtype="bf16",
+                                 adtype="bf16", tokens=6, batch=64, rho=0.8, cap_slots=7),
+    # every sequence routes to both experts: 64 pairs per expert (N = 64); the layers' 6 experts
+    # cycle through 4 slots, so every request misses and evicts
+    "bf16_full": synth.Workload("b_bf16_full", d=256, n_experts=2, top_k=2, d_ff=128, n_layers=3, wdtype="bf16",
+                                adtype="bf16", tokens=4, batch=64, rho=0.8, cap_slots=4),
 }
+TC_SHAPES = ["bf16_wide", "bf16_tc", "bf16_dense", "bf16_full"]
 
 
 @pytest.mark.parametrize("name", list(BATCHED))
 def test_batched_small_shapes(P, name):
     wl = BATCHED[name]
     out, tr = _parity(wl, wl.cap_slots)
-    assert (tr["kind"] == 0).any() and (tr["evicted"] >= 0).any()
+    assert (tr["evicted"] >= 0).any()
+    assert (tr["kind"] == 0).any() or name == "bf16_full"
 
 
-def test_batched_cap_invariance_bit_exact(P):
+@pytest.mark.parametrize("name", TC_SHAPES)
+def test_batched_cuda_core_path_on_tensor_core_shapes(P, name):
+    wl = BATCHED[name]
+    _parity(wl, wl.cap_slots, path="cuda_cores")
+
+
+@pytest.mark.parametrize("name,path", [("bf16_ragged", "auto"), ("bf16_tc", "auto"), ("bf16_dense", "auto"),
+                                       ("bf16_tc", "cuda_cores")])
+def test_batched_cap_invariance_bit_exact(P, name, path):
     # residency only changes where the weights are read from: outputs with a capped pool that
     # evicts every step and with every expert resident are identical
-    wl = BATCHED["bf16_ragged"]
+    wl = BATCHED[name]
     hidden = synth.hidden_all(wl)
     outs = []
     for cap in (wl.cap_slots, wl.n_gid):
-        m = _create(wl, cap)
+        m = _create(wl, cap, batched_path=path)
         try:
             outs.append(run_gpu(m, hidden, wl.adtype)[0])
         finally:
@@ -173,13 +195,14 @@ def test_batch_above_max_is_rejected(P):
         m.destroy()
 
 
-def test_layer_bf16_batch64(P):
+@pytest.mark.parametrize("path", ["auto", "cuda_cores"])
+def test_layer_bf16_batch64(P, path):
     # Qwen3-30B-A3B-shaped layers, 64 sequences: 512 routed pairs per layer-step over ~126 experts
     wl = synth.WORKLOADS["layer_bf16"].replace(name="layer_bf16_b64", n_layers=2, batch=64, tokens=4, cap_slots=200)
     rng = np.random.default_rng(0)
     samples = [(t, l, int(b)) for t in range(wl.tokens) for l in range(wl.n_layers)
                for b in rng.choice(64, size=4, replace=False)]
-    _parity(wl, wl.cap_slots, samples=samples, threads=16)
+    _parity(wl, wl.cap_slots, samples=samples, threads=16, path=path)
 
 
 def test_stack48_batch64_capped_steps(P):
