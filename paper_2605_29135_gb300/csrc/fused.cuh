@@ -123,10 +123,13 @@ struct BatchArgs {
   unsigned* work;              // [2] work-item counters of phases C and D (reset in phase S)
   int touch_shift;
   int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
+  int router_tb;               // sequences per router work item (batched_router_tb)
 };
 
 // Pairs staged per group for this shape, and the co-resident grid (0: shape or cap unsupported).
 int batched_tg(int wdtype, int d, int I);
+// Sequences per router work item (1..8: their activations fit in the kernel's shared memory).
+int batched_router_tb(int wdtype, int d, int I, bool tensor_cores);
 int fused_batched_grid(int wdtype, int d, int I, int64_t cap, int64_t n_gid);
 cudaError_t launch_fused_batched(const BatchArgs& a, int grid, cudaStream_t s);
 

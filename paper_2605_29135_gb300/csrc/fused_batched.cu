@@ -70,28 +70,42 @@ size_t batched_smem(int wdtype, int d, int I, int64_t cap, int64_t n_gid) {
   return std::max((size_t)tg_of(wdtype, d, I) * per, (size_t)sort_n_of(cap, n_gid) * sizeof(unsigned long long));
 }
 
-// ---- phase R: logits of one router row for up to 8 sequences
+// ---- phase R: a CTA work item is (block of up to rtb sequences, block of 8 router rows). The
+// CTA stages the sequences' activations in shared memory; warp w holds row 8 * eb + w in
+// registers (its loads are issued before the staging, so their latency overlaps it) and dots it
+// with every staged activation vector.
 template <int WDR>
-__device__ __forceinline__ void router_item(const BatchArgs& a, int l, int e, int b0, int lane) {
+__device__ __forceinline__ void router_block(const BatchArgs& a, int l, int tb, int eb, int rtb, uint8_t* xs) {
   constexpr int RG = 8;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int xbytes = a.d * (WDR == WD_FP32 ? 4 : 2);
+  const int xpad = (xbytes + 15) & ~15;
   const int nchr = xbytes / 16;
-  const uint8_t* row = a.routers + ((int64_t)l * a.E + e) * xbytes;
-  const int nt = a.B - b0 < 8 ? a.B - b0 : 8;
+  const int e = eb * kBWarps + warp;
+  const bool has_row = e < a.E;
+  const uint8_t* row = a.routers + ((int64_t)l * a.E + (has_row ? e : 0)) * xbytes;
+  const int b0 = tb * rtb;
+  const int nt = a.B - b0 < rtb ? a.B - b0 : rtb;
   uint4 rw[RG];
-  if (nchr <= 32 * RG) {
 #pragma unroll
-    for (int j = 0; j < RG; j++) {
-      const int c = j * 32 + lane;
-      rw[j] = c < nchr ? ld_cg(row + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
-    }
+  for (int j = 0; j < RG; j++) {
+    const int c = j * 32 + lane;
+    rw[j] = (has_row && c < nchr) ? ld_cg(row + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
   }
+  __syncthreads();  // the previous item's readers are done with xs
+  for (int q = threadIdx.x; q < nt * nchr; q += blockDim.x) {
+    const int t = q / nchr, c = q - t * nchr;
+    const uint4* src = reinterpret_cast<const uint4*>((const uint8_t*)a.hidden + ((int64_t)l * a.B + b0 + t) * xbytes);
+    *reinterpret_cast<uint4*>(xs + (int64_t)t * xpad + (int64_t)c * 16) = __ldg(src + c);
+  }
+  __syncthreads();
+  if (!has_row) return;
 #pragma unroll 1
   for (int t = 0; t < nt; t++) {
-    const uint8_t* x = (const uint8_t*)a.hidden + ((int64_t)l * a.B + b0 + t) * xbytes;
+    const uint8_t* x = xs + (int64_t)t * xpad;
     float acc = 0.f;
     for (int c0 = 0; c0 < nchr; c0 += 32 * RG) {
-      if (nchr > 32 * RG) {
+      if (c0 > 0) {  // rows longer than 256 chunks: the next part (L1/L2 hits after the first vector)
 #pragma unroll
         for (int j = 0; j < RG; j++) {
           const int c = c0 + j * 32 + lane;
@@ -100,79 +114,119 @@ __device__ __forceinline__ void router_item(const BatchArgs& a, int l, int e, in
       }
 #pragma unroll
       for (int j = 0; j < RG; j++) {
+        opaque(rw[j]);
         const int c = c0 + j * 32 + lane;
         if (c < nchr) acc = dot_chunk<WDR>(rw[j], x + (int64_t)c * 16, acc);
       }
     }
     acc = warp_sum(acc);
     if (lane == 0) a.z[(int64_t)(b0 + t) * a.E + e] = acc;
+    if (nchr > 32 * RG && t + 1 < nt) {  // back to the row's first part for the next vector
+#pragma unroll
+      for (int j = 0; j < RG; j++) {
+        const int c = j * 32 + lane;
+        rw[j] = c < nchr ? ld_cg(row + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+      }
+    }
   }
 }
 
 // ---- phase S: union of the pairs' experts, one lookup-table step, trace and plan (CTA 0)
 __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t step, unsigned long long* keys) {
-  __shared__ int s_sel[kMaxPairs];
-  __shared__ int s_flag[256];
-  __shared__ int s_need[256];    // needed expert ids (within the layer), ascending
+  constexpr int kChunks = kMaxPairs / 32;
+  __shared__ int s_sel[kMaxPairs];       // expert of pair p
+  __shared__ uint8_t s_rank[kMaxPairs];  // rank of pair p among the pairs of its 32-pair chunk with its expert
+  __shared__ uint8_t s_hist[kChunks][256];  // pairs per (chunk, expert), then their prefix over chunks
+  __shared__ int s_slot_e[256];          // slot of every expert of the layer before the step (-1: not resident)
+  __shared__ int s_tot[256];             // pairs per expert
+  __shared__ int s_q_of_e[256];          // index of expert e among the needed experts
+  __shared__ int s_need[256];            // needed expert ids (within the layer), ascending
   __shared__ int s_slot[256];
   __shared__ int s_miss[256];
-  __shared__ int s_mbefore[256]; // misses among needed[0..q)
+  __shared__ int s_mbefore[256];         // misses among needed[0..q)
   __shared__ int s_evict[256];
-  __shared__ int s_pos[256];     // plan position of needed q: misses first, then hits
-  __shared__ int s_cnt[256];     // pairs per plan position
+  __shared__ int s_pos[256];             // plan position of needed q: misses first, then hits
+  __shared__ int s_cnt[256];             // pairs per plan position
   __shared__ int s_off[256];
   __shared__ int s_n, s_nm, s_nused0, s_nfree, s_nev, s_nevicted;
+  __shared__ unsigned long long s_trace_base;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int E = a.E, P = a.B * a.k;
+  const int nchunks = (P + 31) / 32;
 
+  // every global read this step needs, issued together
   for (int p = tid; p < P; p += blockDim.x) s_sel[p] = __ldcg(a.sel_e + p);
-  for (int e = tid; e < 256; e += blockDim.x) s_flag[e] = 0;
-  if (tid == 0) s_nevicted = 0;
+  for (int e = tid; e < E; e += blockDim.x) s_slot_e[e] = a.slot_of[l * E + e];
+  if (tid == 0) {
+    s_nused0 = *a.n_used;
+    s_trace_base = *(volatile unsigned long long*)a.trace_n;
+    s_nevicted = 0;
+  }
+  for (int i = tid; i < kChunks * 256 / 4; i += blockDim.x) reinterpret_cast<uint32_t*>(s_hist)[i] = 0u;
   __syncthreads();
-  for (int p = tid; p < P; p += blockDim.x) s_flag[s_sel[p]] = 1;
+  // per 32-pair chunk: pairs per expert, and each pair's rank among its chunk's pairs of that expert
+  for (int c = warp; c < nchunks; c += kBWarps) {
+    const int p = c * 32 + lane;
+    const int e = p < P ? s_sel[p] : -1 - lane;  // distinct values for the lanes past the end
+    const unsigned m = __match_any_sync(kFull, e);
+    if (p < P) {
+      s_rank[p] = (uint8_t)__popc(m & ((1u << lane) - 1u));
+      if (lane == __ffs(m) - 1) s_hist[c][e] = (uint8_t)__popc(m);
+    }
+  }
+  __syncthreads();
+  // per expert: the prefix of its chunk counts (its pairs in earlier chunks), and its total
+  for (int e = tid; e < E; e += blockDim.x) {
+    int run = 0;
+    for (int c = 0; c < nchunks; c++) {
+      const int v = s_hist[c][e];
+      s_hist[c][e] = (uint8_t)run;
+      run += v;
+    }
+    s_tot[e] = run;
+  }
   __syncthreads();
   if (warp == 0) {
+    // needed experts (at least one pair) ascending, with their slots; then the misses' ranks
     int base = 0;
     for (int e0 = 0; e0 < E; e0 += 32) {
       const int e = e0 + lane;
-      const bool f = e < E && s_flag[e];
+      const int tot = e < E ? s_tot[e] : 0;
+      const bool f = tot > 0;
       const unsigned m = __ballot_sync(kFull, f);
-      if (f) s_need[base + __popc(m & ((1u << lane) - 1u))] = e;
+      if (f) {
+        const int q = base + __popc(m & ((1u << lane) - 1u));
+        s_need[q] = e;
+        s_q_of_e[e] = q;
+        s_slot[q] = s_slot_e[e];
+        s_miss[q] = s_slot_e[e] < 0;
+        s_evict[q] = -1;
+        s_cnt[q] = tot;  // by needed index for now
+      }
       base += __popc(m);
     }
-    if (lane == 0) s_n = base;
-  }
-  __syncthreads();
-  const int n = s_n;
-  for (int q = tid; q < n; q += blockDim.x) {
-    const int sl = a.slot_of[l * E + s_need[q]];
-    s_slot[q] = sl;
-    s_miss[q] = sl < 0;
-    s_evict[q] = -1;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    int base = 0;
+    const int n = base;
+    __syncwarp();
+    int nm = 0;
     for (int q0 = 0; q0 < n; q0 += 32) {
       const int q = q0 + lane;
       const bool f = q < n && s_miss[q];
       const unsigned m = __ballot_sync(kFull, f);
-      if (q < n) s_mbefore[q] = base + __popc(m & ((1u << lane) - 1u));
-      base += __popc(m);
+      if (q < n) s_mbefore[q] = nm + __popc(m & ((1u << lane) - 1u));
+      nm += __popc(m);
     }
     if (lane == 0) {
-      const int nused = *a.n_used;
-      const int nfree = (int)(a.cap - nused);
-      const int take = base < nfree ? base : nfree;
-      *a.n_used = nused + take;
-      s_nm = base;
-      s_nused0 = nused;
+      const int nfree = (int)(a.cap - s_nused0);
+      const int take = nm < nfree ? nm : nfree;
+      *a.n_used = s_nused0 + take;
+      s_n = n;
+      s_nm = nm;
       s_nfree = nfree;
-      s_nev = base - take;
+      s_nev = nm - take;
     }
   }
   __syncthreads();
-  const int nm = s_nm, nfree = s_nfree, nev = s_nev;
+  const int n = s_n, nm = s_nm, nfree = s_nfree, nev = s_nev;
   if (nev > 0) {
     // Every slot is occupied. Sort the slot keys (last use << 32 | id) ascending, with the slots
     // of this step's hits pinned at the maximum: the first nev keys are the victims.
@@ -201,6 +255,7 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   }
   // place the misses: free slots first, then the victims in ascending key order
   for (int q = tid; q < n; q += blockDim.x) {
+    s_pos[q] = s_miss[q] ? s_mbefore[q] : nm + (q - s_mbefore[q]);
     if (!s_miss[q]) continue;
     const int m = s_mbefore[q];
     int slot = -1;
@@ -220,46 +275,18 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
     s_slot[q] = slot;
   }
   __syncthreads();
-  for (int q = tid; q < n; q += blockDim.x)
-    if (s_evict[q] >= 0) a.slot_of[s_evict[q]] = -1;
-  __syncthreads();
-  const unsigned long long base_rec = *(volatile unsigned long long*)a.trace_n;
   for (int q = tid; q < n; q += blockDim.x) {
-    const int gid = l * E + s_need[q];
-    const int sl = s_slot[q];
-    if (s_miss[q] && sl >= 0) a.slot_of[gid] = sl;
-    if (sl >= 0) a.slot_key[sl] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)gid;
-    if (base_rec + q < (unsigned long long)a.trace_cap) {
-      TraceRec rec;
-      rec.step = (int32_t)step;
-      rec.layer = l;
-      rec.expert = s_need[q];
-      rec.kind = s_miss[q];
-      rec.slot = sl;
-      rec.evicted = s_evict[q];
-      a.trace[base_rec + q] = rec;
-    }
-    s_pos[q] = s_miss[q] ? s_mbefore[q] : nm + (q - s_mbefore[q]);
-  }
-  __syncthreads();
-  // pairs per needed expert, ascending pair order (one warp per expert, a ballot per 32 pairs)
-  for (int q = warp; q < n; q += kBWarps) {
-    const int e = s_need[q];
-    int cnt = 0;
-    for (int p0 = 0; p0 < P; p0 += 32) {
-      const int p = p0 + lane;
-      cnt += __popc(__ballot_sync(kFull, p < P && s_sel[p] == e));
-    }
-    if (lane == 0) s_cnt[s_pos[q]] = cnt;
+    if (s_evict[q] >= 0) a.slot_of[s_evict[q]] = -1;
+    s_off[s_pos[q]] = s_cnt[q];  // pairs per plan position (scanned below)
   }
   __syncthreads();
   if (warp == 0) {
-    // exclusive scan of s_cnt[0..n) in plan order: 8 consecutive entries per lane
+    // exclusive scan of the pair counts in plan order: 8 consecutive entries per lane
     int v[8], sum = 0;
 #pragma unroll
     for (int j = 0; j < 8; j++) {
       const int q = lane * 8 + j;
-      v[j] = q < n ? s_cnt[q] : 0;
+      v[j] = q < n ? s_off[q] : 0;
       sum += v[j];
     }
     int inc = sum;
@@ -268,48 +295,62 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
       const int o = __shfl_up_sync(kFull, inc, off);
       if (lane >= off) inc += o;
     }
+    __syncwarp();
     int run = inc - sum;
 #pragma unroll
     for (int j = 0; j < 8; j++) {
       const int q = lane * 8 + j;
-      if (q < n) s_off[q] = run;
+      if (q < n) {
+        s_off[q] = run;
+        s_cnt[q] = v[j];  // now by plan position
+      }
       run += v[j];
+    }
+  } else {
+    const unsigned long long base_rec = s_trace_base;
+    for (int q = tid - 32; q < n; q += blockDim.x - 32) {
+      const int gid = l * E + s_need[q];
+      const int sl = s_slot[q];
+      if (s_miss[q] && sl >= 0) a.slot_of[gid] = sl;
+      if (sl >= 0) a.slot_key[sl] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)gid;
+      if (base_rec + q < (unsigned long long)a.trace_cap) {
+        TraceRec rec;
+        rec.step = (int32_t)step;
+        rec.layer = l;
+        rec.expert = s_need[q];
+        rec.kind = s_miss[q];
+        rec.slot = sl;
+        rec.evicted = s_evict[q];
+        a.trace[base_rec + q] = rec;
+      }
     }
   }
   __syncthreads();
-  for (int q = warp; q < n; q += kBWarps) {
-    const int e = s_need[q];
+  // the plan: pairs grouped by expert in plan order, ascending pair index within an expert
+  for (int p = tid; p < P; p += blockDim.x) {
+    const int e = s_sel[p];
+    const int pos = s_pos[s_q_of_e[e]];
+    a.plan_tok[s_off[pos] + s_hist[p >> 5][e] + s_rank[p]] = p;
+  }
+  for (int q = tid; q < n; q += blockDim.x) {
     const int pos = s_pos[q];
-    int w = s_off[pos];
-    for (int p0 = 0; p0 < P; p0 += 32) {
-      const int p = p0 + lane;
-      const bool f = p < P && s_sel[p] == e;
-      const unsigned m = __ballot_sync(kFull, f);
-      if (f) a.plan_tok[w + __popc(m & ((1u << lane) - 1u))] = p;
-      w += __popc(m);
-    }
-    if (lane == 0) {
-      const int sl = s_slot[q];
-      a.plan_slot[pos] = sl < 0 ? 0 : sl;
-      a.plan_gid[pos] = l * E + e;
-      a.plan_miss[pos] = s_miss[q];
-      a.plan_off[pos] = s_off[pos];
-      a.plan_cnt[pos] = s_cnt[pos];
-    }
+    const int sl = s_slot[q];
+    a.plan_slot[pos] = sl < 0 ? 0 : sl;
+    a.plan_gid[pos] = l * E + s_need[q];
+    a.plan_miss[pos] = s_miss[q];
+    a.plan_off[pos] = s_off[pos];
+    a.plan_cnt[pos] = s_cnt[pos];
   }
   if (tid == 0) {
     a.plan_n[0] = n;
     a.plan_n[1] = nm;
     a.work[0] = 0u;  // the previous layer's phases C and D are complete (grid barriers since)
     a.work[1] = 0u;
-    a.stats[STAT_HITS] += (unsigned long long)(n - nm);
-    a.stats[STAT_MISSES] += (unsigned long long)nm;
-    a.stats[STAT_LAYER_STEPS] += 1;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    a.stats[STAT_EVICTIONS] += (unsigned long long)s_nevicted;
-    *a.trace_n = base_rec + n;
+    *a.trace_n = s_trace_base + n;
+    atomicAdd(a.stats + STAT_HITS, (unsigned long long)(n - nm));
+    atomicAdd(a.stats + STAT_MISSES, (unsigned long long)nm);
+    atomicAdd(a.stats + STAT_EVICTIONS, (unsigned long long)s_nevicted);
+    atomicAdd(a.stats + STAT_LAYER_STEPS, 1ull);
   }
 }
 
@@ -533,16 +574,17 @@ __device__ void down_item(const BatchArgs& a, int pos, int oblk, float* us, int*
   }
 }
 
-// ---- phase R for all CTAs: one warp per (router row, block of 8 sequences)
-__device__ __forceinline__ void phase_router(const BatchArgs& a, int l, int gw, int W, int lane) {
-  const int nb8 = (a.B + 7) / 8;
-  for (int it = gw; it < a.E * nb8; it += W) {
-    const int e = it / nb8;
-    const int b0 = (it - e * nb8) * 8;
+// ---- phase R for all CTAs: items (block of a.router_tb sequences, block of 8 router rows)
+__device__ __forceinline__ void phase_router(const BatchArgs& a, int l, uint8_t* xs) {
+  const int rtb = a.router_tb;
+  const int ntb = (a.B + rtb - 1) / rtb;
+  const int neb = (a.E + kBWarps - 1) / kBWarps;
+  for (int it = blockIdx.x; it < ntb * neb; it += gridDim.x) {
+    const int eb = it / ntb, tb = it - eb * ntb;
     if (a.wdtype == WD_FP32)
-      router_item<WD_FP32>(a, l, e, b0, lane);
+      router_block<WD_FP32>(a, l, tb, eb, rtb, xs);
     else
-      router_item<WD_BF16>(a, l, e, b0, lane);
+      router_block<WD_BF16>(a, l, tb, eb, rtb, xs);
   }
 }
 
@@ -565,22 +607,32 @@ __device__ __forceinline__ void phase_topk(const BatchArgs& a, int l, int gw, in
   }
 }
 
-// ---- phase E: out[b][o] = sum_r g_{b,r} y_{b*k+r}[o], ranks in order
+// ---- phase E: out[b][o] = sum_r g_{b,r} y_{b*k+r}[o], ranks in order; four outputs per thread
+// (d is a multiple of 4)
 __device__ __forceinline__ void phase_combine(const BatchArgs& a, int l) {
-  const int64_t nout = (int64_t)a.B * a.d;
+  const int d4 = a.d / 4;
+  const int64_t nout = (int64_t)a.B * d4;
   for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nout; q += (int64_t)gridDim.x * blockDim.x) {
-    const int b = (int)(q / a.d);
-    const int o = (int)(q - (int64_t)b * a.d);
-    float acc = 0.f;
+    const int b = (int)(q / d4);
+    const int o = 4 * (int)(q - (int64_t)b * d4);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int r = 0; r < a.k; r++) {
       const int p = b * a.k + r;
-      acc = fmaf(__ldcg(a.sel_g + p), __ldcg(a.y + (int64_t)p * a.d + o), acc);
+      const float g = __ldcg(a.sel_g + p);
+      const float4 y = __ldcg(reinterpret_cast<const float4*>(a.y + (int64_t)p * a.d + o));
+      acc.x = fmaf(g, y.x, acc.x);
+      acc.y = fmaf(g, y.y, acc.y);
+      acc.z = fmaf(g, y.z, acc.z);
+      acc.w = fmaf(g, y.w, acc.w);
     }
     const int64_t oi = ((int64_t)l * a.B + b) * a.d + o;
-    if (a.wdtype == WD_FP32)
-      reinterpret_cast<float*>(a.out)[oi] = acc;
-    else
-      reinterpret_cast<__nv_bfloat16*>(a.out)[oi] = __float2bfloat16_rn(acc);
+    if (a.wdtype == WD_FP32) {
+      *reinterpret_cast<float4*>(reinterpret_cast<float*>(a.out) + oi) = acc;
+    } else {
+      __nv_bfloat162* dst = reinterpret_cast<__nv_bfloat162*>(reinterpret_cast<__nv_bfloat16*>(a.out) + oi);
+      dst[0] = __floats2bfloat162_rn(acc.x, acc.y);
+      dst[1] = __floats2bfloat162_rn(acc.z, acc.w);
+    }
   }
 }
 
@@ -615,7 +667,7 @@ __global__ void __launch_bounds__(kBThreads, 2) k_fused_batched(const __grid_con
 
   for (int l = 0; l < a.L; l++) {
     const int clock = (int)(step * a.L + l + 1);  // 0 is older than every step (preloaded experts)
-    phase_router(a, l, gw, W, lane);
+    phase_router(a, l, smem);
     if (!grid_sync(a, nbar)) return;
     mark(l, 0);
     phase_topk(a, l, gw, W, lane);
@@ -892,7 +944,7 @@ __global__ void __launch_bounds__(kBThreads, 1) k_fused_batched_tc(const __grid_
   auto layers = [&]() -> bool {
     for (int l = 0; l < a.L; l++) {
       const int clock = (int)(step * a.L + l + 1);
-      phase_router(a, l, gw, W, lane);
+      phase_router(a, l, smem);
       if (!grid_sync(a, nbar)) return false;
       mark(l, 0);
       phase_topk(a, l, gw, W, lane);
@@ -1037,6 +1089,14 @@ cudaError_t run_fused_b(const BatchArgs& a, int grid, cudaStream_t s) {
   } while (0)
 
 int batched_tg(int wdtype, int d, int I) { return tg_of(wdtype, d, I); }
+
+int batched_router_tb(int wdtype, int d, int I, bool tensor_cores) {
+  const int xpad = (d * (wdtype == WD_FP32 ? 4 : 2) + 15) & ~15;
+  // the dynamic shared memory without the sort keys (which may be absent)
+  const size_t smem = tensor_cores ? (size_t)kTcStages * kTcStageBytes
+                                   : (size_t)tg_of(wdtype, d, I) * std::max(xpad, ipad_of(I) * 4);
+  return (int)std::max<size_t>(1, std::min<size_t>(8, smem / xpad));
+}
 
 int fused_batched_grid(int wdtype, int d, int I, int64_t cap, int64_t n_gid) {
   if (sort_n_of(cap, n_gid) > kBatchedEvictCap) return 0;

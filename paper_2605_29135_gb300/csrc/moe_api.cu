@@ -646,6 +646,7 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.work = h->d_bar + 2;
   a.touch_shift = h->touch_shift;
   a.tg_max = h->tg_max;
+  a.router_tb = moe::batched_router_tb(c.wdtype, c.d, c.d_ff, h->batched_tc);
   a.map_gu = h->map_gu;
   a.map_d = h->map_d;
   a.map_x = h->map_x;
