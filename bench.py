@@ -212,19 +212,26 @@ def oracle_layer_sample(wl, hidden, budget_s):
                       f"router + top-k expert FFN + combine in fp64, {dt:.1f} s; tok/s = units / layers / s"}
 
 
-def kernel_source_digest() -> str:
-    """Digest of the device-driven kernel's sources (ties a stored ncu traffic figure to them)."""
+KERNEL_SOURCES = {
+    "k_fused": ("fused.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh"),
+    "k_fused_batched": ("fused_batched.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh", "tc.cuh"),
+    "k_fused_batched_tc": ("fused_batched.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh", "tc.cuh"),
+}
+
+
+def kernel_source_digest(kernel: str = "k_fused") -> str:
+    """Digest of a decode kernel's sources (ties a stored ncu traffic figure to them)."""
     import hashlib
 
     h = hashlib.sha256()
-    for f in ("fused.cu", "fused.cuh", "dev.cuh"):
+    for f in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2605_29135_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
 
 
-def stored_traffic(name: str):
-    """Per-launch DRAM traffic of the fused kernel from a committed ncu summary, if it was taken on
+def stored_traffic(name: str, kernel: str):
+    """Per-launch DRAM traffic of a decode kernel from a committed ncu summary, if it was taken on
     the current kernel sources (else None)."""
     p = os.path.join(ROOT, "profiles", name)
     if not os.path.exists(p):
@@ -235,7 +242,7 @@ def stored_traffic(name: str):
             if ":" in line and line.strip().startswith("- "):
                 k, v = line.strip()[2:].split(":", 1)
                 vals[k.strip()] = v.strip().strip("`")
-    if vals.get("kernel_source_digest") != kernel_source_digest():
+    if vals.get("kernel_source_digest") != kernel_source_digest(kernel):
         return None
     try:
         return float(vals["traffic_bytes_per_full_launch"])
@@ -282,13 +289,15 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
     achieved = per_launch / avg_s / 1e9
     phases = {k[len("fused_phase_"):]: round(v["total_ms"] * 1e3 / v["launches"], 2)
               for k, v in prof.items() if k.startswith("fused_phase_") and v["launches"]}
-    kname = ("k_fused_batched" if wl.batch > 1 else "k_fused") if dom == "fused_step" else dom
+    tensor_cores = prof.get("fused_phase_gather", {}).get("launches", 0) > 0
+    kname = (("k_fused_batched_tc" if tensor_cores else "k_fused_batched") if wl.batch > 1 else "k_fused") \
+        if dom == "fused_step" else dom
     traffic_file = f"{kname}_{wl.name}_resident.md".replace("k_fused_stack48_bf16", "k_fused_stack48")
     return {"bound": "hbm", "kernel": kname,
             "workload": f"{wl.name} with all {wl.n_gid} experts resident (preloaded), batch {wl.batch}",
             "achieved": achieved, "peak": peak_hbm, "unit": "GB/s", "frac": achieved / peak_hbm,
             "peak_source": f"{peak_src} hbm_gbs (copy; burst figure: kernel timed per launch)",
-            "traffic": stored_traffic(traffic_file) if dom == "fused_step" else None,
+            "traffic": stored_traffic(traffic_file, kname) if dom == "fused_step" else None,
             "bytes_per_launch": per_launch, "experts_per_step": experts_per_step,
             "avg_launch_us": avg_s * 1e6, "launches": dk["launches"],
             "misses_in_window": s1["misses"] - s0["misses"], "phase_us_per_layer": phases}
