@@ -490,7 +490,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
     // L2 prefetch per page-sized stride, issued by every thread of the grid at once. Without it
     // the streaming warps meet each page's translation miss one after another as they advance
     // through the expert, and the link idles while the translations resolve.
-    if (nm > 0) {
+    if (nm > 0 && a.touch_shift > 0) {
       const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
       const int64_t gt0 = (int64_t)blockIdx.x * kFThreads + threadIdx.x;
       const int64_t GT = (int64_t)gridDim.x * kFThreads;

@@ -56,7 +56,7 @@ struct FusedArgs {
   unsigned long long* phase_ts; // optional [L][4]: global-timer ns at the end of phases R, S, C, D
                                 // (CTA 0, after each barrier); NULL = off
   int miss_ctas;               // CTAs that stream missed experts from the host tier in phase C
-  int touch_shift;             // log2 of the stride of the translation-warming touches (12 = 4 KB)
+  int touch_shift;             // log2 of the stride of the translation-warming touches (12 = 4 KB; 0 = none)
 };
 
 // Maximum co-resident CTAs for the fused kernel of this shape (0 if it cannot launch).
@@ -121,7 +121,7 @@ struct BatchArgs {
   unsigned long long barrier_timeout_ns;
   unsigned long long* phase_ts; // optional [L][kBatchedPhases] + 1
   unsigned* work;              // [2] work-item counters of phases C and D (reset in phase S)
-  int touch_shift;
+  int touch_shift;             // log2 of the translation-warming touch stride (0: no touches)
   int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
   int router_tb;               // sequences per router work item (batched_router_tb)
 };

@@ -858,7 +858,7 @@ __device__ void tc_epilogue(const BatchArgs& a, TcShared& st, const TcGemm& g, i
 __device__ void tc_gather_copy(const BatchArgs& a, int l, int gw, int W, int lane, int* s_item) {
   const int nm = __ldcg(a.plan_n + 1);
   const int P = a.B * a.k;
-  if (nm > 0) {
+  if (nm > 0 && a.touch_shift > 0) {
     const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
     const int64_t gt0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t GT = (int64_t)gridDim.x * blockDim.x;
