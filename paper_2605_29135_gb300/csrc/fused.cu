@@ -41,6 +41,34 @@ __device__ __forceinline__ unsigned long long shfl_min_u64(unsigned long long v)
   return v;
 }
 
+// The k smallest slot keys of a full pool, ascending, into a.cand (CTA 0, all threads; keys are
+// distinct, so round j takes the smallest key above round j - 1's).
+__device__ void find_victim_candidates(const FusedArgs& a) {
+  __shared__ unsigned long long s_min[kFWarps];
+  __shared__ unsigned long long s_last;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  unsigned long long last = 0ull;
+  for (int j = 0; j < a.k; j++) {
+    unsigned long long best = ~0ull;
+    for (int64_t sl = threadIdx.x; sl < a.cap; sl += blockDim.x) {
+      const unsigned long long key = __ldcg(a.slot_key + sl);
+      if ((j == 0 || key > last) && key < best) best = key;
+    }
+    best = shfl_min_u64(best);
+    if (lane == 0) s_min[warp] = best;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned long long m = s_min[0];
+      for (int w = 1; w < kFWarps; w++) m = s_min[w] < m ? s_min[w] : m;
+      a.cand[j] = m;
+      s_last = m;
+    }
+    __syncthreads();
+    last = s_last;
+  }
+  if (threadIdx.x == 0) a.cand[kMaxRanks] = (unsigned long long)a.k;
+}
+
 // Phase S, run by CTA 0 (all its threads).
 __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t step) {
   __shared__ int s_idx[kMaxRanks];
@@ -51,7 +79,7 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   __shared__ int s_evict[kMaxRanks];  // evicted global id per needed id, -1 if none
   __shared__ int s_vslot[kMaxRanks];  // victims in ascending (last use, id): slot and global id
   __shared__ int s_vgid[kMaxRanks];
-  __shared__ int s_nev;
+  __shared__ int s_nev, s_nev_found;
   __shared__ unsigned long long s_ckey[kFWarps][kMaxRanks];  // each warp's smallest candidate keys
   __shared__ int s_cslot[kFWarps][kMaxRanks];
   const int k = a.k, E = a.E;
@@ -102,10 +130,29 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   }
   __syncthreads();
   const int nev = s_nev;
-  if (nev > 0) {
+  if (nev > 0 && threadIdx.x == 0) {
     // Victims: the nev smallest slot keys (last use, id) among slots that hold no expert of this
-    // step (every slot is occupied when eviction is needed). Each warp finds the nev smallest of
-    // its slots, warp 0 takes the nev smallest of those candidates.
+    // step (every slot is occupied when eviction is needed). They are among the k smallest keys
+    // of the pool (at most k - nev of those belong to this step's hits), which phase C of the
+    // previous layer-step left in a.cand. s_nev_found < nev sends phase S to the full scan.
+    const int nc = (int)__ldcg(a.cand + kMaxRanks);
+    int j = 0;
+    for (int c = 0; c < nc && j < nev; c++) {
+      const unsigned long long key = __ldcg(a.cand + c);
+      const int g = (int)(uint32_t)(key & 0xffffffffull);
+      bool needed = false;
+      for (int t = 0; t < k; t++) needed |= (s_need[t] == g);
+      if (needed) continue;
+      s_vgid[j] = g;
+      s_vslot[j] = a.slot_of[g];
+      j++;
+    }
+    s_nev_found = j;
+  }
+  __syncthreads();
+  if (nev > 0 && s_nev_found < nev) {
+    // Full scan: each warp finds the nev smallest of its slots, warp 0 takes the nev smallest of
+    // those candidates.
     for (int j = 0; j < nev; j++) {
       unsigned long long best = ~0ull;
       int bslot = -1;
@@ -201,6 +248,7 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     a.stats[STAT_MISSES] += misses;
     a.stats[STAT_EVICTIONS] += evictions;
     a.stats[STAT_LAYER_STEPS] += 1;
+    a.cand[kMaxRanks] = 0ull;  // the keys changed: phase C finds new candidates if the pool is full
   }
   __syncthreads();
   if (threadIdx.x < k) {
@@ -500,6 +548,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
         asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
       }
     }
+    if (blockIdx.x == 0 && __ldcg(a.n_used) >= a.cap) find_victim_candidates(a);
     const int mctas = nm > 0 ? (a.miss_ctas < (int)gridDim.x - 1 ? a.miss_ctas : (int)gridDim.x - 1) : 0;
     const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;  // the last CTAs (CTA 0 leads phase S)
     if (miss_cta) {

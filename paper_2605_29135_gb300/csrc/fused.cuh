@@ -57,6 +57,10 @@ struct FusedArgs {
                                 // (CTA 0, after each barrier); NULL = off
   int miss_ctas;               // CTAs that stream missed experts from the host tier in phase C
   int touch_shift;             // log2 of the stride of the translation-warming touches (12 = 4 KB; 0 = none)
+  // Victim candidates: the k smallest slot keys of a full pool, ascending, found by CTA 0 during
+  // phase C (off the critical path) for the next layer-step's phase S; cand[kMaxRanks] holds how
+  // many are valid (0: phase S scans every slot).
+  unsigned long long* cand;    // [kMaxRanks + 1]
 };
 
 // Maximum co-resident CTAs for the fused kernel of this shape (0 if it cannot launch).

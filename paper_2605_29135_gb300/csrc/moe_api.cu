@@ -31,8 +31,10 @@ namespace {
 
 constexpr double kWaitTimeoutS = 20.0;
 // CTAs of the fused kernel that stream missed experts: enough warps to keep the host link's
-// bandwidth-delay product in flight, few enough not to flood it with outstanding requests.
-constexpr int kDefaultMissCtas = 24;
+// bandwidth-delay product in flight when a layer-step misses only a few small (int4) experts,
+// few enough not to flood it with outstanding requests when it misses several bf16 experts
+// (measured on the 48-layer stacks: bf16 flat from 24 to 64 CTAs, int4 +8% at 64).
+constexpr int kDefaultMissCtas = 64;
 
 thread_local std::string g_create_error;
 
@@ -113,6 +115,7 @@ struct moe_handle {
   const uint8_t* arena_dev = nullptr;
   int32_t* d_slot_of = nullptr;
   unsigned long long* d_slot_key = nullptr;
+  unsigned long long* d_cand = nullptr;  // batch-1 kernel: victim candidates [kMaxRanks + 1]
   int32_t* d_n_used = nullptr;
   int64_t* d_step = nullptr;
   float* d_z = nullptr;
@@ -205,6 +208,7 @@ void reset_device_state(moe_handle* h) {
   if (!h->dev_mode) return;
   cudaMemset(h->d_slot_of, 0xff, sizeof(int32_t) * h->n_gid);
   cudaMemset(h->d_slot_key, 0xff, sizeof(unsigned long long) * h->cap);
+  cudaMemset(h->d_cand, 0, sizeof(unsigned long long) * (moe::kMaxRanks + 1));
   cudaMemset(h->d_n_used, 0, sizeof(int32_t));
   cudaMemset(h->d_step, 0, sizeof(int64_t));
   cudaMemset(h->d_trace_n, 0, sizeof(unsigned long long));
@@ -684,6 +688,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   a.arena = h->arena_dev;
   a.slot_of = h->d_slot_of;
   a.slot_key = h->d_slot_key;
+  a.cand = h->d_cand;
   a.n_used = h->d_n_used;
   a.step = h->d_step;
   a.z = h->d_z;
@@ -790,7 +795,7 @@ void free_all(moe_handle* h) {
   if (h->routers) cudaFree(h->routers);
   if (h->route) cudaFreeHost(h->route);
   if (h->u) cudaFree(h->u);
-  for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_n_used,
+  for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_cand, (void*)h->d_n_used,
                   (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
                   (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
                   (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y,
@@ -912,6 +917,7 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     const int64_t plan_ints = h->batched ? 2 + 5 * (int64_t)cfg->n_experts + pairs : 3 * (int64_t)k;
     bool ok = cudaMalloc(&h->d_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
               cudaMalloc(&h->d_slot_key, sizeof(unsigned long long) * h->cap) == cudaSuccess &&
+              cudaMalloc(&h->d_cand, sizeof(unsigned long long) * (moe::kMaxRanks + 1)) == cudaSuccess &&
               cudaMalloc(&h->d_n_used, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_step, sizeof(int64_t)) == cudaSuccess &&
               cudaMalloc(&h->d_z, sizeof(float) * 256 * cfg->max_batch) == cudaSuccess &&
@@ -1153,6 +1159,7 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
     // preloaded slots are contiguous [n_used - loaded, n_used)
     MOE_CK(h, cudaMemcpy(h->d_slot_key + kslots.front(), keys.data(), sizeof(unsigned long long) * keys.size(),
                          cudaMemcpyHostToDevice));
+    MOE_CK(h, cudaMemset(h->d_cand, 0, sizeof(unsigned long long) * (moe::kMaxRanks + 1)));  // keys changed
   }
   if (n_loaded) *n_loaded = loaded;
   return MOE_OK;
