@@ -125,6 +125,32 @@ def anon_huge_kb() -> int:
     return 0
 
 
+# ---- multi-rank helpers (one replica per GPU; no data-path collective)
+
+def max_over_ranks(x: float, device) -> float:
+    """The largest value of x over all ranks of the default process group (x itself when there is
+    no group): the whole job takes as long as its slowest replica."""
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, world: int, seconds: float) -> float:
+    """Units all replicas processed per second of the slowest replica (weak scaling)."""
+    return units_per_rank * world / seconds
+
+
+def host_tier_fits(need_bytes_per_replica: float, replicas_per_host: int, available_bytes: int) -> bool:
+    """Whether every replica on this host can page-lock its host tier, with 10% of the available
+    memory left over (0 available = unknown: assume it fits)."""
+    return not available_bytes or need_bytes_per_replica * replicas_per_host <= 0.9 * available_bytes
+
+
 def oracle_cpu_baseline(wl, hidden, budget_s: float = 15.0):
     """Time the fp64 oracle (as it stands) decoding whole tokens of the workload on the host cores.
 
@@ -387,7 +413,7 @@ def main():
     peak_hbm, peak_src = load_peaks()
     need_host = wl.n_gid * synth.expert_bytes(wl.d, wl.d_ff, wl.wdtype) * 1.05 + (2 << 30)
     avail = mem_available_bytes()
-    if avail and need_host * int(os.environ.get("LOCAL_WORLD_SIZE", world)) > 0.9 * avail:
+    if not host_tier_fits(need_host, int(os.environ.get("LOCAL_WORLD_SIZE", world)), avail):
         if rank == 0:
             print(json.dumps({"metric": "MoE decode tok/s at batch 1 under 6 GB expert cap", "value": None,
                               "error": f"host memory: {int(os.environ.get('LOCAL_WORLD_SIZE', world))} replicas need "
@@ -452,12 +478,8 @@ def main():
     clk = clocks.stop()
     # kernel-timing pass over the next steps of the same run: every launch bracketed by CUDA events
     ms_prof, _, prof, _, _ = timed(args.warmup + args.steps, True)
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    tok = args.steps * wl.batch * world
-    value = tok / (ms * 1e-3)
+    ms = max_over_ranks(ms, "cuda")
+    value = whole_job_rate(args.steps * wl.batch, world, ms * 1e-3)
 
     # end to end through the host-buffer entry point (pinned host in, pinned host out)
     e2e_steps = args.e2e_steps or max(8, args.steps // 4)
@@ -471,11 +493,8 @@ def main():
     for i in range(base + 1, base + 1 + e2e_steps):
         m.decode_step_host(hid_host[i % n_tok], out_host, batch=wl.batch)
     e2e_s = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([e2e_s], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e_value = e2e_steps * wl.batch * world / e2e_s
+    e2e_s = max_over_ranks(e2e_s, "cuda")
+    e2e_value = whole_job_rate(e2e_steps * wl.batch, world, e2e_s)
     act_bytes = wl.n_layers * wl.batch * wl.d * (4 if wl.adtype == "fp32" else 2)
 
     # kernel launches of the timed region (phase entries are per-layer timestamps, not launches)

@@ -1,0 +1,73 @@
+"""The multi-rank path of bench.py on CPU (gloo, world size 2): each GPU runs an independent
+replica, the job takes as long as its slowest replica (max over ranks), the job's rate is all
+replicas' units over that time, and the reference arm runs on rank 0 only."""
+import os
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+import bench
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, results):
+    import torch.distributed as dist
+
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        ms_local = [120.0, 95.5][rank]  # rank 0 is the slower replica
+        ms = bench.max_over_ranks(ms_local, "cpu")
+        rate = bench.whole_job_rate(200 * 64, world, ms * 1e-3)
+        dist.barrier()
+        results[rank] = (ms, rate)
+    finally:
+        dist.destroy_process_group()
+
+
+def test_max_over_ranks_and_whole_job_rate_on_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    with ctx.Manager() as mgr:
+        results = mgr.dict()
+        port = _free_port()
+        procs = [ctx.Process(target=_rank_main, args=(r, 2, port, results)) for r in range(2)]
+        for p in procs:
+            p.start()
+        for p in procs:
+            p.join(timeout=120)
+        assert all(p.exitcode == 0 for p in procs)
+        got = dict(results)
+    # both ranks agree on the slowest replica's time and on the job's rate
+    assert got[0] == got[1]
+    ms, rate = got[0]
+    assert ms == 120.0
+    assert rate == pytest.approx(2 * 200 * 64 / 0.120)
+
+
+def test_single_process_needs_no_group():
+    assert bench.max_over_ranks(7.5, "cpu") == 7.5
+    assert bench.whole_job_rate(10, 1, 2.0) == 5.0
+
+
+def test_host_tier_guard():
+    gb = 1e9
+    assert bench.host_tier_fits(60 * gb, 1, int(100 * gb))
+    assert not bench.host_tier_fits(60 * gb, 2, int(100 * gb))  # two replicas of a 58 GB tier
+    assert bench.host_tier_fits(60 * gb, 8, 0)  # available memory unknown
+
+
+def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
+    import argparse
+
+    import synth
+
+    monkeypatch.setenv("RANK", "1")
+    args = argparse.Namespace(warmup=3, steps=4, gpus=2)
+    assert bench.run_reference(args, synth.WORKLOADS["tiny_fp32"]) == 0
+    assert capsys.readouterr().out == ""
