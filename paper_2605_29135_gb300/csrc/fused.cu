@@ -69,7 +69,9 @@ __device__ void find_victim_candidates(const FusedArgs& a) {
   if (threadIdx.x == 0) a.cand[kMaxRanks] = (unsigned long long)a.k;
 }
 
-// Phase S, run by CTA 0 (all its threads).
+// Phase S, run by CTA 0 (all its threads). Every global read the phase needs is issued at its
+// start, side by side: the logits (warp 0), the layer's row of the lookup table, the pool's fill
+// count, the trace position and the victim candidates (warps 1-7).
 __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t step) {
   __shared__ int s_idx[kMaxRanks];
   __shared__ float s_gate[kMaxRanks];
@@ -79,7 +81,10 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   __shared__ int s_evict[kMaxRanks];  // evicted global id per needed id, -1 if none
   __shared__ int s_vslot[kMaxRanks];  // victims in ascending (last use, id): slot and global id
   __shared__ int s_vgid[kMaxRanks];
-  __shared__ int s_nev, s_nev_found;
+  __shared__ int s_nev, s_nev_found, s_nused, s_ncand;
+  __shared__ unsigned long long s_trace_base;
+  __shared__ int s_slot_e[256];       // the layer's row of the lookup table
+  __shared__ int s_cand_gid[kMaxRanks], s_cand_slot[kMaxRanks];
   __shared__ unsigned long long s_ckey[kFWarps][kMaxRanks];  // each warp's smallest candidate keys
   __shared__ int s_cslot[kFWarps][kMaxRanks];
   const int k = a.k, E = a.E;
@@ -105,51 +110,61 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
       s_gate[lane] = my_g;
       s_need[pos] = gid;
     }
-    __syncwarp();
-    if (lane < k) {
-      const int sl = a.slot_of[s_need[lane]];
-      s_slot[lane] = sl;
-      s_miss[lane] = sl < 0;
-      s_evict[lane] = -1;
+  } else {
+    for (int e = threadIdx.x - 32; e < E; e += blockDim.x - 32) s_slot_e[e] = a.slot_of[l * E + e];
+    if (threadIdx.x == 32) {
+      s_nused = *a.n_used;
+      s_trace_base = *(volatile unsigned long long*)a.trace_n;
     }
-    __syncwarp();
-    if (lane == 0) {
-      // misses in ascending id take free slots [n_used, cap) first
-      int n_used = *a.n_used;
-      int nev = 0;
-      for (int t = 0; t < k; t++) {
-        if (s_slot[t] >= 0) continue;
-        if (n_used < a.cap)
-          s_slot[t] = n_used++;
-        else
-          nev++;
+    if (warp == 2 && lane < k) {
+      const int nc = (int)__ldcg(a.cand + kMaxRanks);
+      if (lane == 0) s_ncand = nc;
+      if (lane < nc) {
+        const int g = (int)(uint32_t)(__ldcg(a.cand + lane) & 0xffffffffull);
+        s_cand_gid[lane] = g;
+        s_cand_slot[lane] = a.slot_of[g];
       }
-      *a.n_used = n_used;
-      s_nev = nev;
     }
   }
   __syncthreads();
-  const int nev = s_nev;
-  if (nev > 0 && threadIdx.x == 0) {
+  if (threadIdx.x < k) {
+    const int sl = s_slot_e[s_need[threadIdx.x] - l * E];
+    s_slot[threadIdx.x] = sl;
+    s_miss[threadIdx.x] = sl < 0;
+    s_evict[threadIdx.x] = -1;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    // misses in ascending id take free slots [n_used, cap) first
+    int n_used = s_nused;
+    int nev = 0;
+    for (int t = 0; t < k; t++) {
+      if (s_slot[t] >= 0) continue;
+      if (n_used < a.cap)
+        s_slot[t] = n_used++;
+      else
+        nev++;
+    }
+    if (n_used != s_nused) *a.n_used = n_used;
+    s_nev = nev;
     // Victims: the nev smallest slot keys (last use, id) among slots that hold no expert of this
     // step (every slot is occupied when eviction is needed). They are among the k smallest keys
     // of the pool (at most k - nev of those belong to this step's hits), which phase C of the
-    // previous layer-step left in a.cand. s_nev_found < nev sends phase S to the full scan.
-    const int nc = (int)__ldcg(a.cand + kMaxRanks);
+    // previous layer-step left in a.cand. s_nev_found < nev sends the phase to the full scan.
     int j = 0;
-    for (int c = 0; c < nc && j < nev; c++) {
-      const unsigned long long key = __ldcg(a.cand + c);
-      const int g = (int)(uint32_t)(key & 0xffffffffull);
+    for (int c = 0; c < s_ncand && j < nev; c++) {
+      const int g = s_cand_gid[c];
       bool needed = false;
       for (int t = 0; t < k; t++) needed |= (s_need[t] == g);
       if (needed) continue;
       s_vgid[j] = g;
-      s_vslot[j] = a.slot_of[g];
+      s_vslot[j] = s_cand_slot[c];
       j++;
     }
     s_nev_found = j;
   }
   __syncthreads();
+  const int nev = s_nev;
   if (nev > 0 && s_nev_found < nev) {
     // Full scan: each warp finds the nev smallest of its slots, warp 0 takes the nev smallest of
     // those candidates.
@@ -244,16 +259,16 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     }
     for (int t = 0; t < k; t++)
       if (s_slot[t] >= 0) a.slot_key[s_slot[t]] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)s_need[t];
-    a.stats[STAT_HITS] += hits;
-    a.stats[STAT_MISSES] += misses;
-    a.stats[STAT_EVICTIONS] += evictions;
-    a.stats[STAT_LAYER_STEPS] += 1;
+    atomicAdd(a.stats + STAT_HITS, hits);
+    atomicAdd(a.stats + STAT_MISSES, misses);
+    atomicAdd(a.stats + STAT_EVICTIONS, evictions);
+    atomicAdd(a.stats + STAT_LAYER_STEPS, 1ull);
     a.cand[kMaxRanks] = 0ull;  // the keys changed: phase C finds new candidates if the pool is full
   }
   __syncthreads();
   if (threadIdx.x < k) {
     const int t = threadIdx.x;
-    const unsigned long long base = *(volatile unsigned long long*)a.trace_n;
+    const unsigned long long base = s_trace_base;
     if (base + t < (unsigned long long)a.trace_cap) {
       TraceRec rec;
       rec.step = (int32_t)step;
@@ -276,7 +291,7 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     a.route_gate[l * k + t] = s_gate[t];
   }
   __syncthreads();
-  if (threadIdx.x == 0) *a.trace_n = *(volatile unsigned long long*)a.trace_n + k;
+  if (threadIdx.x == 0) *a.trace_n = s_trace_base + k;
 }
 
 // Copy n bf16 values (scales) from src to dst with 2-byte accesses, one per lane.
@@ -548,8 +563,11 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
         asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
       }
     }
-    if (blockIdx.x == 0 && __ldcg(a.n_used) >= a.cap) find_victim_candidates(a);
-    const int mctas = nm > 0 ? (a.miss_ctas < (int)gridDim.x - 1 ? a.miss_ctas : (int)gridDim.x - 1) : 0;
+    // With a full pool that can evict, CTA 0 finds the next layer-step's victim candidates
+    // instead of computing hit rows.
+    const bool cand_cta0 = a.may_evict && __ldcg(a.n_used) >= a.cap;
+    if (blockIdx.x == 0 && cand_cta0) find_victim_candidates(a);
+    const int mctas = nm > 0 ? (a.miss_ctas < (int)gridDim.x - 2 ? a.miss_ctas : (int)gridDim.x - 2) : 0;
     const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;  // the last CTAs (CTA 0 leads phase S)
     if (miss_cta) {
       const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
@@ -584,9 +602,10 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
         }
         for (; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
       }
-    } else {
-      const int hw = (int)blockIdx.x * kFWarps + (threadIdx.x >> 5);
-      const int HW = ((int)gridDim.x - mctas) * kFWarps;
+    } else if (!(cand_cta0 && blockIdx.x == 0)) {
+      const int c0 = cand_cta0 ? 1 : 0;
+      const int hw = ((int)blockIdx.x - c0) * kFWarps + (threadIdx.x >> 5);
+      const int HW = ((int)gridDim.x - mctas - c0) * kFWarps;
       for (int p = hw; p < nh * a.I; p += HW) {
         const int r = p_hr[p / a.I];
         const int i = p - (p / a.I) * a.I;

@@ -61,6 +61,7 @@ struct FusedArgs {
   // phase C (off the critical path) for the next layer-step's phase S; cand[kMaxRanks] holds how
   // many are valid (0: phase S scans every slot).
   unsigned long long* cand;    // [kMaxRanks + 1]
+  int may_evict;               // cap < experts in the stack (else no step ever evicts)
 };
 
 // Maximum co-resident CTAs for the fused kernel of this shape (0 if it cannot launch).

@@ -689,6 +689,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   a.slot_of = h->d_slot_of;
   a.slot_key = h->d_slot_key;
   a.cand = h->d_cand;
+  a.may_evict = h->cap < h->n_gid;
   a.n_used = h->d_n_used;
   a.step = h->d_step;
   a.z = h->d_z;
