@@ -606,6 +606,20 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
       const int c0 = cand_cta0 ? 1 : 0;
       const int hw = ((int)blockIdx.x - c0) * kFWarps + (threadIdx.x >> 5);
       const int HW = ((int)gridDim.x - mctas - c0) * kFWarps;
+      // When this layer-step also streams misses over the host link, phase C leaves HBM mostly
+      // idle: bring the hit experts' W_d regions into L2 meanwhile, so phase D reads them from L2.
+      // (With every expert a hit the prefetches would compete with the gate/up rows instead.)
+      if (nm > 0) {
+        const int64_t dbytes = a.lay.total - a.lay.d_off;
+        const int64_t nlines = (dbytes + 127) >> 7;
+        const int64_t t0 = (int64_t)hw * 32 + lane;
+        const int64_t T = (int64_t)HW * 32;
+        for (int64_t q = t0; q < (int64_t)nh * nlines; q += T) {
+          const int m = (int)(q / nlines);
+          const uint8_t* pa = a.pool + (int64_t)p_slot[p_hr[m]] * a.slot_stride + a.lay.d_off + ((q - m * nlines) << 7);
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+        }
+      }
       for (int p = hw; p < nh * a.I; p += HW) {
         const int r = p_hr[p / a.I];
         const int i = p - (p / a.I) * a.I;
