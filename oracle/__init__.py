@@ -224,13 +224,13 @@ class Oracle:
         self.token_step = 0
 
     @classmethod
-    def for_workload(cls, wl, cap_slots=None, keep_slot_copies=True, routers=None, experts=None):
+    def for_workload(cls, wl, cap_slots=None, keep_slot_copies=True, routers=None, experts=None, renorm=True):
         import synth
 
         routers = routers if routers is not None else [synth.router_weights(wl, l) for l in range(wl.n_layers)]
         experts = experts if experts is not None else (lambda l, e: synth.expert_weights(wl, l, e))
         return cls(wl.d, wl.n_experts, wl.top_k, wl.d_ff, wl.n_layers, wl.wdtype, wl.adtype,
-                   wl.cap_slots if cap_slots is None else cap_slots, routers, experts,
+                   wl.cap_slots if cap_slots is None else cap_slots, routers, experts, renorm=renorm,
                    keep_slot_copies=keep_slot_copies)
 
     def reset(self):

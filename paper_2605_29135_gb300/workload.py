@@ -24,10 +24,10 @@ def config_for(wl, cap_slots=None, device=0, trace_capacity=1 << 22, renorm=True
 
 
 def create_for_workload(wl, cap_slots=None, device=0, trace_capacity=1 << 22, threads=None,
-                        schedule="device", miss_ctas=0, batched_path="auto") -> MoE:
+                        schedule="device", miss_ctas=0, batched_path="auto", renorm=True) -> MoE:
     import synth
 
-    m = MoE(config_for(wl, cap_slots, device, trace_capacity, schedule=schedule, miss_ctas=miss_ctas,
+    m = MoE(config_for(wl, cap_slots, device, trace_capacity, renorm=renorm, schedule=schedule, miss_ctas=miss_ctas,
                        batched_path=batched_path))
     try:
         for layer in range(wl.n_layers):
