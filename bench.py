@@ -167,7 +167,7 @@ def oracle_cpu_baseline(wl, hidden, budget_s: float = 15.0):
 
     routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
     probe = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers)
-    max_tok = 4
+    max_tok = 12  # ~1 s per token on 16 cores: a sample of ~10 s
     need = set()
     for t in range(max_tok):
         r = probe.decode_step(hidden[t], compute_out=False)
