@@ -79,6 +79,8 @@ def lib():
             L.orc_combine.argtypes = [vp, vp, i32, i32, vp]
             L.orc_lru_step.argtypes = [i64, vp, vp, vp, i64, vp, i32, i32, i32, vp]
             L.orc_lru_step.restype = i32
+            L.orc_rotary_step.argtypes = [i64, vp, vp, vp, vp, vp, i32, i32, i32, vp]
+            L.orc_rotary_step.restype = i32
             _lib = L
     return _lib
 
@@ -190,6 +192,41 @@ class LRUTable:
         return out
 
 
+
+class RotaryTable:
+    """Residency state under the rotary slot-group policy (this build's reading of the paper's
+    rotary residency, Fig. 1/2): a ring of slots with a hand; a miss returns to the slot it was last
+    evicted from when that slot holds no expert of the step (reverse rotation), else takes the next
+    such slot from the hand (forward rotation). See orc_rotary_step."""
+
+    def __init__(self, n_gid: int, cap: int, n_experts: int):
+        self.n_gid, self.cap, self.n_experts = n_gid, cap, n_experts
+        self.slot_of = np.full(n_gid, -1, dtype=np.int32)
+        self.gid_of = np.full(cap, -1, dtype=np.int32)
+        self.prior = np.full(cap, -1, dtype=np.int32)
+        self.hand = np.zeros(1, dtype=np.int64)
+
+    def preload(self):
+        """Warm start: slots 0.. take experts in ascending global id order; the hand stays at slot 0,
+        so forward rotation replaces the preloaded experts first, in id order."""
+        for s in range(min(self.cap, self.n_gid)):
+            if self.gid_of[s] < 0:
+                g = int(np.flatnonzero(self.slot_of < 0)[0])
+                self.gid_of[s] = g
+                self.slot_of[g] = s
+
+    def step(self, clock: int, needed, step: int) -> np.ndarray:
+        needed = np.ascontiguousarray(sorted(set(int(g) for g in needed)), dtype=np.int32)
+        out = np.zeros(len(needed), dtype=REC_DTYPE)
+        n = lib().orc_rotary_step(self.cap, _p(self.slot_of), _p(self.gid_of), _p(self.prior), _p(self.hand),
+                                  _p(needed), len(needed), self.n_experts, step, _p(out))
+        if n < 0:
+            raise RuntimeError("rotary step: capacity below the number of distinct experts in one layer-step")
+        return out
+
+
+TABLES = {"lru": LRUTable, "rotary": RotaryTable}
+
 # ----------------------------------------------------------------------------------------------
 # the full decode step
 
@@ -212,29 +249,31 @@ class Oracle:
     """
 
     def __init__(self, d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots, routers, experts,
-                 renorm=True, keep_slot_copies=True):
+                 renorm=True, keep_slot_copies=True, policy="lru"):
         self.d, self.E, self.k, self.I, self.L = d, n_experts, top_k, d_ff, n_layers
         self.wdtype, self.adtype, self.renorm = wdtype, adtype, renorm
         self.router_dtype = "fp32" if wdtype == "fp32" else "bf16"
         self.routers = [widen(self.router_dtype, routers[l], n_experts, d) for l in range(n_layers)]
         self.experts = experts
         self.keep = keep_slot_copies
-        self.table = LRUTable(n_layers * n_experts, cap_slots, n_experts)
+        self.policy = policy
+        self.table = TABLES[policy](n_layers * n_experts, cap_slots, n_experts)
         self.slots: dict[int, object] = {}
         self.token_step = 0
 
     @classmethod
-    def for_workload(cls, wl, cap_slots=None, keep_slot_copies=True, routers=None, experts=None, renorm=True):
+    def for_workload(cls, wl, cap_slots=None, keep_slot_copies=True, routers=None, experts=None, renorm=True,
+                     policy="lru"):
         import synth
 
         routers = routers if routers is not None else [synth.router_weights(wl, l) for l in range(wl.n_layers)]
         experts = experts if experts is not None else (lambda l, e: synth.expert_weights(wl, l, e))
         return cls(wl.d, wl.n_experts, wl.top_k, wl.d_ff, wl.n_layers, wl.wdtype, wl.adtype,
                    wl.cap_slots if cap_slots is None else cap_slots, routers, experts, renorm=renorm,
-                   keep_slot_copies=keep_slot_copies)
+                   keep_slot_copies=keep_slot_copies, policy=policy)
 
     def reset(self):
-        self.table = LRUTable(self.table.n_gid, self.table.cap, self.E)
+        self.table = TABLES[self.policy](self.table.n_gid, self.table.cap, self.E)
         self.slots = {}
         self.token_step = 0
 

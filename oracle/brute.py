@@ -75,3 +75,40 @@ class RecencyListLRU:
             recs.append((g, 1, s, victim))
         self.order = [v for v in self.order if v not in pinned] + needed
         return recs
+
+
+class RotaryRing:
+    """Independent pure-Python model of the rotary slot group (ring of slots, a hand, and each
+    slot's previous occupant), for checking orc_rotary_step on random request sequences."""
+
+    def __init__(self, cap):
+        self.cap = cap
+        self.ring = [None] * cap  # occupant of each slot
+        self.prev = [None] * cap  # occupant evicted most recently from each slot
+        self.hand = 0
+
+    def step(self, needed):
+        need = sorted(set(needed))
+        pinned = set(need)
+        recs = []
+        for g in need:
+            if g in self.ring:
+                recs.append((g, 0, self.ring.index(g), -1))
+                continue
+            free = lambda s: self.ring[s] is None or self.ring[s] not in pinned
+            back = [s for s in range(self.cap) if self.prev[s] == g and free(s)]
+            if back:
+                s = back[0]
+            else:
+                order = [(self.hand + j) % self.cap for j in range(self.cap)]
+                cand = [s for s in order if free(s)]
+                if not cand:
+                    raise RuntimeError("no slot")
+                s = cand[0]
+                self.hand = (s + 1) % self.cap
+            v = self.ring[s]
+            self.prev = [None if p == g else p for p in self.prev]
+            self.prev[s] = v
+            self.ring[s] = g
+            recs.append((g, 1, s, -1 if v is None else v))
+        return recs

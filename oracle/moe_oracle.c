@@ -249,3 +249,69 @@ int32_t orc_lru_step(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t* la
   for (int32_t i = 0; i < n; i++) last_use[needed[i]] = clock;
   return n;
 }
+
+/*
+ * One layer-step of the rotary slot group: this build's reading of the paper's rotary residency
+ * (Fig. 1 "Rotary Slot Group", Fig. 2 "cyclical forward and reverse rotation"; the paper gives no
+ * algorithm). The cap slots form a ring with a hand; each slot remembers its previous occupant.
+ *
+ * State: slot_of[gid], gid_of[slot] (-1 empty), prior[slot] (the gid last evicted from the slot,
+ * -1 none), *hand (a slot index). needed: distinct gids of the layer-step, ascending.
+ *
+ * For each needed gid g in ascending order: if resident, a hit (nothing moves). Otherwise a miss:
+ *   reverse rotation: if some slot s has prior[s] == g and s holds no gid of `needed`, g returns
+ *     to s;
+ *   forward rotation: otherwise g takes the first slot s at or after *hand (cyclically) that holds
+ *     no gid of `needed`, and *hand moves to s + 1 (mod cap).
+ * The occupant v of s (if any) is evicted: slot_of[v] = -1. Then prior[s] = v (possibly -1), every
+ * other prior entry equal to g is cleared, and g is placed in s. One record per needed gid.
+ *
+ * Returns the number of records, or -1 if no slot is available (cap < |needed|).
+ */
+int32_t orc_rotary_step(int64_t cap, int32_t* slot_of, int32_t* gid_of, int32_t* prior, int64_t* hand,
+                        const int32_t* needed, int32_t n, int32_t n_experts, int32_t step, orc_rec* out) {
+  for (int32_t i = 0; i < n; i++) {
+    int32_t g = needed[i];
+    orc_rec rec;
+    rec.step = step;
+    rec.layer = g / n_experts;
+    rec.expert = g % n_experts;
+    if (slot_of[g] >= 0) {
+      rec.kind = 0;
+      rec.slot = slot_of[g];
+      rec.evicted = -1;
+      out[i] = rec;
+      continue;
+    }
+    int64_t slot = -1;
+    for (int64_t s = 0; s < cap; s++) {
+      if (prior[s] == g && (gid_of[s] < 0 || !in_sorted(needed, n, gid_of[s]))) {
+        slot = s;
+        break;
+      }
+    }
+    if (slot < 0) {
+      for (int64_t j = 0; j < cap; j++) {
+        int64_t s = (*hand + j) % cap;
+        if (gid_of[s] < 0 || !in_sorted(needed, n, gid_of[s])) {
+          slot = s;
+          break;
+        }
+      }
+      if (slot < 0) return -1;
+      *hand = (slot + 1) % cap;
+    }
+    int32_t v = gid_of[slot];
+    if (v >= 0) slot_of[v] = -1;
+    for (int64_t s = 0; s < cap; s++)
+      if (prior[s] == g) prior[s] = -1;
+    prior[slot] = v;
+    gid_of[slot] = g;
+    slot_of[g] = (int32_t)slot;
+    rec.kind = 1;
+    rec.slot = (int32_t)slot;
+    rec.evicted = v;
+    out[i] = rec;
+  }
+  return n;
+}
