@@ -89,6 +89,17 @@ enum { MOE_SCHEDULE_DEVICE = 0, MOE_SCHEDULE_HOST_COPY_ENGINE = 1 };
  *     experts stream from the host tier straight into their slot and the compute. */
 enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
 
+/* Replacement policy of the slot group.
+ *   MOE_POLICY_LRU (default): misses take the lowest free slot, else evict the resident expert not
+ *     needed this layer-step with the smallest (last use, global id). Both schedules.
+ *   MOE_POLICY_ROTARY: this library's reading of the paper's rotary slot group (Fig. 1, Fig. 2;
+ *     the paper gives no algorithm). The slots form a ring with a hand and each slot remembers its
+ *     previous occupant. A miss returns to the slot it was last evicted from when that slot holds no
+ *     expert of the layer-step (reverse rotation), else takes the first such slot at or after the
+ *     hand, which then moves past it (forward rotation). Hits change nothing. Misses in ascending
+ *     global id. MOE_SCHEDULE_HOST_COPY_ENGINE only (the host runs the controller). */
+enum { MOE_POLICY_LRU = 0, MOE_POLICY_ROTARY = 1 };
+
 typedef struct {
   int32_t d;          /* hidden size */
   int32_t n_experts;  /* experts per layer, E (<= 256) */
@@ -112,6 +123,7 @@ typedef struct {
                              host link while the others compute the hits (0: library default). Batched
                              steps hand work items to all CTAs, missed experts first, and ignore it */
   int32_t batched_path;   /* MOE_BATCHED_AUTO (default) or MOE_BATCHED_CUDA_CORES */
+  int32_t policy;         /* MOE_POLICY_LRU (default) or MOE_POLICY_ROTARY */
 } moe_config;
 
 /* One residency record: a requested expert's outcome in one layer-step. */

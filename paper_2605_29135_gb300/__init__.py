@@ -15,7 +15,7 @@ import ctypes
 import numpy as np
 
 from . import _lib
-from ._lib import BATCHED_PATH, DTYPE, SCHEDULE, STATUS, KernelTime, MoeConfig, Stats, TraceRec
+from ._lib import BATCHED_PATH, DTYPE, POLICY, SCHEDULE, STATUS, KernelTime, MoeConfig, Stats, TraceRec
 
 TRACE_DTYPE = np.dtype([("step", np.int32), ("layer", np.int32), ("expert", np.int32), ("kind", np.int32),
                         ("slot", np.int32), ("evicted", np.int32)])
@@ -29,12 +29,12 @@ class MoEError(RuntimeError):
 
 def make_config(d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots=0, cap_bytes=0, renorm=True,
                 device=0, max_batch=1, trace_capacity=1 << 22, device_pool=None, schedule="device",
-                miss_ctas=0, batched_path="auto") -> MoeConfig:
+                miss_ctas=0, batched_path="auto", policy="lru") -> MoeConfig:
     return MoeConfig(d=d, n_experts=n_experts, top_k=top_k, d_ff=d_ff, n_layers=n_layers, max_batch=max_batch,
                      wdtype=DTYPE[wdtype], adtype=DTYPE[adtype], cap_slots=cap_slots, cap_bytes=cap_bytes,
                      renorm=1 if renorm else 0, device=device, device_pool=device_pool,
                      trace_capacity=trace_capacity, schedule=SCHEDULE[schedule], miss_ctas=miss_ctas,
-                     batched_path=BATCHED_PATH[batched_path])
+                     batched_path=BATCHED_PATH[batched_path], policy=POLICY[policy])
 
 
 def expert_bytes(cfg: MoeConfig) -> int:

@@ -18,6 +18,7 @@ STATUS = {0: "MOE_OK", -1: "MOE_ERR_INVALID", -2: "MOE_ERR_OOM", -3: "MOE_ERR_CU
 DTYPE = {"fp32": 0, "bf16": 1, "int4": 2}
 SCHEDULE = {"device": 0, "host_copy_engine": 1}
 BATCHED_PATH = {"auto": 0, "cuda_cores": 1}
+POLICY = {"lru": 0, "rotary": 1}
 
 # Every function the header declares (checked by the CPU test suite).
 EXPORTS = ["moe_expert_bytes", "moe_pool_bytes", "moe_create", "moe_set_router", "moe_register_host_experts",
@@ -32,7 +33,7 @@ class MoeConfig(ctypes.Structure):
                 ("wdtype", ctypes.c_int32), ("adtype", ctypes.c_int32), ("cap_slots", ctypes.c_int64),
                 ("cap_bytes", ctypes.c_int64), ("renorm", ctypes.c_int32), ("device", ctypes.c_int32),
                 ("device_pool", ctypes.c_void_p), ("trace_capacity", ctypes.c_int64), ("schedule", ctypes.c_int32),
-                ("miss_ctas", ctypes.c_int32), ("batched_path", ctypes.c_int32)]
+                ("miss_ctas", ctypes.c_int32), ("batched_path", ctypes.c_int32), ("policy", ctypes.c_int32)]
 
 
 class TraceRec(ctypes.Structure):

@@ -85,6 +85,10 @@ struct moe_handle {
   std::vector<uint8_t> in_step;
   std::set<std::pair<int64_t, int32_t>> lru;  // resident (last_use, gid)
   std::set<int32_t> free_slots;
+  // rotary slot-group policy: each slot's previous occupant, its inverse, and the hand
+  std::vector<int32_t> prior;          // [cap]: gid last evicted from the slot, -1 none
+  std::vector<int32_t> prior_slot_of;  // [n_gid]: the slot whose previous occupant is gid, -1 none
+  int64_t hand = 0;
   int64_t token_step = 0;
   int64_t route_seq = 0;
   std::vector<moe_trace_rec> trace;
@@ -195,6 +199,9 @@ std::string check_config(const moe_config* c) {
   if (c->schedule != MOE_SCHEDULE_DEVICE && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "unknown schedule";
   if (c->miss_ctas < 0) return "miss_ctas must be >= 0";
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
+  if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY) return "unknown policy";
+  if (c->policy == MOE_POLICY_ROTARY && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE)
+    return "the rotary policy runs in the host copy-engine schedule";
   return "";
 }
 
@@ -231,6 +238,9 @@ void reset_state(moe_handle* h) {
   h->lru.clear();
   h->free_slots.clear();
   for (int64_t s = 0; s < h->cap; s++) h->free_slots.insert((int32_t)s);
+  std::fill(h->prior.begin(), h->prior.end(), -1);
+  std::fill(h->prior_slot_of.begin(), h->prior_slot_of.end(), -1);
+  h->hand = 0;
   h->token_step = 0;
   h->trace.clear();
   h->trace_dropped = 0;
@@ -349,6 +359,48 @@ moe_status residency_step(moe_handle* h, int32_t layer, std::vector<Need>& needs
       rec.kind = 0;
       rec.slot = n.slot;
       h->stats.hits++;
+    } else if (h->cfg.policy == MOE_POLICY_ROTARY) {
+      // Rotary slot group (reverse rotation back to the slot the expert was last evicted from
+      // when that slot holds no expert of this step, else forward rotation from the hand).
+      auto open = [&](int32_t s) { return h->gid_of[s] < 0 || !h->in_step[h->gid_of[s]]; };
+      const int32_t ps = h->prior_slot_of[n.gid];
+      int32_t slot = ps >= 0 && open(ps) ? ps : -1;
+      if (slot < 0) {
+        for (int64_t j = 0; j < h->cap; j++) {
+          const int32_t sj = (int32_t)((h->hand + j) % h->cap);
+          if (open(sj)) {
+            slot = sj;
+            break;
+          }
+        }
+        if (slot < 0) {
+          st = fail(h, MOE_ERR_CAPACITY, "no available slot (cap below the step's working set)");
+          break;
+        }
+        h->hand = (slot + 1) % h->cap;
+      }
+      const int32_t victim = h->gid_of[slot];
+      if (victim >= 0) {
+        h->slot_of[victim] = -1;
+        h->stats.evictions++;
+      } else {
+        h->free_slots.erase(slot);
+      }
+      if (ps >= 0) h->prior[ps] = -1;  // n.gid is no longer anyone's previous occupant
+      const int32_t u = h->prior[slot];
+      if (u >= 0) h->prior_slot_of[u] = -1;
+      h->prior[slot] = victim;
+      if (victim >= 0) h->prior_slot_of[victim] = slot;
+      h->prior_slot_of[n.gid] = -1;
+      h->gid_of[slot] = n.gid;
+      h->slot_of[n.gid] = slot;
+      n.slot = slot;
+      n.miss = true;
+      rec.kind = 1;
+      rec.slot = slot;
+      rec.evicted = victim;
+      h->stats.misses++;
+      h->stats.miss_bytes += h->lay.total;
     } else {
       int32_t slot = -1, victim = -1;
       if (!h->free_slots.empty()) {
@@ -389,7 +441,7 @@ moe_status residency_step(moe_handle* h, int32_t layer, std::vector<Need>& needs
   }
   for (auto& n : needs) {
     h->in_step[n.gid] = 0;
-    if (st != MOE_OK) continue;
+    if (st != MOE_OK || h->cfg.policy != MOE_POLICY_LRU) continue;
     if (h->last_use[n.gid] >= 0 && !n.miss) h->lru.erase({h->last_use[n.gid], n.gid});
     h->last_use[n.gid] = clock;
     h->lru.insert({clock, n.gid});
@@ -943,6 +995,8 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   h->gid_of.assign(h->cap, -1);
   h->last_use.assign(h->n_gid, -1);
   h->in_step.assign(h->n_gid, 0);
+  h->prior.assign(h->cap, -1);
+  h->prior_slot_of.assign(h->n_gid, -1);
   if (cfg->trace_capacity > 0) h->trace.reserve((size_t)std::min<int64_t>(cfg->trace_capacity, 1 << 22));
   reset_state(h);
   *out = h;

@@ -37,9 +37,9 @@ def run_gpu(m, hidden: np.ndarray, dtype_out: str):
     return o, idx, gate
 
 
-def oracle_trace(wl, hidden: np.ndarray, cap: int, forced_idx=None, routers=None):
+def oracle_trace(wl, hidden: np.ndarray, cap: int, forced_idx=None, routers=None, policy="lru"):
     """Routing + residency trace of the oracle for all steps (no expert FFN)."""
-    orc = oracle.Oracle.for_workload(wl, cap_slots=cap, keep_slot_copies=False, routers=routers)
+    orc = oracle.Oracle.for_workload(wl, cap_slots=cap, keep_slot_copies=False, routers=routers, policy=policy)
     idx, z, recs = [], [], []
     for t in range(hidden.shape[0]):
         r = orc.decode_step(hidden[t], compute_out=False, forced_idx=None if forced_idx is None else forced_idx[t])

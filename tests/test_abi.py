@@ -41,7 +41,7 @@ def test_config_struct_layout_matches_header(lib):
     from paper_2605_29135_gb300._lib import MoeConfig, TraceRec
 
     # int32 x6, int32 x2, int64 x2, int32 x2, pointer, int64, int32 x2
-    assert ctypes.sizeof(MoeConfig) == 6 * 4 + 2 * 4 + 2 * 8 + 2 * 4 + 8 + 8 + 8 + 8  # batched_path + padding
+    assert ctypes.sizeof(MoeConfig) == 6 * 4 + 2 * 4 + 2 * 8 + 2 * 4 + 8 + 8 + 8 + 8  # batched_path, policy
     assert ctypes.sizeof(TraceRec) == 24
 
 
@@ -74,3 +74,15 @@ def test_null_handle_calls_fail_cleanly(lib):
     assert lib.moe_decode_step(None, None, None, 1, None) == -1
     assert lib.moe_reset_residency(None) == -1
     lib.moe_destroy(None)
+
+
+def test_create_rejects_rotary_policy_outside_the_host_schedule():
+    # the configuration is checked before any device is touched
+    import paper_2605_29135_gb300 as P
+    from paper_2605_29135_gb300.buildsys import build
+
+    build()
+    cfg = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4, schedule="device", policy="rotary")
+    with pytest.raises(P.MoEError) as ei:
+        P.MoE(cfg)
+    assert ei.value.status == -1 and "rotary" in str(ei.value)
