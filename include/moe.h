@@ -97,7 +97,7 @@ enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
  *     previous occupant. A miss returns to the slot it was last evicted from when that slot holds no
  *     expert of the layer-step (reverse rotation), else takes the first such slot at or after the
  *     hand, which then moves past it (forward rotation). Hits change nothing. Misses in ascending
- *     global id. MOE_SCHEDULE_HOST_COPY_ENGINE only (the host runs the controller). */
+ *     global id. Both schedules, max_batch 1. */
 enum { MOE_POLICY_LRU = 0, MOE_POLICY_ROTARY = 1 };
 
 typedef struct {

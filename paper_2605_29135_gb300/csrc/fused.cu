@@ -69,6 +69,112 @@ __device__ void find_victim_candidates(const FusedArgs& a) {
   if (threadIdx.x == 0) a.cand[kMaxRanks] = (unsigned long long)a.k;
 }
 
+// Rotary slot-group step for the misses of one layer-step (thread 0 of CTA 0; at most k misses,
+// in ascending id). A miss returns to the slot it was last evicted from when that slot holds no
+// expert of the step (reverse rotation), else takes the first such slot at or after the hand, which
+// moves past it (forward rotation). Uses what phase S read up front: the layer's previous-slot
+// entries with those slots' occupants, and the min(cap, 2k + 1) slots from the hand (a step skips
+// at most k pinned slots and takes at most k), updated here as the step places experts.
+__device__ void rotary_place(const FusedArgs& a, int l, int clock, int k, int E, const int* need, const int* miss,
+                             int* slot_out, int* evict_out, const int* ps_e, const int* ps_gid, int* win_gid,
+                             int* win_prior, int hand0, int nused0) {
+  const int nw = 2 * k + 1 < a.cap ? 2 * k + 1 : (int)a.cap;
+  int placed_slot[kMaxRanks], placed_gid[kMaxRanks];
+  int np = 0;
+  auto in_need = [&](int g) {
+    bool f = false;
+    for (int t = 0; t < k; t++) f |= need[t] == g;
+    return f;
+  };
+  auto win_index = [&](int sl) {  // position of slot sl in the window, -1 outside
+    const int j = (int)(((int64_t)sl - hand0 + a.cap) % a.cap);
+    return j < nw ? j : -1;
+  };
+  int hand = hand0, nused = nused0;
+  unsigned long long misses = 0, evictions = 0;
+  for (int t = 0; t < k; t++) {
+    if (!miss[t]) continue;
+    misses++;
+    const int g = need[t];
+    const int e = g - l * E;
+    // current occupant of a slot: this step's placements first, then what was read up front
+    auto occupant = [&](int sl, int fallback) {
+      int o = fallback;
+      for (int q = 0; q < np; q++)
+        if (placed_slot[q] == sl) o = placed_gid[q];
+      return o;
+    };
+    int slot = -1, occ = -1;
+    // g's return slot, while that slot's previous occupant is still g (an earlier miss of this
+    // step may have taken the slot; slots outside the window change only by a return of g itself)
+    int ps = ps_e[e];
+    if (ps >= 0) {
+      const int wj = win_index(ps);
+      if (wj >= 0 && win_prior[wj] != g) ps = -1;
+    }
+    if (ps >= 0) {
+      const int wj = win_index(ps);
+      const int o = occupant(ps, wj >= 0 ? win_gid[wj] : ps_gid[e]);
+      if (o < 0 || !in_need(o)) {
+        slot = ps;
+        occ = o;
+      }
+    }
+    if (slot < 0) {
+      for (int j = 0; j < nw; j++) {
+        const int sl = (int)((hand + (int64_t)j) % a.cap);
+        const int wj = win_index(sl);
+        if (wj < 0) break;  // cannot happen (see above); reported as no available slot
+        const int o = occupant(sl, win_gid[wj]);
+        if (o < 0 || !in_need(o)) {
+          slot = sl;
+          occ = o;
+          break;
+        }
+      }
+      if (slot < 0) {
+        atomicOr(a.err, FERR_NO_VICTIM);
+        slot_out[t] = -1;
+        continue;
+      }
+      hand = (int)((slot + 1) % a.cap);
+    }
+    // evict the occupant; bookkeeping of previous occupants
+    if (occ >= 0) {
+      a.slot_of[occ] = -1;
+      evictions++;
+    } else {
+      nused++;
+    }
+    if (ps >= 0) {
+      a.prior[ps] = -1;
+      const int wj = win_index(ps);
+      if (wj >= 0) win_prior[wj] = -1;
+    }
+    const int wj = win_index(slot);
+    const int u = slot == ps ? -1 : (wj >= 0 ? win_prior[wj] : -1);
+    if (u >= 0) a.prior_slot_of[u] = -1;
+    a.prior[slot] = occ;
+    if (wj >= 0) win_prior[wj] = occ;
+    if (occ >= 0) a.prior_slot_of[occ] = slot;
+    a.prior_slot_of[g] = -1;
+    a.slot_of[g] = slot;
+    placed_slot[np] = slot;
+    placed_gid[np] = g;
+    np++;
+    slot_out[t] = slot;
+    evict_out[t] = occ;
+  }
+  for (int t = 0; t < k; t++)
+    if (slot_out[t] >= 0) a.slot_key[slot_out[t]] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)need[t];
+  if (hand != hand0) *a.hand = hand;
+  if (nused != nused0) *a.n_used = nused;
+  atomicAdd(a.stats + STAT_HITS, (unsigned long long)k - misses);
+  atomicAdd(a.stats + STAT_MISSES, misses);
+  atomicAdd(a.stats + STAT_EVICTIONS, evictions);
+  atomicAdd(a.stats + STAT_LAYER_STEPS, 1ull);
+}
+
 // Phase S, run by CTA 0 (all its threads). Every global read the phase needs is issued at its
 // start, side by side: the logits (warp 0), the layer's row of the lookup table, the pool's fill
 // count, the trace position and the victim candidates (warps 1-7).
@@ -85,6 +191,12 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   __shared__ unsigned long long s_trace_base;
   __shared__ int s_slot_e[256];       // the layer's row of the lookup table
   __shared__ int s_cand_gid[kMaxRanks], s_cand_slot[kMaxRanks];
+  // rotary: the layer's previous-slot entries and those slots' occupants, the window of slots from
+  // the hand (occupant, previous occupant)
+  constexpr int kWin = 2 * kMaxRanks + 1;
+  __shared__ int s_ps_e[256], s_ps_gid[256];
+  __shared__ int s_win_gid[kWin], s_win_prior[kWin];
+  __shared__ int s_hand;
   __shared__ unsigned long long s_ckey[kFWarps][kMaxRanks];  // each warp's smallest candidate keys
   __shared__ int s_cslot[kFWarps][kMaxRanks];
   const int k = a.k, E = a.E;
@@ -116,6 +228,28 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
       s_nused = *a.n_used;
       s_trace_base = *(volatile unsigned long long*)a.trace_n;
     }
+    if (a.policy == 1) {
+      // occupant of slot s: the low 32 bits of its key, or -1 when empty (key all ones)
+      auto occupant = [&](int64_t sl) {
+        const unsigned long long key = __ldcg(a.slot_key + sl);
+        return key == ~0ull ? -1 : (int)(uint32_t)(key & 0xffffffffull);
+      };
+      for (int e = threadIdx.x - 32; e < E; e += blockDim.x - 32) {
+        const int ps = a.prior_slot_of[l * E + e];
+        s_ps_e[e] = ps;
+        s_ps_gid[e] = ps >= 0 ? occupant(ps) : -1;
+      }
+      if (warp == 3) {
+        const int h0 = *a.hand;
+        if (lane == 0) s_hand = h0;
+        const int nw = 2 * k + 1 < a.cap ? 2 * k + 1 : (int)a.cap;
+        for (int j = lane; j < nw; j += 32) {
+          const int64_t sl = (h0 + j) % a.cap;
+          s_win_gid[j] = occupant(sl);
+          s_win_prior[j] = a.prior[sl];
+        }
+      }
+    }
     if (warp == 2 && lane < k) {
       const int nc = (int)__ldcg(a.cand + kMaxRanks);
       if (lane == 0) s_ncand = nc;
@@ -134,7 +268,12 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     s_evict[threadIdx.x] = -1;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (a.policy == 1) {
+    if (threadIdx.x == 0) rotary_place(a, l, clock, k, E, s_need, s_miss, s_slot, s_evict, s_ps_e, s_ps_gid, s_win_gid,
+                                       s_win_prior, s_hand, s_nused);
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && a.policy == 0) {
     // misses in ascending id take free slots [n_used, cap) first
     int n_used = s_nused;
     int nev = 0;
@@ -164,8 +303,8 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     s_nev_found = j;
   }
   __syncthreads();
-  const int nev = s_nev;
-  if (nev > 0 && s_nev_found < nev) {
+  const int nev = a.policy == 0 ? s_nev : 0;
+  if (nev > 0 && s_nev_found < nev) {  // (LRU only: nev is 0 under the rotary policy)
     // Full scan: each warp finds the nev smallest of its slots, warp 0 takes the nev smallest of
     // those candidates.
     for (int j = 0; j < nev; j++) {
@@ -234,7 +373,7 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     }
     __syncthreads();
   }
-  if (threadIdx.x == 0) {
+  if (threadIdx.x == 0 && a.policy == 0) {
     int j = 0;
     unsigned long long hits = 0, misses = 0, evictions = 0;
     for (int t = 0; t < k; t++) {

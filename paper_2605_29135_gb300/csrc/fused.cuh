@@ -61,7 +61,12 @@ struct FusedArgs {
   // phase C (off the critical path) for the next layer-step's phase S; cand[kMaxRanks] holds how
   // many are valid (0: phase S scans every slot).
   unsigned long long* cand;    // [kMaxRanks + 1]
-  int may_evict;               // cap < experts in the stack (else no step ever evicts)
+  int may_evict;               // LRU with cap < experts in the stack (else no victim search is needed)
+  // Rotary slot-group policy (policy == 1): each slot's previous occupant, its inverse, the hand.
+  int policy;                  // 0 LRU, 1 rotary
+  int32_t* prior;              // [cap]: global id last evicted from the slot, -1 none
+  int32_t* prior_slot_of;      // [L*E]: the slot whose previous occupant is the id, -1 none
+  int32_t* hand;               // [1]
 };
 
 // Maximum co-resident CTAs for the fused kernel of this shape (0 if it cannot launch).

@@ -120,6 +120,9 @@ struct moe_handle {
   int32_t* d_slot_of = nullptr;
   unsigned long long* d_slot_key = nullptr;
   unsigned long long* d_cand = nullptr;  // batch-1 kernel: victim candidates [kMaxRanks + 1]
+  int32_t* d_prior = nullptr;            // rotary policy: previous occupant per slot [cap]
+  int32_t* d_prior_slot_of = nullptr;    // rotary policy: its inverse [n_gid]
+  int32_t* d_hand = nullptr;             // rotary policy: the hand [1]
   int32_t* d_n_used = nullptr;
   int64_t* d_step = nullptr;
   float* d_z = nullptr;
@@ -200,8 +203,7 @@ std::string check_config(const moe_config* c) {
   if (c->miss_ctas < 0) return "miss_ctas must be >= 0";
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
   if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY) return "unknown policy";
-  if (c->policy == MOE_POLICY_ROTARY && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE)
-    return "the rotary policy runs in the host copy-engine schedule";
+  if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
   return "";
 }
 
@@ -216,6 +218,9 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_slot_of, 0xff, sizeof(int32_t) * h->n_gid);
   cudaMemset(h->d_slot_key, 0xff, sizeof(unsigned long long) * h->cap);
   cudaMemset(h->d_cand, 0, sizeof(unsigned long long) * (moe::kMaxRanks + 1));
+  cudaMemset(h->d_prior, 0xff, sizeof(int32_t) * h->cap);
+  cudaMemset(h->d_prior_slot_of, 0xff, sizeof(int32_t) * h->n_gid);
+  cudaMemset(h->d_hand, 0, sizeof(int32_t));
   cudaMemset(h->d_n_used, 0, sizeof(int32_t));
   cudaMemset(h->d_step, 0, sizeof(int64_t));
   cudaMemset(h->d_trace_n, 0, sizeof(unsigned long long));
@@ -741,7 +746,11 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   a.slot_of = h->d_slot_of;
   a.slot_key = h->d_slot_key;
   a.cand = h->d_cand;
-  a.may_evict = h->cap < h->n_gid;
+  a.policy = c.policy;
+  a.may_evict = h->cap < h->n_gid && c.policy == MOE_POLICY_LRU;
+  a.prior = h->d_prior;
+  a.prior_slot_of = h->d_prior_slot_of;
+  a.hand = h->d_hand;
   a.n_used = h->d_n_used;
   a.step = h->d_step;
   a.z = h->d_z;
@@ -848,7 +857,8 @@ void free_all(moe_handle* h) {
   if (h->routers) cudaFree(h->routers);
   if (h->route) cudaFreeHost(h->route);
   if (h->u) cudaFree(h->u);
-  for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_cand, (void*)h->d_n_used,
+  for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_cand, (void*)h->d_prior,
+                  (void*)h->d_prior_slot_of, (void*)h->d_hand, (void*)h->d_n_used,
                   (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
                   (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
                   (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y,
@@ -971,6 +981,9 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     bool ok = cudaMalloc(&h->d_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
               cudaMalloc(&h->d_slot_key, sizeof(unsigned long long) * h->cap) == cudaSuccess &&
               cudaMalloc(&h->d_cand, sizeof(unsigned long long) * (moe::kMaxRanks + 1)) == cudaSuccess &&
+              cudaMalloc(&h->d_prior, sizeof(int32_t) * h->cap) == cudaSuccess &&
+              cudaMalloc(&h->d_prior_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
+              cudaMalloc(&h->d_hand, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_n_used, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_step, sizeof(int64_t)) == cudaSuccess &&
               cudaMalloc(&h->d_z, sizeof(float) * 256 * cfg->max_batch) == cudaSuccess &&

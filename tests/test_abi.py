@@ -76,13 +76,13 @@ def test_null_handle_calls_fail_cleanly(lib):
     lib.moe_destroy(None)
 
 
-def test_create_rejects_rotary_policy_outside_the_host_schedule():
+def test_create_rejects_rotary_policy_for_batches():
     # the configuration is checked before any device is touched
     import paper_2605_29135_gb300 as P
     from paper_2605_29135_gb300.buildsys import build
 
     build()
-    cfg = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4, schedule="device", policy="rotary")
+    cfg = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4, max_batch=4, policy="rotary")
     with pytest.raises(P.MoEError) as ei:
         P.MoE(cfg)
     assert ei.value.status == -1 and "rotary" in str(ei.value)
