@@ -194,7 +194,7 @@ class LRUTable:
 
 
 class RotaryTable:
-    """Residency state under the rotary slot-group policy (this build's reading of the paper's
+    """Residency state under the rotary slot-group policy (one reading of the paper's
     rotary residency, Fig. 1/2): a ring of slots with a hand; a miss returns to the slot it was last
     evicted from when that slot holds no expert of the step (reverse rotation), else takes the next
     such slot from the hand (forward rotation). See orc_rotary_step."""

@@ -251,7 +251,7 @@ int32_t orc_lru_step(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t* la
 }
 
 /*
- * One layer-step of the rotary slot group: this build's reading of the paper's rotary residency
+ * One layer-step of the rotary slot group: one reading of the paper's rotary residency
  * (Fig. 1 "Rotary Slot Group", Fig. 2 "cyclical forward and reverse rotation"; the paper gives no
  * algorithm). The cap slots form a ring with a hand; each slot remembers its previous occupant.
  *

@@ -1,4 +1,4 @@
-"""Pins of the oracle's rotary slot-group step (this build's reading of the paper's rotary
+"""Pins of the oracle's rotary slot-group step (one reading of the paper's rotary
 residency, Fig. 1 "Rotary Slot Group" and Fig. 2 "cyclical forward and reverse rotation").
 
 Checked against: a hand-simulated 4-slot trace (tests/golden/rotary_hand_trace_4slot.txt), an
