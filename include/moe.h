@@ -226,9 +226,10 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded);
 /* Profiling: with on = 1, every kernel launch and miss copy of later steps is bracketed by
  * CUDA events on its stream. moe_profile_read waits for the recorded work, then reports one
  * entry per kernel class (router, gateup, down_combine, miss_copy, fused_step) and, for the
- * device schedule, per phase of the fused kernel (fused_phase_router, _select, _gateup, _down,
- * and for batches _topk, _combine: per layer-step durations from the kernel's global timer),
- * accumulated since the last read, and clears the accumulators. */
+ * device schedule, per phase of the fused kernel (fused_phase_router, _select, _gateup, _down;
+ * for batches also _topk and _combine, and _gather in the tensor-core variant: per layer-step
+ * durations from the kernel's global timer), accumulated since the last read, and clears the
+ * accumulators. */
 moe_status moe_profile_enable(moe_handle* h, int32_t on);
 moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, int32_t* n_out);
 
