@@ -233,6 +233,17 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded);
 moe_status moe_profile_enable(moe_handle* h, int32_t on);
 moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, int32_t* n_out);
 
+/* ---- Fault injection (test hook; the paper has no counterpart) --------------------------------
+ * Arms one fault for the next decode step, to exercise the error paths without faulting a GPU:
+ *   MOE_FAULT_BARRIER_TIMEOUT (device schedule): the step's grid barriers wait for an arrival
+ *     count no launch reaches, with a 0.2 s limit. Every wait runs out, the kernel exits, and the
+ *     step (or the next call that synchronises) returns MOE_ERR_TIMEOUT with the pool emptied.
+ *   MOE_FAULT_COPY_ERROR (host copy-engine schedule): the step's first miss copy reports a CUDA
+ *     error before it is issued; the step returns MOE_ERR_CUDA with the pool emptied.
+ *   MOE_FAULT_NONE disarms. MOE_ERR_INVALID for a kind the handle's schedule cannot take. */
+enum { MOE_FAULT_NONE = 0, MOE_FAULT_BARRIER_TIMEOUT = 1, MOE_FAULT_COPY_ERROR = 2 };
+moe_status moe_inject_fault(moe_handle* h, int32_t kind);
+
 /* ---- Allocation-free routing --------------------------------------------------------------
  * The paper has no counterpart to this call; it exists for callers that cannot allocate device
  * memory at the point where they route (an inference runtime that reserves all device memory at

@@ -124,6 +124,10 @@ class MoE:
     def reset_residency(self):
         self._check(self.lib.moe_reset_residency(self.h))
 
+    def inject_fault(self, kind: str):
+        """Test hook: arm one fault ("barrier_timeout", "copy_error" or "none") for the next step."""
+        self._check(self.lib.moe_inject_fault(self.h, _lib.FAULT[kind]))
+
     def preload(self) -> int:
         n = ctypes.c_int64()
         self._check(self.lib.moe_preload(self.h, ctypes.byref(n)))

@@ -19,12 +19,13 @@ DTYPE = {"fp32": 0, "bf16": 1, "int4": 2}
 SCHEDULE = {"device": 0, "host_copy_engine": 1}
 BATCHED_PATH = {"auto": 0, "cuda_cores": 1}
 POLICY = {"lru": 0, "rotary": 1}
+FAULT = {"none": 0, "barrier_timeout": 1, "copy_error": 2}
 
 # Every function the header declares (checked by the CPU test suite).
 EXPORTS = ["moe_expert_bytes", "moe_pool_bytes", "moe_create", "moe_set_router", "moe_register_host_experts",
            "moe_decode_step", "moe_decode_step_host", "moe_get_residency_trace", "moe_get_last_routing",
            "moe_get_stats", "moe_reset_residency", "moe_profile_enable", "moe_profile_read", "moe_last_error",
-           "moe_destroy", "moe_route_noalloc", "moe_preload"]
+           "moe_destroy", "moe_route_noalloc", "moe_preload", "moe_inject_fault"]
 
 
 class MoeConfig(ctypes.Structure):
@@ -102,5 +103,7 @@ def load(path: str | None = None):
         L.moe_route_noalloc.restype = ctypes.c_int
         L.moe_preload.argtypes = [vp, ctypes.POINTER(i64)]
         L.moe_preload.restype = ctypes.c_int
+        L.moe_inject_fault.argtypes = [vp, i32]
+        L.moe_inject_fault.restype = ctypes.c_int
         _lib = L
         return L

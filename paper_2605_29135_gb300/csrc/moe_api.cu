@@ -141,6 +141,7 @@ struct moe_handle {
   cudaEvent_t err_ev = nullptr;
   bool err_pending = false;
   int64_t steps_launched = 0;
+  int fault = MOE_FAULT_NONE;  // armed by moe_inject_fault for the next decode step
   std::string err;
 };
 
@@ -496,6 +497,10 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     for (auto& n : needs) {
       if (!n.miss) continue;
       ProfScope ps(h, h->copy_stream, PC_COPY, h->lay.total);
+      if (h->fault == MOE_FAULT_COPY_ERROR) {  // an armed copy fault: this copy "fails"
+        h->fault = MOE_FAULT_NONE;
+        return cuda_fail(h, cudaErrorInvalidValue, "miss copy (injected fault)");
+      }
       MOE_CK(h, cudaMemcpyAsync(h->pool + (int64_t)n.slot * h->slot_stride, h->arena + (int64_t)n.gid * h->slot_stride,
                                 h->lay.total, cudaMemcpyHostToDevice, h->copy_stream));
       ps.done();
@@ -641,6 +646,16 @@ unsigned long long* phase_buffer(moe_handle* h) {
   return h->d_phase_ts;
 }
 
+// An armed barrier fault: the step's grid barriers wait for an arrival count that no launch
+// reaches, with a 0.2 s limit, so every CTA's bounded wait runs out and the step reports
+// MOE_ERR_TIMEOUT (the kernels exit normally; nothing waits without a limit).
+void arm_barrier_fault(moe_handle* h, unsigned& bar_base, unsigned long long& timeout_ns) {
+  if (h->fault != MOE_FAULT_BARRIER_TIMEOUT) return;
+  h->fault = MOE_FAULT_NONE;
+  bar_base += 0x40000000u;
+  timeout_ns = 200000000ull;
+}
+
 moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
   const moe_config& c = h->cfg;
   const int k = c.top_k, E = c.n_experts;
@@ -689,6 +704,7 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.bar_base = h->bar_epoch;
   a.err = h->d_err;
   a.barrier_timeout_ns = 2000000000ull;
+  arm_barrier_fault(h, a.bar_base, a.barrier_timeout_ns);
   a.phase_ts = phase_buffer(h);
   a.work = h->d_bar + 2;
   a.touch_shift = h->touch_shift;
@@ -769,6 +785,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   a.bar_base = h->bar_epoch;
   a.err = h->d_err;
   a.barrier_timeout_ns = 2000000000ull;
+  arm_barrier_fault(h, a.bar_base, a.barrier_timeout_ns);
   a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
   a.touch_shift = h->touch_shift;
   a.phase_ts = phase_buffer(h);
@@ -1259,6 +1276,18 @@ moe_status moe_profile_read(moe_handle* h, moe_kernel_time* out, int32_t cap, in
 }
 
 const char* moe_last_error(const moe_handle* h) { return h ? h->err.c_str() : g_create_error.c_str(); }
+
+moe_status moe_inject_fault(moe_handle* h, int32_t kind) {
+  if (!h) return MOE_ERR_INVALID;
+  if (kind == MOE_FAULT_BARRIER_TIMEOUT && !h->dev_mode)
+    return fail(h, MOE_ERR_INVALID, "barrier faults need the device schedule");
+  if (kind == MOE_FAULT_COPY_ERROR && h->dev_mode)
+    return fail(h, MOE_ERR_INVALID, "copy faults need the host copy-engine schedule");
+  if (kind != MOE_FAULT_NONE && kind != MOE_FAULT_BARRIER_TIMEOUT && kind != MOE_FAULT_COPY_ERROR)
+    return fail(h, MOE_ERR_INVALID, "unknown fault kind");
+  h->fault = kind;
+  return MOE_OK;
+}
 
 void moe_destroy(moe_handle* h) {
   if (!h) return;
