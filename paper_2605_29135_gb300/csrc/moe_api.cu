@@ -1,5 +1,10 @@
 // C ABI of the capped-residency MoE decode library: handle, pinned host tier, slot pool,
-// residency table (LRU with lower-id ties), miss-copy pipeline and the per-layer schedule.
+// residency table (LRU with lower-id ties, or the rotary slot group), miss-copy pipeline and the
+// per-layer schedules.
+//
+// Device schedule: one cooperative kernel per decode step runs every layer (fused.cu at batch 1,
+// fused_batched.cu for batches, on tensor cores where the shape allows); the lookup table lives in
+// device memory. This file sets up its state, launches it and reads back its error flag.
 //
 // Host-driven schedule of one layer (the routing result reaches the host through mapped
 // pinned memory; the host owns the lookup table and issues the selective loads):
