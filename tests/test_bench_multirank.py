@@ -1,4 +1,4 @@
-"""The multi-rank path of bench.py on CPU (gloo, world size 2): each GPU runs an independent
+"""Host logic of bench.py on CPU. The multi-rank path (gloo, world size 2): each GPU runs an independent
 replica, the job takes as long as its slowest replica (max over ranks), the job's rate is all
 replicas' units over that time, and the reference arm runs on rank 0 only."""
 import os
@@ -71,3 +71,28 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
     args = argparse.Namespace(warmup=3, steps=4, gpus=2)
     assert bench.run_reference(args, synth.WORKLOADS["tiny_fp32"]) == 0
     assert capsys.readouterr().out == ""
+
+
+def test_stored_traffic_only_for_matching_kernel_sources(tmp_path, monkeypatch):
+    # a committed ncu summary is used only while the kernel's sources hash to its recorded digest
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    good = bench.kernel_source_digest("k_fused")
+    (prof / "k_ok.md").write_text(f"- kernel_source_digest: `{good}`\n- traffic_bytes_per_full_launch: `12345`\n")
+    (prof / "k_stale.md").write_text("- kernel_source_digest: `0000000000000000`\n"
+                                     "- traffic_bytes_per_full_launch: `12345`\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    monkeypatch.setattr(bench, "kernel_source_digest", lambda kernel="k_fused": good)
+    assert bench.stored_traffic("k_ok.md", "k_fused") == 12345.0
+    assert bench.stored_traffic("k_stale.md", "k_fused") is None
+    assert bench.stored_traffic("missing.md", "k_fused") is None
+
+
+def test_sample_units_walk_sequences_then_layers_then_tokens():
+    import synth
+
+    wl = synth.WORKLOADS["stack48_batch64"]
+    u = bench.sample_units(wl, 130)
+    assert u[0] == (0, 0, 0) and u[63] == (0, 0, 63) and u[64] == (0, 1, 0) and u[129] == (0, 2, 1)
+    wl1 = synth.WORKLOADS["stack48_bf16"]
+    assert bench.sample_units(wl1, 50)[-1] == (1, 1, 0)
