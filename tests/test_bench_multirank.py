@@ -1,6 +1,9 @@
-"""Host logic of bench.py on CPU. The multi-rank path (gloo, world size 2): each GPU runs an independent
-replica, the job takes as long as its slowest replica (max over ranks), the job's rate is all
-replicas' units over that time, and the reference arm runs on rank 0 only."""
+"""Host logic of bench.py on CPU.
+
+The multi-rank path (gloo, world size 2): each GPU runs an independent replica, the job takes as
+long as its slowest replica (max over ranks), the job's rate is all replicas' units over that time,
+and the reference arm runs on rank 0 only. Also: stored ncu traffic figures are used only for the
+kernel sources they were captured on, and the oracle's sample walks units in decode order."""
 import os
 import socket
 
