@@ -325,19 +325,18 @@ int pick_chd(int nch) {
   return -1;
 }
 
+// Opt the kernel in to `smem` bytes of dynamic shared memory on the current device when that is
+// above the default 48 KB (the attribute is per device, so it is set at every such launch).
 template <typename K>
-cudaError_t allow_smem(K kernel, size_t smem, size_t& granted) {
-  if (smem <= granted) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess) granted = smem;
-  return e;
+cudaError_t allow_smem(K kernel, size_t smem) {
+  if (smem <= 48 * 1024) return cudaSuccess;
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
 template <int WD, int CH>
 cudaError_t run_router(const RouterArgs& a, cudaStream_t s) {
-  static size_t granted = 48 * 1024;
   const size_t smem = (size_t)a.d * (WD == WD_FP32 ? 4 : 2);
-  cudaError_t e = allow_smem(k_router<WD, CH>, smem, granted);
+  cudaError_t e = allow_smem(k_router<WD, CH>, smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(kRouterCtas);
@@ -358,9 +357,8 @@ template <int WD, int CH>
 cudaError_t run_gateup(const GateUpArgs& a, cudaStream_t s) {
   const int total = a.n_tasks * a.I;
   if (total <= 0) return cudaSuccess;
-  static size_t granted = 48 * 1024;
   const size_t smem = (size_t)a.d * (WD == WD_FP32 ? 4 : 2);
-  cudaError_t e = allow_smem(k_gateup<WD, CH>, smem, granted);
+  cudaError_t e = allow_smem(k_gateup<WD, CH>, smem);
   if (e != cudaSuccess) return e;
   k_gateup<WD, CH><<<(total + kGuWarps - 1) / kGuWarps, kGuWarps * 32, smem, s>>>(a);
   return cudaGetLastError();
@@ -368,9 +366,8 @@ cudaError_t run_gateup(const GateUpArgs& a, cudaStream_t s) {
 
 template <int WD, int CHD>
 cudaError_t run_down(const DownArgs& a, cudaStream_t s) {
-  static size_t granted = 48 * 1024;
   const size_t smem = (size_t)a.k * ipad_of(a.I) * sizeof(float);
-  cudaError_t e = allow_smem(k_down_combine<WD, CHD>, smem, granted);
+  cudaError_t e = allow_smem(k_down_combine<WD, CHD>, smem);
   if (e != cudaSuccess) return e;
   k_down_combine<WD, CHD><<<(a.d + kDnWarps - 1) / kDnWarps, kDnWarps * 32, smem, s>>>(a);
   return cudaGetLastError();

@@ -814,18 +814,18 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   return MOE_OK;
 }
 
+// The driver's tensor-map encoder, looked up once per process (thread-safe static initialisation).
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static bool tried = false;
-  if (!tried) {
-    tried = true;
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
+    PFN_cuTensorMapEncodeTiled_v12000 f = nullptr;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+      f = (PFN_cuTensorMapEncodeTiled_v12000)p;
     cudaGetLastError();
-  }
+    return f;
+  }();
   return fn;
 }
 
