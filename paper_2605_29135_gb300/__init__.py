@@ -49,11 +49,37 @@ def _ptr(a) -> ctypes.c_void_p:
     if a is None:
         return None
     if isinstance(a, np.ndarray):
-        assert a.flags["C_CONTIGUOUS"], "arrays passed to libmoe must be C-contiguous"
+        if not a.flags["C_CONTIGUOUS"]:
+            raise ValueError("arrays passed to libmoe must be C-contiguous")
         return ctypes.c_void_p(a.ctypes.data)
     # torch tensor
-    assert a.is_contiguous(), "tensors passed to libmoe must be contiguous"
+    if not a.is_contiguous():
+        raise ValueError("tensors passed to libmoe must be contiguous")
     return ctypes.c_void_p(a.data_ptr())
+
+
+def _nbytes(a) -> int:
+    return a.nbytes if isinstance(a, np.ndarray) else a.numel() * a.element_size()
+
+
+def _check_buffer(name: str, a, need: int, where: str, device: int = 0):
+    """Refuse a buffer the library would read or write past its end, or on the wrong side."""
+    if a is None:
+        raise ValueError(f"{name} is None")
+    if not (a.flags["C_CONTIGUOUS"] if isinstance(a, np.ndarray) else a.is_contiguous()):
+        raise ValueError(f"{name} must be contiguous")
+    on_gpu = not isinstance(a, np.ndarray) and a.is_cuda
+    if where == "device" and (not on_gpu or a.device.index != device):
+        raise ValueError(f"{name} must be a tensor on cuda:{device}")
+    if where == "host" and on_gpu:
+        raise ValueError(f"{name} must be in host memory")
+    if _nbytes(a) < need:
+        raise ValueError(f"{name} holds {_nbytes(a)} bytes, the call needs {need}")
+
+
+def _weight_bytes(wdtype: int, n: int) -> int:
+    """Bytes of n stored weight elements (int4: two per byte)."""
+    return {DTYPE["fp32"]: 4 * n, DTYPE["bf16"]: 2 * n, DTYPE["int4"]: n // 2}[wdtype]
 
 
 class MoE:
@@ -78,18 +104,33 @@ class MoE:
 
     # -- ABI
     def set_router(self, layer: int, w_r: np.ndarray):
-        self._check(self.lib.moe_set_router(self.h, layer, _ptr(np.ascontiguousarray(w_r))))
+        c = self.cfg
+        w = np.ascontiguousarray(w_r)
+        _check_buffer("w_r", w, (4 if c.wdtype == DTYPE["fp32"] else 2) * c.n_experts * c.d, "host")
+        self._check(self.lib.moe_set_router(self.h, layer, _ptr(w)))
 
     def register_host_experts(self, layer: int, expert: int, gate, up, down, scales=None):
+        c = self.cfg
         g, u, dn = (np.ascontiguousarray(a) for a in (gate, up, down))
+        for name, a in (("gate", g), ("up", u), ("down", dn)):
+            _check_buffer(name, a, _weight_bytes(c.wdtype, c.d * c.d_ff), "host")
         sc = None if scales is None else np.ascontiguousarray(scales, dtype=np.uint16)
+        if sc is not None:
+            _check_buffer("scales", sc, 2 * (2 * c.d_ff * (c.d // 128) + c.d * (c.d_ff // 128)), "host")
         self._check(self.lib.moe_register_host_experts(self.h, layer, expert, _ptr(g), _ptr(u), _ptr(dn), _ptr(sc)))
+
+    def _act_bytes(self, batch: int) -> int:
+        c = self.cfg
+        return c.n_layers * batch * c.d * (4 if c.adtype == DTYPE["fp32"] else 2)
 
     def decode_step(self, hidden, out, batch: int = 1, stream=None):
         """hidden, out: contiguous device tensors [n_layers x batch x d]; stream: torch.cuda.Stream or None
         (torch's current stream)."""
         import torch
 
+        need = self._act_bytes(batch)
+        _check_buffer("hidden", hidden, need, "device", self.cfg.device)
+        _check_buffer("out", out, need, "device", self.cfg.device)
         if stream is None:
             stream = torch.cuda.current_stream(hidden.device)
         self._check(self.lib.moe_decode_step(self.h, _ptr(hidden), _ptr(out), batch,
@@ -97,6 +138,9 @@ class MoE:
 
     def decode_step_host(self, hidden, out, batch: int = 1):
         """hidden, out: host buffers (numpy arrays or CPU tensors, ideally pinned)."""
+        need = self._act_bytes(batch)
+        _check_buffer("hidden", hidden, need, "host")
+        _check_buffer("out", out, need, "host")
         self._check(self.lib.moe_decode_step_host(self.h, _ptr(hidden), _ptr(out), batch))
 
     def get_residency_trace(self) -> np.ndarray:
