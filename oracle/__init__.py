@@ -15,6 +15,10 @@ a deterministic LRU with lower-id ties):
    LRU step (``orc_lru_step``), which yields one hit/miss record per id;
    every miss copies the expert's stored weights from the host tier into
    its slot (the oracle keeps those slot copies and computes from them);
+2b. optional prefetch admission (``prefetch=m``, LRU only): after the step,
+   the m experts each sequence's router ranks right after its top k are
+   admitted into the slot group if absent (``orc_lru_admit``, records of kind
+   2), evicting only experts this layer-step does not need;
 3. expert FFN from the slot copy: u = silu(W_g x) * (W_u x), y_r = W_d u;
 4. combine: out = sum_r g_r y_r in rank order.
 
@@ -81,6 +85,8 @@ def lib():
             L.orc_lru_step.restype = i32
             L.orc_rotary_step.argtypes = [i64, vp, vp, vp, vp, vp, i32, i32, i32, vp]
             L.orc_rotary_step.restype = i32
+            L.orc_lru_admit.argtypes = [i64, vp, vp, vp, i64, vp, i32, vp, i32, i32, i32, vp]
+            L.orc_lru_admit.restype = i32
             _lib = L
     return _lib
 
@@ -137,6 +143,16 @@ def router(Wr: np.ndarray, h: np.ndarray, k: int, renorm: bool = True, forced_id
     return idx, gate, z, p
 
 
+def prefetch_candidates(z: np.ndarray, idx, m: int):
+    """The m experts the router ranks highest after the selected ones: descending logit z, ties to
+    the lower id, skipping the ids in idx (ranks k .. k + m - 1 when idx is the router's own top k).
+    One reading of the paper's principle that residency decisions may use information produced
+    during execution (Sec. 3; the routing result of Fig. 1 feeds the residency decision)."""
+    sel = set(int(e) for e in idx)
+    order = sorted(range(len(z)), key=lambda e: (-float(z[e]), e))
+    return [e for e in order if e not in sel][:m]
+
+
 def expert_ffn(Wg: np.ndarray, Wu: np.ndarray, Wd: np.ndarray, x: np.ndarray):
     """SwiGLU expert FFN in fp64 -> (y [d], u [I])."""
     Wg, Wu, Wd = (np.ascontiguousarray(a, dtype=np.float64) for a in (Wg, Wu, Wd))
@@ -191,6 +207,14 @@ class LRUTable:
             raise RuntimeError("LRU step: capacity below the number of distinct experts in one layer-step")
         return out
 
+    def admit(self, clock: int, pinned, admit, step: int) -> np.ndarray:
+        """Prefetch admission after a layer-step (see orc_lru_admit): records of kind 2."""
+        pinned = np.ascontiguousarray(sorted(set(int(g) for g in pinned)), dtype=np.int32)
+        admit = np.ascontiguousarray(sorted(set(int(g) for g in admit)), dtype=np.int32)
+        out = np.zeros(len(admit), dtype=REC_DTYPE)
+        n = lib().orc_lru_admit(self.cap, _p(self.slot_of), _p(self.gid_of), _p(self.last_use), clock, _p(pinned),
+                                len(pinned), _p(admit), len(admit), self.n_experts, step, _p(out))
+        return out[:n]
 
 
 class RotaryTable:
@@ -249,7 +273,7 @@ class Oracle:
     """
 
     def __init__(self, d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots, routers, experts,
-                 renorm=True, keep_slot_copies=True, policy="lru"):
+                 renorm=True, keep_slot_copies=True, policy="lru", prefetch=0):
         self.d, self.E, self.k, self.I, self.L = d, n_experts, top_k, d_ff, n_layers
         self.wdtype, self.adtype, self.renorm = wdtype, adtype, renorm
         self.router_dtype = "fp32" if wdtype == "fp32" else "bf16"
@@ -257,20 +281,23 @@ class Oracle:
         self.experts = experts
         self.keep = keep_slot_copies
         self.policy = policy
+        if prefetch and policy != "lru":
+            raise ValueError("prefetch admission is defined for the LRU policy")
+        self.prefetch = prefetch  # router ranks k .. k + prefetch - 1 admitted after each layer-step
         self.table = TABLES[policy](n_layers * n_experts, cap_slots, n_experts)
         self.slots: dict[int, object] = {}
         self.token_step = 0
 
     @classmethod
     def for_workload(cls, wl, cap_slots=None, keep_slot_copies=True, routers=None, experts=None, renorm=True,
-                     policy="lru"):
+                     policy="lru", prefetch=0):
         import synth
 
         routers = routers if routers is not None else [synth.router_weights(wl, l) for l in range(wl.n_layers)]
         experts = experts if experts is not None else (lambda l, e: synth.expert_weights(wl, l, e))
         return cls(wl.d, wl.n_experts, wl.top_k, wl.d_ff, wl.n_layers, wl.wdtype, wl.adtype,
                    wl.cap_slots if cap_slots is None else cap_slots, routers, experts, renorm=renorm,
-                   keep_slot_copies=keep_slot_copies, policy=policy)
+                   keep_slot_copies=keep_slot_copies, policy=policy, prefetch=prefetch)
 
     def reset(self):
         self.table = TABLES[self.policy](self.table.n_gid, self.table.cap, self.E)
@@ -329,9 +356,14 @@ class Oracle:
                 idx[l, b], gate[l, b], z[l, b], _ = router(self.routers[l], h[l, b], self.k, self.renorm, fi)
             needed = sorted(set(int(l * self.E + e) for e in idx[l].ravel()))
             r = self.table.step(clock, needed, self.token_step)
+            if self.prefetch:
+                admit = set()
+                for b in range(B):
+                    admit.update(l * self.E + e for e in prefetch_candidates(z[l, b], idx[l, b], self.prefetch))
+                r = np.concatenate([r, self.table.admit(clock, needed, sorted(admit - set(needed)), self.token_step)])
             recs.append(r)
             for rec in r:
-                if rec["kind"] == 1:
+                if rec["kind"] in (1, 2):
                     gid = int(l * self.E + rec["expert"])
                     if self.keep:
                         w = self.experts(l, int(rec["expert"]))

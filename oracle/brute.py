@@ -77,6 +77,54 @@ class RecencyListLRU:
         return recs
 
 
+def admit_brute(lru, needed, admit):
+    """Prefetch admission on a RecencyListLRU right after its step(needed).
+
+    Written on the recency list: ids in admit (ascending) that are absent take the lowest free
+    slot, else the slot of the oldest resident outside needed and admit; when there is none the
+    rest are dropped. Newly admitted ids join the needed ones at the newest use time, the group
+    ordered by id. Returns records (id, 2, slot, evicted).
+    """
+    needed = sorted(set(needed))
+    admit = sorted(set(admit))
+    keep = set(needed) | set(admit)
+    recs = []
+    new = []
+    for g in admit:
+        if g in lru.slot:
+            continue
+        if lru.free:
+            s = min(lru.free)
+            lru.free.remove(s)
+            victim = -1
+        else:
+            victim = next((v for v in lru.order if v not in keep), None)
+            if victim is None:
+                break
+            lru.order.remove(victim)
+            s = lru.slot.pop(victim)
+        lru.slot[g] = s
+        new.append(g)
+        recs.append((g, 2, s, victim))
+    newest = set(needed) | set(new)
+    lru.order = [v for v in lru.order if v not in newest] + sorted(newest)
+    return recs
+
+
+def prefetch_candidates_brute(z, sel, m):
+    """The m largest logits outside sel, by repeated arg-max with ties to the lower id."""
+    left = [e for e in range(len(z)) if e not in set(sel)]
+    out = []
+    for _ in range(min(m, len(left))):
+        best = left[0]
+        for e in left[1:]:
+            if z[e] > z[best]:
+                best = e
+        out.append(best)
+        left.remove(best)
+    return out
+
+
 class RotaryRing:
     """Independent pure-Python model of the rotary slot group (ring of slots, a hand, and each
     slot's previous occupant), for checking orc_rotary_step on random request sequences."""

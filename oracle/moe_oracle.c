@@ -177,7 +177,7 @@ typedef struct {
   int32_t step;    /* decode step (token index) */
   int32_t layer;
   int32_t expert;  /* expert id within the layer */
-  int32_t kind;    /* 0 hit, 1 miss */
+  int32_t kind;    /* 0 hit, 1 miss, 2 prefetch admission (orc_lru_admit) */
   int32_t slot;    /* slot that holds the expert after the step */
   int32_t evicted; /* global id of the evicted expert, -1 if a free slot was used or on a hit */
 } orc_rec;
@@ -312,6 +312,59 @@ int32_t orc_rotary_step(int64_t cap, int32_t* slot_of, int32_t* gid_of, int32_t*
     rec.slot = (int32_t)slot;
     rec.evicted = v;
     out[i] = rec;
+  }
+  return n;
+}
+
+/*
+ * Prefetch admission after a layer-step's lookup (one reading of the paper's hidden-state-guided
+ * residency: experts the router ranks just below the top k are likely needed by the next token).
+ * admit: the global ids to bring in, ascending. pinned: the layer-step's needed ids, ascending.
+ * For each admitted id g in ascending order: if resident, nothing happens (no record). Otherwise
+ * g takes the lowest free slot, else the resident v with the smallest (last_use[v], v) that is
+ * neither pinned nor admitted in this call; the record has kind 2. If no slot is available the
+ * remaining ids are not admitted. Admitted ids get last_use = clock.
+ *
+ * Returns the number of records written to out.
+ */
+int32_t orc_lru_admit(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t* last_use, int64_t clock,
+                      const int32_t* pinned, int32_t npinned, const int32_t* admit, int32_t nadmit, int32_t n_experts,
+                      int32_t step, orc_rec* out) {
+  int32_t n = 0;
+  for (int32_t i = 0; i < nadmit; i++) {
+    int32_t g = admit[i];
+    if (slot_of[g] >= 0) continue;
+    int64_t slot = -1;
+    for (int64_t s = 0; s < cap; s++) {
+      if (gid_of[s] < 0) {
+        slot = s;
+        break;
+      }
+    }
+    int32_t victim = -1;
+    if (slot < 0) {
+      for (int64_t s = 0; s < cap; s++) {
+        int32_t v = gid_of[s];
+        if (v < 0 || in_sorted(pinned, npinned, v) || in_sorted(admit, nadmit, v)) continue;
+        if (victim < 0 || last_use[v] < last_use[victim] || (last_use[v] == last_use[victim] && v < victim)) {
+          victim = v;
+          slot = s;
+        }
+      }
+      if (victim < 0) break;
+      slot_of[victim] = -1;
+    }
+    gid_of[slot] = g;
+    slot_of[g] = (int32_t)slot;
+    last_use[g] = clock;
+    orc_rec rec;
+    rec.step = step;
+    rec.layer = g / n_experts;
+    rec.expert = g % n_experts;
+    rec.kind = 2;
+    rec.slot = (int32_t)slot;
+    rec.evicted = victim;
+    out[n++] = rec;
   }
   return n;
 }
