@@ -131,7 +131,7 @@ typedef struct {
   int32_t step;    /* decode step index since create/reset */
   int32_t layer;
   int32_t expert;  /* expert id within the layer */
-  int32_t kind;    /* 0 hit, 1 miss */
+  int32_t kind;    /* 0 hit, 1 miss, 2 prefetch admission (residency planner only) */
   int32_t slot;    /* slot holding the expert after the step */
   int32_t evicted; /* global id (layer * E + expert) of the evicted expert; -1 if none */
 } moe_trace_rec;
@@ -272,6 +272,45 @@ moe_status moe_inject_fault(moe_handle* h, int32_t kind);
 #define MOE_NOALLOC_MAX_EXPERTS 256
 moe_status moe_route_noalloc(const void* w_r, const void* hidden, int32_t rows, int32_t n_experts, int32_t d,
                              int32_t top_k, int32_t renorm, int32_t wdtype, int32_t* idx, float* gate, void* stream);
+
+/* ---- Residency planner ------------------------------------------------------------------------
+ * The library's host slot table (the code the MOE_SCHEDULE_HOST_COPY_ENGINE schedule runs, and
+ * the same rules the device schedule's kernel applies) driven by expert selections the caller
+ * supplies. It touches no GPU and holds no weights. Use it to size a cap or compare policies on
+ * a recorded routing sequence: it returns the hit / miss / eviction records a decode step would
+ * produce (paper Sec. 3, Fig. 1: slot group, lookup table, selective load and evict).
+ *
+ * moe_planner_create: n_layers * n_experts global ids (gid = layer * n_experts + expert), a slot
+ *   group of min(cap_slots, n_layers * n_experts) slots, all free; policy MOE_POLICY_LRU or
+ *   MOE_POLICY_ROTARY (rules as for moe_config.policy). MOE_ERR_INVALID for bad sizes (the
+ *   message is moe_planner_last_error(NULL)); *out is NULL on failure.
+ * moe_planner_preload: as moe_preload: free slots take absent ids in ascending order; those
+ *   count as used before every step. *n_loaded (optional) = ids placed.
+ * moe_planner_step: one layer-step. (step, layer) must increase from call to call (layer in
+ *   [0, n_layers)) and orders the layer-steps for recency, as in a decode step. experts: the n expert ids (within
+ *   the layer) the step uses; duplicates are merged, as the union of a batch's selections is.
+ *   prefetch (LRU only, else MOE_ERR_INVALID): n_prefetch candidate ids admitted after the step,
+ *   one reading of the paper's residency decisions that use information produced during
+ *   execution (Sec. 3), e.g. the experts the router ranks right after its top k: ids that are
+ *   absent take the lowest free slot, else the slot of the resident with the smallest
+ *   (last use, gid) that is neither used by this step nor a candidate; when none is left the rest
+ *   are dropped; an admitted id counts as used by this step. recs (recs_cap >= n + n_prefetch)
+ *   receives one record per distinct used id (ascending gid, kind 0 or 1) followed by one per
+ *   admitted candidate (ascending, kind 2); *n_recs = records written. MOE_ERR_CAPACITY when a
+ *   used id finds no slot (cap below the step's distinct ids): the records decided before it are
+ *   written and the planner refuses further steps. Argument errors change nothing.
+ * One planner is used by one host thread at a time. */
+typedef struct moe_planner moe_planner;
+moe_status moe_planner_create(int32_t n_layers, int32_t n_experts, int64_t cap_slots, int32_t policy,
+                              moe_planner** out);
+moe_status moe_planner_preload(moe_planner* p, int64_t* n_loaded);
+moe_status moe_planner_step(moe_planner* p, int64_t step, int32_t layer, const int32_t* experts, int32_t n,
+                            const int32_t* prefetch, int32_t n_prefetch, moe_trace_rec* recs, int32_t recs_cap,
+                            int32_t* n_recs);
+/* Message of the last failure on p (or of the last failed moe_planner_create if p is NULL). */
+const char* moe_planner_last_error(const moe_planner* p);
+/* NULL is a no-op. */
+void moe_planner_destroy(moe_planner* p);
 
 /* Message of the last failure on h (or of the last failed moe_create if h is NULL). */
 const char* moe_last_error(const moe_handle* h);

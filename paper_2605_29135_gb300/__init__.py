@@ -207,6 +207,63 @@ class MoE:
         self.destroy()
 
 
+class Planner:
+    """Residency planner (moe_planner_*): the library's host slot table driven by expert
+    selections, with no GPU. step() returns the layer-step's records (TRACE_DTYPE): hits and
+    misses of the used experts, then prefetch admissions (kind 2, LRU only)."""
+
+    def __init__(self, n_layers: int, n_experts: int, cap_slots: int, policy: str = "lru"):
+        self.lib = _lib.load()
+        self.n_layers, self.n_experts = n_layers, n_experts
+        h = ctypes.c_void_p()
+        st = self.lib.moe_planner_create(n_layers, n_experts, cap_slots, _lib.POLICY[policy], ctypes.byref(h))
+        if st != 0:
+            raise MoEError(st, (self.lib.moe_planner_last_error(None) or b"").decode())
+        self.h = h
+
+    def _check(self, st):
+        if st != 0:
+            raise MoEError(st, (self.lib.moe_planner_last_error(self.h) or b"").decode())
+
+    def preload(self) -> int:
+        n = ctypes.c_int64()
+        self._check(self.lib.moe_planner_preload(self.h, ctypes.byref(n)))
+        return n.value
+
+    def step(self, step: int, layer: int, experts, prefetch=()) -> np.ndarray:
+        ex = np.ascontiguousarray(np.asarray(experts, dtype=np.int32).ravel())
+        pf = np.ascontiguousarray(np.asarray(prefetch, dtype=np.int32).ravel())
+        out = np.zeros(max(1, ex.size + pf.size), dtype=TRACE_DTYPE)
+        n = ctypes.c_int32()
+        st = self.lib.moe_planner_step(self.h, step, layer, _ptr(ex) if ex.size else None, ex.size,
+                                       _ptr(pf) if pf.size else None, pf.size, _ptr(out), out.size, ctypes.byref(n))
+        recs = out[:n.value]
+        if st != 0:
+            err = MoEError(st, (self.lib.moe_planner_last_error(self.h) or b"").decode())
+            err.records = recs
+            raise err
+        return recs
+
+    def destroy(self):
+        if getattr(self, "h", None):
+            self.lib.moe_planner_destroy(self.h)
+            self.h = None
+
+    close = destroy
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.destroy()
+
+
 def route_noalloc(w_r, hidden, top_k: int, renorm: bool = True, stream=None):
     """Routing without any device allocation by the library (moe_route_noalloc).
 

@@ -25,7 +25,8 @@ FAULT = {"none": 0, "barrier_timeout": 1, "copy_error": 2}
 EXPORTS = ["moe_expert_bytes", "moe_pool_bytes", "moe_create", "moe_set_router", "moe_register_host_experts",
            "moe_decode_step", "moe_decode_step_host", "moe_get_residency_trace", "moe_get_last_routing",
            "moe_get_stats", "moe_reset_residency", "moe_profile_enable", "moe_profile_read", "moe_last_error",
-           "moe_destroy", "moe_route_noalloc", "moe_preload", "moe_inject_fault"]
+           "moe_destroy", "moe_route_noalloc", "moe_preload", "moe_inject_fault", "moe_planner_create",
+           "moe_planner_preload", "moe_planner_step", "moe_planner_last_error", "moe_planner_destroy"]
 
 
 class MoeConfig(ctypes.Structure):
@@ -105,5 +106,15 @@ def load(path: str | None = None):
         L.moe_preload.restype = ctypes.c_int
         L.moe_inject_fault.argtypes = [vp, i32]
         L.moe_inject_fault.restype = ctypes.c_int
+        L.moe_planner_create.argtypes = [i32, i32, i64, i32, ctypes.POINTER(vp)]
+        L.moe_planner_create.restype = ctypes.c_int
+        L.moe_planner_preload.argtypes = [vp, ctypes.POINTER(i64)]
+        L.moe_planner_preload.restype = ctypes.c_int
+        L.moe_planner_step.argtypes = [vp, i64, i32, vp, i32, vp, i32, vp, i32, ctypes.POINTER(i32)]
+        L.moe_planner_step.restype = ctypes.c_int
+        L.moe_planner_last_error.argtypes = [vp]
+        L.moe_planner_last_error.restype = ctypes.c_char_p
+        L.moe_planner_destroy.argtypes = [vp]
+        L.moe_planner_destroy.restype = None
         _lib = L
         return L

@@ -22,7 +22,6 @@
 #include <chrono>
 #include <cstdio>
 #include <cstring>
-#include <set>
 #include <thread>
 #include <string>
 #include <utility>
@@ -31,6 +30,7 @@
 #include "fused.cuh"
 #include "kernels.cuh"
 #include "moe.h"
+#include "slot_table.h"
 
 namespace {
 
@@ -84,16 +84,10 @@ struct moe_handle {
   std::vector<cudaEvent_t> copy_ev;
   void* hid_dev = nullptr;
   void* out_dev = nullptr;
-  // residency state
-  std::vector<int32_t> slot_of, gid_of;
-  std::vector<int64_t> last_use;
-  std::vector<uint8_t> in_step;
-  std::set<std::pair<int64_t, int32_t>> lru;  // resident (last_use, gid)
-  std::set<int32_t> free_slots;
-  // rotary slot-group policy: each slot's previous occupant, its inverse, and the hand
-  std::vector<int32_t> prior;          // [cap]: gid last evicted from the slot, -1 none
-  std::vector<int32_t> prior_slot_of;  // [n_gid]: the slot whose previous occupant is gid, -1 none
-  int64_t hand = 0;
+  // residency state of the host-driven schedule
+  moe::SlotTable table;
+  std::vector<int32_t> need_gids;
+  std::vector<moe::SlotDecision> decisions;
   int64_t token_step = 0;
   int64_t route_seq = 0;
   std::vector<moe_trace_rec> trace;
@@ -242,16 +236,7 @@ void reset_device_state(moe_handle* h) {
 
 void reset_state(moe_handle* h) {
   reset_device_state(h);
-  std::fill(h->slot_of.begin(), h->slot_of.end(), -1);
-  std::fill(h->gid_of.begin(), h->gid_of.end(), -1);
-  std::fill(h->last_use.begin(), h->last_use.end(), -1);
-  std::fill(h->in_step.begin(), h->in_step.end(), 0);
-  h->lru.clear();
-  h->free_slots.clear();
-  for (int64_t s = 0; s < h->cap; s++) h->free_slots.insert((int32_t)s);
-  std::fill(h->prior.begin(), h->prior.end(), -1);
-  std::fill(h->prior_slot_of.begin(), h->prior_slot_of.end(), -1);
-  h->hand = 0;
+  h->table.reset();
   h->token_step = 0;
   h->trace.clear();
   h->trace_dropped = 0;
@@ -354,110 +339,35 @@ struct Need {
   bool miss;
 };
 
-// One layer-step of the lookup table: same rules as the reference definition (misses in
-// ascending gid; lowest free slot first, else the unpinned resident with the smallest
-// (last_use, gid); all needed experts pinned; last_use = clock afterwards), kept in an ordered
-// set so each decision is O(log cap).
+// One layer-step of the lookup table (rules in slot_table.h; needs in ascending gid). Fills each
+// need's slot and miss flag, the stats and the trace.
 moe_status residency_step(moe_handle* h, int32_t layer, std::vector<Need>& needs, int64_t clock) {
   const int32_t E = h->cfg.n_experts;
-  for (auto& n : needs) h->in_step[n.gid] = 1;
-  moe_status st = MOE_OK;
-  for (auto& n : needs) {
-    moe_trace_rec rec{(int32_t)h->token_step, layer, n.gid - layer * E, 0, 0, -1};
-    if (h->slot_of[n.gid] >= 0) {
-      n.slot = h->slot_of[n.gid];
-      n.miss = false;
-      rec.kind = 0;
-      rec.slot = n.slot;
-      h->stats.hits++;
-    } else if (h->cfg.policy == MOE_POLICY_ROTARY) {
-      // Rotary slot group (reverse rotation back to the slot the expert was last evicted from
-      // when that slot holds no expert of this step, else forward rotation from the hand).
-      auto open = [&](int32_t s) { return h->gid_of[s] < 0 || !h->in_step[h->gid_of[s]]; };
-      const int32_t ps = h->prior_slot_of[n.gid];
-      int32_t slot = ps >= 0 && open(ps) ? ps : -1;
-      if (slot < 0) {
-        for (int64_t j = 0; j < h->cap; j++) {
-          const int32_t sj = (int32_t)((h->hand + j) % h->cap);
-          if (open(sj)) {
-            slot = sj;
-            break;
-          }
-        }
-        if (slot < 0) {
-          st = fail(h, MOE_ERR_CAPACITY, "no available slot (cap below the step's working set)");
-          break;
-        }
-        h->hand = (slot + 1) % h->cap;
-      }
-      const int32_t victim = h->gid_of[slot];
-      if (victim >= 0) {
-        h->slot_of[victim] = -1;
-        h->stats.evictions++;
-      } else {
-        h->free_slots.erase(slot);
-      }
-      if (ps >= 0) h->prior[ps] = -1;  // n.gid is no longer anyone's previous occupant
-      const int32_t u = h->prior[slot];
-      if (u >= 0) h->prior_slot_of[u] = -1;
-      h->prior[slot] = victim;
-      if (victim >= 0) h->prior_slot_of[victim] = slot;
-      h->prior_slot_of[n.gid] = -1;
-      h->gid_of[slot] = n.gid;
-      h->slot_of[n.gid] = slot;
-      n.slot = slot;
-      n.miss = true;
-      rec.kind = 1;
-      rec.slot = slot;
-      rec.evicted = victim;
+  h->need_gids.clear();
+  for (auto& n : needs) h->need_gids.push_back(n.gid);
+  h->decisions.clear();
+  const bool ok = h->table.step(h->need_gids.data(), (int32_t)h->need_gids.size(), clock, h->decisions);
+  for (size_t i = 0; i < h->decisions.size(); i++) {
+    const moe::SlotDecision& d = h->decisions[i];
+    Need& n = needs[i];
+    n.slot = d.slot;
+    n.miss = d.kind == moe::SLOT_MISS;
+    if (n.miss) {
       h->stats.misses++;
       h->stats.miss_bytes += h->lay.total;
+      if (d.evicted >= 0) h->stats.evictions++;
     } else {
-      int32_t slot = -1, victim = -1;
-      if (!h->free_slots.empty()) {
-        slot = *h->free_slots.begin();
-        h->free_slots.erase(h->free_slots.begin());
-      } else {
-        for (auto it = h->lru.begin(); it != h->lru.end(); ++it) {
-          if (!h->in_step[it->second]) {
-            victim = it->second;
-            h->lru.erase(it);
-            break;
-          }
-        }
-        if (victim < 0) {
-          st = fail(h, MOE_ERR_CAPACITY, "no evictable slot (cap below the step's working set)");
-          break;
-        }
-        slot = h->slot_of[victim];
-        h->slot_of[victim] = -1;
-        h->stats.evictions++;
-      }
-      h->gid_of[slot] = n.gid;
-      h->slot_of[n.gid] = slot;
-      n.slot = slot;
-      n.miss = true;
-      rec.kind = 1;
-      rec.slot = slot;
-      rec.evicted = victim;
-      h->stats.misses++;
-      h->stats.miss_bytes += h->lay.total;
+      h->stats.hits++;
     }
     if (h->cfg.trace_capacity > 0) {
       if ((int64_t)h->trace.size() < h->cfg.trace_capacity)
-        h->trace.push_back(rec);
+        h->trace.push_back(moe_trace_rec{(int32_t)h->token_step, layer, d.gid - layer * E, d.kind, d.slot, d.evicted});
       else
         h->trace_dropped++;
     }
   }
-  for (auto& n : needs) {
-    h->in_step[n.gid] = 0;
-    if (st != MOE_OK || h->cfg.policy != MOE_POLICY_LRU) continue;
-    if (h->last_use[n.gid] >= 0 && !n.miss) h->lru.erase({h->last_use[n.gid], n.gid});
-    h->last_use[n.gid] = clock;
-    h->lru.insert({clock, n.gid});
-  }
-  return st;
+  if (!ok) return fail(h, MOE_ERR_CAPACITY, "no slot available (cap below the layer-step's working set)");
+  return MOE_OK;
 }
 
 moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_t s) {
@@ -512,7 +422,7 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       MOE_CK(h, cudaEventRecord(h->copy_ev[n_miss], h->copy_stream));
       n_miss++;
     }
-    auto slot_ptr = [&](int32_t gid) { return h->pool + (int64_t)h->slot_of[gid] * h->slot_stride; };
+    auto slot_ptr = [&](int32_t gid) { return h->pool + (int64_t)h->table.slot_of(gid) * h->slot_stride; };
     // gate-up on the hits
     moe::GateUpArgs ga{};
     ga.d = c.d;
@@ -1026,12 +936,7 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   }
   h->registered.assign(h->n_gid, 0);
   h->router_set.assign(cfg->n_layers, 0);
-  h->slot_of.assign(h->n_gid, -1);
-  h->gid_of.assign(h->cap, -1);
-  h->last_use.assign(h->n_gid, -1);
-  h->in_step.assign(h->n_gid, 0);
-  h->prior.assign(h->cap, -1);
-  h->prior_slot_of.assign(h->n_gid, -1);
+  h->table.init(h->n_gid, h->cap, cfg->policy);
   if (cfg->trace_capacity > 0) h->trace.reserve((size_t)std::min<int64_t>(cfg->trace_capacity, 1 << 22));
   reset_state(h);
   *out = h;
@@ -1212,16 +1117,28 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
   } else {
     MOE_CK(h, cudaDeviceSynchronize());
   }
-  // current lookup table
+  if (!h->dev_mode) {
+    // the host table decides the placements; a failed copy empties the pool again
+    std::vector<std::pair<int32_t, int32_t>> placed;
+    h->table.preload(placed);
+    for (const auto& gs : placed) {
+      cudaError_t e = cudaMemcpyAsync(h->pool + (int64_t)gs.second * h->slot_stride,
+                                      h->arena + (int64_t)gs.first * h->slot_stride, h->lay.total,
+                                      cudaMemcpyHostToDevice, h->copy_stream);
+      if (e == cudaSuccess) continue;
+      cudaStreamSynchronize(h->copy_stream);
+      reset_state(h);
+      return cuda_fail(h, e, "preload copy");
+    }
+    MOE_CK(h, cudaStreamSynchronize(h->copy_stream));
+    if (n_loaded) *n_loaded = (int64_t)placed.size();
+    return MOE_OK;
+  }
+  // device lookup table: free slots are [n_used, cap), filled in ascending gid
   std::vector<int32_t> slot_of(h->n_gid);
   int32_t n_used = 0;
-  if (h->dev_mode) {
-    MOE_CK(h, cudaMemcpy(slot_of.data(), h->d_slot_of, sizeof(int32_t) * h->n_gid, cudaMemcpyDeviceToHost));
-    MOE_CK(h, cudaMemcpy(&n_used, h->d_n_used, sizeof n_used, cudaMemcpyDeviceToHost));
-  } else {
-    slot_of = h->slot_of;
-    n_used = (int32_t)(h->cap - (int64_t)h->free_slots.size());
-  }
+  MOE_CK(h, cudaMemcpy(slot_of.data(), h->d_slot_of, sizeof(int32_t) * h->n_gid, cudaMemcpyDeviceToHost));
+  MOE_CK(h, cudaMemcpy(&n_used, h->d_n_used, sizeof n_used, cudaMemcpyDeviceToHost));
   int64_t loaded = 0;
   std::vector<unsigned long long> keys;
   std::vector<int32_t> kslots;
@@ -1233,17 +1150,10 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
     slot_of[g] = slot;
     keys.push_back((unsigned long long)(uint32_t)g);  // last use 0: older than every decode step
     kslots.push_back(slot);
-    if (!h->dev_mode) {
-      h->free_slots.erase(slot);
-      h->gid_of[slot] = (int32_t)g;
-      h->slot_of[g] = slot;
-      h->last_use[g] = 0;
-      h->lru.insert({0, (int32_t)g});
-    }
     loaded++;
   }
   MOE_CK(h, cudaStreamSynchronize(h->copy_stream));
-  if (h->dev_mode && loaded > 0) {
+  if (loaded > 0) {
     MOE_CK(h, cudaMemcpy(h->d_slot_of, slot_of.data(), sizeof(int32_t) * h->n_gid, cudaMemcpyHostToDevice));
     MOE_CK(h, cudaMemcpy(h->d_n_used, &n_used, sizeof n_used, cudaMemcpyHostToDevice));
     // preloaded slots are contiguous [n_used - loaded, n_used)
