@@ -15,6 +15,9 @@ a deterministic LRU with lower-id ties):
    LRU step (``orc_lru_step``), which yields one hit/miss record per id;
    every miss copies the expert's stored weights from the host tier into
    its slot (the oracle keeps those slot copies and computes from them);
+   Policies: ``lru`` (above), ``rotary`` (``orc_rotary_step``), ``guided``
+   (``orc_guided_step``: evict the resident with the worst rank in its
+   layer's most recent routing, refreshed before each lookup);
 2b. optional prefetch admission (``prefetch=m``, LRU only): after the step,
    the m experts each sequence's router ranks right after its top k are
    admitted into the slot group if absent (``orc_lru_admit``, records of kind
@@ -87,6 +90,8 @@ def lib():
             L.orc_rotary_step.restype = i32
             L.orc_lru_admit.argtypes = [i64, vp, vp, vp, i64, vp, i32, vp, i32, i32, i32, vp]
             L.orc_lru_admit.restype = i32
+            L.orc_guided_step.argtypes = [i64, vp, vp, vp, vp, i64, vp, i32, i32, i32, vp]
+            L.orc_guided_step.restype = i32
             _lib = L
     return _lib
 
@@ -249,7 +254,46 @@ class RotaryTable:
         return out
 
 
-TABLES = {"lru": LRUTable, "rotary": RotaryTable}
+def route_ranks(z: np.ndarray) -> np.ndarray:
+    """Rank of every expert in one routing: 0 for the highest logit, ties to the lower id."""
+    order = sorted(range(len(z)), key=lambda e: (-float(z[e]), e))
+    rank = np.empty(len(z), dtype=np.int32)
+    rank[order] = np.arange(len(z), dtype=np.int32)
+    return rank
+
+
+class GuidedTable:
+    """Residency state under router-guided replacement (one reading of the paper's residency
+    decisions that use information produced during execution, Sec. 3): every layer keeps the rank of
+    each of its experts in its most recent routing (the best rank over a batch's sequences; E before
+    the layer is first routed). A miss takes the lowest free slot, else evicts the resident outside
+    the layer-step's needed set with the largest rank, ties to the least recent use, then to the
+    lower global id. See orc_guided_step."""
+
+    def __init__(self, n_gid: int, cap: int, n_experts: int):
+        self.n_gid, self.cap, self.n_experts = n_gid, cap, n_experts
+        self.slot_of = np.full(n_gid, -1, dtype=np.int32)
+        self.gid_of = np.full(cap, -1, dtype=np.int32)
+        self.last_use = np.full(n_gid, -1, dtype=np.int64)
+        self.rank = np.full(n_gid, n_experts, dtype=np.int32)
+
+    preload = LRUTable.preload
+
+    def set_layer_ranks(self, layer: int, ranks):
+        E = self.n_experts
+        self.rank[layer * E:(layer + 1) * E] = np.asarray(ranks, dtype=np.int32)
+
+    def step(self, clock: int, needed, step: int) -> np.ndarray:
+        needed = np.ascontiguousarray(sorted(set(int(g) for g in needed)), dtype=np.int32)
+        out = np.zeros(len(needed), dtype=REC_DTYPE)
+        n = lib().orc_guided_step(self.cap, _p(self.slot_of), _p(self.gid_of), _p(self.last_use), _p(self.rank),
+                                  clock, _p(needed), len(needed), self.n_experts, step, _p(out))
+        if n < 0:
+            raise RuntimeError("guided step: capacity below the number of distinct experts in one layer-step")
+        return out
+
+
+TABLES = {"lru": LRUTable, "rotary": RotaryTable, "guided": GuidedTable}
 
 # ----------------------------------------------------------------------------------------------
 # the full decode step
@@ -355,6 +399,8 @@ class Oracle:
                 fi = None if forced_idx is None else forced_idx[l, b]
                 idx[l, b], gate[l, b], z[l, b], _ = router(self.routers[l], h[l, b], self.k, self.renorm, fi)
             needed = sorted(set(int(l * self.E + e) for e in idx[l].ravel()))
+            if self.policy == "guided":
+                self.table.set_layer_ranks(l, np.min([route_ranks(z[l, b]) for b in range(B)], axis=0))
             r = self.table.step(clock, needed, self.token_step)
             if self.prefetch:
                 admit = set()

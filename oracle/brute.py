@@ -125,6 +125,56 @@ def prefetch_candidates_brute(z, sel, m):
     return out
 
 
+def ranks_brute(z):
+    """Rank of e = how many experts beat it: a higher logit, or an equal logit and a lower id."""
+    return [sum(1 for j in range(len(z)) if z[j] > z[e] or (z[j] == z[e] and j < e)) for e in range(len(z))]
+
+
+class GuidedResidents:
+    """Router-guided replacement kept as a dict of residents and a free list.
+
+    The victim is chosen by comparing every evictable resident's (rank, age, id) in one max():
+    largest rank first, then the oldest use, then the lowest id. Misses in ascending id take the
+    lowest free slot first; every needed id is stamped with the step counter afterwards.
+    """
+
+    def __init__(self, cap, n_experts):
+        self.cap, self.E = cap, n_experts
+        self.slot = {}
+        self.last = {}
+        self.rank = {}
+        self.free = list(range(cap))
+        self.t = 0
+
+    def set_ranks(self, layer, ranks):
+        for e, r in enumerate(ranks):
+            self.rank[layer * self.E + e] = r
+
+    def step(self, needed):
+        needed = sorted(set(needed))
+        recs = []
+        for g in needed:
+            if g in self.slot:
+                recs.append((g, 0, self.slot[g], -1))
+                continue
+            if self.free:
+                s = min(self.free)
+                self.free.remove(s)
+                victim = -1
+            else:
+                cands = [v for v in self.slot if v not in needed]
+                if not cands:
+                    raise RuntimeError("capacity below the step's working set")
+                victim = max(cands, key=lambda v: (self.rank.get(v, self.E), -self.last.get(v, -1), -v))
+                s = self.slot.pop(victim)
+            self.slot[g] = s
+            recs.append((g, 1, s, victim))
+        for g in needed:
+            self.last[g] = self.t
+        self.t += 1
+        return recs
+
+
 class RotaryRing:
     """Independent pure-Python model of the rotary slot group (ring of slots, a hand, and each
     slot's previous occupant), for checking orc_rotary_step on random request sequences."""

@@ -368,3 +368,70 @@ int32_t orc_lru_admit(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t* l
   }
   return n;
 }
+
+/*
+ * One layer-step under router-guided replacement (one reading of the paper's residency decisions
+ * that use information produced during execution, Sec. 3, with the routing result of Fig. 1 as
+ * that information). rank[gid]: the expert's rank in its layer's most recent routing (0 = highest
+ * logit), n_experts for a layer not routed yet; the caller refreshes the layer's ranks before the
+ * call. For each needed gid in ascending order: if resident, a hit. Otherwise the lowest free
+ * slot, else the slot of the resident v outside `needed` with the largest rank[v], ties to the
+ * smaller last_use[v], then to the lower v. Afterwards last_use[x] = clock for every needed x.
+ *
+ * Returns the number of records, or -1 if no victim exists (cap < |needed|).
+ */
+int32_t orc_guided_step(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t* last_use, const int32_t* rank,
+                        int64_t clock, const int32_t* needed, int32_t n, int32_t n_experts, int32_t step,
+                        orc_rec* out) {
+  for (int32_t i = 0; i < n; i++) {
+    int32_t g = needed[i];
+    orc_rec rec;
+    rec.step = step;
+    rec.layer = g / n_experts;
+    rec.expert = g % n_experts;
+    rec.evicted = -1;
+    if (slot_of[g] >= 0) {
+      rec.kind = 0;
+      rec.slot = slot_of[g];
+      out[i] = rec;
+      continue;
+    }
+    int64_t slot = -1;
+    for (int64_t s = 0; s < cap; s++) {
+      if (gid_of[s] < 0) {
+        slot = s;
+        break;
+      }
+    }
+    if (slot < 0) {
+      int32_t victim = -1;
+      for (int64_t s = 0; s < cap; s++) {
+        int32_t v = gid_of[s];
+        if (v < 0 || in_sorted(needed, n, v)) continue;
+        int better = 0;
+        if (victim < 0)
+          better = 1;
+        else if (rank[v] != rank[victim])
+          better = rank[v] > rank[victim];
+        else if (last_use[v] != last_use[victim])
+          better = last_use[v] < last_use[victim];
+        else
+          better = v < victim;
+        if (better) {
+          victim = v;
+          slot = s;
+        }
+      }
+      if (victim < 0) return -1;
+      slot_of[victim] = -1;
+      rec.evicted = victim;
+    }
+    gid_of[slot] = g;
+    slot_of[g] = (int32_t)slot;
+    rec.kind = 1;
+    rec.slot = (int32_t)slot;
+    out[i] = rec;
+  }
+  for (int32_t i = 0; i < n; i++) last_use[needed[i]] = clock;
+  return n;
+}
