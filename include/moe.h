@@ -98,7 +98,13 @@ enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
  *     expert of the layer-step (reverse rotation), else takes the first such slot at or after the
  *     hand, which then moves past it (forward rotation). Hits change nothing. Misses in ascending
  *     global id. Both schedules, max_batch 1. */
-enum { MOE_POLICY_LRU = 0, MOE_POLICY_ROTARY = 1 };
+/*   MOE_POLICY_GUIDED: router-guided replacement, one reading of the paper's residency decisions
+ *     that use information produced during execution (Sec. 3). Each layer keeps the rank of every
+ *     expert in its most recent routing (0 = highest logit; for a batch, the best rank over its
+ *     sequences). A miss takes the lowest free slot, else evicts the resident not needed this
+ *     layer-step with the largest rank, ties to the older use, then to the lower global id.
+ *     Residency planner only for now (moe_create rejects it). */
+enum { MOE_POLICY_LRU = 0, MOE_POLICY_ROTARY = 1, MOE_POLICY_GUIDED = 2 };
 
 typedef struct {
   int32_t d;          /* hidden size */
@@ -281,8 +287,8 @@ moe_status moe_route_noalloc(const void* w_r, const void* hidden, int32_t rows, 
  * produce (paper Sec. 3, Fig. 1: slot group, lookup table, selective load and evict).
  *
  * moe_planner_create: n_layers * n_experts global ids (gid = layer * n_experts + expert), a slot
- *   group of min(cap_slots, n_layers * n_experts) slots, all free; policy MOE_POLICY_LRU or
- *   MOE_POLICY_ROTARY (rules as for moe_config.policy). MOE_ERR_INVALID for bad sizes (the
+ *   group of min(cap_slots, n_layers * n_experts) slots, all free; policy MOE_POLICY_LRU,
+ *   MOE_POLICY_ROTARY or MOE_POLICY_GUIDED (rules as for moe_config.policy). MOE_ERR_INVALID for bad sizes (the
  *   message is moe_planner_last_error(NULL)); *out is NULL on failure.
  * moe_planner_preload: as moe_preload: free slots take absent ids in ascending order; those
  *   count as used before every step. *n_loaded (optional) = ids placed.
@@ -294,7 +300,10 @@ moe_status moe_route_noalloc(const void* w_r, const void* hidden, int32_t rows, 
  *   execution (Sec. 3), e.g. the experts the router ranks right after its top k: ids that are
  *   absent take the lowest free slot, else the slot of the resident with the smallest
  *   (last use, gid) that is neither used by this step nor a candidate; when none is left the rest
- *   are dropped; an admitted id counts as used by this step. recs (recs_cap >= n + n_prefetch)
+ *   are dropped; an admitted id counts as used by this step. ranks: MOE_POLICY_GUIDED only (NULL
+ *   otherwise), the rank in [0, n_experts] of each of the layer's n_experts experts in this step's
+ *   routing (0 = highest logit; the best rank over a batch), applied before the lookup; a layer
+ *   counts every expert at rank n_experts until its first step. recs (recs_cap >= n + n_prefetch)
  *   receives one record per distinct used id (ascending gid, kind 0 or 1) followed by one per
  *   admitted candidate (ascending, kind 2); *n_recs = records written. MOE_ERR_CAPACITY when a
  *   used id finds no slot (cap below the step's distinct ids): the records decided before it are
@@ -305,8 +314,8 @@ moe_status moe_planner_create(int32_t n_layers, int32_t n_experts, int64_t cap_s
                               moe_planner** out);
 moe_status moe_planner_preload(moe_planner* p, int64_t* n_loaded);
 moe_status moe_planner_step(moe_planner* p, int64_t step, int32_t layer, const int32_t* experts, int32_t n,
-                            const int32_t* prefetch, int32_t n_prefetch, moe_trace_rec* recs, int32_t recs_cap,
-                            int32_t* n_recs);
+                            const int32_t* prefetch, int32_t n_prefetch, const int32_t* ranks, moe_trace_rec* recs,
+                            int32_t recs_cap, int32_t* n_recs);
 /* Message of the last failure on p (or of the last failed moe_planner_create if p is NULL). */
 const char* moe_planner_last_error(const moe_planner* p);
 /* NULL is a no-op. */

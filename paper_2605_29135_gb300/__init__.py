@@ -230,13 +230,21 @@ class Planner:
         self._check(self.lib.moe_planner_preload(self.h, ctypes.byref(n)))
         return n.value
 
-    def step(self, step: int, layer: int, experts, prefetch=()) -> np.ndarray:
+    def step(self, step: int, layer: int, experts, prefetch=(), ranks=None) -> np.ndarray:
+        """ranks: the "guided" policy's [n_experts] ranks of the layer's experts in this step's
+        routing (0 = highest logit; the best rank over a batch)."""
         ex = np.ascontiguousarray(np.asarray(experts, dtype=np.int32).ravel())
         pf = np.ascontiguousarray(np.asarray(prefetch, dtype=np.int32).ravel())
+        rk = None
+        if ranks is not None:
+            rk = np.ascontiguousarray(np.asarray(ranks, dtype=np.int32).ravel())
+            if rk.size != self.n_experts:
+                raise ValueError(f"ranks has {rk.size} entries, expected n_experts = {self.n_experts}")
         out = np.zeros(max(1, ex.size + pf.size), dtype=TRACE_DTYPE)
         n = ctypes.c_int32()
         st = self.lib.moe_planner_step(self.h, step, layer, _ptr(ex) if ex.size else None, ex.size,
-                                       _ptr(pf) if pf.size else None, pf.size, _ptr(out), out.size, ctypes.byref(n))
+                                       _ptr(pf) if pf.size else None, pf.size, _ptr(rk), _ptr(out), out.size,
+                                       ctypes.byref(n))
         recs = out[:n.value]
         if st != 0:
             err = MoEError(st, (self.lib.moe_planner_last_error(self.h) or b"").decode())

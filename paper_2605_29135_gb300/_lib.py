@@ -18,7 +18,7 @@ STATUS = {0: "MOE_OK", -1: "MOE_ERR_INVALID", -2: "MOE_ERR_OOM", -3: "MOE_ERR_CU
 DTYPE = {"fp32": 0, "bf16": 1, "int4": 2}
 SCHEDULE = {"device": 0, "host_copy_engine": 1}
 BATCHED_PATH = {"auto": 0, "cuda_cores": 1}
-POLICY = {"lru": 0, "rotary": 1}
+POLICY = {"lru": 0, "rotary": 1, "guided": 2}
 FAULT = {"none": 0, "barrier_timeout": 1, "copy_error": 2}
 
 # Every function the header declares (checked by the CPU test suite).
@@ -110,7 +110,7 @@ def load(path: str | None = None):
         L.moe_planner_create.restype = ctypes.c_int
         L.moe_planner_preload.argtypes = [vp, ctypes.POINTER(i64)]
         L.moe_planner_preload.restype = ctypes.c_int
-        L.moe_planner_step.argtypes = [vp, i64, i32, vp, i32, vp, i32, vp, i32, ctypes.POINTER(i32)]
+        L.moe_planner_step.argtypes = [vp, i64, i32, vp, i32, vp, i32, vp, vp, i32, ctypes.POINTER(i32)]
         L.moe_planner_step.restype = ctypes.c_int
         L.moe_planner_last_error.argtypes = [vp]
         L.moe_planner_last_error.restype = ctypes.c_char_p

@@ -202,6 +202,7 @@ std::string check_config(const moe_config* c) {
   if (c->schedule != MOE_SCHEDULE_DEVICE && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "unknown schedule";
   if (c->miss_ctas < 0) return "miss_ctas must be >= 0";
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
+  if (c->policy == MOE_POLICY_GUIDED) return "the router-guided policy is available in the residency planner only";
   if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY) return "unknown policy";
   if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
   return "";
@@ -936,7 +937,7 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   }
   h->registered.assign(h->n_gid, 0);
   h->router_set.assign(cfg->n_layers, 0);
-  h->table.init(h->n_gid, h->cap, cfg->policy);
+  h->table.init(h->n_gid, h->cap, cfg->policy, cfg->n_experts);
   if (cfg->trace_capacity > 0) h->trace.reserve((size_t)std::min<int64_t>(cfg->trace_capacity, 1 << 22));
   reset_state(h);
   *out = h;

@@ -58,7 +58,7 @@ moe_status moe_planner_create(int32_t n_layers, int32_t n_experts, int64_t cap_s
     bad = "n_layers * n_experts must fit in int32";
   else if (cap_slots < 1 || cap_slots > INT32_MAX)
     bad = "cap_slots must be in [1, 2^31)";
-  else if (policy != MOE_POLICY_LRU && policy != MOE_POLICY_ROTARY)
+  else if (policy != MOE_POLICY_LRU && policy != MOE_POLICY_ROTARY && policy != MOE_POLICY_GUIDED)
     bad = "unknown policy";
   if (bad) {
     g_planner_create_error = bad;
@@ -71,7 +71,7 @@ moe_status moe_planner_create(int32_t n_layers, int32_t n_experts, int64_t cap_s
   }
   const int64_t n_gid = (int64_t)n_layers * n_experts;
   try {
-    p->table.init(n_gid, std::min(cap_slots, n_gid), policy);
+    p->table.init(n_gid, std::min(cap_slots, n_gid), policy, n_experts);
   } catch (const std::bad_alloc&) {
     delete p;
     g_planner_create_error = "host allocation failed";
@@ -98,8 +98,8 @@ moe_status moe_planner_preload(moe_planner* p, int64_t* n_loaded) {
 }
 
 moe_status moe_planner_step(moe_planner* p, int64_t step, int32_t layer, const int32_t* experts, int32_t n,
-                            const int32_t* prefetch, int32_t n_prefetch, moe_trace_rec* recs, int32_t recs_cap,
-                            int32_t* n_recs) {
+                            const int32_t* prefetch, int32_t n_prefetch, const int32_t* ranks, moe_trace_rec* recs,
+                            int32_t recs_cap, int32_t* n_recs) {
   if (!p) return MOE_ERR_INVALID;
   if (n_recs) *n_recs = 0;
   if (p->broken) return planner_fail(p, MOE_ERR_INVALID, "the planner failed a step earlier");
@@ -114,12 +114,20 @@ moe_status moe_planner_step(moe_planner* p, int64_t step, int32_t layer, const i
   if ((int64_t)recs_cap < (int64_t)n + n_prefetch)
     return planner_fail(p, MOE_ERR_INVALID, "recs_cap below n + n_prefetch");
   const int32_t E = p->n_experts;
+  const bool guided = p->table.policy() == MOE_POLICY_GUIDED;
+  if (guided != (ranks != nullptr))
+    return planner_fail(p, MOE_ERR_INVALID, "ranks are required by the guided policy and taken by no other");
+  if (guided) {
+    for (int32_t e = 0; e < E; e++)
+      if (ranks[e] < 0 || ranks[e] > E) return planner_fail(p, MOE_ERR_INVALID, "a rank is outside [0, n_experts]");
+  }
   bool ok = false;
   try {
     if (!gather_ids(experts, n, layer, E, p->needed) || !gather_ids(prefetch, n_prefetch, layer, E, p->cand))
       return planner_fail(p, MOE_ERR_INVALID, "an expert id is outside [0, n_experts)");
     const int64_t clock = step * p->n_layers + layer + 1;  // 0: preloaded, older than every step
     p->dec.clear();
+    if (guided) p->table.set_ranks(layer, ranks);
     ok = p->table.step(p->needed.data(), (int32_t)p->needed.size(), clock, p->dec);
     if (ok && !p->cand.empty())
       p->table.admit(p->needed.data(), (int32_t)p->needed.size(), p->cand.data(), (int32_t)p->cand.size(), clock,

@@ -7,10 +7,11 @@
 
 namespace moe {
 
-void SlotTable::init(int64_t n_gid, int64_t cap, int32_t policy) {
+void SlotTable::init(int64_t n_gid, int64_t cap, int32_t policy, int32_t n_experts) {
   n_gid_ = n_gid;
   cap_ = cap;
   policy_ = policy;
+  n_experts_ = n_experts;
   reset();
 }
 
@@ -25,6 +26,11 @@ void SlotTable::reset() {
   prior_.assign(cap_, -1);
   prior_slot_of_.assign(n_gid_, -1);
   hand_ = 0;
+  rank_.assign(n_gid_, n_experts_);
+}
+
+void SlotTable::set_ranks(int32_t layer, const int32_t* ranks) {
+  std::copy(ranks, ranks + n_experts_, rank_.begin() + (int64_t)layer * n_experts_);
 }
 
 int32_t SlotTable::take_free() {
@@ -42,6 +48,19 @@ int32_t SlotTable::lru_victim() {
     }
   }
   return -1;
+}
+
+int32_t SlotTable::guided_victim() {
+  int32_t victim = -1;
+  for (int64_t s = 0; s < cap_; s++) {
+    const int32_t v = gid_of_[s];
+    if (v < 0 || mark_[v]) continue;
+    if (victim < 0 || rank_[v] > rank_[victim] ||
+        (rank_[v] == rank_[victim] &&
+         (last_use_[v] < last_use_[victim] || (last_use_[v] == last_use_[victim] && v < victim))))
+      victim = v;
+  }
+  return victim;
 }
 
 bool SlotTable::step(const int32_t* needed, int32_t n, int64_t clock, std::vector<SlotDecision>& out) {
@@ -87,7 +106,7 @@ bool SlotTable::step(const int32_t* needed, int32_t n, int64_t clock, std::vecto
     } else if (!free_.empty()) {
       slot = take_free();
     } else {
-      victim = lru_victim();
+      victim = policy_ == MOE_POLICY_GUIDED ? guided_victim() : lru_victim();
       if (victim < 0) {
         ok = false;
         break;
@@ -100,12 +119,12 @@ bool SlotTable::step(const int32_t* needed, int32_t n, int64_t clock, std::vecto
     out.push_back(SlotDecision{g, SLOT_MISS, slot, victim});
   }
   for (int32_t i = 0; i < n; i++) mark_[needed[i]] = 0;
-  if (!ok || policy_ != MOE_POLICY_LRU) return ok;
+  if (!ok || policy_ == MOE_POLICY_ROTARY) return ok;
   for (int32_t i = 0; i < n; i++) {
     const int32_t g = needed[i];
-    if (out[first + i].kind == SLOT_HIT) lru_.erase({last_use_[g], g});
+    if (policy_ == MOE_POLICY_LRU && out[first + i].kind == SLOT_HIT) lru_.erase({last_use_[g], g});
     last_use_[g] = clock;
-    lru_.insert({clock, g});
+    if (policy_ == MOE_POLICY_LRU) lru_.insert({clock, g});
   }
   return true;
 }

@@ -1,7 +1,7 @@
 // Host residency table: a fixed group of `cap` slots, the lookup table global expert id -> slot
 // and its replacement policy (paper Sec. 3, Fig. 1: slot group, lookup table, selective load and
 // evict driven by the routing result). The host-driven decode schedule and the residency planner
-// both run this code; the device schedule runs the same rules inside its kernel.
+// both run this code; the device schedule applies the LRU and rotary rules inside its kernel.
 //
 // Rules of one layer-step (needed: the distinct global ids the step uses, ascending):
 //   LRU (MOE_POLICY_LRU): a resident id is a hit. A missing id takes the lowest free slot, else
@@ -11,6 +11,11 @@
 //     last evicted from it. A missing id returns to the slot it was last evicted from when that
 //     slot holds nothing the step needs (reverse rotation), else takes the first such slot at or
 //     after the hand, which then moves past it (forward rotation). Hits change nothing.
+//   Router-guided (MOE_POLICY_GUIDED): each id carries its rank in its layer's most recent routing
+//     (set_ranks, before the layer's step; n_experts until the layer is first routed). A missing
+//     id takes the lowest free slot, else the slot of the resident the step does not need with the
+//     largest rank, ties to the smaller last use, then to the lower id. Every needed id then gets
+//     the step's clock as its last use.
 // Prefetch admission (LRU only; one reading of the paper's residency decisions that use
 // information produced during execution, Sec. 3): after a step, candidate ids (ascending) that are
 // absent take the lowest free slot, else the slot of the resident with the smallest (last use, id)
@@ -35,10 +40,14 @@ struct SlotDecision {
 
 class SlotTable {
  public:
-  // policy: MOE_POLICY_LRU or MOE_POLICY_ROTARY. Starts empty.
-  void init(int64_t n_gid, int64_t cap, int32_t policy);
-  // Every slot free, hand at slot 0, no remembered occupants.
+  // policy: MOE_POLICY_LRU, MOE_POLICY_ROTARY or MOE_POLICY_GUIDED; ids are layer * n_experts +
+  // expert. Starts empty.
+  void init(int64_t n_gid, int64_t cap, int32_t policy, int32_t n_experts);
+  // Every slot free, hand at slot 0, no remembered occupants, no layer routed.
   void reset();
+
+  // Router-guided policy: ranks [n_experts] of the layer's experts in its latest routing.
+  void set_ranks(int32_t layer, const int32_t* ranks);
 
   // One layer-step: appends one decision per needed id (ascending, distinct, in [0, n_gid)).
   // Returns false when a missing id finds no slot (cap below the step's working set); the
@@ -64,10 +73,13 @@ class SlotTable {
 
  private:
   int32_t take_free();
-  int32_t lru_victim();  // resident with the smallest (last use, id) not marked; -1 when none
+  int32_t lru_victim();     // resident with the smallest (last use, id) not marked; -1 when none
+  int32_t guided_victim();  // resident with the largest (rank, -last use, -id) not marked; -1 when none
 
   int64_t n_gid_ = 0, cap_ = 0;
   int32_t policy_ = 0;
+  int32_t n_experts_ = 1;
+  std::vector<int32_t> rank_;  // router-guided policy: [n_gid]
   std::vector<int32_t> slot_of_, gid_of_;
   std::vector<int64_t> last_use_;
   std::vector<uint8_t> mark_;                  // needed (or admitted) in the current call

@@ -1,6 +1,6 @@
 """The library's host slot table, through the residency planner (moe_planner_*), against the
-oracle on the CPU: the same records, bit for bit, for the LRU and rotary policies, with preload,
-batched unions and prefetch admission, and the planner's argument and capacity errors. The host
+oracle on the CPU: the same records, bit for bit, for the LRU, rotary and router-guided policies,
+with preload, batched unions and prefetch admission, and the planner's argument and capacity errors. The host
 copy-engine decode schedule runs this same table, so this checks its decisions without a GPU."""
 import numpy as np
 import pytest
@@ -176,3 +176,74 @@ def test_empty_layer_step_is_allowed():
     with Planner(1, 8, 4) as p:
         assert len(p.step(0, 0, [])) == 0
         assert len(p.step(1, 0, [3])) == 1
+
+
+def _ranks_of(order):
+    r = np.empty(len(order), dtype=np.int32)
+    r[list(order)] = np.arange(len(order))
+    return r
+
+
+@pytest.mark.parametrize("seed", range(4))
+@pytest.mark.parametrize("n_layers,E,k,cap,B,preload", [(1, 8, 2, 4, 1, False), (3, 8, 2, 5, 1, False),
+                                                        (4, 16, 4, 9, 1, False), (3, 4, 1, 5, 1, False),
+                                                        (3, 16, 3, 14, 4, False), (3, 4, 1, 7, 1, True)])
+def test_guided_policy_matches_the_oracle(seed, n_layers, E, k, cap, B, preload):
+    rng = np.random.default_rng(400 + seed)
+    table = oracle.GuidedTable(n_layers * E, cap, E)
+    with Planner(n_layers, E, cap, "guided") as p:
+        if preload:
+            table.preload()
+            p.preload()
+        for tok in range(40):
+            for l in range(n_layers):
+                used, best = set(), np.full(E, E, dtype=np.int32)
+                for _ in range(B):
+                    order = [int(e) for e in rng.permutation(E)]
+                    used.update(order[:k])
+                    best = np.minimum(best, _ranks_of(order))
+                table.set_layer_ranks(l, best)
+                want = _tuples(table.step(tok * n_layers + l, [l * E + e for e in used], tok), E)
+                got = _tuples(p.step(tok, l, sorted(used), ranks=best), E)
+                assert got == want, f"token {tok} layer {l}"
+
+
+def test_guided_golden_traces():
+    from tests.test_oracle_guided import read_guided_golden
+
+    for name, (E, L, k, cap, preload, steps) in read_guided_golden().items():
+        with Planner(L, E, cap, "guided") as p:
+            if preload:
+                p.preload()
+            for (tok, l, order), expect in steps:
+                recs = p.step(tok, l, order[:k], ranks=_ranks_of(order))
+                got = [(int(r["expert"]), int(r["kind"]), int(r["slot"]), int(r["evicted"])) for r in recs]
+                assert got == expect, f"case {name} token {tok} layer {l}"
+
+
+def test_guided_policy_on_the_oracle_routing_of_a_stack():
+    wl = synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, tokens=20)
+    hidden = synth.hidden_all(wl)
+    cap, E, L = 8, wl.n_experts, wl.n_layers
+    orc = oracle.Oracle.for_workload(wl, cap_slots=cap, keep_slot_copies=False, policy="guided")
+    with Planner(L, E, cap, "guided") as p:
+        for t in range(wl.tokens):
+            st = orc.decode_step(hidden[t], compute_out=False)
+            got = []
+            for l in range(L):
+                got += _tuples(p.step(t, l, st.idx[l, 0], ranks=oracle.route_ranks(st.z[l, 0])), E)
+            assert got == _tuples(st.records, E), f"token {t}"
+
+
+def test_guided_rank_arguments_are_checked():
+    with Planner(1, 8, 4, "guided") as p:
+        for kw in ({}, {"ranks": [0, 1, 2, 3, 4, 5, 6, 9]}, {"ranks": [-1, 1, 2, 3, 4, 5, 6, 7]}):
+            with pytest.raises(MoEError) as ei:
+                p.step(0, 0, [1, 2], **kw)
+            assert ei.value.status == -1
+        with pytest.raises(ValueError):
+            p.step(0, 0, [1, 2], ranks=[0, 1])
+        assert len(p.step(0, 0, [1, 2], ranks=np.arange(8))) == 2
+    with Planner(1, 8, 4, "lru") as p:
+        with pytest.raises(MoEError):
+            p.step(0, 0, [1, 2], ranks=np.arange(8))
