@@ -394,46 +394,63 @@ class Oracle:
         out = np.zeros((L, B, self.d), dtype=np.float64) if compute_out else None
         recs = []
         for l in range(L):
-            clock = self.token_step * L + l
-            for b in range(B):
-                fi = None if forced_idx is None else forced_idx[l, b]
-                idx[l, b], gate[l, b], z[l, b], _ = router(self.routers[l], h[l, b], self.k, self.renorm, fi)
-            needed = sorted(set(int(l * self.E + e) for e in idx[l].ravel()))
-            if self.policy == "guided":
-                self.table.set_layer_ranks(l, np.min([route_ranks(z[l, b]) for b in range(B)], axis=0))
-            r = self.table.step(clock, needed, self.token_step)
-            if self.prefetch:
-                admit = set()
-                for b in range(B):
-                    admit.update(l * self.E + e for e in prefetch_candidates(z[l, b], idx[l, b], self.prefetch))
-                r = np.concatenate([r, self.table.admit(clock, needed, sorted(admit - set(needed)), self.token_step)])
-            recs.append(r)
-            for rec in r:
-                if rec["kind"] in (1, 2):
-                    gid = int(l * self.E + rec["expert"])
-                    if self.keep:
-                        w = self.experts(l, int(rec["expert"]))
-                        self.slots[int(rec["slot"])] = (gid, _copy_expert(w))
+            o, idx[l], gate[l], z[l], r = self.layer_step(l, h[l], compute_out,
+                                                          None if forced_idx is None else forced_idx[l])
             if compute_out:
-                cache = {}
-                for b in range(B):
-                    ys = np.empty((self.k, self.d), dtype=np.float64)
-                    for rk in range(self.k):
-                        e = int(idx[l, b, rk])
-                        gid = l * self.E + e
-                        if gid not in cache:
-                            if self.keep:
-                                slot = int(self.table.slot_of[gid])
-                                held_gid, w = self.slots[slot]
-                                assert held_gid == gid, "slot holds another expert"
-                            else:
-                                w = self.experts(l, e)
-                            cache[gid] = self._widen_expert(w)
-                        Wg, Wu, Wd = cache[gid]
-                        ys[rk], _ = expert_ffn(Wg, Wu, Wd, h[l, b])
-                    out[l, b] = combine(ys, gate[l, b])
+                out[l] = o
+            recs.append(r)
         self.token_step += 1
         return StepResult(out, np.concatenate(recs), idx, gate, z)
+
+    def layer_step(self, l: int, h: np.ndarray, compute_out: bool = True, forced_idx=None):
+        """Layer l of the current decode step on fp64 inputs h [B x d]: routing, one residency step,
+        expert FFNs from the slot copies and the combine. The clock is token_step * L + l; the
+        caller advances token_step once per decode step (decode_step does).
+        Returns (out [B x d] or None, idx [B x k], gate [B x k], z [B x E], records)."""
+        B = h.shape[0]
+        idx = np.empty((B, self.k), dtype=np.int32)
+        gate = np.empty((B, self.k), dtype=np.float64)
+        z = np.empty((B, self.E), dtype=np.float64)
+        clock = self.token_step * self.L + l
+        for b in range(B):
+            fi = None if forced_idx is None else forced_idx[b]
+            idx[b], gate[b], z[b], _ = router(self.routers[l], h[b], self.k, self.renorm, fi)
+        needed = sorted(set(int(l * self.E + e) for e in idx.ravel()))
+        if self.policy == "guided":
+            self.table.set_layer_ranks(l, np.min([route_ranks(z[b]) for b in range(B)], axis=0))
+        r = self.table.step(clock, needed, self.token_step)
+        if self.prefetch:
+            admit = set()
+            for b in range(B):
+                admit.update(l * self.E + e for e in prefetch_candidates(z[b], idx[b], self.prefetch))
+            r = np.concatenate([r, self.table.admit(clock, needed, sorted(admit - set(needed)), self.token_step)])
+        for rec in r:
+            if rec["kind"] in (1, 2):
+                gid = int(l * self.E + rec["expert"])
+                if self.keep:
+                    w = self.experts(l, int(rec["expert"]))
+                    self.slots[int(rec["slot"])] = (gid, _copy_expert(w))
+        out = None
+        if compute_out:
+            out = np.zeros((B, self.d), dtype=np.float64)
+            cache = {}
+            for b in range(B):
+                ys = np.empty((self.k, self.d), dtype=np.float64)
+                for rk in range(self.k):
+                    e = int(idx[b, rk])
+                    gid = l * self.E + e
+                    if gid not in cache:
+                        if self.keep:
+                            slot = int(self.table.slot_of[gid])
+                            held_gid, w = self.slots[slot]
+                            assert held_gid == gid, "slot holds another expert"
+                        else:
+                            w = self.experts(l, e)
+                        cache[gid] = self._widen_expert(w)
+                    Wg, Wu, Wd = cache[gid]
+                    ys[rk], _ = expert_ffn(Wg, Wu, Wd, h[b])
+                out[b] = combine(ys, gate[b])
+        return out, idx, gate, z, r
 
 
 def _copy_expert(w):
