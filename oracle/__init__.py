@@ -26,7 +26,8 @@ a deterministic LRU with lower-id ties):
 4. combine: out = sum_r g_r y_r in rank order.
 
 All arithmetic is fp64 on exactly widened inputs (bf16/fp32 values, int4
-dequantised to q * scale). Every function here is pinned by ``tests/test_oracle_*``
+dequantised to q * scale). ``oracle.decoder`` chains this MoE layer into a
+stack of decoder blocks (attention over a KV cache, norms, residual stream). Every function here is pinned by ``tests/test_oracle_*``
 against brute force, closed forms, invariants and a hand-simulated LRU trace.
 """
 from __future__ import annotations
@@ -92,6 +93,13 @@ def lib():
             L.orc_lru_admit.restype = i32
             L.orc_guided_step.argtypes = [i64, vp, vp, vp, vp, i64, vp, i32, i32, i32, vp]
             L.orc_guided_step.restype = i32
+            f64 = ctypes.c_double
+            L.orc_rmsnorm.argtypes = [vp, vp, i32, f64, vp]
+            L.orc_rmsnorm.restype = None
+            L.orc_rope.argtypes = [vp, i32, i64, f64, vp]
+            L.orc_rope.restype = None
+            L.orc_attend.argtypes = [vp, vp, vp, i32, i32, i64, i64, i32, vp, vp]
+            L.orc_attend.restype = None
             _lib = L
     return _lib
 

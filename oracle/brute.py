@@ -6,6 +6,7 @@ list instead of timestamps; the expert FFN is explicit Python loops.
 """
 from __future__ import annotations
 
+import cmath
 import math
 
 
@@ -210,3 +211,37 @@ class RotaryRing:
             self.ring[s] = g
             recs.append((g, 1, s, -1 if v is None else v))
         return recs
+
+
+def rmsnorm_brute(x, w, eps):
+    """Explicit loop: divide by the root of the mean square plus eps, then scale by w."""
+    ms = sum(v * v for v in x) / len(x)
+    r = math.sqrt(ms + eps)
+    return [w[i] * x[i] / r for i in range(len(x))]
+
+
+def rope_brute(x, pos, theta):
+    """Rotary embedding as complex multiplication: the pair (x_i, x_{i+D/2}) is the complex number
+    x_i + j x_{i+D/2}, multiplied by exp(j pos theta^(-2i/D))."""
+    D = len(x)
+    h = D // 2
+    out = [0.0] * D
+    for i in range(h):
+        c = complex(x[i], x[i + h]) * cmath.exp(1j * pos * theta ** (-2.0 * i / D))
+        out[i], out[i + h] = c.real, c.imag
+    return out
+
+
+def attend_brute(q, K, V, T):
+    """q [Hq][D], K/V [Hkv][>=T][D]: per query head, scores over positions, a softmax written out
+    with math.exp, and the weighted sum of value rows."""
+    Hq, Hkv, D = len(q), len(K), len(q[0])
+    out = []
+    for h in range(Hq):
+        g = h * Hkv // Hq
+        s = [sum(q[h][i] * K[g][j][i] for i in range(D)) / math.sqrt(D) for j in range(T)]
+        m = max(s)
+        e = [math.exp(v - m) for v in s]
+        tot = sum(e)
+        out.append([sum(e[j] / tot * V[g][j][i] for j in range(T)) for i in range(D)])
+    return out

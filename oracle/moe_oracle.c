@@ -435,3 +435,66 @@ int32_t orc_guided_step(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t*
   for (int32_t i = 0; i < n; i++) last_use[needed[i]] = clock;
   return n;
 }
+
+/* ---------------------------------------------------------------------------------------------
+ * The decoder block around the MoE layer (a chained stack: attention with a KV cache, then the
+ * MoE layer, each on a residual stream). The paper ran a whole MoE decoder with a 4096-token
+ * context; it prints no architecture, so these follow a Qwen3-MoE-class block.
+ * ------------------------------------------------------------------------------------------- */
+
+/* RMSNorm: out_i = w_i * x_i / sqrt(mean_j x_j^2 + eps). */
+void orc_rmsnorm(const double* x, const double* w, int32_t n, double eps, double* out) {
+  double ss = 0.0;
+  for (int32_t i = 0; i < n; i++) ss += x[i] * x[i];
+  const double r = 1.0 / sqrt(ss / (double)n + eps);
+  for (int32_t i = 0; i < n; i++) out[i] = w[i] * (x[i] * r);
+}
+
+/* Rotary position embedding of one head vector of even length D at position pos, pairing
+ * element i with element i + D/2 (rotate-half layout): with a_i = pos * theta^(-2i/D),
+ *   out_i       = x_i cos a_i - x_{i+D/2} sin a_i
+ *   out_{i+D/2} = x_{i+D/2} cos a_i + x_i sin a_i            for 0 <= i < D/2. */
+void orc_rope(const double* x, int32_t D, int64_t pos, double theta, double* out) {
+  const int32_t h = D / 2;
+  for (int32_t i = 0; i < h; i++) {
+    const double a = (double)pos * pow(theta, -2.0 * (double)i / (double)D);
+    const double c = cos(a), s = sin(a);
+    const double x0 = x[i], x1 = x[i + h];
+    out[i] = x0 * c - x1 * s;
+    out[i + h] = x1 * c + x0 * s;
+  }
+}
+
+/* Grouped-query attention of one query token over T cached positions.
+ * q [Hq x D]; K, V [Hkv x Tmax x D] (position j of kv head g at (g * Tmax + j) * D); Hq a multiple
+ * of Hkv, query head h reads kv head h / (Hq / Hkv). s_j = (q_h . K_gj) / sqrt(D) for j < T;
+ * w = softmax(s) (maximum subtracted); out_h = sum_j w_j V_gj. scratch holds T doubles. */
+void orc_attend(const double* q, const double* K, const double* V, int32_t Hq, int32_t Hkv, int64_t T, int64_t Tmax,
+                int32_t D, double* out, double* scratch) {
+  const int32_t group = Hq / Hkv;
+  const double scale = 1.0 / sqrt((double)D);
+  for (int32_t h = 0; h < Hq; h++) {
+    const int32_t g = h / group;
+    const double* qh = q + (int64_t)h * D;
+    double m = -INFINITY;
+    for (int64_t j = 0; j < T; j++) {
+      const double* kj = K + ((int64_t)g * Tmax + j) * D;
+      double acc = 0.0;
+      for (int32_t i = 0; i < D; i++) acc += qh[i] * kj[i];
+      scratch[j] = acc * scale;
+      if (scratch[j] > m) m = scratch[j];
+    }
+    double tot = 0.0;
+    for (int64_t j = 0; j < T; j++) {
+      scratch[j] = exp(scratch[j] - m);
+      tot += scratch[j];
+    }
+    double* oh = out + (int64_t)h * D;
+    for (int32_t i = 0; i < D; i++) oh[i] = 0.0;
+    for (int64_t j = 0; j < T; j++) {
+      const double wj = scratch[j] / tot;
+      const double* vj = V + ((int64_t)g * Tmax + j) * D;
+      for (int32_t i = 0; i < D; i++) oh[i] += wj * vj[i];
+    }
+  }
+}

@@ -287,3 +287,107 @@ def act_to_f64(raw: np.ndarray, adtype: str) -> np.ndarray:
     if adtype == "fp32":
         return raw.astype(np.float64)
     return bf16_bits_to_f32(raw).astype(np.float64)
+
+
+# ----------------------------------------------------------------------------------------------
+# decoder blocks around the MoE layer (attention with a KV cache, norms, a residual stream)
+
+# matrix ids of a layer's attention weights in the weight streams (experts use 0-2, the router 3)
+_ATTN_MATRIX = {"wq": 4, "wk": 5, "wv": 6, "wo": 7}
+_NORM_MATRIX = {"in": 8, "post": 9, "q": 10, "k": 11}
+_KV_MATRIX = {"k": 12, "v": 13}
+TOKEN_INPUT_SEED = 1 << 20  # seed of the token-input streams (layers use seeds 0..L-1)
+
+
+@dataclass(frozen=True)
+class DecoderWorkload:
+    """A chained stack of decoder blocks: per layer, x += W_o attn(...) then x += MoE(...).
+
+    moe: the MoE layer's workload (its n_layers is the stack depth, its wdtype/adtype the storage
+    of every weight and of the KV cache). ctx: positions already in the KV cache when the first
+    decode token arrives (a seeded N(0, 1) prefix). The attention follows a Qwen3-MoE-class block:
+    grouped-query heads with per-head RMSNorm on q and k and rotary positions.
+    """
+
+    name: str
+    moe: Workload
+    n_heads: int
+    n_kv_heads: int
+    head_dim: int
+    ctx: int
+    eps: float = 1e-6
+    rope_theta: float = 1e6
+    norm_std: float = 0.1  # RMSNorm weights are 1 + N(0, norm_std^2)
+    description: str = field(default="", compare=False)
+
+    def replace(self, **kw) -> "DecoderWorkload":
+        from dataclasses import replace
+
+        return replace(self, **kw)
+
+
+DECODERS = {
+    "tiny_block_fp32": DecoderWorkload(
+        "tiny_block_fp32", WORKLOADS["tiny_fp32"].replace(n_layers=2, tokens=8, cap_slots=6),
+        n_heads=4, n_kv_heads=2, head_dim=64, ctx=24,
+        description="2 tiny fp32 decoder blocks (d=256, 4 query / 2 kv heads of 64, E=8, top-2), 24 cached positions"),
+    "block48_bf16": DecoderWorkload(
+        "block48_bf16", WORKLOADS["stack48_bf16"], n_heads=32, n_kv_heads=4, head_dim=128, ctx=4095,
+        description="48 Qwen3-30B-A3B-class decoder blocks, bf16, 4095 cached positions (context 4096), 6 GB pool"),
+}
+
+
+def _store(x: np.ndarray, dtype: str) -> np.ndarray:
+    """fp32 values -> raw storage of dtype (float32, or bf16 bits)."""
+    if dtype == "fp32":
+        return np.ascontiguousarray(x, dtype=np.float32)
+    return f32_to_bf16_bits(x)
+
+
+def attention_weights(dw: DecoderWorkload, layer: int) -> dict:
+    """Raw storage of one layer's attention and norm weights: wq [Hq*Dh x d], wk and wv
+    [Hkv*Dh x d], wo [d x Hq*Dh] (out x in, N(0, 1/fan_in)); norm_in and norm_post [d], norm_q and
+    norm_k [Dh] (1 + N(0, norm_std^2)). fp32 workloads: float32; otherwise bf16 bits."""
+    wl = dw.moe
+    dt = "fp32" if wl.wdtype == "fp32" else "bf16"
+    code = WDTYPES[dt]
+    d, qd, kd = wl.d, dw.n_heads * dw.head_dim, dw.n_kv_heads * dw.head_dim
+    out = {}
+    for name, (rows, cols) in (("wq", (qd, d)), ("wk", (kd, d)), ("wv", (kd, d)), ("wo", (d, qd))):
+        w = np.empty((rows, cols), dtype=np.float32 if code == 0 else np.uint16)
+        tmp = np.empty(rows * cols, dtype=np.float32)
+        rc = lib().synth_weight(wl.weight_seed, layer, 0, _ATTN_MATRIX[name], rows, cols, code, _p(w), None, _p(tmp))
+        assert rc == 0
+        out[name] = w
+    for name, n in (("in", d), ("post", d), ("q", dw.head_dim), ("k", dw.head_dim)):
+        stream = lib().synth_weight_stream(layer, 0, _NORM_MATRIX[name])
+        out["norm_" + name] = _store(1.0 + normal(wl.weight_seed, stream, 0, n, dw.norm_std), dt)
+    return out
+
+
+def kv_prefix(dw: DecoderWorkload, layer: int) -> tuple[np.ndarray, np.ndarray]:
+    """The KV cache contents of one layer before the first decode token: K and V [Hkv x ctx x Dh],
+    N(0, 1), in the activation storage (float32, or bf16 bits)."""
+    wl = dw.moe
+    n = dw.n_kv_heads * dw.ctx * dw.head_dim
+    kv = []
+    for name in ("k", "v"):
+        stream = lib().synth_weight_stream(layer, 0, _KV_MATRIX[name])
+        kv.append(_store(normal(wl.weight_seed, stream, 0, n, 1.0), wl.adtype).reshape(
+            dw.n_kv_heads, dw.ctx, dw.head_dim))
+    return kv[0], kv[1]
+
+
+def token_inputs(dw: DecoderWorkload, tokens: int | None = None, seq: int = 0) -> np.ndarray:
+    """The residual stream entering layer 0 at each decode token: an AR(1) stream (the MoE
+    workload's rho) [T x d] in the activation storage."""
+    wl = dw.moe
+    T = wl.tokens if tokens is None else tokens
+    h = ar1(TOKEN_INPUT_SEED, HIDDEN_STREAM_TAG | seq, T, wl.d, wl.rho)
+    if wl.adtype == "fp32":
+        out = np.empty(h.shape, dtype=np.float32)
+        lib().synth_f64_to_f32(_p(h), _p(out), h.size)
+    else:
+        out = np.empty(h.shape, dtype=np.uint16)
+        lib().synth_f64_to_bf16(_p(h), _p(out), h.size)
+    return out
