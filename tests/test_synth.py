@@ -112,3 +112,41 @@ def test_weight_shapes_and_scale():
     r = synth.bf16_bits_to_f32(synth.router_weights(wb, 0)).astype(np.float64)
     assert r.shape == (wb.n_experts, wb.d)
     assert abs(r.std() * math.sqrt(wb.d) - 1.0) < 0.01  # std = 1 / sqrt(fan_in)
+
+
+def test_decoder_inputs_shapes_scales_and_independence():
+    dw = synth.DECODERS["tiny_block_fp32"]
+    wl = dw.moe
+    a0, a1 = synth.attention_weights(dw, 0), synth.attention_weights(dw, 1)
+    qd, kd = dw.n_heads * dw.head_dim, dw.n_kv_heads * dw.head_dim
+    assert a0["wq"].shape == (qd, wl.d) and a0["wk"].shape == (kd, wl.d) and a0["wo"].shape == (wl.d, qd)
+    # N(0, 1/fan_in) projections, 1 + N(0, 0.1^2) norm weights
+    np.testing.assert_allclose(a0["wq"].std() * np.sqrt(wl.d), 1.0, rtol=0.05)
+    np.testing.assert_allclose(a0["wo"].std() * np.sqrt(qd), 1.0, rtol=0.05)
+    np.testing.assert_allclose(a0["norm_in"].mean(), 1.0, atol=0.03)
+    np.testing.assert_allclose(a0["norm_in"].std(), dw.norm_std, rtol=0.2)
+    # layers and matrices draw from different streams; none collides with the router or experts
+    assert not np.array_equal(a0["wq"], a1["wq"])
+    assert not np.array_equal(a0["wk"][:, :], a0["wv"][:, :])
+    r0 = synth.router_weights(wl, 0)
+    assert not np.array_equal(a0["wq"][:wl.n_experts], r0)
+    K, V = synth.kv_prefix(dw, 0)
+    assert K.shape == V.shape == (dw.n_kv_heads, dw.ctx, dw.head_dim)
+    assert not np.array_equal(K, V)
+    x = synth.token_inputs(dw, 200).astype(np.float64)
+    # AR(1): lag-1 correlation rho, unit variance
+    c = (x[1:] * x[:-1]).mean() / (x * x).mean()
+    np.testing.assert_allclose(c, wl.rho, atol=0.05)
+    np.testing.assert_allclose(x.var(), 1.0, atol=0.15)
+    np.testing.assert_array_equal(synth.token_inputs(dw, 5), synth.token_inputs(dw, 200)[:5])
+
+
+def test_decoder_inputs_bf16_storage():
+    dw = synth.DECODERS["tiny_block_fp32"].replace(
+        moe=synth.WORKLOADS["tiny_fp32"].replace(wdtype="bf16", adtype="bf16", n_layers=2))
+    a = synth.attention_weights(dw, 0)
+    assert a["wq"].dtype == np.uint16 and a["norm_q"].dtype == np.uint16
+    f = synth.attention_weights(synth.DECODERS["tiny_block_fp32"], 0)
+    np.testing.assert_array_equal(a["wq"], synth.f32_to_bf16_bits(f["wq"]))
+    K, _ = synth.kv_prefix(dw, 1)
+    assert K.dtype == np.uint16
