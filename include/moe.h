@@ -102,7 +102,7 @@ enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
  *     that use information produced during execution (Sec. 3). Each layer keeps the rank of every
  *     expert in its most recent routing (0 = highest logit; for a batch, the best rank over its
  *     sequences). A miss takes the lowest free slot, else evicts the resident not needed this
- *     layer-step with the largest rank, ties to the older use, then to the lower global id.
+ *     layer-step with the largest rank, ties to the more recent use, then to the lower global id.
  *     Residency planner only for now (moe_create rejects it). */
 enum { MOE_POLICY_LRU = 0, MOE_POLICY_ROTARY = 1, MOE_POLICY_GUIDED = 2 };
 

@@ -275,7 +275,7 @@ class GuidedTable:
     decisions that use information produced during execution, Sec. 3): every layer keeps the rank of
     each of its experts in its most recent routing (the best rank over a batch's sequences; E before
     the layer is first routed). A miss takes the lowest free slot, else evicts the resident outside
-    the layer-step's needed set with the largest rank, ties to the least recent use, then to the
+    the layer-step's needed set with the largest rank, ties to the most recent use, then to the
     lower global id. See orc_guided_step."""
 
     def __init__(self, n_gid: int, cap: int, n_experts: int):

@@ -134,9 +134,9 @@ def ranks_brute(z):
 class GuidedResidents:
     """Router-guided replacement kept as a dict of residents and a free list.
 
-    The victim is chosen by comparing every evictable resident's (rank, age, id) in one max():
-    largest rank first, then the oldest use, then the lowest id. Misses in ascending id take the
-    lowest free slot first; every needed id is stamped with the step counter afterwards.
+    The victim is chosen by comparing every evictable resident's (rank, last use, id) in one max():
+    largest rank first, then the most recent use, then the lowest id. Misses in ascending id take
+    the lowest free slot first; every needed id is stamped with the step counter afterwards.
     """
 
     def __init__(self, cap, n_experts):
@@ -166,13 +166,56 @@ class GuidedResidents:
                 cands = [v for v in self.slot if v not in needed]
                 if not cands:
                     raise RuntimeError("capacity below the step's working set")
-                victim = max(cands, key=lambda v: (self.rank.get(v, self.E), -self.last.get(v, -1), -v))
+                victim = max(cands, key=lambda v: (self.rank.get(v, self.E), self.last.get(v, -1), -v))
                 s = self.slot.pop(victim)
             self.slot[g] = s
             recs.append((g, 1, s, victim))
         for g in needed:
             self.last[g] = self.t
         self.t += 1
+        return recs
+
+
+class RecencyListMRU(RecencyListLRU):
+    """The recency list with the most recent evictable resident as the victim (newest first; among
+    ids of the same step, the lowest id)."""
+
+    def __init__(self, cap):
+        super().__init__(cap)
+        self.t = 0
+        self.stamp = {}  # id -> the step it was last used in
+
+    def step(self, needed):
+        needed = sorted(set(needed))
+        pinned = set(needed)
+        recs = []
+        for g in needed:
+            if g in self.slot:
+                recs.append((g, 0, self.slot[g], -1))
+                continue
+            if self.free:
+                s = min(self.free)
+                self.free.remove(s)
+                victim = -1
+            else:
+                group = []  # the newest step's evictable ids, then older steps
+                for v in reversed(self.order):
+                    if v in pinned:
+                        continue
+                    if group and self.stamp[v] != self.stamp[group[0]]:
+                        break
+                    group.append(v)
+                if not group:
+                    raise RuntimeError("capacity below the step's working set")
+                victim = min(group)
+                self.order.remove(victim)
+                s = self.slot.pop(victim)
+            self.slot[g] = s
+            recs.append((g, 1, s, victim))
+        self.t += 1
+        for g in needed:
+            self.stamp[g] = self.t
+        self.order = [v for v in self.order if v not in pinned] + needed
         return recs
 
 

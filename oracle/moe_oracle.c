@@ -376,7 +376,8 @@ int32_t orc_lru_admit(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t* l
  * logit), n_experts for a layer not routed yet; the caller refreshes the layer's ranks before the
  * call. For each needed gid in ascending order: if resident, a hit. Otherwise the lowest free
  * slot, else the slot of the resident v outside `needed` with the largest rank[v], ties to the
- * smaller last_use[v], then to the lower v. Afterwards last_use[x] = clock for every needed x.
+ * larger last_use[v] (the more recent use), then to the lower v. Afterwards last_use[x] = clock
+ * for every needed x.
  *
  * Returns the number of records, or -1 if no victim exists (cap < |needed|).
  */
@@ -414,7 +415,7 @@ int32_t orc_guided_step(int64_t cap, int32_t* slot_of, int32_t* gid_of, int64_t*
         else if (rank[v] != rank[victim])
           better = rank[v] > rank[victim];
         else if (last_use[v] != last_use[victim])
-          better = last_use[v] < last_use[victim];
+          better = last_use[v] > last_use[victim];
         else
           better = v < victim;
         if (better) {

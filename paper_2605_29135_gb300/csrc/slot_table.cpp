@@ -57,7 +57,7 @@ int32_t SlotTable::guided_victim() {
     if (v < 0 || mark_[v]) continue;
     if (victim < 0 || rank_[v] > rank_[victim] ||
         (rank_[v] == rank_[victim] &&
-         (last_use_[v] < last_use_[victim] || (last_use_[v] == last_use_[victim] && v < victim))))
+         (last_use_[v] > last_use_[victim] || (last_use_[v] == last_use_[victim] && v < victim))))
       victim = v;
   }
   return victim;

@@ -14,8 +14,8 @@
 //   Router-guided (MOE_POLICY_GUIDED): each id carries its rank in its layer's most recent routing
 //     (set_ranks, before the layer's step; n_experts until the layer is first routed). A missing
 //     id takes the lowest free slot, else the slot of the resident the step does not need with the
-//     largest rank, ties to the smaller last use, then to the lower id. Every needed id then gets
-//     the step's clock as its last use.
+//     largest rank, ties to the larger (more recent) last use, then to the lower id. Every needed
+//     id then gets the step's clock as its last use.
 // Prefetch admission (LRU only; one reading of the paper's residency decisions that use
 // information produced during execution, Sec. 3): after a step, candidate ids (ascending) that are
 // absent take the lowest free slot, else the slot of the resident with the smallest (last use, id)
@@ -74,7 +74,7 @@ class SlotTable {
  private:
   int32_t take_free();
   int32_t lru_victim();     // resident with the smallest (last use, id) not marked; -1 when none
-  int32_t guided_victim();  // resident with the largest (rank, -last use, -id) not marked; -1 when none
+  int32_t guided_victim();  // resident with the largest (rank, last use, -id) not marked; -1 when none
 
   int64_t n_gid_ = 0, cap_ = 0;
   int32_t policy_ = 0;
