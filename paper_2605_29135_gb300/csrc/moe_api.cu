@@ -17,6 +17,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <chrono>
@@ -33,6 +34,26 @@
 #include "slot_table.h"
 
 namespace {
+
+// NVTX range over a scope, optionally tagged with an integer (a layer): visible to nsys and to
+// ncu --nvtx, a no-op when no tool is attached.
+struct NvtxRange {
+  explicit NvtxRange(const char* name, int tag = -1) {
+    nvtxEventAttributes_t a{};
+    a.version = NVTX_VERSION;
+    a.size = NVTX_EVENT_ATTRIB_STRUCT_SIZE;
+    a.messageType = NVTX_MESSAGE_TYPE_ASCII;
+    a.message.ascii = name;
+    if (tag >= 0) {
+      a.payloadType = NVTX_PAYLOAD_TYPE_INT32;
+      a.payload.iValue = tag;
+    }
+    nvtxRangePushEx(&a);
+  }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 constexpr double kWaitTimeoutS = 20.0;
 // CTAs of the fused kernel that stream missed experts: enough warps to keep the host link's
@@ -386,7 +407,11 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
   std::vector<int32_t> rank_gid(k);
   for (int32_t l = 0; l < L; l++) {
     const void* hid_l = (const uint8_t*)hidden + (int64_t)l * act_row;
-    st = wait_route(h, h->route_seq, s);
+    NvtxRange layer_range("layer", l);
+    {
+      NvtxRange r("wait for routing", l);
+      st = wait_route(h, h->route_seq, s);
+    }
     if (st != MOE_OK) return st;
     if (h->prof) harvest(h, false);
     // routing result of layer l
@@ -405,7 +430,10 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     for (size_t i = 1; i < needs.size(); i++)
       if (needs[i].gid == needs[i - 1].gid) return fail(h, MOE_ERR_INVALID, "router produced duplicate expert ids");
     const int64_t clock = h->token_step * L + l + 1;  // 0 is older than every step (preloaded experts)
-    st = residency_step(h, l, needs, clock);
+    {
+      NvtxRange r("slot lookup", l);
+      st = residency_step(h, l, needs, clock);
+    }
     if (st != MOE_OK) return st;
     h->stats.layer_steps++;
     // selective loads: misses in ascending gid on the copy stream
@@ -1004,6 +1032,7 @@ moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t
                                                    std::to_string(g / h->cfg.n_experts) + " not registered");
     h->all_registered = true;
   }
+  NvtxRange range(h->dev_mode ? "moe_decode_step (device schedule)" : "moe_decode_step (host schedule)");
   moe_status st = h->dev_mode ? decode_device(h, hidden, out, batch, (cudaStream_t)stream)
                               : decode_impl(h, hidden, out, (cudaStream_t)stream);
   if (st != MOE_OK) {
@@ -1023,11 +1052,13 @@ moe_status moe_decode_step_host(moe_handle* h, const void* hidden_host, void* ou
   if (!hidden_host || !out_host) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
   if (batch < 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be in [1, max_batch]");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
+  NvtxRange range("moe_decode_step_host");
   const int64_t bytes = (int64_t)h->cfg.n_layers * batch * h->cfg.d * h->asize;
   MOE_CK(h, cudaMemcpyAsync(h->hid_dev, hidden_host, bytes, cudaMemcpyHostToDevice, h->host_stream));
   moe_status st = moe_decode_step(h, h->hid_dev, h->out_dev, batch, h->host_stream);
   if (st != MOE_OK) return st;
   MOE_CK(h, cudaMemcpyAsync(out_host, h->out_dev, bytes, cudaMemcpyDeviceToHost, h->host_stream));
+  NvtxRange wait_range("wait for the step and its copies");
   MOE_CK(h, cudaStreamSynchronize(h->host_stream));
   return MOE_OK;
 }
@@ -1107,6 +1138,7 @@ moe_status moe_reset_residency(moe_handle* h) {
 
 moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
   if (!h) return MOE_ERR_INVALID;
+  NvtxRange range("moe_preload");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   if (!h->all_registered) {
     for (int64_t g = 0; g < h->n_gid; g++)
