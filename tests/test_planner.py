@@ -247,3 +247,46 @@ def test_guided_rank_arguments_are_checked():
     with Planner(1, 8, 4, "lru") as p:
         with pytest.raises(MoEError):
             p.step(0, 0, [1, 2], ranks=np.arange(8))
+
+
+def test_random_configurations_match_the_oracle():
+    # property check over random shapes, caps, policies, batches and prefetch depths
+    hyp = pytest.importorskip("hypothesis")
+    st = hyp.strategies
+
+    @hyp.settings(max_examples=60, deadline=None, derandomize=True)
+    @hyp.given(L=st.integers(1, 4), E=st.integers(2, 24), data=st.data(), policy=st.sampled_from(["lru", "rotary", "guided"]),
+               seed=st.integers(0, 2 ** 31 - 1))
+    def check(L, E, data, policy, seed):
+        k = data.draw(st.integers(1, E))
+        B = data.draw(st.integers(1, 3))
+        need_max = min(E, k * B)
+        cap = data.draw(st.integers(need_max, L * E + 2))
+        m = data.draw(st.integers(0, E - k)) if policy == "lru" else 0
+        preload = data.draw(st.booleans())
+        rng = np.random.default_rng(seed)
+        table = oracle.TABLES[policy](L * E, min(cap, L * E), E)
+        with Planner(L, E, cap, policy) as p:
+            if preload:
+                table.preload()
+                p.preload()
+            for tok in range(6):
+                for l in range(L):
+                    used, pf, best = set(), set(), np.full(E, E, dtype=np.int32)
+                    for _ in range(B):
+                        order = [int(e) for e in rng.permutation(E)]
+                        used.update(order[:k])
+                        pf.update(order[k:k + m])
+                        best = np.minimum(best, _ranks_of(order))
+                    pf -= used
+                    clock = tok * L + l
+                    if policy == "guided":
+                        table.set_layer_ranks(l, best)
+                    want = table.step(clock, [l * E + e for e in used], tok)
+                    if pf:
+                        want = np.concatenate([want, table.admit(clock, [l * E + e for e in used],
+                                                                 [l * E + e for e in pf], tok)])
+                    got = p.step(tok, l, sorted(used), sorted(pf), ranks=best if policy == "guided" else None)
+                    assert _tuples(got, E) == _tuples(want, E)
+
+    check()
