@@ -13,6 +13,18 @@
  * paper does not disclose its replacement policy, so the residency step here
  * is a deterministic LRU with lower-id ties (see orc_lru_step).
  *
+ * Contents, in file order:
+ *   widening of stored weights; matvec, softmax, top-k, the router; the SwiGLU
+ *     expert FFN and the combine (one MoE layer);
+ *   residency steps: LRU (orc_lru_step), our reading of the rotary slot group
+ *     (orc_rotary_step, Fig. 1/2), prefetch admission after an LRU step
+ *     (orc_lru_admit) and router-guided replacement (orc_guided_step), the
+ *     last two readings of the paper's residency decisions that use
+ *     information produced during execution (Sec. 3);
+ *   the decoder block around the MoE layer: RMSNorm, rotary positions and
+ *     grouped-query attention over a KV cache (orc_rmsnorm, orc_rope,
+ *     orc_attend), chained by oracle/decoder.py.
+ *
  * Everything is plain fp64 arithmetic on exactly widened inputs, one rounded
  * operation at a time (built with -ffp-contract=off, no fast-math), sums in
  * ascending index order. Rows of a matrix-vector product may be spread over
