@@ -58,16 +58,51 @@ REC_DTYPE = np.dtype([("step", np.int32), ("layer", np.int32), ("expert", np.int
                       ("slot", np.int32), ("evicted", np.int32)])
 
 
+def compile_source(src: str, out: str) -> str:
+    """Compile an oracle C source to a shared library (plain C, fp64, OpenMP over matrix rows)."""
+    tmp = out + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-fPIC", "-shared", "-o", tmp, src, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
 def build(force: bool = False) -> str:
-    """Compile liboracle.so in-tree (plain C, fp64, OpenMP over matrix rows)."""
+    """Compile liboracle.so in-tree."""
     if not force and os.path.exists(_LIB_PATH) and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC):
         return _LIB_PATH
-    tmp = _LIB_PATH + f".tmp{os.getpid()}"
-    cmd = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-fPIC", "-shared", "-o", tmp, _SRC,
-           "-lm"]
-    subprocess.run(cmd, check=True)
-    os.replace(tmp, _LIB_PATH)
-    return _LIB_PATH
+    return compile_source(_SRC, _LIB_PATH)
+
+
+def load_library(path: str):
+    """Load a compiled oracle library and declare its signatures (used by lib(); tests also load
+    deliberately broken builds of the same source through it)."""
+    L = ctypes.CDLL(path)
+    vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    L.orc_widen.argtypes = [ctypes.c_int, vp, vp, i64, i64, vp]
+    L.orc_widen.restype = ctypes.c_int
+    L.orc_matvec.argtypes = [vp, vp, i64, i64, vp]
+    L.orc_softmax.argtypes = [vp, i64, vp]
+    L.orc_topk.argtypes = [vp, i64, i32, vp, vp]
+    L.orc_router.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp]
+    L.orc_expert_ffn.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp]
+    L.orc_combine.argtypes = [vp, vp, i32, i32, vp]
+    L.orc_lru_step.argtypes = [i64, vp, vp, vp, i64, vp, i32, i32, i32, vp]
+    L.orc_lru_step.restype = i32
+    L.orc_rotary_step.argtypes = [i64, vp, vp, vp, vp, vp, i32, i32, i32, vp]
+    L.orc_rotary_step.restype = i32
+    L.orc_lru_admit.argtypes = [i64, vp, vp, vp, i64, vp, i32, vp, i32, i32, i32, vp]
+    L.orc_lru_admit.restype = i32
+    L.orc_guided_step.argtypes = [i64, vp, vp, vp, vp, i64, vp, i32, i32, i32, vp]
+    L.orc_guided_step.restype = i32
+    f64 = ctypes.c_double
+    L.orc_rmsnorm.argtypes = [vp, vp, i32, f64, vp]
+    L.orc_rmsnorm.restype = None
+    L.orc_rope.argtypes = [vp, i32, i64, f64, vp]
+    L.orc_rope.restype = None
+    L.orc_attend.argtypes = [vp, vp, vp, i32, i32, i64, i64, i32, vp, vp]
+    L.orc_attend.restype = None
+    return L
 
 
 def lib():
@@ -75,31 +110,7 @@ def lib():
     with _lock:
         if _lib is None:
             build()
-            L = ctypes.CDLL(_LIB_PATH)
-            vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
-            L.orc_widen.argtypes = [ctypes.c_int, vp, vp, i64, i64, vp]
-            L.orc_widen.restype = ctypes.c_int
-            L.orc_matvec.argtypes = [vp, vp, i64, i64, vp]
-            L.orc_softmax.argtypes = [vp, i64, vp]
-            L.orc_topk.argtypes = [vp, i64, i32, vp, vp]
-            L.orc_router.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp]
-            L.orc_expert_ffn.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp]
-            L.orc_combine.argtypes = [vp, vp, i32, i32, vp]
-            L.orc_lru_step.argtypes = [i64, vp, vp, vp, i64, vp, i32, i32, i32, vp]
-            L.orc_lru_step.restype = i32
-            L.orc_rotary_step.argtypes = [i64, vp, vp, vp, vp, vp, i32, i32, i32, vp]
-            L.orc_rotary_step.restype = i32
-            L.orc_lru_admit.argtypes = [i64, vp, vp, vp, i64, vp, i32, vp, i32, i32, i32, vp]
-            L.orc_lru_admit.restype = i32
-            L.orc_guided_step.argtypes = [i64, vp, vp, vp, vp, i64, vp, i32, i32, i32, vp]
-            L.orc_guided_step.restype = i32
-            f64 = ctypes.c_double
-            L.orc_rmsnorm.argtypes = [vp, vp, i32, f64, vp]
-            L.orc_rmsnorm.restype = None
-            L.orc_rope.argtypes = [vp, i32, i64, f64, vp]
-            L.orc_rope.restype = None
-            L.orc_attend.argtypes = [vp, vp, vp, i32, i32, i64, i64, i32, vp, vp]
-            L.orc_attend.restype = None
+            L = load_library(_LIB_PATH)
             _lib = L
     return _lib
 
