@@ -99,3 +99,60 @@ def test_pins_catch_the_planted_mistake(name, tmp_path):
     finally:
         oracle._lib = real
     RTR.test_ties_break_toward_lower_id()  # the real build is back
+
+
+def _decoder_mutants():
+    """Mistakes in the decoder stack's Python orchestration, as replacement methods."""
+    import numpy as np
+
+    from oracle import decoder as D
+
+    orig_attention = D.DecoderOracle.attention
+
+    def rope_position_off_by_one(self, l, x):
+        orig = D.rope
+        D.rope = lambda v, pos, theta: orig(v, pos + 1, theta)
+        try:
+            return orig_attention(self, l, x)
+        finally:
+            D.rope = orig
+
+    def value_not_cached(self, l, x):
+        out = orig_attention(self, l, x)
+        self.V[l, :, self.pos] = 0.0  # the new position's value row is lost for later tokens
+        return out
+
+    def wrong_norm_weights(self, l, x):
+        w = self.attn_w[l]
+        saved = w["norm_in"]
+        w["norm_in"] = w["norm_post"]
+        try:
+            return orig_attention(self, l, x)
+        finally:
+            w["norm_in"] = saved
+
+    def no_qk_norm(self, l, x):
+        orig = D.rmsnorm
+        calls = {"n": 0}
+
+        def rms(v, w, eps):
+            calls["n"] += 1
+            return orig(v, w, eps) if calls["n"] == 1 else np.asarray(v, dtype=np.float64)
+
+        D.rmsnorm = rms
+        try:
+            return orig_attention(self, l, x)
+        finally:
+            D.rmsnorm = orig
+
+    return {"rotary position off by one": rope_position_off_by_one, "value row not cached": value_not_cached,
+            "input norm uses the post-attention weights": wrong_norm_weights, "no q/k norm": no_qk_norm}
+
+
+@pytest.mark.parametrize("name", list(_decoder_mutants()))
+def test_decoder_pin_catches_the_planted_mistake(name, monkeypatch):
+    from oracle import decoder as D
+
+    monkeypatch.setattr(D.DecoderOracle, "attention", _decoder_mutants()[name])
+    with pytest.raises(Exception):
+        DEC.test_incremental_decode_equals_the_matrix_form()
