@@ -252,6 +252,29 @@ class Planner:
             raise err
         return recs
 
+    def run(self, idx, ranks=None, prefetch=None, first_step: int = 0) -> dict:
+        """Replay a recorded routing sequence: idx int [T x L x B x k] (or [T x L x k]) expert ids,
+        as moe_get_last_routing returns them step by step; ranks [T x L x E] for the "guided"
+        policy; prefetch [T x L x m] candidates (LRU only). Returns the records and per-step counts:
+        {"records", "hits", "misses", "prefetches", "evictions", "hit_rate"}."""
+        idx = np.asarray(idx)
+        if idx.ndim == 3:
+            idx = idx[:, :, None, :]
+        T, L = idx.shape[0], idx.shape[1]
+        if L != self.n_layers:
+            raise ValueError(f"idx has {L} layers, the planner {self.n_layers}")
+        recs = []
+        for t in range(T):
+            for l in range(L):
+                recs.append(self.step(first_step + t, l, idx[t, l].ravel(),
+                                      () if prefetch is None else np.asarray(prefetch[t][l]).ravel(),
+                                      None if ranks is None else ranks[t][l]))
+        records = np.concatenate(recs) if recs else np.zeros(0, dtype=TRACE_DTYPE)
+        kind = records["kind"]
+        hits, misses = int((kind == 0).sum()), int((kind == 1).sum())
+        return {"records": records, "hits": hits, "misses": misses, "prefetches": int((kind == 2).sum()),
+                "evictions": int((records["evicted"] >= 0).sum()), "hit_rate": hits / max(1, hits + misses)}
+
     def destroy(self):
         if getattr(self, "h", None):
             self.lib.moe_planner_destroy(self.h)

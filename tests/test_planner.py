@@ -290,3 +290,22 @@ def test_random_configurations_match_the_oracle():
                     assert _tuples(got, E) == _tuples(want, E)
 
     check()
+
+
+def test_run_replays_a_recorded_routing_like_the_oracle():
+    # the oracle's routing of a small stack, replayed in one call: same records, counts from them
+    wl = synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, tokens=16)
+    hidden = synth.hidden_all(wl)
+    orc = oracle.Oracle.for_workload(wl, cap_slots=6, keep_slot_copies=False, policy="guided")
+    steps = [orc.decode_step(hidden[t], compute_out=False) for t in range(wl.tokens)]
+    idx = np.stack([s.idx for s in steps])  # [T x L x B x k]
+    ranks = np.stack([[oracle.route_ranks(s.z[l, 0]) for l in range(wl.n_layers)] for s in steps])
+    with Planner(wl.n_layers, wl.n_experts, 6, "guided") as p:
+        res = p.run(idx, ranks=ranks)
+    want = np.concatenate([s.records for s in steps])
+    assert _tuples(res["records"], wl.n_experts) == _tuples(want, wl.n_experts)
+    assert res["hits"] == int((want["kind"] == 0).sum()) and res["misses"] == int((want["kind"] == 1).sum())
+    assert 0.0 < res["hit_rate"] < 1.0 and res["prefetches"] == 0
+    with Planner(wl.n_layers, wl.n_experts, 6) as p:
+        with pytest.raises(ValueError):
+            p.run(idx[:, :2])
