@@ -98,3 +98,18 @@ def test_create_rejects_the_guided_policy_for_decoding():
     with pytest.raises(P.MoEError) as ei:
         P.MoE(cfg)
     assert ei.value.status == -1 and "planner" in str(ei.value)
+
+
+@pytest.mark.parametrize("lang,std", [("c", "c99"), ("c++", "c++11")])
+def test_header_compiles_as_plain_c_and_cpp(lang, std, tmp_path):
+    # the boundary is a C ABI: the header must stand alone in C as well as C++
+    import shutil
+    import subprocess
+
+    cc = shutil.which("gcc" if lang == "c" else "g++")
+    if cc is None:
+        pytest.skip("no host compiler")
+    src = tmp_path / ("use.c" if lang == "c" else "use.cpp")
+    src.write_text('#include "moe.h"\nint main(void) { moe_config c; (void)c; return (int)sizeof(moe_trace_rec) - 24; }\n')
+    subprocess.run([cc, f"-std={std}", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", os.path.join(ROOT, "include"),
+                    "-fsyntax-only", str(src)], check=True)
