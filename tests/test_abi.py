@@ -113,3 +113,15 @@ def test_header_compiles_as_plain_c_and_cpp(lang, std, tmp_path):
     src.write_text('#include "moe.h"\nint main(void) { moe_config c; (void)c; return (int)sizeof(moe_trace_rec) - 24; }\n')
     subprocess.run([cc, f"-std={std}", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", os.path.join(ROOT, "include"),
                     "-fsyntax-only", str(src)], check=True)
+
+
+def test_binding_argument_counts_match_the_header(lib):
+    # every prototype in include/moe.h takes as many arguments as the ctypes declaration passes
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    protos = re.findall(r"\b(moe_[a-z_]+)\s*\(([^)]*)\)\s*;", src)
+    assert len(protos) == len(_declared())
+    for name, params in protos:
+        params = " ".join(params.split())
+        n = 0 if params in ("", "void") else params.count(",") + 1
+        assert len(getattr(lib, name).argtypes) == n, name
