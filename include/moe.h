@@ -273,7 +273,9 @@ moe_status moe_inject_fault(moe_handle* h, int32_t kind);
  * streams or host threads) race on it and must be serialised by the caller.
  * Returns MOE_ERR_CAPACITY if rows > MOE_NOALLOC_MAX_ROWS or n_experts > MOE_NOALLOC_MAX_EXPERTS,
  * MOE_ERR_INVALID for other bad arguments (top_k > 16 or > n_experts, d * element bytes not a
- * multiple of 16 or above 48 KiB, NULL pointers), MOE_ERR_CUDA if a launch fails. */
+ * multiple of 16 or above 48 KiB, NULL pointers, w_r or hidden not 16-byte aligned, idx or gate
+ * not 4-byte aligned), MOE_ERR_CUDA if a launch fails. Every argument check runs before any CUDA
+ * call. A logit that is NaN still yields expert ids inside [0, n_experts). */
 #define MOE_NOALLOC_MAX_ROWS 64
 #define MOE_NOALLOC_MAX_EXPERTS 256
 moe_status moe_route_noalloc(const void* w_r, const void* hidden, int32_t rows, int32_t n_experts, int32_t d,

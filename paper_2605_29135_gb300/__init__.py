@@ -324,22 +324,36 @@ def route_noalloc(w_r, hidden, top_k: int, renorm: bool = True, stream=None):
     """Routing without any device allocation by the library (moe_route_noalloc).
 
     For callers that cannot allocate device memory at routing time: the logits go to a fixed
-    scratch array inside the library, and the caller passes its own outputs. w_r: device tensor
-    [E x d] (float32 or bfloat16); hidden: device tensor [rows x d] of the same dtype. Returns
-    (idx int32 [rows x top_k], gate float32 [rows x top_k]) as device tensors allocated by the
-    caller side here (torch), never by the library.
+    scratch array inside the library, and the caller passes its own outputs. w_r: contiguous
+    device tensor [E x d]; hidden: contiguous device tensor [rows x d] on the same device, both
+    float32 or both bfloat16. Returns (idx int32 [rows x top_k], gate float32 [rows x top_k]) as
+    device tensors allocated by the caller side here (torch), never by the library. The call runs
+    with hidden's device current (the library resolves its scratch array on the current device).
     """
     import torch
 
+    if not (isinstance(w_r, torch.Tensor) and isinstance(hidden, torch.Tensor)):
+        raise ValueError("w_r and hidden must be torch tensors")
+    if w_r.dim() != 2 or hidden.dim() != 2:
+        raise ValueError("w_r must be [E x d] and hidden [rows x d]")
+    if w_r.dtype != hidden.dtype or w_r.dtype not in (torch.float32, torch.bfloat16):
+        raise ValueError("w_r and hidden must both be float32 or both bfloat16")
+    if not (w_r.is_cuda and hidden.is_cuda) or w_r.device != hidden.device:
+        raise ValueError("w_r and hidden must be on one CUDA device")
+    if not (w_r.is_contiguous() and hidden.is_contiguous()):
+        raise ValueError("w_r and hidden must be contiguous")
     rows, d = hidden.shape
     E = w_r.shape[0]
+    if w_r.shape[1] != d:
+        raise ValueError(f"w_r has {w_r.shape[1]} columns, hidden has {d}")
     wd = DTYPE["fp32"] if w_r.dtype == torch.float32 else DTYPE["bf16"]
-    idx = torch.empty((rows, top_k), dtype=torch.int32, device=hidden.device)
-    gate = torch.empty((rows, top_k), dtype=torch.float32, device=hidden.device)
-    if stream is None:
-        stream = torch.cuda.current_stream(hidden.device)
-    st = _lib.load().moe_route_noalloc(_ptr(w_r), _ptr(hidden), rows, E, d, top_k, 1 if renorm else 0, wd,
-                                        _ptr(idx), _ptr(gate), ctypes.c_void_p(stream.cuda_stream))
+    with torch.cuda.device(hidden.device):
+        idx = torch.empty((rows, top_k), dtype=torch.int32, device=hidden.device)
+        gate = torch.empty((rows, top_k), dtype=torch.float32, device=hidden.device)
+        if stream is None:
+            stream = torch.cuda.current_stream(hidden.device)
+        st = _lib.load().moe_route_noalloc(_ptr(w_r), _ptr(hidden), rows, E, d, top_k, 1 if renorm else 0, wd,
+                                            _ptr(idx), _ptr(gate), ctypes.c_void_p(stream.cuda_stream))
     if st != 0:
         raise MoEError(st, "moe_route_noalloc rejected the arguments" if st != -3 else "moe_route_noalloc launch failed")
     return idx, gate

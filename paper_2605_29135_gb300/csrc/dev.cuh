@@ -110,7 +110,11 @@ __device__ __forceinline__ void stage16(uint4* dst, const void* src, int nbytes,
 // Order-preserving map of a float to uint32 (larger float -> larger key; -0 treated as +0).
 __device__ __forceinline__ uint32_t ord_key(float f) {
   uint32_t u = __float_as_uint(f == 0.0f ? 0.0f : f);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  const uint32_t key = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  // key 0 is reserved: the top-k selections use it for "taken or absent". The one float that
+  // would map to it, the negative NaN with every bit set, takes key 1 and sorts with the other
+  // negative NaNs, below -inf.
+  return key > 1u ? key : 1u;
 }
 __device__ __forceinline__ float key_value(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);

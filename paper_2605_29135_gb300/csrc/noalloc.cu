@@ -21,6 +21,7 @@
 
 #include "dev.cuh"
 #include "moe.h"
+#include "topk.cuh"
 
 namespace {
 
@@ -54,54 +55,17 @@ __global__ void __launch_bounds__(256) k_route_logits(const uint8_t* w, const ui
   if (lane == 0) z[b * MOE_NOALLOC_MAX_EXPERTS + e] = acc;
 }
 
-// Top-k and gates of row blockIdx.x, one warp.
+// Top-k and gates of row blockIdx.x, one warp: the decode kernels' own selection code.
 __global__ void __launch_bounds__(32) k_route_select(const float* z, int E, int k, int renorm, int32_t* idx,
                                                     float* gate) {
   const int b = blockIdx.x;
   const int lane = threadIdx.x;
-  const float* zb = z + b * MOE_NOALLOC_MAX_EXPERTS;
-  constexpr int PER = MOE_NOALLOC_MAX_EXPERTS / 32;
-  uint32_t key[PER];
-#pragma unroll
-  for (int j = 0; j < PER; j++) {
-    const int e = j * 32 + lane;
-    key[j] = e < E ? ord_key(zb[e]) : 0u;
-  }
-  float my_z = 0.f;
-  int my_i = -1;
-  for (int r = 0; r < k; r++) {
-    uint32_t bk = 0u;
-    int bi = 0x7fffffff;
-#pragma unroll
-    for (int j = 0; j < PER; j++) {
-      if (key[j] > bk) {
-        bk = key[j];
-        bi = j * 32 + lane;
-      }
-    }
-    const uint32_t mk = __reduce_max_sync(kFull, bk);
-    const int win = (int)__reduce_min_sync(kFull, bk == mk ? (uint32_t)bi : 0xffffffffu);
-    if (lane == r) {
-      my_z = key_value(mk);
-      my_i = win;
-    }
-#pragma unroll
-    for (int j = 0; j < PER; j++)
-      if (win == j * 32 + lane) key[j] = 0u;
-  }
-  const float m = __shfl_sync(kFull, my_z, 0);
-  const float ex = lane < k ? expf(my_z - m) : 0.f;
-  float denom;
-  if (renorm) {
-    denom = warp_sum(ex);
-  } else {
-    float part = 0.f;
-    for (int e = lane; e < E; e += 32) part += expf(zb[e] - m);
-    denom = warp_sum(part);
-  }
+  int my_i;
+  float my_g;
+  warp_topk(z + b * MOE_NOALLOC_MAX_EXPERTS, E, k, renorm, lane, my_i, my_g);
   if (lane < k) {
     idx[b * k + lane] = my_i;
-    gate[b * k + lane] = ex / denom;
+    gate[b * k + lane] = my_g;
   }
 }
 
@@ -135,6 +99,10 @@ extern "C" moe_status moe_route_noalloc(const void* w_r, const void* hidden, int
   if (wdtype != MOE_DTYPE_FP32 && wdtype != MOE_DTYPE_BF16) return MOE_ERR_INVALID;
   const int xbytes = d * (wdtype == MOE_DTYPE_FP32 ? 4 : 2);
   if (xbytes % 16 != 0 || xbytes > 48 * 1024) return MOE_ERR_INVALID;
+  // w_r and hidden are read as 16-byte vectors, idx and gate written as 4-byte words: a
+  // misaligned pointer is refused here rather than faulting the launch
+  if ((((uintptr_t)w_r | (uintptr_t)hidden) & 15) != 0 || (((uintptr_t)idx | (uintptr_t)gate) & 3) != 0)
+    return MOE_ERR_INVALID;
   float* z = nullptr;
   if (scratch_for_current_device(&z) != cudaSuccess) return MOE_ERR_CUDA;
   cudaStream_t s = (cudaStream_t)stream;

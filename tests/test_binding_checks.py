@@ -53,3 +53,18 @@ def test_none_buffers_are_refused():
     m = _handleless()
     with pytest.raises(ValueError, match="None"):
         m.decode_step_host(None, np.zeros(4096, dtype=np.uint16), batch=1)
+
+
+def test_route_noalloc_refuses_mismatched_or_host_tensors_before_calling_the_library():
+    w = torch.zeros((8, 256), dtype=torch.bfloat16)
+    h = torch.zeros((2, 256), dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="CUDA device"):
+        P.route_noalloc(w, h, 2)
+    with pytest.raises(ValueError, match="float32 or both bfloat16"):
+        P.route_noalloc(w, h.float(), 2)
+    with pytest.raises(ValueError, match="float32 or both bfloat16"):
+        P.route_noalloc(w.half(), h.half(), 2)
+    with pytest.raises(ValueError, match=r"\[E x d\]"):
+        P.route_noalloc(w, h[0], 2)
+    with pytest.raises(ValueError, match="torch tensors"):
+        P.route_noalloc(np.zeros((8, 256), np.float32), h, 2)
