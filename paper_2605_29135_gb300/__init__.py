@@ -160,6 +160,12 @@ class MoE:
         shape = (self.cfg.n_layers, self.cfg.max_batch, self.cfg.top_k)
         return idx.reshape(shape), gate.reshape(shape)
 
+    def get_last_logits(self) -> np.ndarray:
+        """Router logits of the last step, float32 [n_layers x n_experts] (device schedule, batch 1)."""
+        z = np.empty(self.cfg.n_layers * self.cfg.n_experts, dtype=np.float32)
+        self._check(self.lib.moe_get_last_logits(self.h, _ptr(z), z.size))
+        return z.reshape(self.cfg.n_layers, self.cfg.n_experts)
+
     def get_stats(self) -> dict:
         s = Stats()
         self._check(self.lib.moe_get_stats(self.h, ctypes.byref(s)))

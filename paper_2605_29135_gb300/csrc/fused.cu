@@ -4,8 +4,11 @@
 //   R  router logits z = W_r h, one warp per expert row;
 //   S  CTA 0: top-k (ties -> lower id) and gates, then one step of the lookup table: hits keep
 //      their slot, misses (ascending global id) take the lowest free slot, else the unpinned
-//      resident with the smallest (last use, global id); records go to the trace buffer and the
-//      per-rank plan (slot, miss flag, gate) to global memory;
+//      resident with the smallest key: (last use, global id) under LRU; under router-guided
+//      replacement the largest rank in its layer's latest routing first (this layer's ranks are
+//      refreshed from z before the lookup), then the most recent use; the rotary ring otherwise.
+//      Records go to the trace buffer and the per-rank plan (slot, miss flag, gate) to global
+//      memory;
 //   C  gate-up rows of every rank, u_r[i] = silu(W_g[i] . h) * (W_u[i] . h). A few "miss CTAs"
 //      stream every missed expert from the page-locked host tier over NVLink-C2C: its gate/up
 //      rows are stored into the freed slot and used for u in the same pass, and its W_d region
@@ -199,13 +202,20 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   __shared__ int s_hand;
   __shared__ unsigned long long s_ckey[kFWarps][kMaxRanks];  // each warp's smallest candidate keys
   __shared__ int s_cslot[kFWarps][kMaxRanks];
+  // router-guided: the layer's logits and ranks, the refreshed keys of its residents that the step
+  // does not use (~0 otherwise), their nev smallest, and the candidates' keys
+  __shared__ float s_z[256];
+  __shared__ int s_rank[256];
+  __shared__ unsigned long long s_lkey[256];
+  __shared__ unsigned long long s_lsel[kMaxRanks];
+  __shared__ unsigned long long s_cand_key[kMaxRanks];
   const int k = a.k, E = a.E;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (warp == 0) {
     int my_i;
     float my_g;
-    warp_topk(a.z, E, k, a.renorm, lane, my_i, my_g);
+    warp_topk(a.z + (int64_t)l * E, E, k, a.renorm, lane, my_i, my_g);
     if (lane < k && (my_i < 0 || my_i >= E)) {
       atomicOr(a.err, FERR_BAD_ROUTE);
       my_i = lane;  // keep the step well-defined; the host reports the error
@@ -254,11 +264,16 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
       const int nc = (int)__ldcg(a.cand + kMaxRanks);
       if (lane == 0) s_ncand = nc;
       if (lane < nc) {
-        const int g = (int)(uint32_t)(__ldcg(a.cand + lane) & 0xffffffffull);
-        s_cand_gid[lane] = g;
-        s_cand_slot[lane] = a.slot_of[g];
+        const unsigned long long key = __ldcg(a.cand + lane);
+        const int g = slot_key_gid(key, a.policy);
+        const bool ok = g >= 0 && g < a.L * E;  // a free slot's key (~0) names no expert
+        s_cand_key[lane] = ok ? key : ~0ull;
+        s_cand_gid[lane] = ok ? g : -1;
+        s_cand_slot[lane] = ok ? a.slot_of[g] : -1;
       }
     }
+    if (a.policy == 2)
+      for (int e = threadIdx.x - 32; e < E; e += blockDim.x - 32) s_z[e] = __ldcg(a.z + (int64_t)l * E + e);
   }
   __syncthreads();
   if (threadIdx.x < k) {
@@ -273,7 +288,33 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
                                        s_win_prior, s_hand, s_nused);
     __syncthreads();
   }
-  if (threadIdx.x == 0 && a.policy == 0) {
+  if (a.policy == 2) {
+    // Refresh the layer's ranks from this routing (rank = logits that beat the expert's, ties to the
+    // lower id, in the top-k's order), and the keys of its residents this step does not use; the
+    // used ones get their keys below, with this step's clock.
+    for (int e = threadIdx.x; e < E; e += blockDim.x) {
+      const uint32_t ke = ord_key(s_z[e]);
+      int rank = 0;
+      for (int j = 0; j < E; j++) {
+        const uint32_t kj = ord_key(s_z[j]);
+        rank += (kj > ke || (kj == ke && j < e)) ? 1 : 0;
+      }
+      s_rank[e] = rank;
+      a.rank[l * E + e] = rank;
+      const int g = l * E + e;
+      const int sl = s_slot_e[e];
+      bool used = false;
+      for (int t = 0; t < k; t++) used |= s_need[t] == g;
+      unsigned long long lk = ~0ull;
+      if (sl >= 0 && !used) {
+        lk = guided_key(E, rank, guided_key_last_use(__ldcg(a.slot_key + sl)), g);
+        a.slot_key[sl] = lk;
+      }
+      s_lkey[e] = lk;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && (a.policy == 0 || a.policy == 2)) {
     // misses in ascending id take free slots [n_used, cap) first
     int n_used = s_nused;
     int nev = 0;
@@ -286,25 +327,84 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     }
     if (n_used != s_nused) *a.n_used = n_used;
     s_nev = nev;
+    if (a.policy == 2) s_nev_found = 0;  // the guided merge below decides
     // Victims: the nev smallest slot keys (last use, id) among slots that hold no expert of this
     // step (every slot is occupied when eviction is needed). They are among the k smallest keys
     // of the pool (at most k - nev of those belong to this step's hits), which phase C of the
     // previous layer-step left in a.cand. s_nev_found < nev sends the phase to the full scan.
-    int j = 0;
-    for (int c = 0; c < s_ncand && j < nev; c++) {
-      const int g = s_cand_gid[c];
-      bool needed = false;
-      for (int t = 0; t < k; t++) needed |= (s_need[t] == g);
-      if (needed) continue;
-      s_vgid[j] = g;
-      s_vslot[j] = s_cand_slot[c];
-      j++;
+    if (a.policy == 0) {
+      int j = 0;
+      for (int c = 0; c < s_ncand && j < nev; c++) {
+        const int g = s_cand_gid[c];
+        if (g < 0) break;  // ascending keys: only free slots' keys follow
+        bool needed = false;
+        for (int t = 0; t < k; t++) needed |= (s_need[t] == g);
+        if (needed) continue;
+        s_vgid[j] = g;
+        s_vslot[j] = s_cand_slot[c];
+        j++;
+      }
+      s_nev_found = j;
     }
-    s_nev_found = j;
   }
   __syncthreads();
-  const int nev = a.policy == 0 ? s_nev : 0;
-  if (nev > 0 && s_nev_found < nev) {  // (LRU only: nev is 0 under the rotary policy)
+  const int nev = (a.policy == 0 || a.policy == 2) ? s_nev : 0;
+  if (a.policy == 2 && nev > 0) {
+    // Victims: the nev smallest keys among residents this step does not use. Only this layer's keys
+    // changed since phase C of the previous layer-step left the pool's k smallest keys in a.cand,
+    // so the candidates of other layers, ascending, are still the smallest keys of other layers;
+    // merge them with the nev smallest refreshed keys of this layer. Running out of candidates
+    // before nev victims sends the phase to the full scan.
+    if (warp == 0) {
+      unsigned long long lk[8];
+#pragma unroll
+      for (int q = 0; q < 8; q++) {
+        const int e = q * 32 + lane;
+        lk[q] = e < E ? s_lkey[e] : ~0ull;
+      }
+      for (int j = 0; j < nev; j++) {
+        unsigned long long best = ~0ull;
+        int bq = 0;
+#pragma unroll
+        for (int q = 0; q < 8; q++)
+          if (lk[q] < best) {
+            best = lk[q];
+            bq = q;
+          }
+        const unsigned long long wmin = shfl_min_u64(best);
+        const unsigned win = __ballot_sync(kFull, best == wmin && wmin != ~0ull);
+        if (win && lane == __ffs(win) - 1) {
+#pragma unroll
+          for (int q = 0; q < 8; q++)
+            if (q == bq) lk[q] = ~0ull;
+        }
+        if (lane == 0) s_lsel[j] = wmin;
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int c = 0, li = 0, j = 0;
+      for (; j < nev; j++) {
+        while (c < s_ncand && s_cand_gid[c] >= 0 && s_cand_gid[c] / E == l) c++;  // this layer's are stale
+        if (c >= s_ncand || s_cand_gid[c] < 0) break;  // other layers' next key unknown: full scan
+        const unsigned long long ck = s_cand_key[c];
+        const unsigned long long lk = s_lsel[li];
+        if (lk < ck) {
+          const int g = slot_key_gid(lk, 2);
+          s_vgid[j] = g;
+          s_vslot[j] = s_slot_e[g - l * E];
+          li++;
+        } else {
+          s_vgid[j] = s_cand_gid[c];
+          s_vslot[j] = s_cand_slot[c];
+          c++;
+        }
+      }
+      s_nev_found = j;
+    }
+    __syncthreads();
+  }
+  if (nev > 0 && s_nev_found < nev) {  // (LRU and router-guided: nev is 0 under the rotary policy)
     // Full scan: each warp finds the nev smallest of its slots, warp 0 takes the nev smallest of
     // those candidates.
     for (int j = 0; j < nev; j++) {
@@ -367,13 +467,13 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
         if (lane == 0) {
           if (!win) atomicOr(a.err, FERR_NO_VICTIM);
           s_vslot[j] = win ? vslot : -1;
-          s_vgid[j] = win ? (int)(uint32_t)(wmin & 0xffffffffull) : -1;
+          s_vgid[j] = win ? slot_key_gid(wmin, a.policy) : -1;
         }
       }
     }
     __syncthreads();
   }
-  if (threadIdx.x == 0 && a.policy == 0) {
+  if (threadIdx.x == 0 && (a.policy == 0 || a.policy == 2)) {
     int j = 0;
     unsigned long long hits = 0, misses = 0, evictions = 0;
     for (int t = 0; t < k; t++) {
@@ -396,8 +496,12 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
       }
       if (s_slot[t] >= 0) a.slot_of[g] = s_slot[t];
     }
-    for (int t = 0; t < k; t++)
-      if (s_slot[t] >= 0) a.slot_key[s_slot[t]] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)s_need[t];
+    for (int t = 0; t < k; t++) {
+      if (s_slot[t] < 0) continue;
+      a.slot_key[s_slot[t]] = a.policy == 2
+                                  ? guided_key(E, s_rank[s_need[t] - l * E], (uint32_t)clock, s_need[t])
+                                  : ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)s_need[t];
+    }
     atomicAdd(a.stats + STAT_HITS, hits);
     atomicAdd(a.stats + STAT_MISSES, misses);
     atomicAdd(a.stats + STAT_EVICTIONS, evictions);
@@ -658,7 +762,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
           }
         }
         acc = warp_sum(acc);
-        if (lane == 0) a.z[gw] = acc;
+        if (lane == 0) a.z[(int64_t)l * a.E + gw] = acc;
       }
     }
     if (!grid_sync(a, nbar)) return;

@@ -88,13 +88,14 @@ def test_create_rejects_rotary_policy_for_batches():
     assert ei.value.status == -1 and "rotary" in str(ei.value)
 
 
-def test_create_rejects_the_guided_policy_for_decoding():
-    # router-guided replacement is a planner policy for now; the check runs before any device call
+@pytest.mark.parametrize("kw", [{"schedule": "host_copy_engine"}, {"max_batch": 4}])
+def test_create_rejects_the_guided_policy_outside_batch1_device_schedule(kw):
+    # the check runs before any device call
     import paper_2605_29135_gb300 as P
     from paper_2605_29135_gb300.buildsys import build
 
     build()
-    cfg = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4, policy="guided")
+    cfg = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4, policy="guided", **kw)
     with pytest.raises(P.MoEError) as ei:
         P.MoE(cfg)
-    assert ei.value.status == -1 and "planner" in str(ei.value)
+    assert ei.value.status == -1 and "guided" in str(ei.value)
