@@ -161,10 +161,11 @@ class MoE:
         return idx.reshape(shape), gate.reshape(shape)
 
     def get_last_logits(self) -> np.ndarray:
-        """Router logits of the last step, float32 [n_layers x n_experts] (device schedule, batch 1)."""
-        z = np.empty(self.cfg.n_layers * self.cfg.n_experts, dtype=np.float32)
+        """Router logits of the last step, float32 [n_layers x max_batch x n_experts] (device schedule)."""
+        c = self.cfg
+        z = np.empty(c.n_layers * c.max_batch * c.n_experts, dtype=np.float32)
         self._check(self.lib.moe_get_last_logits(self.h, _ptr(z), z.size))
-        return z.reshape(self.cfg.n_layers, self.cfg.n_experts)
+        return z.reshape(c.n_layers, c.max_batch, c.n_experts)
 
     def get_stats(self) -> dict:
         s = Stats()

@@ -128,7 +128,7 @@ struct BatchArgs {
   int32_t* n_used;
   int64_t* step;
   // per-layer scratch
-  float* z;                    // [B][E]
+  float* z;                    // [L][Bmax][E] router logits of the current decode step
   int32_t* sel_e;              // [B*k] expert of pair p = b*k + r
   float* sel_g;                // [B*k] its gate
   int32_t* plan_n;             // [2] distinct experts needed this layer-step, and how many missed
@@ -155,6 +155,9 @@ struct BatchArgs {
   int touch_shift;             // log2 of the translation-warming touch stride (0: no touches)
   int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
   int router_tb;               // sequences per router work item (batched_router_tb)
+  int policy;                  // 0 LRU, 2 router-guided
+  int32_t* rank;               // [L*E] router-guided: rank in the layer's latest routing (best over the batch)
+  int32_t* rank_best;          // [E] router-guided scratch: this layer-step's best rank over the batch
 };
 
 // Pairs staged per group for this shape, and the co-resident grid (0: shape or cap unsupported).

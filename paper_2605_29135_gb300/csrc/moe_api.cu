@@ -143,6 +143,7 @@ struct moe_handle {
   int32_t* d_prior = nullptr;            // rotary policy: previous occupant per slot [cap]
   int32_t* d_prior_slot_of = nullptr;    // rotary policy: its inverse [n_gid]
   int32_t* d_rank = nullptr;             // router-guided policy: rank in the layer's latest routing [n_gid]
+  int32_t* d_rank_best = nullptr;        // router-guided, batched: the layer-step's best rank [256]
   int32_t* d_hand = nullptr;             // rotary policy: the hand [1]
   int32_t* d_n_used = nullptr;
   int64_t* d_step = nullptr;
@@ -226,8 +227,8 @@ std::string check_config(const moe_config* c) {
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
   if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY && c->policy != MOE_POLICY_GUIDED)
     return "unknown policy";
-  if (c->policy == MOE_POLICY_GUIDED && (c->schedule != MOE_SCHEDULE_DEVICE || c->max_batch != 1))
-    return "the router-guided policy runs in the device schedule at batch 1";
+  if (c->policy == MOE_POLICY_GUIDED && c->schedule != MOE_SCHEDULE_DEVICE)
+    return "the router-guided policy runs in the device schedule";
   if (c->policy == MOE_POLICY_GUIDED && (int64_t)c->n_layers * c->n_experts >= (1LL << moe::kGuidedGidBits))
     return "the router-guided policy needs n_layers * n_experts < 2^23";
   if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
@@ -663,6 +664,9 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.touch_shift = h->touch_shift;
   a.tg_max = h->tg_max;
   a.router_tb = moe::batched_router_tb(c.wdtype, c.d, c.d_ff, h->batched_tc);
+  a.policy = c.policy;
+  a.rank = h->d_rank;
+  a.rank_best = h->d_rank_best;
   a.map_gu = h->map_gu;
   a.map_d = h->map_d;
   a.map_x = h->map_x;
@@ -829,7 +833,8 @@ void free_all(moe_handle* h) {
   if (h->route) cudaFreeHost(h->route);
   if (h->u) cudaFree(h->u);
   for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_cand, (void*)h->d_prior,
-                  (void*)h->d_prior_slot_of, (void*)h->d_rank, (void*)h->d_hand, (void*)h->d_n_used,
+                  (void*)h->d_prior_slot_of, (void*)h->d_rank, (void*)h->d_rank_best, (void*)h->d_hand,
+                  (void*)h->d_n_used,
                   (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
                   (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
                   (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y,
@@ -955,11 +960,12 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
               cudaMalloc(&h->d_prior, sizeof(int32_t) * h->cap) == cudaSuccess &&
               cudaMalloc(&h->d_prior_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
               cudaMalloc(&h->d_rank, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
+              cudaMalloc(&h->d_rank_best, sizeof(int32_t) * 256) == cudaSuccess &&
               cudaMalloc(&h->d_hand, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_n_used, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_step, sizeof(int64_t)) == cudaSuccess &&
-              cudaMalloc(&h->d_z, sizeof(float) * std::max<int64_t>(256 * (int64_t)cfg->max_batch, h->n_gid)) ==
-                  cudaSuccess &&
+              cudaMalloc(&h->d_z, sizeof(float) * std::max<int64_t>(256 * (int64_t)cfg->max_batch,
+                                                                    h->n_gid * cfg->max_batch)) == cudaSuccess &&
               cudaMalloc(&h->d_plan, sizeof(int32_t) * plan_ints) == cudaSuccess &&
               cudaMalloc(&h->d_plan_gate, sizeof(float) * pairs) == cudaSuccess &&
               (!h->batched || cudaMalloc(&h->d_sel_e, sizeof(int32_t) * pairs) == cudaSuccess) &&
@@ -1122,13 +1128,13 @@ moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_
 
 moe_status moe_get_last_logits(moe_handle* h, float* z, int64_t n) {
   if (!h || !z) return MOE_ERR_INVALID;
-  if (!h->dev_mode || h->batched)
-    return fail(h, MOE_ERR_INVALID, "router logits are kept by the device schedule at batch 1 only");
-  if (n < h->n_gid) return fail(h, MOE_ERR_INVALID, "buffer below n_layers * n_experts");
+  if (!h->dev_mode) return fail(h, MOE_ERR_INVALID, "router logits are kept by the device schedule only");
+  const int64_t need = h->n_gid * h->cfg.max_batch;
+  if (n < need) return fail(h, MOE_ERR_INVALID, "buffer below n_layers * max_batch * n_experts");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   moe_status st = check_device_error(h, true);
   if (st != MOE_OK) return st;
-  MOE_CK(h, cudaMemcpy(z, h->d_z, sizeof(float) * h->n_gid, cudaMemcpyDeviceToHost));
+  MOE_CK(h, cudaMemcpy(z, h->d_z, sizeof(float) * need, cudaMemcpyDeviceToHost));
   return MOE_OK;
 }
 

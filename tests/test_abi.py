@@ -88,8 +88,8 @@ def test_create_rejects_rotary_policy_for_batches():
     assert ei.value.status == -1 and "rotary" in str(ei.value)
 
 
-@pytest.mark.parametrize("kw", [{"schedule": "host_copy_engine"}, {"max_batch": 4}])
-def test_create_rejects_the_guided_policy_outside_batch1_device_schedule(kw):
+@pytest.mark.parametrize("kw", [{"schedule": "host_copy_engine"}])
+def test_create_rejects_the_guided_policy_outside_the_device_schedule(kw):
     # the check runs before any device call
     import paper_2605_29135_gb300 as P
     from paper_2605_29135_gb300.buildsys import build

@@ -1,5 +1,5 @@
-"""Router-guided replacement (MOE_POLICY_GUIDED, device schedule, batch 1) through the C ABI against
-the oracle's guided step.
+"""Router-guided replacement (MOE_POLICY_GUIDED, device schedule, batch 1 and batched) through the C
+ABI against the oracle's guided step.
 
 The device ranks experts by its fp32 logits (moe_get_last_logits). Those ranks must agree with the
 oracle's fp64 logits up to swaps of experts whose oracle logits lie within the near-tie bound. The
@@ -24,32 +24,32 @@ def P():
     return P
 
 
-def _run(wl, cap, policy, preload=False):
+def _run(wl, cap, policy, preload=False, batched_path="auto"):
     """Decode every token on the device; returns hidden, outputs, selections, logits, trace, stats."""
     import torch
 
     from paper_2605_29135_gb300.workload import create_for_workload
 
     hidden = synth.hidden_all(wl)
-    T = hidden.shape[0]
+    T, B = hidden.shape[0], hidden.shape[2]
     dev = torch.device("cuda", 0)
     fp32 = wl.adtype == "fp32"
     hid = torch.from_numpy(hidden.view(np.float32) if fp32 else hidden.view(np.int16)).to(dev)
     if not fp32:
         hid = hid.view(torch.bfloat16)
     out = torch.empty(hid.shape, dtype=hid.dtype, device=dev)
-    idx = np.empty((T, wl.n_layers, 1, wl.top_k), dtype=np.int32)
-    z = np.empty((T, wl.n_layers, wl.n_experts), dtype=np.float32)
-    m = create_for_workload(wl, cap_slots=cap, schedule="device", policy=policy)
+    idx = np.empty((T, wl.n_layers, B, wl.top_k), dtype=np.int32)
+    z = np.empty((T, wl.n_layers, B, wl.n_experts), dtype=np.float32)
+    m = create_for_workload(wl, cap_slots=cap, schedule="device", policy=policy, batched_path=batched_path)
     try:
         if preload:
             m.preload()
         for t in range(T):
-            m.decode_step(hid[t], out[t], batch=1)
+            m.decode_step(hid[t], out[t], batch=B)
             i, _ = m.get_last_routing()
-            idx[t] = i[:, :1]
+            idx[t] = i[:, :B]
             if policy == "guided":
-                z[t] = m.get_last_logits()
+                z[t] = m.get_last_logits()[:, :B]
         torch.cuda.synchronize()
         tr = m.get_residency_trace()
         stats = m.get_stats()
@@ -69,10 +69,10 @@ def _device_ranks(z32):
 
 
 def _check_ranks(ranks, z64, idx):
-    """The device's order of every layer-step's experts is the oracle's up to near-ties, and its
-    top-k selection is the head of that order."""
+    """Per sequence: the device's order of a layer-step's experts is the oracle's up to near-ties,
+    and its top-k selection is the head of that order."""
     k = idx.shape[-1]
-    np.testing.assert_array_equal(idx[:, :, 0, :], np.argsort(ranks, axis=-1)[..., :k])
+    np.testing.assert_array_equal(idx, np.argsort(ranks, axis=-1)[..., :k])
     for pos in np.ndindex(*ranks.shape[:-1]):
         order = np.argsort(ranks[pos])
         zs = z64[pos][order]
@@ -80,17 +80,19 @@ def _check_ranks(ranks, z64, idx):
 
 
 def _replay(wl, cap, hidden, idx, ranks, preload=False, compute_out=True):
+    """The oracle with the device's selections and, per layer-step, its best rank over the batch."""
     orc = oracle.Oracle.for_workload(wl, cap_slots=cap, policy="guided", keep_slot_copies=compute_out)
     if preload:
         orc.preload()
-    res = [orc.decode_step(hidden[t], compute_out=compute_out, forced_idx=idx[t], forced_ranks=ranks[t])
+    best = ranks.min(axis=2)  # [T x L x E]
+    res = [orc.decode_step(hidden[t], compute_out=compute_out, forced_idx=idx[t], forced_ranks=best[t])
            for t in range(hidden.shape[0])]
     return res
 
 
 def _oracle_z(wl, hidden):
     orc = oracle.Oracle.for_workload(wl, keep_slot_copies=False, policy="guided")
-    return np.stack([orc.decode_step(hidden[t], compute_out=False).z[:, 0] for t in range(hidden.shape[0])])
+    return np.stack([orc.decode_step(hidden[t], compute_out=False).z for t in range(hidden.shape[0])])
 
 
 @pytest.mark.parametrize("cap", [2, 3, 5])
@@ -142,3 +144,28 @@ def test_stack48_guided_512_tokens(P, name):
     # the point of the policy: fewer misses than LRU on the same tokens
     _, _, _, _, _, stats_lru = _run(wl, wl.cap_slots, "lru")
     assert stats["misses"] < stats_lru["misses"]
+
+
+@pytest.mark.parametrize("path", ["auto", "cuda_cores"])
+def test_tiny_batched_guided(P, path):
+    # bf16, d = 256, d_ff = 128: "auto" takes the tensor-core kernel, "cuda_cores" the GEMV one
+    wl = synth.WORKLOADS["tiny_fp32"].replace(wdtype="bf16", adtype="bf16", n_layers=3, batch=4, tokens=24)
+    cap = 8
+    hidden, out, idx, z, tr, stats = _run(wl, cap, "guided", batched_path=path)
+    ranks = _device_ranks(z)
+    _check_ranks(ranks, _oracle_z(wl, hidden), idx)
+    res = _replay(wl, cap, hidden, idx, ranks)
+    np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate([r.records for r in res])))
+    assert rel_l2_rows(out, np.stack([r.out for r in res])).max() <= TOL["bf16"]
+
+
+def test_batch64_guided_keeps_part_of_the_pool(P):
+    # 64 sequences put nearly every expert of a layer at rank 0, so ties to the more recent use
+    # decide; unlike LRU, part of the pool then survives from one token to the next
+    wl = synth.WORKLOADS["stack48_batch64"].replace(tokens=6)
+    hidden, out, idx, z, tr, stats = _run(wl, wl.cap_slots, "guided")
+    ranks = _device_ranks(z)
+    _check_ranks(ranks, _oracle_z(wl, hidden), idx)
+    res = _replay(wl, wl.cap_slots, hidden, idx, ranks, compute_out=False)
+    np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate([r.records for r in res])))
+    assert stats["hits"] > 0
