@@ -116,6 +116,8 @@ struct moe_handle {
   moe_stats stats{};
   std::vector<int32_t> last_idx;
   std::vector<float> last_gate;
+  std::vector<float> last_z;      // host schedule, router-guided: [L][E] logits of the last step
+  std::vector<int32_t> ranks;     // host schedule, router-guided: scratch [E]
   // profiling
   bool prof = false;
   std::vector<PendingTime> pending;
@@ -227,8 +229,6 @@ std::string check_config(const moe_config* c) {
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
   if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY && c->policy != MOE_POLICY_GUIDED)
     return "unknown policy";
-  if (c->policy == MOE_POLICY_GUIDED && c->schedule != MOE_SCHEDULE_DEVICE)
-    return "the router-guided policy runs in the device schedule";
   if (c->policy == MOE_POLICY_GUIDED && (int64_t)c->n_layers * c->n_experts >= (1LL << moe::kGuidedGidBits))
     return "the router-guided policy needs n_layers * n_experts < 2^23";
   if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
@@ -358,6 +358,7 @@ moe_status launch_router(moe_handle* h, int32_t layer, const void* hidden_l, cud
   a.wdtype = h->cfg.wdtype == MOE_DTYPE_FP32 ? moe::WD_FP32 : moe::WD_BF16;
   a.out = h->route_dev;
   a.seq = ++h->route_seq;
+  a.want_z = h->cfg.policy == MOE_POLICY_GUIDED;
   ProfScope ps(h, s, PC_ROUTER, (int64_t)a.E * a.d * h->router_eb + (int64_t)a.d * h->asize);
   cudaError_t e = moe::launch_router(a, s);
   ps.done();
@@ -411,6 +412,7 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
   if (h->prof) harvest(h, false);
   h->last_idx.assign((size_t)L * k, -1);
   h->last_gate.assign((size_t)L * k, 0.f);
+  if (c.policy == MOE_POLICY_GUIDED) h->last_z.assign((size_t)L * E, 0.f);
   moe_status st = launch_router(h, 0, hidden, s);
   if (st != MOE_OK) return st;
   std::vector<Need> needs;
@@ -437,6 +439,20 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       needs.push_back(Need{l * E + e, -1, false});
     }
     std::sort(needs.begin(), needs.end(), [](const Need& a, const Need& b) { return a.gid < b.gid; });
+    if (c.policy == MOE_POLICY_GUIDED) {
+      // the layer's ranks from this routing: the logits that beat each expert's, ties to the
+      // lower id (the router's own order)
+      float* zl = h->last_z.data() + (size_t)l * E;
+      const volatile float* rz = h->route->z;
+      for (int32_t e = 0; e < E; e++) zl[e] = rz[e];
+      h->ranks.resize(E);
+      for (int32_t e = 0; e < E; e++) {
+        int32_t r = 0;
+        for (int32_t j = 0; j < E; j++) r += (zl[j] > zl[e] || (zl[j] == zl[e] && j < e)) ? 1 : 0;
+        h->ranks[e] = r;
+      }
+      h->table.set_ranks(l, h->ranks.data());
+    }
     for (size_t i = 1; i < needs.size(); i++)
       if (needs[i].gid == needs[i - 1].gid) return fail(h, MOE_ERR_INVALID, "router produced duplicate expert ids");
     const int64_t clock = h->token_step * L + l + 1;  // 0 is older than every step (preloaded experts)
@@ -1128,9 +1144,15 @@ moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_
 
 moe_status moe_get_last_logits(moe_handle* h, float* z, int64_t n) {
   if (!h || !z) return MOE_ERR_INVALID;
-  if (!h->dev_mode) return fail(h, MOE_ERR_INVALID, "router logits are kept by the device schedule only");
   const int64_t need = h->n_gid * h->cfg.max_batch;
   if (n < need) return fail(h, MOE_ERR_INVALID, "buffer below n_layers * max_batch * n_experts");
+  if (!h->dev_mode) {
+    if (h->cfg.policy != MOE_POLICY_GUIDED)
+      return fail(h, MOE_ERR_INVALID, "the host schedule keeps router logits under the router-guided policy only");
+    std::fill(z, z + need, 0.f);
+    std::copy(h->last_z.begin(), h->last_z.end(), z);
+    return MOE_OK;
+  }
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   moe_status st = check_device_error(h, true);
   if (st != MOE_OK) return st;

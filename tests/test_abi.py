@@ -87,15 +87,3 @@ def test_create_rejects_rotary_policy_for_batches():
         P.MoE(cfg)
     assert ei.value.status == -1 and "rotary" in str(ei.value)
 
-
-@pytest.mark.parametrize("kw", [{"schedule": "host_copy_engine"}])
-def test_create_rejects_the_guided_policy_outside_the_device_schedule(kw):
-    # the check runs before any device call
-    import paper_2605_29135_gb300 as P
-    from paper_2605_29135_gb300.buildsys import build
-
-    build()
-    cfg = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4, policy="guided", **kw)
-    with pytest.raises(P.MoEError) as ei:
-        P.MoE(cfg)
-    assert ei.value.status == -1 and "guided" in str(ei.value)

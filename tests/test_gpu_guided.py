@@ -24,7 +24,7 @@ def P():
     return P
 
 
-def _run(wl, cap, policy, preload=False, batched_path="auto"):
+def _run(wl, cap, policy, preload=False, batched_path="auto", schedule="device"):
     """Decode every token on the device; returns hidden, outputs, selections, logits, trace, stats."""
     import torch
 
@@ -40,7 +40,7 @@ def _run(wl, cap, policy, preload=False, batched_path="auto"):
     out = torch.empty(hid.shape, dtype=hid.dtype, device=dev)
     idx = np.empty((T, wl.n_layers, B, wl.top_k), dtype=np.int32)
     z = np.empty((T, wl.n_layers, B, wl.n_experts), dtype=np.float32)
-    m = create_for_workload(wl, cap_slots=cap, schedule="device", policy=policy, batched_path=batched_path)
+    m = create_for_workload(wl, cap_slots=cap, schedule=schedule, policy=policy, batched_path=batched_path)
     try:
         if preload:
             m.preload()
@@ -95,23 +95,28 @@ def _oracle_z(wl, hidden):
     return np.stack([orc.decode_step(hidden[t], compute_out=False).z for t in range(hidden.shape[0])])
 
 
+SCHEDULES = ["device", "host_copy_engine"]
+
+
+@pytest.mark.parametrize("schedule", SCHEDULES)
 @pytest.mark.parametrize("cap", [2, 3, 5])
-def test_tiny_guided_trace_and_outputs(P, cap):
+def test_tiny_guided_trace_and_outputs(P, cap, schedule):
     wl = synth.WORKLOADS["tiny_fp32"].replace(n_layers=2)
-    hidden, out, idx, z, tr, stats = _run(wl, cap, "guided")
+    hidden, out, idx, z, tr, stats = _run(wl, cap, "guided", schedule=schedule)
     ranks = _device_ranks(z)
     _check_ranks(ranks, _oracle_z(wl, hidden), idx)
     res = _replay(wl, cap, hidden, idx, ranks)
     np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate([r.records for r in res])))
     assert rel_l2_rows(out, np.stack([r.out for r in res])).max() <= TOL["fp32"]
     assert stats["misses"] == int((tr["kind"] == 1).sum()) and stats["evictions"] == int((tr["evicted"] >= 0).sum())
-    _, out_lru, _, _, tr_lru, _ = _run(wl, cap, "lru")
+    _, out_lru, _, _, tr_lru, _ = _run(wl, cap, "lru", schedule=schedule)
     np.testing.assert_array_equal(out, out_lru)  # same arithmetic whatever the slot contents
 
 
-def test_guided_preload(P):
+@pytest.mark.parametrize("schedule", SCHEDULES)
+def test_guided_preload(P, schedule):
     wl = synth.WORKLOADS["tiny_fp32"].replace(n_layers=2, tokens=32)
-    hidden, out, idx, z, tr, _ = _run(wl, 6, "guided", preload=True)
+    hidden, out, idx, z, tr, _ = _run(wl, 6, "guided", preload=True, schedule=schedule)
     res = _replay(wl, 6, hidden, idx, _device_ranks(z), preload=True, compute_out=False)
     np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate([r.records for r in res])))
 
@@ -129,10 +134,11 @@ def test_layer_bf16_guided(P):
         assert rel_l2_rows(out[t, 0, 0], ref) <= TOL["bf16"]
 
 
+@pytest.mark.parametrize("schedule", SCHEDULES)
 @pytest.mark.parametrize("name", ["stack48_bf16", "stack48_int4"])
-def test_stack48_guided_512_tokens(P, name):
+def test_stack48_guided_512_tokens(P, name, schedule):
     wl = synth.WORKLOADS[name].replace(tokens=512)
-    hidden, out, idx, z, tr, stats = _run(wl, wl.cap_slots, "guided")
+    hidden, out, idx, z, tr, stats = _run(wl, wl.cap_slots, "guided", schedule=schedule)
     ranks = _device_ranks(z)
     _check_ranks(ranks, _oracle_z(wl, hidden), idx)
     res = _replay(wl, wl.cap_slots, hidden, idx, ranks, compute_out=False)
@@ -142,7 +148,7 @@ def test_stack48_guided_512_tokens(P, name):
         ref, _, _ = orc.moe_layer(l, hidden[t, l, 0], forced_idx=idx[t, l, 0])
         assert rel_l2_rows(out[t, l, 0], ref) <= TOL[wl.wdtype]
     # the point of the policy: fewer misses than LRU on the same tokens
-    _, _, _, _, _, stats_lru = _run(wl, wl.cap_slots, "lru")
+    _, _, _, _, _, stats_lru = _run(wl, wl.cap_slots, "lru", schedule=schedule)
     assert stats["misses"] < stats_lru["misses"]
 
 
