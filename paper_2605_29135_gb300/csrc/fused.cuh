@@ -73,6 +73,7 @@ struct FusedArgs {
   // Router-guided policy (policy == 2): every expert's rank in its layer's latest routing
   // (0 = highest logit, ties to the lower id; E before the layer's first routing).
   int32_t* rank;               // [L*E]
+  unsigned* plan_flag;         // clock of the last layer-step whose plan CTA 0 has published (0: none)
 };
 
 // Router-guided replacement key: the victim is the smallest key, i.e. the largest rank, then the

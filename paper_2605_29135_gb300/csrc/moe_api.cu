@@ -741,6 +741,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   a.prior = h->d_prior;
   a.prior_slot_of = h->d_prior_slot_of;
   a.hand = h->d_hand;
+  a.plan_flag = h->d_bar + 1;  // cleared with the barrier counter
   a.n_used = h->d_n_used;
   a.step = h->d_step;
   a.z = h->d_z;
@@ -774,7 +775,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   MOE_CK(h, cudaEventRecord(h->err_ev, s));
   h->err_pending = true;
   h->steps_launched++;
-  h->bar_epoch += 4u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 4 barriers per layer
+  h->bar_epoch += 3u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
   if (a.phase_ts) {
     // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
     static const int cls[4] = {PC_PH_R, PC_PH_S, PC_PH_C, PC_PH_D};
