@@ -381,8 +381,8 @@ def main():
     ap.add_argument("--layers", type=int, default=None, help="layer count override (small profiling cases)")
     ap.add_argument("--preload", action="store_true", help="fill the pool (moe_preload) before the warm-up")
     ap.add_argument("--miss-ctas", type=int, default=0, help="CTAs streaming missed experts (0: library default)")
-    ap.add_argument("--policy", default="lru", choices=["lru", "rotary"],
-                    help="slot-group replacement policy (rotary: host copy-engine schedule only)")
+    ap.add_argument("--policy", default="lru", choices=["lru", "rotary", "guided"],
+                    help="slot-group replacement policy (rotary: batch 1; guided: device schedule, batch 1)")
     ap.add_argument("--batched-path", default="auto", choices=["auto", "cuda_cores"],
                     help="expert FFN of batched steps: tensor cores where the shape allows, or CUDA cores")
     args = ap.parse_args()

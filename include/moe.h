@@ -103,7 +103,7 @@ enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
  *     expert in its most recent routing (0 = highest logit; for a batch, the best rank over its
  *     sequences). A miss takes the lowest free slot, else evicts the resident not needed this
  *     layer-step with the largest rank, ties to the more recent use, then to the lower global id.
- *     Residency planner only for now (moe_create rejects it). */
+ *     Both schedules (device: n_layers * n_experts < 2^23), and the residency planner. */
 enum { MOE_POLICY_LRU = 0, MOE_POLICY_ROTARY = 1, MOE_POLICY_GUIDED = 2 };
 
 typedef struct {
@@ -219,6 +219,13 @@ moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* 
 moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_t n);
 
 moe_status moe_get_stats(moe_handle* h, moe_stats* out);
+
+/* Router logits of the last decode step, fp32 [n_layers x max_batch x n_experts] (z = W_r h as the
+ * device computed it; the router-guided policy ranks experts by them; rows b >= the step's batch
+ * are stale). MOE_SCHEDULE_DEVICE, or MOE_SCHEDULE_HOST_COPY_ENGINE under MOE_POLICY_GUIDED
+ * (MOE_ERR_INVALID otherwise, or if n is below n_layers * max_batch * n_experts). Waits for the
+ * step. */
+moe_status moe_get_last_logits(moe_handle* h, float* z, int64_t n);
 
 /* Empty the slot pool (all experts non-resident), step clock 0, trace and stats cleared. */
 moe_status moe_reset_residency(moe_handle* h);

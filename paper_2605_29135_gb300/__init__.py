@@ -160,6 +160,13 @@ class MoE:
         shape = (self.cfg.n_layers, self.cfg.max_batch, self.cfg.top_k)
         return idx.reshape(shape), gate.reshape(shape)
 
+    def get_last_logits(self) -> np.ndarray:
+        """Router logits of the last step, float32 [n_layers x max_batch x n_experts] (device schedule)."""
+        c = self.cfg
+        z = np.empty(c.n_layers * c.max_batch * c.n_experts, dtype=np.float32)
+        self._check(self.lib.moe_get_last_logits(self.h, _ptr(z), z.size))
+        return z.reshape(c.n_layers, c.max_batch, c.n_experts)
+
     def get_stats(self) -> dict:
         s = Stats()
         self._check(self.lib.moe_get_stats(self.h, ctypes.byref(s)))

@@ -116,6 +116,8 @@ struct moe_handle {
   moe_stats stats{};
   std::vector<int32_t> last_idx;
   std::vector<float> last_gate;
+  std::vector<float> last_z;      // host schedule, router-guided: [L][E] logits of the last step
+  std::vector<int32_t> ranks;     // host schedule, router-guided: scratch [E]
   // profiling
   bool prof = false;
   std::vector<PendingTime> pending;
@@ -142,6 +144,8 @@ struct moe_handle {
   unsigned long long* d_cand = nullptr;  // batch-1 kernel: victim candidates [kMaxRanks + 1]
   int32_t* d_prior = nullptr;            // rotary policy: previous occupant per slot [cap]
   int32_t* d_prior_slot_of = nullptr;    // rotary policy: its inverse [n_gid]
+  int32_t* d_rank = nullptr;             // router-guided policy: rank in the layer's latest routing [n_gid]
+  int32_t* d_rank_best = nullptr;        // router-guided, batched: the layer-step's best rank [256]
   int32_t* d_hand = nullptr;             // rotary policy: the hand [1]
   int32_t* d_n_used = nullptr;
   int64_t* d_step = nullptr;
@@ -223,8 +227,10 @@ std::string check_config(const moe_config* c) {
   if (c->schedule != MOE_SCHEDULE_DEVICE && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "unknown schedule";
   if (c->miss_ctas < 0) return "miss_ctas must be >= 0";
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
-  if (c->policy == MOE_POLICY_GUIDED) return "the router-guided policy is available in the residency planner only";
-  if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY) return "unknown policy";
+  if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY && c->policy != MOE_POLICY_GUIDED)
+    return "unknown policy";
+  if (c->policy == MOE_POLICY_GUIDED && (int64_t)c->n_layers * c->n_experts >= (1LL << moe::kGuidedGidBits))
+    return "the router-guided policy needs n_layers * n_experts < 2^23";
   if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
   return "";
 }
@@ -242,6 +248,10 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_cand, 0, sizeof(unsigned long long) * (moe::kMaxRanks + 1));
   cudaMemset(h->d_prior, 0xff, sizeof(int32_t) * h->cap);
   cudaMemset(h->d_prior_slot_of, 0xff, sizeof(int32_t) * h->n_gid);
+  {
+    const std::vector<int32_t> unrouted((size_t)h->n_gid, h->cfg.n_experts);  // rank E: not routed yet
+    cudaMemcpy(h->d_rank, unrouted.data(), sizeof(int32_t) * h->n_gid, cudaMemcpyHostToDevice);
+  }
   cudaMemset(h->d_hand, 0, sizeof(int32_t));
   cudaMemset(h->d_n_used, 0, sizeof(int32_t));
   cudaMemset(h->d_step, 0, sizeof(int64_t));
@@ -348,6 +358,7 @@ moe_status launch_router(moe_handle* h, int32_t layer, const void* hidden_l, cud
   a.wdtype = h->cfg.wdtype == MOE_DTYPE_FP32 ? moe::WD_FP32 : moe::WD_BF16;
   a.out = h->route_dev;
   a.seq = ++h->route_seq;
+  a.want_z = h->cfg.policy == MOE_POLICY_GUIDED;
   ProfScope ps(h, s, PC_ROUTER, (int64_t)a.E * a.d * h->router_eb + (int64_t)a.d * h->asize);
   cudaError_t e = moe::launch_router(a, s);
   ps.done();
@@ -401,6 +412,7 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
   if (h->prof) harvest(h, false);
   h->last_idx.assign((size_t)L * k, -1);
   h->last_gate.assign((size_t)L * k, 0.f);
+  if (c.policy == MOE_POLICY_GUIDED) h->last_z.assign((size_t)L * E, 0.f);
   moe_status st = launch_router(h, 0, hidden, s);
   if (st != MOE_OK) return st;
   std::vector<Need> needs;
@@ -427,6 +439,20 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       needs.push_back(Need{l * E + e, -1, false});
     }
     std::sort(needs.begin(), needs.end(), [](const Need& a, const Need& b) { return a.gid < b.gid; });
+    if (c.policy == MOE_POLICY_GUIDED) {
+      // the layer's ranks from this routing: the logits that beat each expert's, ties to the
+      // lower id (the router's own order)
+      float* zl = h->last_z.data() + (size_t)l * E;
+      const volatile float* rz = h->route->z;
+      for (int32_t e = 0; e < E; e++) zl[e] = rz[e];
+      h->ranks.resize(E);
+      for (int32_t e = 0; e < E; e++) {
+        int32_t r = 0;
+        for (int32_t j = 0; j < E; j++) r += (zl[j] > zl[e] || (zl[j] == zl[e] && j < e)) ? 1 : 0;
+        h->ranks[e] = r;
+      }
+      h->table.set_ranks(l, h->ranks.data());
+    }
     for (size_t i = 1; i < needs.size(); i++)
       if (needs[i].gid == needs[i - 1].gid) return fail(h, MOE_ERR_INVALID, "router produced duplicate expert ids");
     const int64_t clock = h->token_step * L + l + 1;  // 0 is older than every step (preloaded experts)
@@ -654,6 +680,9 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.touch_shift = h->touch_shift;
   a.tg_max = h->tg_max;
   a.router_tb = moe::batched_router_tb(c.wdtype, c.d, c.d_ff, h->batched_tc);
+  a.policy = c.policy;
+  a.rank = h->d_rank;
+  a.rank_best = h->d_rank_best;
   a.map_gu = h->map_gu;
   a.map_d = h->map_d;
   a.map_x = h->map_x;
@@ -707,10 +736,12 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   a.slot_key = h->d_slot_key;
   a.cand = h->d_cand;
   a.policy = c.policy;
-  a.may_evict = h->cap < h->n_gid && c.policy == MOE_POLICY_LRU;
+  a.may_evict = h->cap < h->n_gid && c.policy != MOE_POLICY_ROTARY;
+  a.rank = h->d_rank;
   a.prior = h->d_prior;
   a.prior_slot_of = h->d_prior_slot_of;
   a.hand = h->d_hand;
+  a.plan_flag = h->d_bar + 1;  // cleared with the barrier counter
   a.n_used = h->d_n_used;
   a.step = h->d_step;
   a.z = h->d_z;
@@ -744,7 +775,7 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   MOE_CK(h, cudaEventRecord(h->err_ev, s));
   h->err_pending = true;
   h->steps_launched++;
-  h->bar_epoch += 4u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 4 barriers per layer
+  h->bar_epoch += 3u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
   if (a.phase_ts) {
     // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
     static const int cls[4] = {PC_PH_R, PC_PH_S, PC_PH_C, PC_PH_D};
@@ -819,7 +850,8 @@ void free_all(moe_handle* h) {
   if (h->route) cudaFreeHost(h->route);
   if (h->u) cudaFree(h->u);
   for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_cand, (void*)h->d_prior,
-                  (void*)h->d_prior_slot_of, (void*)h->d_hand, (void*)h->d_n_used,
+                  (void*)h->d_prior_slot_of, (void*)h->d_rank, (void*)h->d_rank_best, (void*)h->d_hand,
+                  (void*)h->d_n_used,
                   (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
                   (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
                   (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y,
@@ -944,10 +976,13 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
               cudaMalloc(&h->d_cand, sizeof(unsigned long long) * (moe::kMaxRanks + 1)) == cudaSuccess &&
               cudaMalloc(&h->d_prior, sizeof(int32_t) * h->cap) == cudaSuccess &&
               cudaMalloc(&h->d_prior_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
+              cudaMalloc(&h->d_rank, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
+              cudaMalloc(&h->d_rank_best, sizeof(int32_t) * 256) == cudaSuccess &&
               cudaMalloc(&h->d_hand, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_n_used, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_step, sizeof(int64_t)) == cudaSuccess &&
-              cudaMalloc(&h->d_z, sizeof(float) * 256 * cfg->max_batch) == cudaSuccess &&
+              cudaMalloc(&h->d_z, sizeof(float) * std::max<int64_t>(256 * (int64_t)cfg->max_batch,
+                                                                    h->n_gid * cfg->max_batch)) == cudaSuccess &&
               cudaMalloc(&h->d_plan, sizeof(int32_t) * plan_ints) == cudaSuccess &&
               cudaMalloc(&h->d_plan_gate, sizeof(float) * pairs) == cudaSuccess &&
               (!h->batched || cudaMalloc(&h->d_sel_e, sizeof(int32_t) * pairs) == cudaSuccess) &&
@@ -1108,6 +1143,24 @@ moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_
   return MOE_OK;
 }
 
+moe_status moe_get_last_logits(moe_handle* h, float* z, int64_t n) {
+  if (!h || !z) return MOE_ERR_INVALID;
+  const int64_t need = h->n_gid * h->cfg.max_batch;
+  if (n < need) return fail(h, MOE_ERR_INVALID, "buffer below n_layers * max_batch * n_experts");
+  if (!h->dev_mode) {
+    if (h->cfg.policy != MOE_POLICY_GUIDED)
+      return fail(h, MOE_ERR_INVALID, "the host schedule keeps router logits under the router-guided policy only");
+    std::fill(z, z + need, 0.f);
+    std::copy(h->last_z.begin(), h->last_z.end(), z);
+    return MOE_OK;
+  }
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  moe_status st = check_device_error(h, true);
+  if (st != MOE_OK) return st;
+  MOE_CK(h, cudaMemcpy(z, h->d_z, sizeof(float) * need, cudaMemcpyDeviceToHost));
+  return MOE_OK;
+}
+
 moe_status moe_get_stats(moe_handle* h, moe_stats* out) {
   if (!h || !out) return MOE_ERR_INVALID;
   if (h->dev_mode) {
@@ -1172,6 +1225,12 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
   int32_t n_used = 0;
   MOE_CK(h, cudaMemcpy(slot_of.data(), h->d_slot_of, sizeof(int32_t) * h->n_gid, cudaMemcpyDeviceToHost));
   MOE_CK(h, cudaMemcpy(&n_used, h->d_n_used, sizeof n_used, cudaMemcpyDeviceToHost));
+  const bool guided = h->cfg.policy == MOE_POLICY_GUIDED;
+  std::vector<int32_t> rank;
+  if (guided) {
+    rank.resize(h->n_gid);
+    MOE_CK(h, cudaMemcpy(rank.data(), h->d_rank, sizeof(int32_t) * h->n_gid, cudaMemcpyDeviceToHost));
+  }
   int64_t loaded = 0;
   std::vector<unsigned long long> keys;
   std::vector<int32_t> kslots;
@@ -1181,7 +1240,8 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
     MOE_CK(h, cudaMemcpyAsync(h->pool + (int64_t)slot * h->slot_stride, h->arena + g * h->slot_stride, h->lay.total,
                               cudaMemcpyHostToDevice, h->copy_stream));
     slot_of[g] = slot;
-    keys.push_back((unsigned long long)(uint32_t)g);  // last use 0: older than every decode step
+    // last use 0: older than every decode step
+    keys.push_back(guided ? moe::guided_key(h->cfg.n_experts, rank[g], 0u, (int32_t)g) : (unsigned long long)(uint32_t)g);
     kslots.push_back(slot);
     loaded++;
   }

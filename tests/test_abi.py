@@ -88,18 +88,6 @@ def test_create_rejects_rotary_policy_for_batches():
     assert ei.value.status == -1 and "rotary" in str(ei.value)
 
 
-def test_create_rejects_the_guided_policy_for_decoding():
-    # router-guided replacement is a planner policy for now; the check runs before any device call
-    import paper_2605_29135_gb300 as P
-    from paper_2605_29135_gb300.buildsys import build
-
-    build()
-    cfg = P.make_config(256, 8, 2, 128, 1, "fp32", "fp32", cap_slots=4, policy="guided")
-    with pytest.raises(P.MoEError) as ei:
-        P.MoE(cfg)
-    assert ei.value.status == -1 and "planner" in str(ei.value)
-
-
 @pytest.mark.parametrize("lang,std", [("c", "c99"), ("c++", "c++11")])
 def test_header_compiles_as_plain_c_and_cpp(lang, std, tmp_path):
     # the boundary is a C ABI: the header must stand alone in C as well as C++
