@@ -285,7 +285,7 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
 
     wr = wl.replace(cap_slots=wl.n_gid)
     m = create_for_workload(wr, device=device, trace_capacity=0, schedule=args.schedule,
-                            batched_path=args.batched_path, policy=args.policy)
+                            batched_path=args.batched_path, policy=args.policy, lookahead=args.lookahead)
     try:
         m.preload()
         n_tok = hid_dev.shape[0]
@@ -383,6 +383,8 @@ def main():
     ap.add_argument("--miss-ctas", type=int, default=0, help="CTAs streaming missed experts (0: library default)")
     ap.add_argument("--policy", default="lru", choices=["lru", "rotary", "guided"],
                     help="slot-group replacement policy (rotary: batch 1; guided: device schedule, batch 1)")
+    ap.add_argument("--lookahead", action="store_true",
+                    help="host copy-engine schedule: route layer l + 1 and issue its copies while layer l computes")
     ap.add_argument("--batched-path", default="auto", choices=["auto", "cuda_cores"],
                     help="expert FFN of batched steps: tensor cores where the shape allows, or CUDA cores")
     args = ap.parse_args()
@@ -430,7 +432,7 @@ def main():
     thp0 = anon_huge_kb()
     t_setup = time.perf_counter()
     m = create_for_workload(wl, device=local, trace_capacity=0, schedule=args.schedule, miss_ctas=args.miss_ctas,
-                            batched_path=args.batched_path, policy=args.policy)
+                            batched_path=args.batched_path, policy=args.policy, lookahead=args.lookahead)
     t_setup = time.perf_counter() - t_setup
     thp_gb = (anon_huge_kb() - thp0) / 1e6
     eb = P.expert_bytes(m.cfg)
@@ -523,6 +525,7 @@ def main():
                    "parallelism": "replicas" if world > 1 else "single GPU", "schedule": args.schedule,
                    "miss_ctas": args.miss_ctas or "default",
                    "batched_path": args.batched_path if wl.batch > 1 else None, "policy": args.policy,
+                   "lookahead": args.lookahead,
                    "l2": f"inputs larger than L2 ({wl.cap_slots * eb / 1e9:.1f} GB pool, "
                          f"{hbm_bytes_step / 1e9:.1f} GB of expert weights read per step)"},
         "step_roofline": {"bound": "h2d" if t_h2d >= t_hbm else "hbm", "t_star_ms": t_star * 1e3,

@@ -130,6 +130,11 @@ typedef struct {
                              steps hand work items to all CTAs, missed experts first, and ignore it */
   int32_t batched_path;   /* MOE_BATCHED_AUTO (default) or MOE_BATCHED_CUDA_CORES */
   int32_t policy;         /* MOE_POLICY_LRU (default) or MOE_POLICY_ROTARY */
+  int32_t lookahead;      /* MOE_SCHEDULE_HOST_COPY_ENGINE only. 1: route layer l + 1 as soon as layer l's
+                             routing has reached the host, and issue its miss copies while layer l computes
+                             (the layers' inputs are all given with the step, so the decisions, the trace and
+                             the outputs are those of 0); a copy into a slot layer l still reads waits for
+                             layer l's kernels. 0 (default): one layer after another. */
 } moe_config;
 
 /* One residency record: a requested expert's outcome in one layer-step. */

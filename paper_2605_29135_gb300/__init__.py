@@ -29,12 +29,13 @@ class MoEError(RuntimeError):
 
 def make_config(d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots=0, cap_bytes=0, renorm=True,
                 device=0, max_batch=1, trace_capacity=1 << 22, device_pool=None, schedule="device",
-                miss_ctas=0, batched_path="auto", policy="lru") -> MoeConfig:
+                miss_ctas=0, batched_path="auto", policy="lru", lookahead=False) -> MoeConfig:
     return MoeConfig(d=d, n_experts=n_experts, top_k=top_k, d_ff=d_ff, n_layers=n_layers, max_batch=max_batch,
                      wdtype=DTYPE[wdtype], adtype=DTYPE[adtype], cap_slots=cap_slots, cap_bytes=cap_bytes,
                      renorm=1 if renorm else 0, device=device, device_pool=device_pool,
                      trace_capacity=trace_capacity, schedule=SCHEDULE[schedule], miss_ctas=miss_ctas,
-                     batched_path=BATCHED_PATH[batched_path], policy=POLICY[policy])
+                     batched_path=BATCHED_PATH[batched_path], policy=POLICY[policy],
+                     lookahead=1 if lookahead else 0)
 
 
 def expert_bytes(cfg: MoeConfig) -> int:

@@ -36,7 +36,8 @@ class MoeConfig(ctypes.Structure):
                 ("wdtype", ctypes.c_int32), ("adtype", ctypes.c_int32), ("cap_slots", ctypes.c_int64),
                 ("cap_bytes", ctypes.c_int64), ("renorm", ctypes.c_int32), ("device", ctypes.c_int32),
                 ("device_pool", ctypes.c_void_p), ("trace_capacity", ctypes.c_int64), ("schedule", ctypes.c_int32),
-                ("miss_ctas", ctypes.c_int32), ("batched_path", ctypes.c_int32), ("policy", ctypes.c_int32)]
+                ("miss_ctas", ctypes.c_int32), ("batched_path", ctypes.c_int32), ("policy", ctypes.c_int32),
+                ("lookahead", ctypes.c_int32)]
 
 
 class TraceRec(ctypes.Structure):

@@ -103,6 +103,7 @@ struct moe_handle {
   cudaStream_t copy_stream = nullptr;
   cudaStream_t host_stream = nullptr;
   std::vector<cudaEvent_t> copy_ev;
+  cudaEvent_t layer_ev[2] = {nullptr, nullptr};  // host schedule with lookahead: layer l's last kernel done
   void* hid_dev = nullptr;
   void* out_dev = nullptr;
   // residency state of the host-driven schedule
@@ -232,6 +233,8 @@ std::string check_config(const moe_config* c) {
   if (c->policy == MOE_POLICY_GUIDED && (int64_t)c->n_layers * c->n_experts >= (1LL << moe::kGuidedGidBits))
     return "the router-guided policy needs n_layers * n_experts < 2^23";
   if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
+  if (c->lookahead != 0 && c->lookahead != 1) return "lookahead must be 0 or 1";
+  if (c->lookahead && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "lookahead needs the host copy-engine schedule";
   return "";
 }
 
@@ -370,6 +373,7 @@ struct Need {
   int32_t gid;
   int32_t slot;
   bool miss;
+  int32_t evicted;  // global id the miss evicted, -1 if none
 };
 
 // One layer-step of the lookup table (rules in slot_table.h; needs in ascending gid). Fills each
@@ -385,6 +389,7 @@ moe_status residency_step(moe_handle* h, int32_t layer, std::vector<Need>& needs
     Need& n = needs[i];
     n.slot = d.slot;
     n.miss = d.kind == moe::SLOT_MISS;
+    n.evicted = d.evicted;
     if (n.miss) {
       h->stats.misses++;
       h->stats.miss_bytes += h->lay.total;
@@ -417,6 +422,7 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
   if (st != MOE_OK) return st;
   std::vector<Need> needs;
   std::vector<int32_t> rank_gid(k);
+  std::vector<int32_t> prev_needed;  // lookahead: the global ids layer l - 1 reads
   for (int32_t l = 0; l < L; l++) {
     const void* hid_l = (const uint8_t*)hidden + (int64_t)l * act_row;
     NvtxRange layer_range("layer", l);
@@ -436,7 +442,7 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       h->last_idx[(size_t)l * k + r] = e;
       h->last_gate[(size_t)l * k + r] = rgate[r];
       rank_gid[r] = l * E + e;
-      needs.push_back(Need{l * E + e, -1, false});
+      needs.push_back(Need{l * E + e, -1, false, -1});
     }
     std::sort(needs.begin(), needs.end(), [](const Need& a, const Need& b) { return a.gid < b.gid; });
     if (c.policy == MOE_POLICY_GUIDED) {
@@ -455,6 +461,13 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     }
     for (size_t i = 1; i < needs.size(); i++)
       if (needs[i].gid == needs[i - 1].gid) return fail(h, MOE_ERR_INVALID, "router produced duplicate expert ids");
+    // Lookahead: layer l's routing is in host arrays now, so layer l + 1's router may overwrite the
+    // routing buffer. Launched here, it runs on the GPU before layer l's kernels enqueued below,
+    // and the next iteration issues layer l + 1's miss copies while layer l computes.
+    if (c.lookahead && l + 1 < L) {
+      st = launch_router(h, l + 1, (const uint8_t*)hidden + (int64_t)(l + 1) * act_row, s);
+      if (st != MOE_OK) return st;
+    }
     const int64_t clock = h->token_step * L + l + 1;  // 0 is older than every step (preloaded experts)
     {
       NvtxRange r("slot lookup", l);
@@ -464,8 +477,17 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     h->stats.layer_steps++;
     // selective loads: misses in ascending gid on the copy stream
     int n_miss = 0;
+    bool waited_prev = false;
     for (auto& n : needs) {
       if (!n.miss) continue;
+      // Lookahead: layer l - 1's kernels may still be running. A victim they read is overwritten
+      // only after its last kernel (every layer before it has finished: layer l's router ran
+      // after it). With cap >= 2 x a layer-step's experts an LRU victim is never such an expert.
+      if (c.lookahead && !waited_prev && n.evicted >= 0 &&
+          std::find(prev_needed.begin(), prev_needed.end(), n.evicted) != prev_needed.end()) {
+        MOE_CK(h, cudaStreamWaitEvent(h->copy_stream, h->layer_ev[(l - 1) & 1], 0));
+        waited_prev = true;
+      }
       ProfScope ps(h, h->copy_stream, PC_COPY, h->lay.total);
       if (h->fault == MOE_FAULT_COPY_ERROR) {  // an armed copy fault: this copy "fails"
         h->fault = MOE_FAULT_NONE;
@@ -536,7 +558,11 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       ps.done();
       if (e != cudaSuccess) return cuda_fail(h, e, "down/combine launch");
     }
-    if (l + 1 < L) {
+    if (c.lookahead) {
+      MOE_CK(h, cudaEventRecord(h->layer_ev[l & 1], s));
+      prev_needed.clear();
+      for (auto& n : needs) prev_needed.push_back(n.gid);
+    } else if (l + 1 < L) {
       st = launch_router(h, l + 1, (const uint8_t*)hidden + (int64_t)(l + 1) * act_row, s);
       if (st != MOE_OK) return st;
     }
@@ -842,6 +868,8 @@ void free_all(moe_handle* h) {
   harvest(h, true);
   for (auto e : h->ev_pool) cudaEventDestroy(e);
   for (auto e : h->copy_ev) cudaEventDestroy(e);
+  for (auto e : h->layer_ev)
+    if (e) cudaEventDestroy(e);
   if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   if (h->host_stream) cudaStreamDestroy(h->host_stream);
   if (h->own_pool && h->pool) cudaFree(h->pool);
@@ -943,6 +971,8 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     return bail(MOE_ERR_CUDA, "stream creation failed");
   h->copy_ev.resize((size_t)cfg->top_k * cfg->max_batch, nullptr);
   for (auto& e : h->copy_ev)
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
+  for (auto& e : h->layer_ev)
     if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
   h->dev_mode = cfg->schedule == MOE_SCHEDULE_DEVICE;
   h->batched = h->dev_mode && cfg->max_batch > 1;

@@ -16,19 +16,20 @@ from . import MoE, make_config
 
 
 def config_for(wl, cap_slots=None, device=0, trace_capacity=1 << 22, renorm=True, schedule="device", miss_ctas=0,
-               batched_path="auto", policy="lru"):
+               batched_path="auto", policy="lru", lookahead=False):
     return make_config(wl.d, wl.n_experts, wl.top_k, wl.d_ff, wl.n_layers, wl.wdtype, wl.adtype,
                        cap_slots=wl.cap_slots if cap_slots is None else cap_slots, renorm=renorm, device=device,
                        max_batch=wl.batch, trace_capacity=trace_capacity, schedule=schedule, miss_ctas=miss_ctas,
-                       batched_path=batched_path, policy=policy)
+                       batched_path=batched_path, policy=policy, lookahead=lookahead)
 
 
 def create_for_workload(wl, cap_slots=None, device=0, trace_capacity=1 << 22, threads=None,
-                        schedule="device", miss_ctas=0, batched_path="auto", renorm=True, policy="lru") -> MoE:
+                        schedule="device", miss_ctas=0, batched_path="auto", renorm=True, policy="lru",
+                        lookahead=False) -> MoE:
     import synth
 
     m = MoE(config_for(wl, cap_slots, device, trace_capacity, renorm=renorm, schedule=schedule, miss_ctas=miss_ctas,
-                       batched_path=batched_path, policy=policy))
+                       batched_path=batched_path, policy=policy, lookahead=lookahead))
     try:
         for layer in range(wl.n_layers):
             m.set_router(layer, synth.router_weights(wl, layer))

@@ -40,8 +40,9 @@ def test_library_exports_every_declared_symbol(lib):
 def test_config_struct_layout_matches_header(lib):
     from paper_2605_29135_gb300._lib import MoeConfig, TraceRec
 
-    # int32 x6, int32 x2, int64 x2, int32 x2, pointer, int64, int32 x2
-    assert ctypes.sizeof(MoeConfig) == 6 * 4 + 2 * 4 + 2 * 8 + 2 * 4 + 8 + 8 + 8 + 8  # batched_path, policy
+    # int32 x6, int32 x2, int64 x2, int32 x2, pointer, int64, int32 x5 (+ 4 bytes of tail padding)
+    assert ctypes.sizeof(MoeConfig) == 6 * 4 + 2 * 4 + 2 * 8 + 2 * 4 + 8 + 8 + 5 * 4 + 4
+    assert MoeConfig.lookahead.offset == 88
     assert ctypes.sizeof(TraceRec) == 24
 
 

@@ -51,6 +51,8 @@ BAD = [
     (dict(raw_batched_path=3), "unknown batched_path"),
     (dict(raw_policy=9), "unknown policy"),
     (dict(policy="rotary", max_batch=4), "rotary policy runs at batch 1"),
+    (dict(raw_lookahead=2), "lookahead must be 0 or 1"),
+    (dict(lookahead=True), "lookahead needs the host copy-engine schedule"),
 ]
 
 

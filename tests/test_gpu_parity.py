@@ -27,13 +27,17 @@ def P():
     return P
 
 
-SCHEDULES = ["device", "host_copy_engine"]
+# "host_lookahead": the host copy-engine schedule routing layer l + 1 while layer l computes; it
+# must give the same trace and outputs as the others
+SCHEDULES = ["device", "host_copy_engine", "host_lookahead"]
 _ORACLE_CACHE = {}
 
 
 def _create(wl, cap, schedule="device"):
     from paper_2605_29135_gb300.workload import create_for_workload
 
+    if schedule == "host_lookahead":
+        return create_for_workload(wl, cap_slots=cap, schedule="host_copy_engine", lookahead=True)
     return create_for_workload(wl, cap_slots=cap, schedule=schedule)
 
 
@@ -99,7 +103,8 @@ def test_cap_invariance_bit_exact_across_schedules(P, name):
     tokens = min(wl.tokens, 96)
     hidden = synth.hidden_all(wl, tokens)
     outs = []
-    for cap, schedule in ((wl.cap_slots, "device"), (wl.n_gid, "device"), (wl.cap_slots, "host_copy_engine")):
+    for cap, schedule in ((wl.cap_slots, "device"), (wl.n_gid, "device"), (wl.cap_slots, "host_copy_engine"),
+                          (wl.cap_slots, "host_lookahead")):
         m = _create(wl, cap, schedule)
         try:
             outs.append(run_gpu(m, hidden, wl.adtype)[0])
@@ -107,6 +112,7 @@ def test_cap_invariance_bit_exact_across_schedules(P, name):
             m.destroy()
     np.testing.assert_array_equal(outs[0], outs[1])
     np.testing.assert_array_equal(outs[0], outs[2])
+    np.testing.assert_array_equal(outs[0], outs[3])
 
 
 RAGGED = {

@@ -20,14 +20,18 @@ def P():
     return P
 
 
-SCHEDULES = ["device", "host_copy_engine"]
+# "host_lookahead": the host schedule routing layer l + 1 while layer l computes. Rotary victims can
+# be experts the previous layer still reads, so this also covers the copy that must wait for them.
+SCHEDULES = ["device", "host_copy_engine", "host_lookahead"]
 
 
 def _run(wl, cap, policy, preload=False, schedule="device"):
     from paper_2605_29135_gb300.workload import create_for_workload
 
     hidden = synth.hidden_all(wl)
-    m = create_for_workload(wl, cap_slots=cap, schedule=schedule, policy=policy)
+    look = schedule == "host_lookahead"
+    m = create_for_workload(wl, cap_slots=cap, schedule="host_copy_engine" if look else schedule, policy=policy,
+                            lookahead=look)
     try:
         if preload:
             m.preload()
