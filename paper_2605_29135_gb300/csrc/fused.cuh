@@ -134,6 +134,11 @@ struct BatchArgs {
   int touch_shift;             // log2 of the translation-warming touch stride (0: no touches)
   int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
   int router_tb;               // sequences per router work item (batched_router_tb)
+  // Rotary slot-group policy (policy == 1), as in FusedArgs
+  int policy;                  // 0 LRU, 1 rotary
+  int32_t* prior;              // [cap]
+  int32_t* prior_slot_of;      // [n_gid]
+  int32_t* hand;               // [1]
 };
 
 // Pairs staged per group for this shape, and the co-resident grid (0: shape or cap unsupported).

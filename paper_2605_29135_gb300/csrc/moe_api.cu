@@ -225,7 +225,6 @@ std::string check_config(const moe_config* c) {
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
   if (c->policy == MOE_POLICY_GUIDED) return "the router-guided policy is available in the residency planner only";
   if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY) return "unknown policy";
-  if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
   return "";
 }
 
@@ -654,6 +653,10 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.touch_shift = h->touch_shift;
   a.tg_max = h->tg_max;
   a.router_tb = moe::batched_router_tb(c.wdtype, c.d, c.d_ff, h->batched_tc);
+  a.policy = c.policy;
+  a.prior = h->d_prior;
+  a.prior_slot_of = h->d_prior_slot_of;
+  a.hand = h->d_hand;
   a.map_gu = h->map_gu;
   a.map_d = h->map_d;
   a.map_x = h->map_x;
