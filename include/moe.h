@@ -97,7 +97,8 @@ enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
  *     previous occupant. A miss returns to the slot it was last evicted from when that slot holds no
  *     expert of the layer-step (reverse rotation), else takes the first such slot at or after the
  *     hand, which then moves past it (forward rotation). Hits change nothing. Misses in ascending
- *     global id. Both schedules, max_batch 1. */
+ *     global id. Both schedules; a batched step (device schedule) applies it to the union of the
+ *     batch's experts. */
 /*   MOE_POLICY_GUIDED: router-guided replacement, one reading of the paper's residency decisions
  *     that use information produced during execution (Sec. 3). Each layer keeps the rank of every
  *     expert in its most recent routing (0 = highest logit; for a batch, the best rank over its

@@ -156,9 +156,13 @@ struct BatchArgs {
   int touch_shift;             // log2 of the translation-warming touch stride (0: no touches)
   int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
   int router_tb;               // sequences per router work item (batched_router_tb)
-  int policy;                  // 0 LRU, 2 router-guided
+  int policy;                  // 0 LRU, 1 rotary, 2 router-guided
   int32_t* rank;               // [L*E] router-guided: rank in the layer's latest routing (best over the batch)
   int32_t* rank_best;          // [E] router-guided scratch: this layer-step's best rank over the batch
+  // Rotary slot-group policy (policy == 1), as in FusedArgs
+  int32_t* prior;              // [cap]
+  int32_t* prior_slot_of;      // [n_gid]
+  int32_t* hand;               // [1]
 };
 
 // Pairs staged per group for this shape, and the co-resident grid (0: shape or cap unsupported).

@@ -132,6 +132,81 @@ __device__ __forceinline__ void router_block(const BatchArgs& a, int l, int tb, 
 }
 
 // ---- phase S: union of the pairs' experts, one lookup-table step, trace and plan (CTA 0)
+// Rotary slot-group step for the misses of a batched layer-step (thread 0 of CTA 0): the rule of
+// the batch-1 kernel applied to the union of the batch's experts, misses in ascending id. A miss
+// returns to the slot it was last evicted from when that slot holds no expert of the step
+// (reverse rotation), else takes the first such slot at or after the hand, which moves past it
+// (forward rotation); the occupant is evicted and remembered as the slot's previous occupant, and
+// the placed expert stops being anyone's previous occupant. Up to E misses per step, so the slot
+// state is read and written in global memory as it goes rather than staged: the occupant of a slot
+// is the low half of its key (all ones: empty), and each placement writes its key at once.
+// needed(o): o belongs to layer l and has pairs this step (tot[o - l * E] > 0).
+__device__ void batched_rotary_place(const BatchArgs& a, int l, int clock, int n, const int* need_e,
+                                     const int* miss, const int* tot, int* slot_out, int* evict_out,
+                                     int* n_evicted) {
+  const int E = a.E;
+  const int64_t cap = a.cap;
+  auto occupant = [&](int64_t sl) {
+    const unsigned long long key = __ldcg(a.slot_key + sl);
+    return key == ~0ull ? -1 : (int)(uint32_t)(key & 0xffffffffull);
+  };
+  auto needed = [&](int o) { return o >= l * E && o < (l + 1) * E && tot[o - l * E] > 0; };
+  int hand = *(volatile int32_t*)a.hand;
+  int nused = *(volatile int32_t*)a.n_used;
+  int evicted = 0;
+  for (int q = 0; q < n; q++) {
+    if (!miss[q]) continue;
+    const int g = l * E + need_e[q];
+    int slot = -1, occ = -1;
+    int ps = __ldcg(a.prior_slot_of + g);
+    if (ps >= 0 && __ldcg(a.prior + ps) != g) ps = -1;  // the inverse entry is stale
+    if (ps >= 0) {
+      const int o = occupant(ps);
+      if (o < 0 || !needed(o)) {
+        slot = ps;
+        occ = o;
+      }
+    }
+    if (slot < 0) {
+      for (int64_t j = 0; j < cap; j++) {
+        const int64_t sl = (hand + j) % cap;
+        const int o = occupant(sl);
+        if (o < 0 || !needed(o)) {
+          slot = (int)sl;
+          occ = o;
+          break;
+        }
+      }
+      if (slot < 0) {
+        atomicOr(a.err, FERR_NO_VICTIM);
+        slot_out[q] = -1;
+        continue;
+      }
+      hand = (int)((slot + 1) % cap);
+    }
+    if (occ >= 0) {
+      a.slot_of[occ] = -1;
+      evicted++;
+    } else {
+      nused++;
+    }
+    if (ps >= 0) a.prior[ps] = -1;  // g is placed: no longer a previous occupant
+    const int u = __ldcg(a.prior + slot);  // the slot's previous occupant loses its return slot
+    if (u >= 0) a.prior_slot_of[u] = -1;
+    a.prior[slot] = occ;
+    if (occ >= 0) a.prior_slot_of[occ] = slot;
+    a.prior_slot_of[g] = -1;
+    a.slot_of[g] = slot;
+    a.slot_key[slot] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)g;
+    __threadfence_block();
+    slot_out[q] = slot;
+    evict_out[q] = occ;
+  }
+  *a.hand = hand;
+  *a.n_used = nused;
+  *n_evicted = evicted;
+}
+
 __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t step, unsigned long long* keys) {
   constexpr int kChunks = kMaxPairs / 32;
   __shared__ int s_sel[kMaxPairs];       // expert of pair p
@@ -233,7 +308,7 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
     if (lane == 0) {
       const int nfree = (int)(a.cap - s_nused0);
       const int take = nm < nfree ? nm : nfree;
-      *a.n_used = s_nused0 + take;
+      if (a.policy != 1) *a.n_used = s_nused0 + take;
       s_n = n;
       s_nm = nm;
       s_nfree = nfree;
@@ -242,7 +317,10 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   }
   __syncthreads();
   const int n = s_n, nm = s_nm, nfree = s_nfree, nev = s_nev;
-  if (nev > 0) {
+  if (a.policy == 1) {
+    if (tid == 0 && nm > 0) batched_rotary_place(a, l, clock, n, s_need, s_miss, s_tot, s_slot, s_evict, &s_nevicted);
+    __syncthreads();
+  } else if (nev > 0) {
     // Every slot is occupied. Sort the slot keys (last use << 32 | id) ascending, with the slots
     // of this step's hits pinned at the maximum: the first nev keys are the victims.
     int N2 = 1;
@@ -271,7 +349,7 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   // place the misses: free slots first, then the victims in ascending key order
   for (int q = tid; q < n; q += blockDim.x) {
     s_pos[q] = s_miss[q] ? s_mbefore[q] : nm + (q - s_mbefore[q]);
-    if (!s_miss[q]) continue;
+    if (!s_miss[q] || a.policy == 1) continue;
     const int m = s_mbefore[q];
     int slot = -1;
     if (m < nfree) {

@@ -232,7 +232,6 @@ std::string check_config(const moe_config* c) {
     return "unknown policy";
   if (c->policy == MOE_POLICY_GUIDED && (int64_t)c->n_layers * c->n_experts >= (1LL << moe::kGuidedGidBits))
     return "the router-guided policy needs n_layers * n_experts < 2^23";
-  if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
   if (c->lookahead != 0 && c->lookahead != 1) return "lookahead must be 0 or 1";
   if (c->lookahead && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "lookahead needs the host copy-engine schedule";
   return "";
@@ -709,6 +708,9 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.policy = c.policy;
   a.rank = h->d_rank;
   a.rank_best = h->d_rank_best;
+  a.prior = h->d_prior;
+  a.prior_slot_of = h->d_prior_slot_of;
+  a.hand = h->d_hand;
   a.map_gu = h->map_gu;
   a.map_d = h->map_d;
   a.map_x = h->map_x;
