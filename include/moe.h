@@ -279,6 +279,25 @@ moe_status moe_inject_fault(moe_handle* h, int32_t kind);
 moe_status moe_route_noalloc(const void* w_r, const void* hidden, int32_t rows, int32_t n_experts, int32_t d,
                              int32_t top_k, int32_t renorm, int32_t wdtype, int32_t* idx, float* gate, void* stream);
 
+/* ---- Attention of the decoder block around the MoE layer ------------------------------------
+ * Grouped-query attention of one decode token over a KV cache (the decoder the paper ran kept a
+ * 4096-token context). No handle; nothing is allocated.
+ *   q        device fp32 [n_heads x head_dim], already normalised, rotated (scale 1/sqrt(head_dim)
+ *            is applied inside)
+ *   k_cache, v_cache  device bf16 [n_kv_heads x max_pos x head_dim], 16-byte aligned; positions
+ *            [0, n_pos) are read
+ *   out      device fp32 [n_heads x head_dim]: query head h reads kv head h / (n_heads / n_kv_heads);
+ *            out_h = sum_j softmax_j(q_h . k_j / sqrt(head_dim)) v_j
+ *   scratch  device fp32 of at least moe_attention_scratch_floats(...) floats (per-split partials)
+ *   stream   cudaStream_t the two kernels are ordered on (NULL = legacy default stream)
+ * head_dim 64 or 128; n_heads / n_kv_heads in {1, 2, 4, 8}; 1 <= n_pos <= max_pos. MOE_ERR_INVALID
+ * for other arguments (moe_attention_scratch_floats returns -1 for them), MOE_ERR_CUDA if a
+ * launch fails. */
+int64_t moe_attention_scratch_floats(int32_t n_heads, int32_t n_kv_heads, int32_t head_dim, int64_t n_pos);
+moe_status moe_attention_decode(const float* q, const void* k_cache, const void* v_cache, int32_t n_heads,
+                                int32_t n_kv_heads, int32_t head_dim, int64_t max_pos, int64_t n_pos, float* out,
+                                float* scratch, int64_t scratch_floats, void* stream);
+
 /* ---- Residency planner ------------------------------------------------------------------------
  * The library's host slot table (the code the MOE_SCHEDULE_HOST_COPY_ENGINE schedule runs, and
  * the same rules the device schedule's kernel applies) driven by expert selections the caller

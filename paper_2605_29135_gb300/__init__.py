@@ -295,6 +295,33 @@ class Planner:
         self.destroy()
 
 
+def attention_decode(q, k_cache, v_cache, n_pos: int, stream=None):
+    """Grouped-query attention of one decode token (moe_attention_decode). q: device float32
+    [n_heads x head_dim]; k_cache, v_cache: device bfloat16 [n_kv_heads x max_pos x head_dim].
+    Returns out, device float32 [n_heads x head_dim]."""
+    import torch
+
+    Hq, D = q.shape
+    Hkv, Tmax, D2 = k_cache.shape
+    if D2 != D or tuple(v_cache.shape) != tuple(k_cache.shape):
+        raise ValueError("q, k_cache and v_cache shapes disagree")
+    if q.dtype != torch.float32 or k_cache.dtype != torch.bfloat16 or v_cache.dtype != torch.bfloat16:
+        raise ValueError("q must be float32, the caches bfloat16")
+    lib = _lib.load()
+    n = lib.moe_attention_scratch_floats(Hq, Hkv, D, n_pos)
+    if n < 0:
+        raise MoEError(-1, "moe_attention_decode does not take this shape")
+    scratch = torch.empty(n, dtype=torch.float32, device=q.device)
+    out = torch.empty((Hq, D), dtype=torch.float32, device=q.device)
+    if stream is None:
+        stream = torch.cuda.current_stream(q.device)
+    st = lib.moe_attention_decode(_ptr(q), _ptr(k_cache), _ptr(v_cache), Hq, Hkv, D, Tmax, n_pos, _ptr(out),
+                                  _ptr(scratch), n, ctypes.c_void_p(stream.cuda_stream))
+    if st != 0:
+        raise MoEError(st, "moe_attention_decode rejected the arguments" if st == -1 else "launch failed")
+    return out
+
+
 def route_noalloc(w_r, hidden, top_k: int, renorm: bool = True, stream=None):
     """Routing without any device allocation by the library (moe_route_noalloc).
 

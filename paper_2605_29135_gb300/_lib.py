@@ -26,7 +26,8 @@ EXPORTS = ["moe_expert_bytes", "moe_pool_bytes", "moe_create", "moe_set_router",
            "moe_decode_step", "moe_decode_step_host", "moe_get_residency_trace", "moe_get_last_routing",
            "moe_get_stats", "moe_reset_residency", "moe_profile_enable", "moe_profile_read", "moe_last_error",
            "moe_destroy", "moe_route_noalloc", "moe_preload", "moe_inject_fault", "moe_planner_create",
-           "moe_planner_preload", "moe_planner_step", "moe_planner_last_error", "moe_planner_destroy"]
+           "moe_planner_preload", "moe_planner_step", "moe_planner_last_error", "moe_planner_destroy",
+           "moe_attention_scratch_floats", "moe_attention_decode"]
 
 
 class MoeConfig(ctypes.Structure):
@@ -114,6 +115,10 @@ def load(path: str | None = None):
         L.moe_planner_step.restype = ctypes.c_int
         L.moe_planner_last_error.argtypes = [vp]
         L.moe_planner_last_error.restype = ctypes.c_char_p
+        L.moe_attention_scratch_floats.argtypes = [i32, i32, i32, i64]
+        L.moe_attention_scratch_floats.restype = i64
+        L.moe_attention_decode.argtypes = [vp, vp, vp, i32, i32, i32, i64, i64, vp, vp, i64, vp]
+        L.moe_attention_decode.restype = ctypes.c_int
         L.moe_planner_destroy.argtypes = [vp]
         L.moe_planner_destroy.restype = None
         _lib = L

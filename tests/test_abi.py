@@ -113,3 +113,14 @@ def test_header_compiles_as_plain_c_and_cpp(lang, std, tmp_path):
     src.write_text('#include "moe.h"\nint main(void) { moe_config c; (void)c; return (int)sizeof(moe_trace_rec) - 24; }\n')
     subprocess.run([cc, f"-std={std}", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", os.path.join(ROOT, "include"),
                     "-fsyntax-only", str(src)], check=True)
+
+
+def test_attention_scratch_size_and_argument_checks_without_gpu(lib):
+    # splits: about 304 CTAs over the kv heads, at least 16 positions each, none empty
+    assert lib.moe_attention_scratch_floats(32, 4, 128, 4095) == 32 * 76 * 130
+    assert lib.moe_attention_scratch_floats(8, 2, 64, 100) == 8 * 7 * 66
+    assert lib.moe_attention_scratch_floats(4, 4, 128, 1) == 4 * 1 * 130
+    for args in [(32, 4, 96, 10), (32, 5, 128, 10), (48, 3, 128, 10), (4, 4, 128, 0), (64, 4, 128, 10)]:
+        assert lib.moe_attention_scratch_floats(*args) == -1
+    # NULL buffers are refused before any device work
+    assert lib.moe_attention_decode(None, None, None, 32, 4, 128, 4096, 10, None, None, 0, None) == -1
