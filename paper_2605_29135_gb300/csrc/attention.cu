@@ -5,14 +5,15 @@
 // positions (each K and V row is read once for all of those heads), and a second kernel merges the
 // splits with their maxima.
 //
-// Arithmetic: fp32 throughout on bf16 K/V and fp32 q; scores are q . k / sqrt(D) with the scale
-// folded into q; exponentials by expf against the running maximum.
+// Arithmetic: fp32 throughout on bf16 or fp32 K/V and fp32 q; scores are q . k / sqrt(D) with the
+// scale folded into q; exponentials by expf against the running maximum.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
 
 #include "moe.h"
+#include "moe_internal.h"
 
 namespace {
 
@@ -25,7 +26,23 @@ __device__ __forceinline__ float warp_allsum(float v) {
   return v;
 }
 
-// VPL consecutive bf16 of a row (VPL = 2 or 4), widened exactly to fp32.
+// VPL consecutive elements of a row (VPL = 2 or 4), widened exactly to fp32.
+template <int VPL>
+__device__ __forceinline__ void load_row(const float* p, float (&f)[VPL]) {
+  static_assert(VPL == 2 || VPL == 4, "head_dim 64 or 128");
+  if constexpr (VPL == 4) {
+    const float4 w = __ldg(reinterpret_cast<const float4*>(p));
+    f[0] = w.x;
+    f[1] = w.y;
+    f[2] = w.z;
+    f[3] = w.w;
+  } else {
+    const float2 w = __ldg(reinterpret_cast<const float2*>(p));
+    f[0] = w.x;
+    f[1] = w.y;
+  }
+}
+
 template <int VPL>
 __device__ __forceinline__ void load_row(const __nv_bfloat16* p, float (&f)[VPL]) {
   static_assert(VPL == 2 || VPL == 4, "head_dim 64 or 128");
@@ -45,10 +62,10 @@ __device__ __forceinline__ void load_row(const __nv_bfloat16* p, float (&f)[VPL]
 // Split sp of kv head g: positions [sp * per, min(T, (sp + 1) * per)). Warp w takes positions
 // p0 + w, p0 + w + 8, ...; lane holds dims [lane * VPL, lane * VPL + VPL) of every vector. The CTA's
 // warps are merged in shared memory into part[g][sp][h] = (acc[D], max, sum).
-template <int VPL, int G>
-__global__ void __launch_bounds__(kAttnWarps * 32) k_attn_split(const float* q, const __nv_bfloat16* K,
-                                                                const __nv_bfloat16* V, int64_t Tmax, int64_t T,
-                                                                int64_t per, int nsplit, float* part) {
+template <typename CT, int VPL, int G>
+__global__ void __launch_bounds__(kAttnWarps * 32) k_attn_split(const float* q, const CT* K, const CT* V,
+                                                                int64_t Tmax, int64_t T, int64_t per, int nsplit,
+                                                                float* part) {
   constexpr int D = 32 * VPL;
   __shared__ float s_m[kAttnWarps][G], s_l[kAttnWarps][G];
   __shared__ float s_acc[kAttnWarps][G][D];
@@ -70,8 +87,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_split(const float* q, 
   }
   const int64_t p0 = (int64_t)sp * per;
   const int64_t p1 = p0 + per < T ? p0 + per : T;
-  const __nv_bfloat16* Kg = K + (int64_t)g * Tmax * D + lane * VPL;
-  const __nv_bfloat16* Vg = V + (int64_t)g * Tmax * D + lane * VPL;
+  const CT* Kg = K + (int64_t)g * Tmax * D + lane * VPL;
+  const CT* Vg = V + (int64_t)g * Tmax * D + lane * VPL;
   for (int64_t j = p0 + warp; j < p1; j += kAttnWarps) {
     float kf[VPL], vf[VPL];
     load_row<VPL>(Kg + j * D, kf);
@@ -154,17 +171,34 @@ void split_plan(int32_t n_kv_heads, int64_t n_pos, int* nsplit, int64_t* per) {
   *per = p;
 }
 
-template <int VPL>
-cudaError_t launch_split(int G, const float* q, const __nv_bfloat16* K, const __nv_bfloat16* V, int Hkv,
-                         int64_t Tmax, int64_t T, int64_t per, int nsplit, float* part, cudaStream_t s) {
+template <typename CT, int VPL>
+cudaError_t launch_split(int G, const float* q, const CT* K, const CT* V, int Hkv, int64_t Tmax, int64_t T,
+                         int64_t per, int nsplit, float* part, cudaStream_t s) {
   const dim3 grid(nsplit, Hkv), block(kAttnWarps * 32);
   switch (G) {
-    case 1: k_attn_split<VPL, 1><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
-    case 2: k_attn_split<VPL, 2><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
-    case 4: k_attn_split<VPL, 4><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
-    case 8: k_attn_split<VPL, 8><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
+    case 1: k_attn_split<CT, VPL, 1><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
+    case 2: k_attn_split<CT, VPL, 2><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
+    case 4: k_attn_split<CT, VPL, 4><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
+    case 8: k_attn_split<CT, VPL, 8><<<grid, block, 0, s>>>(q, K, V, Tmax, T, per, nsplit, part); break;
     default: return cudaErrorInvalidValue;
   }
+  return cudaGetLastError();
+}
+
+template <typename CT>
+cudaError_t launch_attention(const float* q, const void* k_cache, const void* v_cache, int32_t n_heads,
+                             int32_t n_kv_heads, int32_t head_dim, int64_t max_pos, int64_t n_pos, float* out,
+                             float* scratch, cudaStream_t s) {
+  int nsplit;
+  int64_t per;
+  split_plan(n_kv_heads, n_pos, &nsplit, &per);
+  const int G = n_heads / n_kv_heads;
+  const CT* K = (const CT*)k_cache;
+  const CT* V = (const CT*)v_cache;
+  cudaError_t e = head_dim == 128 ? launch_split<CT, 4>(G, q, K, V, n_kv_heads, max_pos, n_pos, per, nsplit, scratch, s)
+                                  : launch_split<CT, 2>(G, q, K, V, n_kv_heads, max_pos, n_pos, per, nsplit, scratch, s);
+  if (e != cudaSuccess) return e;
+  k_attn_merge<<<n_heads, head_dim, 0, s>>>(scratch, head_dim, G, nsplit, out);
   return cudaGetLastError();
 }
 
@@ -177,6 +211,33 @@ bool valid_shape(int32_t n_heads, int32_t n_kv_heads, int32_t head_dim) {
 
 }  // namespace
 
+namespace moe {
+
+bool attention_shape_ok(int32_t n_heads, int32_t n_kv_heads, int32_t head_dim) {
+  return valid_shape(n_heads, n_kv_heads, head_dim);
+}
+
+// split_plan gives at most min(304 / n_kv_heads, ceil(n_pos / 16)) splits (and at least one), a
+// bound that only grows with n_pos, so this many partials serve every n_pos <= max_pos.
+int64_t attention_scratch_bound(int32_t n_heads, int32_t n_kv_heads, int32_t head_dim, int64_t max_pos) {
+  int64_t ns = 304 / n_kv_heads;
+  const int64_t by_len = (max_pos + 15) / 16;
+  if (ns > by_len) ns = by_len;
+  if (ns < 1) ns = 1;
+  return (int64_t)n_heads * ns * (head_dim + 2);
+}
+
+cudaError_t attention_launch(int32_t cache_dtype, const float* q, const void* k_cache, const void* v_cache,
+                             int32_t n_heads, int32_t n_kv_heads, int32_t head_dim, int64_t max_pos, int64_t n_pos,
+                             float* out, float* scratch, cudaStream_t s) {
+  if (cache_dtype == MOE_DTYPE_FP32)
+    return launch_attention<float>(q, k_cache, v_cache, n_heads, n_kv_heads, head_dim, max_pos, n_pos, out, scratch, s);
+  return launch_attention<__nv_bfloat16>(q, k_cache, v_cache, n_heads, n_kv_heads, head_dim, max_pos, n_pos, out,
+                                         scratch, s);
+}
+
+}  // namespace moe
+
 extern "C" {
 
 int64_t moe_attention_scratch_floats(int32_t n_heads, int32_t n_kv_heads, int32_t head_dim, int64_t n_pos) {
@@ -187,25 +248,17 @@ int64_t moe_attention_scratch_floats(int32_t n_heads, int32_t n_kv_heads, int32_
   return (int64_t)n_heads * nsplit * (head_dim + 2);
 }
 
-moe_status moe_attention_decode(const float* q, const void* k_cache, const void* v_cache, int32_t n_heads,
-                                int32_t n_kv_heads, int32_t head_dim, int64_t max_pos, int64_t n_pos, float* out,
-                                float* scratch, int64_t scratch_floats, void* stream) {
+moe_status moe_attention_decode(const float* q, const void* k_cache, const void* v_cache, int32_t cache_dtype,
+                                int32_t n_heads, int32_t n_kv_heads, int32_t head_dim, int64_t max_pos, int64_t n_pos,
+                                float* out, float* scratch, int64_t scratch_floats, void* stream) {
   if (!q || !k_cache || !v_cache || !out || !scratch) return MOE_ERR_INVALID;
+  if (cache_dtype != MOE_DTYPE_FP32 && cache_dtype != MOE_DTYPE_BF16) return MOE_ERR_INVALID;
   if (!valid_shape(n_heads, n_kv_heads, head_dim) || n_pos < 1 || n_pos > max_pos) return MOE_ERR_INVALID;
   if (((uintptr_t)k_cache | (uintptr_t)v_cache) & 15) return MOE_ERR_INVALID;
   if (scratch_floats < moe_attention_scratch_floats(n_heads, n_kv_heads, head_dim, n_pos)) return MOE_ERR_INVALID;
-  int nsplit;
-  int64_t per;
-  split_plan(n_kv_heads, n_pos, &nsplit, &per);
-  const int G = n_heads / n_kv_heads;
-  cudaStream_t s = (cudaStream_t)stream;
-  const __nv_bfloat16* K = (const __nv_bfloat16*)k_cache;
-  const __nv_bfloat16* V = (const __nv_bfloat16*)v_cache;
-  cudaError_t e = head_dim == 128 ? launch_split<4>(G, q, K, V, n_kv_heads, max_pos, n_pos, per, nsplit, scratch, s)
-                                  : launch_split<2>(G, q, K, V, n_kv_heads, max_pos, n_pos, per, nsplit, scratch, s);
-  if (e != cudaSuccess) return MOE_ERR_CUDA;
-  k_attn_merge<<<n_heads, head_dim, 0, s>>>(scratch, head_dim, G, nsplit, out);
-  return cudaGetLastError() == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+  const cudaError_t e = moe::attention_launch(cache_dtype, q, k_cache, v_cache, n_heads, n_kv_heads, head_dim, max_pos,
+                                              n_pos, out, scratch, (cudaStream_t)stream);
+  return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
 }
 
 }  // extern "C"
