@@ -1,5 +1,6 @@
 """The decoder block's attention (moe_attention_decode) through the C ABI against the fp64 oracle's
-grouped-query attention on the same inputs: fp32 q, bf16 K/V (widened exactly for the oracle).
+grouped-query attention on the same inputs: fp32 q, bf16 or fp32 K/V (widened exactly for the
+oracle).
 Relative L2 error per query head <= 1e-5 (fp32 arithmetic over up to 4096 positions); a single
 cached position returns its value row exactly; the kv-head grouping and the split merge are
 covered by shapes whose position counts leave ragged splits."""
@@ -28,13 +29,14 @@ def P():
     return P
 
 
-def _inputs(Hq, Hkv, D, Tmax, seed):
+def _inputs(Hq, Hkv, D, Tmax, seed, cache="bf16"):
     import torch
 
     g = torch.Generator().manual_seed(seed)
+    cdt = torch.bfloat16 if cache == "bf16" else torch.float32
     q = torch.randn(Hq, D, generator=g, dtype=torch.float32) * 2.0
-    K = torch.randn(Hkv, Tmax, D, generator=g, dtype=torch.float32).to(torch.bfloat16)
-    V = torch.randn(Hkv, Tmax, D, generator=g, dtype=torch.float32).to(torch.bfloat16)
+    K = torch.randn(Hkv, Tmax, D, generator=g, dtype=torch.float32).to(cdt)
+    V = torch.randn(Hkv, Tmax, D, generator=g, dtype=torch.float32).to(cdt)
     return q, K, V
 
 
@@ -43,6 +45,15 @@ def test_attention_matches_oracle(P, Hq, Hkv, D, Tmax, T):
     q, K, V = _inputs(Hq, Hkv, D, Tmax, seed=T)
     out = P.attention_decode(q.cuda(), K.cuda(), V.cuda(), T).cpu().numpy().astype(np.float64)
     ref = attend(q.double().numpy(), K.float().double().numpy(), V.float().double().numpy(), T)
+    err = np.linalg.norm(out - ref, axis=1) / np.linalg.norm(ref, axis=1)
+    assert err.max() <= 1e-5, f"max rel L2 {err.max():.3e}"
+
+
+@pytest.mark.parametrize("Hq,Hkv,D,Tmax,T", [(4, 2, 64, 40, 33), (8, 1, 128, 600, 599)])
+def test_fp32_cache_matches_oracle(P, Hq, Hkv, D, Tmax, T):
+    q, K, V = _inputs(Hq, Hkv, D, Tmax, seed=T + 1, cache="fp32")
+    out = P.attention_decode(q.cuda(), K.cuda(), V.cuda(), T).cpu().numpy().astype(np.float64)
+    ref = attend(q.double().numpy(), K.double().numpy(), V.double().numpy(), T)
     err = np.linalg.norm(out - ref, axis=1) / np.linalg.norm(ref, axis=1)
     assert err.max() <= 1e-5, f"max rel L2 {err.max():.3e}"
 
