@@ -747,7 +747,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
   unsigned nbar = 0;  // grid barriers passed in this launch
   if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[a.L * 4] = gtimer();
 
-  for (int l = 0; l < a.L; l++) {
+  for (int l = a.l_begin; l < a.l_end; l++) {
     const int clock = (int)(step * a.L + l + 1);  // 0 is older than every step (preloaded experts)
     // ---- phase R: router logits. A warp's row loads (8 chunks per lane at a time) are issued
     // before the CTA stages h, so their latency overlaps the staging.
@@ -958,7 +958,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
     if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 3] = gtimer();
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
+  if (a.l_end == a.L && blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
 }
 
 size_t fused_smem(int wdtype, int d, int I, int k) {

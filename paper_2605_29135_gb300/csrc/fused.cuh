@@ -22,6 +22,9 @@ constexpr int FERR_FATAL = FERR_BARRIER_TIMEOUT | FERR_PIPE_TIMEOUT;
 
 struct FusedArgs {
   int L, E, k, d, I, renorm, wdtype;
+  int l_begin, l_end;          // layers [l_begin, l_end) run in this launch; the launch that ends at
+                               // layer L completes the decode step (a chained decoder launches one
+                               // layer at a time, each after the attention that produces its input)
   BlobLayout lay;
   int64_t slot_stride;
   int64_t cap;

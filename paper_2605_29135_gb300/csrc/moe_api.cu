@@ -31,6 +31,7 @@
 #include "fused.cuh"
 #include "kernels.cuh"
 #include "moe.h"
+#include "moe_internal.h"
 #include "slot_table.h"
 
 namespace {
@@ -738,14 +739,17 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   return MOE_OK;
 }
 
-moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
-  moe_status st = check_device_error(h, false);
-  if (st != MOE_OK) return st;
-  if (h->batched) return decode_batched(h, hidden, out, batch, s);
+// Layers [l0, l1) of a batch-1 decode step in one launch of the fused kernel; the launch that
+// reaches the last layer completes the step. Per-phase profiling covers whole-step launches only.
+moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, int32_t l0, int32_t l1,
+                                cudaStream_t s) {
   const moe_config& c = h->cfg;
   const int k = c.top_k;
+  const bool whole = l0 == 0 && l1 == c.n_layers;
   moe::FusedArgs a{};
   a.L = c.n_layers;
+  a.l_begin = l0;
+  a.l_end = l1;
   a.E = c.n_experts;
   a.k = k;
   a.d = c.d;
@@ -791,10 +795,10 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   arm_barrier_fault(h, a.bar_base, a.barrier_timeout_ns);
   a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
   a.touch_shift = h->touch_shift;
-  a.phase_ts = phase_buffer(h);
+  a.phase_ts = whole ? phase_buffer(h) : nullptr;
   {
     ProfScope ps(h, s, PC_FUSED,
-                 (int64_t)c.n_layers * (k * h->lay.total + (int64_t)c.n_experts * c.d * h->router_eb));
+                 (int64_t)(l1 - l0) * (k * h->lay.total + (int64_t)c.n_experts * c.d * h->router_eb));
     cudaError_t e = moe::launch_fused(a, h->fgrid, s);
     ps.done();
     if (e != cudaSuccess) return cuda_fail(h, e, "fused decode step launch");
@@ -802,14 +806,43 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   MOE_CK(h, cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, s));
   MOE_CK(h, cudaEventRecord(h->err_ev, s));
   h->err_pending = true;
-  h->steps_launched++;
-  h->bar_epoch += 3u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
+  if (l1 == c.n_layers) h->steps_launched++;
+  h->bar_epoch += 3u * (unsigned)(l1 - l0) * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
   if (a.phase_ts) {
     // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
     static const int cls[4] = {PC_PH_R, PC_PH_S, PC_PH_C, PC_PH_D};
     return harvest_phases(h, a.phase_ts, 4, cls, s);
   }
   return MOE_OK;
+}
+
+moe_status check_registered(moe_handle* h) {
+  if (h->all_registered) return MOE_OK;
+  for (int32_t l = 0; l < h->cfg.n_layers; l++)
+    if (!h->router_set[l]) return fail(h, MOE_ERR_NOT_REGISTERED, "router of layer " + std::to_string(l) + " not set");
+  for (int64_t g = 0; g < h->n_gid; g++)
+    if (!h->registered[g])
+      return fail(h, MOE_ERR_NOT_REGISTERED, "expert " + std::to_string(g % h->cfg.n_experts) + " of layer " +
+                                                 std::to_string(g / h->cfg.n_experts) + " not registered");
+  h->all_registered = true;
+  return MOE_OK;
+}
+
+// The pool contents are unknown after a failed step: wait for the streams, empty the pool.
+void recover_after_failure(moe_handle* h, cudaStream_t s) {
+  std::string keep = h->err;
+  cudaStreamSynchronize(s);
+  cudaStreamSynchronize(h->copy_stream);
+  cudaGetLastError();
+  reset_state(h);
+  h->err = keep;
+}
+
+moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
+  moe_status st = check_device_error(h, false);
+  if (st != MOE_OK) return st;
+  if (h->batched) return decode_batched(h, hidden, out, batch, s);
+  return decode_device_layers(h, hidden, out, 0, h->cfg.n_layers, s);
 }
 
 // The driver's tensor-map encoder, looked up once per process (thread-safe static initialisation).
@@ -1090,27 +1123,12 @@ moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t
   if (!hidden || !out) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
   if (batch < 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be in [1, max_batch]");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
-  if (!h->all_registered) {
-    for (int32_t l = 0; l < h->cfg.n_layers; l++)
-      if (!h->router_set[l]) return fail(h, MOE_ERR_NOT_REGISTERED, "router of layer " + std::to_string(l) + " not set");
-    for (int64_t g = 0; g < h->n_gid; g++)
-      if (!h->registered[g])
-        return fail(h, MOE_ERR_NOT_REGISTERED, "expert " + std::to_string(g % h->cfg.n_experts) + " of layer " +
-                                                   std::to_string(g / h->cfg.n_experts) + " not registered");
-    h->all_registered = true;
-  }
+  moe_status st = check_registered(h);
+  if (st != MOE_OK) return st;
   NvtxRange range(h->dev_mode ? "moe_decode_step (device schedule)" : "moe_decode_step (host schedule)");
-  moe_status st = h->dev_mode ? decode_device(h, hidden, out, batch, (cudaStream_t)stream)
-                              : decode_impl(h, hidden, out, (cudaStream_t)stream);
-  if (st != MOE_OK) {
-    // The pool contents are unknown after a failed step: wait for the streams, empty the pool.
-    std::string keep = h->err;
-    cudaStreamSynchronize((cudaStream_t)stream);
-    cudaStreamSynchronize(h->copy_stream);
-    cudaGetLastError();
-    reset_state(h);
-    h->err = keep;
-  }
+  st = h->dev_mode ? decode_device(h, hidden, out, batch, (cudaStream_t)stream)
+                   : decode_impl(h, hidden, out, (cudaStream_t)stream);
+  if (st != MOE_OK) recover_after_failure(h, (cudaStream_t)stream);
   return st;
 }
 
@@ -1336,3 +1354,40 @@ void moe_destroy(moe_handle* h) {
 }
 
 }  // extern "C"
+
+namespace moe {
+
+bool moe_shape(const moe_handle* h, MoeShape* out) {
+  if (!h || !out) return false;
+  const moe_config& c = h->cfg;
+  out->d = c.d;
+  out->n_layers = c.n_layers;
+  out->top_k = c.top_k;
+  out->n_experts = c.n_experts;
+  out->wdtype = c.wdtype;
+  out->adtype = c.adtype;
+  out->device = c.device;
+  out->device_batch1 = h->dev_mode && !h->batched && c.max_batch == 1;
+  return true;
+}
+
+moe_status moe_run_layer(moe_handle* h, const void* hidden, void* out, int32_t layer, cudaStream_t s) {
+  if (!h) return MOE_ERR_INVALID;
+  if (!h->dev_mode || h->batched) return fail(h, MOE_ERR_INVALID, "a chained decoder needs the batch-1 device schedule");
+  if (layer < 0 || layer >= h->cfg.n_layers) return fail(h, MOE_ERR_INVALID, "layer out of range");
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  moe_status st = MOE_OK;
+  if (layer == 0) {
+    st = check_registered(h);
+    if (st != MOE_OK) return st;
+    st = check_device_error(h, false);
+    if (st != MOE_OK) return st;
+  }
+  st = decode_device_layers(h, hidden, out, layer, layer + 1, s);
+  if (st != MOE_OK) recover_after_failure(h, s);
+  return st;
+}
+
+const char* moe_error_text(const moe_handle* h) { return h ? h->err.c_str() : ""; }
+
+}  // namespace moe

@@ -101,3 +101,35 @@ def test_header_compiles_as_plain_c_and_cpp(lang, std, tmp_path):
     src.write_text('#include "moe.h"\nint main(void) { moe_config c; (void)c; return (int)sizeof(moe_trace_rec) - 24; }\n')
     subprocess.run([cc, f"-std={std}", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", os.path.join(ROOT, "include"),
                     "-fsyntax-only", str(src)], check=True)
+
+
+def test_attention_scratch_size_and_argument_checks_without_gpu(lib):
+    # splits: about 304 CTAs over the kv heads, at least 16 positions each, none empty
+    assert lib.moe_attention_scratch_floats(32, 4, 128, 4095) == 32 * 76 * 130
+    assert lib.moe_attention_scratch_floats(8, 2, 64, 100) == 8 * 7 * 66
+    assert lib.moe_attention_scratch_floats(4, 4, 128, 1) == 4 * 1 * 130
+    for args in [(32, 4, 96, 10), (32, 5, 128, 10), (48, 3, 128, 10), (4, 4, 128, 0), (64, 4, 128, 10)]:
+        assert lib.moe_attention_scratch_floats(*args) == -1
+    # NULL buffers are refused before any device work
+    assert lib.moe_attention_decode(None, None, None, 1, 32, 4, 128, 4096, 10, None, None, 0, None) == -1
+    # an unknown cache element type is refused too
+    dummy = ctypes.c_void_p(16)
+    assert lib.moe_attention_decode(dummy, dummy, dummy, 2, 32, 4, 128, 4096, 10, dummy, dummy, 1 << 30, None) == -1
+
+
+def test_decoder_config_layout_and_argument_checks_without_gpu(lib):
+    from paper_2605_29135_gb300._lib import DecoderConfig
+
+    # int32 x4, int64, double x2
+    assert ctypes.sizeof(DecoderConfig) == 4 * 4 + 8 + 2 * 8
+    assert DecoderConfig.max_pos.offset == 16 and DecoderConfig.eps.offset == 24
+    cfg = DecoderConfig(n_heads=32, n_kv_heads=4, head_dim=128, reserved=0, max_pos=4160, eps=1e-6, rope_theta=1e6)
+    out = ctypes.c_void_p(1)
+    assert lib.moe_decoder_create(None, ctypes.byref(cfg), ctypes.byref(out)) == -1
+    assert out.value is None  # *out is cleared on failure
+    assert b"NULL" in lib.moe_decoder_last_error(None)
+    assert lib.moe_decoder_position(None) == -1
+    assert lib.moe_decoder_step(None, None, None, None, None) == -1
+    assert lib.moe_decoder_set_layer(None, 0, *([None] * 8)) == -1
+    assert lib.moe_decoder_set_cache(None, 0, None, None, 0) == -1
+    lib.moe_decoder_destroy(None)
