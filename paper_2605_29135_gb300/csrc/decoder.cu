@@ -239,7 +239,7 @@ struct moe_decoder {
 
 namespace {
 
-std::string g_create_err;
+thread_local std::string g_create_err;
 
 moe_status dfail(moe_decoder* dec, moe_status st, const std::string& msg) {
   if (dec)
