@@ -240,6 +240,7 @@ def oracle_layer_sample(wl, hidden, budget_s):
 
 KERNEL_SOURCES = {
     "k_fused": ("fused.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh"),
+    "k_fused_la": ("fused.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh"),
     "k_fused_batched": ("fused_batched.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh", "tc.cuh"),
     "k_fused_batched_tc": ("fused_batched.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh", "tc.cuh"),
 }
@@ -316,8 +317,9 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
     phases = {k[len("fused_phase_"):]: round(v["total_ms"] * 1e3 / v["launches"], 2)
               for k, v in prof.items() if k.startswith("fused_phase_") and v["launches"]}
     tensor_cores = prof.get("fused_phase_gather", {}).get("launches", 0) > 0
-    kname = (("k_fused_batched_tc" if tensor_cores else "k_fused_batched") if wl.batch > 1 else "k_fused") \
-        if dom == "fused_step" else dom
+    la_dev = args.lookahead and args.schedule == "device" and wl.batch == 1
+    kname = (("k_fused_batched_tc" if tensor_cores else "k_fused_batched") if wl.batch > 1 else
+             ("k_fused_la" if la_dev else "k_fused")) if dom == "fused_step" else dom
     traffic_file = f"{kname}_{wl.name}_resident.md".replace("k_fused_stack48_bf16", "k_fused_stack48")
     return {"bound": "hbm", "kernel": kname,
             "workload": f"{wl.name} with all {wl.n_gid} experts resident (preloaded), batch {wl.batch}",
@@ -522,7 +524,9 @@ def main():
     ap.add_argument("--policy", default="lru", choices=["lru", "rotary", "guided"],
                     help="slot-group replacement policy (rotary: batch 1; guided: device schedule, batch 1)")
     ap.add_argument("--lookahead", action="store_true",
-                    help="host copy-engine schedule: route layer l + 1 and issue its copies while layer l computes")
+                    help="exact layer lookahead: host copy-engine schedule, route layer l + 1 and issue its copies "
+                         "while layer l computes; device schedule, one kernel routes every layer, then CTA 0 runs "
+                         "the lookups up to two layers ahead of the compute")
     ap.add_argument("--batched-path", default="auto", choices=["auto", "cuda_cores"],
                     help="expert FFN of batched steps: tensor cores where the shape allows, or CUDA cores")
     args = ap.parse_args()

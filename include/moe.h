@@ -131,11 +131,16 @@ typedef struct {
                              steps hand work items to all CTAs, missed experts first, and ignore it */
   int32_t batched_path;   /* MOE_BATCHED_AUTO (default) or MOE_BATCHED_CUDA_CORES */
   int32_t policy;         /* MOE_POLICY_LRU (default) or MOE_POLICY_ROTARY */
-  int32_t lookahead;      /* MOE_SCHEDULE_HOST_COPY_ENGINE only. 1: route layer l + 1 as soon as layer l's
-                             routing has reached the host, and issue its miss copies while layer l computes
-                             (the layers' inputs are all given with the step, so the decisions, the trace and
-                             the outputs are those of 0); a copy into a slot layer l still reads waits for
-                             layer l's kernels. 0 (default): one layer after another. */
+  int32_t lookahead;      /* 1: exact layer lookahead (the layers' inputs are all given with the step, so the
+                             decisions, the trace and the outputs are those of 0). MOE_SCHEDULE_HOST_COPY_ENGINE:
+                             route layer l + 1 as soon as layer l's routing has reached the host, and issue its
+                             miss copies while layer l computes; a copy into a slot layer l still reads waits
+                             for layer l's kernels. MOE_SCHEDULE_DEVICE (max_batch 1, MOE_POLICY_LRU): one kernel
+                             routes every layer first, then CTA 0 runs the layers' lookups in order, at most two
+                             layers ahead of the other CTAs, which compute each layer with one barrier among
+                             them; needs cap_slots >= 4 * top_k unless every expert is resident. Steps of a
+                             chained decoder (moe_decoder_step) run layer by layer whatever this says.
+                             0 (default): one layer after another. */
 } moe_config;
 
 /* One residency record: a requested expert's outcome in one layer-step. */

@@ -204,7 +204,8 @@ __device__ void rotary_place(const FusedArgs& a, int l, int clock, int k, int E,
 // Phase S, run by CTA 0 (all its threads). Every global read the phase needs is issued at its
 // start, side by side: the logits (warp 0), the layer's row of the lookup table, the pool's fill
 // count, the trace position and the victim candidates (warps 1-7).
-__device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t step, PendingTable& pend) {
+__device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t step, PendingTable& pend,
+                                  int64_t po = 0) {
   __shared__ int s_idx[kMaxRanks];
   __shared__ float s_gate[kMaxRanks];
   __shared__ int s_need[kMaxRanks];   // needed global ids, ascending
@@ -549,10 +550,10 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     const int g = l * E + s_idx[t];
     int q = 0;
     while (s_need[q] != g) q++;
-    a.plan_slot[t] = s_slot[q] < 0 ? 0 : s_slot[q];
-    a.plan_gid[t] = g;
-    a.plan_miss[t] = s_miss[q];
-    a.plan_gate[t] = s_gate[t];
+    a.plan_slot[po + t] = s_slot[q] < 0 ? 0 : s_slot[q];
+    a.plan_gid[po + t] = g;
+    a.plan_miss[po + t] = s_miss[q];
+    a.plan_gate[po + t] = s_gate[t];
     a.route_idx[l * k + t] = s_idx[t];
     a.route_gate[l * k + t] = s_gate[t];
   }
@@ -575,7 +576,7 @@ __device__ __forceinline__ float scale_at(const uint16_t* p, bool from_host) {
 // u_r[i] = silu(W_g[i] . x) * (W_u[i] . x) with x staged in shared memory.
 template <int WD, int CH>
 __device__ __forceinline__ void gateup_row(const FusedArgs& a, const uint8_t* src, uint8_t* slot, bool from_host,
-                                           const uint8_t* xs, int r, int i, int lane) {
+                                           const uint8_t* xs, int r, int i, int lane, float* u = nullptr) {
   const int64_t rb = a.lay.row_bytes_gu;
   const int nch = (int)(rb / 16);
   const int G = a.d / 128;
@@ -635,13 +636,13 @@ __device__ __forceinline__ void gateup_row(const FusedArgs& a, const uint8_t* sr
   }
   ag = warp_sum(ag);
   au = warp_sum(au);
-  if (lane == 0) a.u[(int64_t)r * a.I + i] = ag / (1.0f + expf(-ag)) * au;
+  if (lane == 0) (u ? u : a.u)[(int64_t)r * a.I + i] = ag / (1.0f + expf(-ag)) * au;
 }
 
 // Stage the k u vectors ([k x I] fp32, rank-major) into shared memory, padded by 4 floats per
 // 32 so the 16-byte reads of a warp spread over all banks.
-__device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad) {
-  const float4* u4 = reinterpret_cast<const float4*>(a.u);
+__device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad, const float* u = nullptr) {
+  const float4* u4 = reinterpret_cast<const float4*>(u ? u : a.u);
   const int n4 = a.k * a.I / 4;
 #pragma unroll 4
   for (int q = threadIdx.x; q < n4; q += blockDim.x) {
@@ -657,7 +658,7 @@ __device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad)
 // the CTA stages u, so the HBM latency overlaps the staging.
 template <int WD, int CHD>
 __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, const float* pgate, int l, int gw,
-                           int W) {
+                           int W, const float* u = nullptr) {
   constexpr int E = Tr<WD>::epc;
   constexpr int KR = 24 / CHD > 8 ? 8 : (24 / CHD < 1 ? 1 : 24 / CHD);
   const int lane = threadIdx.x & 31;
@@ -691,7 +692,7 @@ __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, cons
     }
   };
   issue(gw, 0);
-  stage_u(a, us, ipad);
+  stage_u(a, us, ipad, u);
   __syncthreads();
   for (int o = gw; o < a.d; o += W) {
     float acc = 0.f;
@@ -961,6 +962,217 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
   if (a.l_end == a.L && blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
 }
 
+// Barrier among the worker CTAs (1 .. gridDim.x - 1) of the lookahead kernel, bounded like grid_sync.
+__device__ bool worker_sync(const FusedArgs& a, unsigned& nbar) {
+  __shared__ int s_abort;
+  __syncthreads();
+  nbar++;
+  if (threadIdx.x == 0) {
+    const unsigned target = a.wbar_base + nbar * (gridDim.x - 1);
+    __threadfence();
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a.wbar_count), "r"(1u) : "memory");
+    if ((int)(ld_acquire_u32(a.wbar_count) - target) < 0) {
+      const uint64_t t0 = gtimer();
+      while ((int)(ld_acquire_u32(a.wbar_count) - target) < 0) {
+        if (*(volatile int*)a.err & FERR_FATAL) break;
+        if (gtimer() - t0 > a.barrier_timeout_ns) {
+          atomicOr(a.err, FERR_BARRIER_TIMEOUT);
+          break;
+        }
+        __nanosleep(20);
+      }
+    }
+    s_abort = *(volatile int*)a.err & FERR_FATAL;
+  }
+  __syncthreads();
+  return s_abort == 0;
+}
+
+// Thread 0 waits (bounded) until the counter p has reached target (wrapping compare); false on a
+// timeout (sets FERR_BARRIER_TIMEOUT) or when another CTA has flagged a fatal error.
+__device__ bool wait_count(const FusedArgs& a, const unsigned* p, unsigned target) {
+  if ((int)(ld_acquire_u32(p) - target) >= 0) return true;
+  const uint64_t t0 = gtimer();
+  while ((int)(ld_acquire_u32(p) - target) < 0) {
+    if (*(volatile int*)a.err & FERR_FATAL) return false;
+    if (gtimer() - t0 > a.barrier_timeout_ns) {
+      atomicOr(a.err, FERR_BARRIER_TIMEOUT);
+      return false;
+    }
+    __nanosleep(20);
+  }
+  return true;
+}
+
+// Exact layer lookahead, batch 1, LRU. One launch per decode step:
+//   R   router logits of every layer (row l * E + e per warp, hidden read from global memory), then
+//       one grid barrier;
+//   CTA 0: the lookup step of layers 0 .. L-1 in order (the same calls, clocks, trace and table as
+//       the layer-by-layer kernel), layer m's plan going to plan[m][k] and plan_flag = its clock.
+//       Layer m is decided only after the workers have passed their barrier of layer
+//       m - kLookaheadDepth; with cap >= (kLookaheadDepth + 2) k every victim then has a last use
+//       older than any layer whose rows may still be read (checked by the host);
+//   workers (CTAs 1 ..): per layer, wait for its plan, gate-up rows (the last miss_ctas workers
+//       stream the missed experts from the host tier into their slots), a barrier among the
+//       workers, then the down rows + combine. No barrier follows the down rows: the next layer's
+//       gate-up rows start beside them, writing the other half of the layer-parity u buffer.
+template <int WD, int CH>
+__global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant__ FusedArgs a) {
+  extern __shared__ uint4 smem4[];
+  __shared__ int p_slot[kMaxRanks], p_gid[kMaxRanks], p_miss[kMaxRanks];
+  __shared__ float p_gate[kMaxRanks];
+  __shared__ int p_mr[kMaxRanks], p_hr[kMaxRanks], p_nm, p_nh;
+  __shared__ PendingTable pend;
+  __shared__ int s_ok;
+  const int asize = WD == WD_FP32 ? 4 : 2;
+  const int xbytes = a.d * asize;
+  uint8_t* xs = reinterpret_cast<uint8_t*>(smem4);
+  float* us = reinterpret_cast<float*>(xs + ((xbytes + 15) & ~15));
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * kFWarps + (threadIdx.x >> 5);
+  const int W = gridDim.x * kFWarps;
+  const int64_t step = *(volatile int64_t*)a.step;
+  const int nchr = xbytes / 16;
+  const int chd_need = (int)((a.lay.row_bytes_d / 16 + 31) / 32);
+  const int k = a.k;
+  unsigned nbar = 0, nwbar = 0;
+
+  // ---- phase R, every layer: one router row per warp at a time, h_l read through L2
+  for (int row = gw; row < a.L * a.E; row += W) {
+    const int l = row / a.E;
+    const uint8_t* wr = a.routers + (int64_t)row * xbytes;
+    const uint8_t* hl = (const uint8_t*)a.hidden + (int64_t)l * xbytes;
+    float acc = 0.f;
+    for (int c = lane; c < nchr; c += 32) {
+      const uint4 w = ld_stream(wr + (int64_t)c * 16);
+      const uint4 h = ld_cg(hl + (int64_t)c * 16);
+      if (WD == WD_FP32)
+        acc = dot_chunk<WD_FP32>(w, reinterpret_cast<const uint8_t*>(&h), acc);
+      else
+        acc = dot_chunk<WD_BF16>(w, reinterpret_cast<const uint8_t*>(&h), acc);
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) a.z[row] = acc;
+  }
+  if (!grid_sync(a, nbar)) return;
+
+  if (blockIdx.x == 0) {
+    // ---- the lookup steps, in layer order, each at most kLookaheadDepth layers ahead
+    for (int m = 0; m < a.L; m++) {
+      const int clock = (int)(step * a.L + m + 1);
+      if (threadIdx.x == 0) {
+        int ok = 1;
+        if (m >= kLookaheadDepth)
+          ok = wait_count(a, a.wbar_count, a.wbar_base + (unsigned)(m - kLookaheadDepth + 1) * (gridDim.x - 1));
+        s_ok = ok;
+        pend.n = 0;
+      }
+      __syncthreads();
+      if (!s_ok) return;
+      select_and_lookup(a, m, clock, step, pend, (int64_t)m * k);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        pend.apply(a);  // nothing else reads the table in this kernel
+        __threadfence();
+        asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(a.plan_flag), "r"((unsigned)clock) : "memory");
+      }
+      __syncthreads();
+      if (a.may_evict && __ldcg(a.n_used) >= a.cap) find_victim_candidates(a);
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) *a.step = step + 1;
+    return;
+  }
+
+  // ---- workers
+  const int wgw = ((int)blockIdx.x - 1) * kFWarps + (threadIdx.x >> 5);
+  const int WW = ((int)gridDim.x - 1) * kFWarps;
+  for (int l = 0; l < a.L; l++) {
+    const int clock = (int)(step * a.L + l + 1);
+    float* u = a.u + (int64_t)(l & 1) * k * a.I;
+    __syncthreads();  // the previous layer's down rows are done with p_slot / p_gate in this CTA
+    if (threadIdx.x == 0) s_ok = wait_count(a, a.plan_flag, (unsigned)clock);
+    __syncthreads();
+    if (!s_ok) return;
+    if (threadIdx.x < k) {
+      const int64_t q = (int64_t)l * k + threadIdx.x;
+      p_slot[threadIdx.x] = __ldcg(a.plan_slot + q);
+      p_gid[threadIdx.x] = __ldcg(a.plan_gid + q);
+      p_miss[threadIdx.x] = __ldcg(a.plan_miss + q);
+      p_gate[threadIdx.x] = __ldcg(a.plan_gate + q);
+    }
+    stage16(reinterpret_cast<uint4*>(xs), (const uint8_t*)a.hidden + (int64_t)l * xbytes, xbytes, threadIdx.x,
+            blockDim.x);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int nm = 0, nh = 0;
+      for (int r = 0; r < k; r++) {
+        if (p_miss[r])
+          p_mr[nm++] = r;
+        else
+          p_hr[nh++] = r;
+      }
+      p_nm = nm;
+      p_nh = nh;
+    }
+    __syncthreads();
+    const int nm = p_nm, nh = p_nh;
+    const int workers = (int)gridDim.x - 1;
+    const int mctas = nm > 0 ? (a.miss_ctas < workers - 1 ? a.miss_ctas : workers - 1) : 0;
+    const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;
+    if (nm > 0 && a.touch_shift > 0) {
+      const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
+      const int64_t gt0 = ((int64_t)blockIdx.x - 1) * kFThreads + threadIdx.x;
+      const int64_t GT = (int64_t)workers * kFThreads;
+      for (int64_t q = gt0; q < (int64_t)nm * pages; q += GT) {
+        const int mi = (int)(q / pages);
+        const uint8_t* pa = a.arena + (int64_t)p_gid[p_mr[mi]] * a.slot_stride + ((q - (int64_t)mi * pages) << a.touch_shift);
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+      }
+    }
+    if (miss_cta) {
+      const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
+      const int MW = mctas * kFWarps;
+      for (int p = mw; p < nm * a.I; p += MW) {
+        const int r = p_mr[p / a.I];
+        const int i = p - (p / a.I) * a.I;
+        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
+        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride;
+        gateup_row<WD, CH>(a, src, slot, true, xs, r, i, lane, u);
+      }
+      const int64_t dbytes = a.lay.total - a.lay.d_off;
+      const int64_t nq = dbytes / 16;
+      const int mt = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFThreads + threadIdx.x;
+      const int MT = mctas * kFThreads;
+      for (int mi = 0; mi < nm; mi++) {
+        const int r = p_mr[mi];
+        uint8_t* dst = a.pool + (int64_t)p_slot[r] * a.slot_stride + a.lay.d_off;
+        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride + a.lay.d_off;
+        for (int64_t q = mt; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
+      }
+    } else {
+      const int hw = wgw;
+      const int HW = (workers - mctas) * kFWarps;
+      for (int p = hw; p < nh * a.I; p += HW) {
+        const int r = p_hr[p / a.I];
+        const int i = p - (p / a.I) * a.I;
+        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
+        gateup_row<WD, CH>(a, slot, slot, false, xs, r, i, lane, u);
+      }
+    }
+    if (!worker_sync(a, nwbar)) return;
+    switch (chd_need) {
+      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+      case 5:
+      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+    }
+  }
+}
+
 size_t fused_smem(int wdtype, int d, int I, int k) {
   const int xbytes = d * (wdtype == WD_FP32 ? 4 : 2);
   return (size_t)((xbytes + 15) & ~15) + (size_t)k * ipad_of(I) * sizeof(float);
@@ -1041,6 +1253,39 @@ int pick_ch_f(int64_t rb) {
     }                                                              \
   } while (0)
 
+template <int WD, int CH>
+int grid_of_la(size_t smem) {
+  static int occ = -1;
+  static size_t occ_smem = 0;
+  if (occ < 0 || occ_smem != smem) {
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(k_fused_la<WD, CH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    int o = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, k_fused_la<WD, CH>, kFThreads, smem) != cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    occ = o;
+    occ_smem = smem;
+  }
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = sms * (occ < 2 ? occ : 2);
+  return grid >= 3 ? grid : 0;  // CTA 0 and at least two workers
+}
+
+template <int WD, int CH>
+cudaError_t run_fused_la(const FusedArgs& a, int grid, cudaStream_t s) {
+  const size_t smem = fused_smem(a.wdtype, a.d, a.I, a.k);
+  void* params[] = {(void*)&a};
+  return cudaLaunchCooperativeKernel((const void*)k_fused_la<WD, CH>, dim3(grid), dim3(kFThreads), params, smem, s);
+}
+
 int fused_grid(int wdtype, int d, int I, int k) {
   const BlobLayout lay = make_layout(wdtype, d, I);
   const int ch = pick_ch_f(lay.row_bytes_gu);
@@ -1053,6 +1298,21 @@ int fused_grid(int wdtype, int d, int I, int k) {
 cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s) {
   const int ch = pick_ch_f(a.lay.row_bytes_gu);
   MOE_F_DISPATCH(run_fused, a.wdtype, ch, a, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+int fused_la_grid(int wdtype, int d, int I, int k) {
+  const BlobLayout lay = make_layout(wdtype, d, I);
+  const int ch = pick_ch_f(lay.row_bytes_gu);
+  const size_t smem = fused_smem(wdtype, d, I, k);
+  if (smem > 200 * 1024) return 0;
+  MOE_F_DISPATCH(grid_of_la, wdtype, ch, smem);
+  return 0;
+}
+
+cudaError_t launch_fused_la(const FusedArgs& a, int grid, cudaStream_t s) {
+  const int ch = pick_ch_f(a.lay.row_bytes_gu);
+  MOE_F_DISPATCH(run_fused_la, a.wdtype, ch, a, grid, s);
   return cudaErrorInvalidValue;
 }
 

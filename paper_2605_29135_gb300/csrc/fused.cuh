@@ -77,6 +77,10 @@ struct FusedArgs {
   // (0 = highest logit, ties to the lower id; E before the layer's first routing).
   int32_t* rank;               // [L*E]
   unsigned* plan_flag;         // clock of the last layer-step whose plan CTA 0 has published (0: none)
+  // Exact layer lookahead (k_fused_la): the worker CTAs' barrier counter and its value at launch.
+  // The plan arrays then hold every layer's plan, [L][k].
+  unsigned* wbar_count;
+  unsigned wbar_base;
 };
 
 // Router-guided replacement key: the victim is the smallest key, i.e. the largest rank, then the
@@ -97,6 +101,15 @@ __host__ __device__ __forceinline__ int slot_key_gid(unsigned long long key, int
 // Maximum co-resident CTAs for the fused kernel of this shape (0 if it cannot launch).
 int fused_grid(int wdtype, int d, int I, int k);
 cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s);
+
+// Exact layer lookahead at batch 1 under LRU (layers' inputs all given with the step): CTA 0 runs
+// the lookup steps of every layer in order while the other CTAs compute, at most
+// kLookaheadDepth layers ahead of them; needs cap >= (kLookaheadDepth + 2) * k (then no slot is
+// re-assigned while a reader of its old contents may still run). Same decisions, trace and
+// outputs as k_fused.
+constexpr int kLookaheadDepth = 2;
+int fused_la_grid(int wdtype, int d, int I, int k);
+cudaError_t launch_fused_la(const FusedArgs& a, int grid, cudaStream_t s);
 
 // Batched decode step: B sequences per step, one cooperative kernel over all layers. Per layer
 // the needed experts are the union of every sequence's top k; each needed expert is read once

@@ -140,6 +140,9 @@ struct moe_handle {
   int tg_max = 0;
   int touch_shift = 12;
   unsigned bar_epoch = 0;  // grid-barrier counter value at the start of the next fused launch
+  bool lookahead_dev = false;  // device schedule with exact layer lookahead (k_fused_la) for whole steps
+  int fgrid_la = 0;
+  unsigned wbar_epoch = 0;     // its worker-barrier counter value at the start of the next launch
   const uint8_t* arena_dev = nullptr;
   int32_t* d_slot_of = nullptr;
   unsigned long long* d_slot_key = nullptr;
@@ -234,7 +237,8 @@ std::string check_config(const moe_config* c) {
   if (c->policy == MOE_POLICY_GUIDED && (int64_t)c->n_layers * c->n_experts >= (1LL << moe::kGuidedGidBits))
     return "the router-guided policy needs n_layers * n_experts < 2^23";
   if (c->lookahead != 0 && c->lookahead != 1) return "lookahead must be 0 or 1";
-  if (c->lookahead && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "lookahead needs the host copy-engine schedule";
+  if (c->lookahead && c->schedule == MOE_SCHEDULE_DEVICE && (c->max_batch != 1 || c->policy != MOE_POLICY_LRU))
+    return "lookahead in the device schedule needs max_batch 1 and the LRU policy";
   return "";
 }
 
@@ -262,6 +266,7 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_stats, 0, sizeof(unsigned long long) * moe::STAT_N);
   cudaMemset(h->d_bar, 0, sizeof(unsigned) * 4);
   h->bar_epoch = 0;
+  h->wbar_epoch = 0;
   cudaMemset(h->d_err, 0, sizeof(int));
   cudaDeviceSynchronize();
   *h->h_err = 0;
@@ -795,11 +800,21 @@ moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, in
   arm_barrier_fault(h, a.bar_base, a.barrier_timeout_ns);
   a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
   a.touch_shift = h->touch_shift;
-  a.phase_ts = whole ? phase_buffer(h) : nullptr;
+  // whole steps of a lookahead handle: every layer's plan at plan[l][k], one grid barrier per launch
+  const bool la = whole && h->lookahead_dev;
+  if (la) {
+    const int64_t Lk = (int64_t)c.n_layers * k;
+    a.plan_gid = h->d_plan + Lk;
+    a.plan_miss = h->d_plan + 2 * Lk;
+    a.wbar_count = h->d_bar + 2;
+    a.wbar_base = h->wbar_epoch;
+    a.may_evict = a.may_evict && c.policy == MOE_POLICY_LRU;
+  }
+  a.phase_ts = whole && !la ? phase_buffer(h) : nullptr;
   {
     ProfScope ps(h, s, PC_FUSED,
                  (int64_t)(l1 - l0) * (k * h->lay.total + (int64_t)c.n_experts * c.d * h->router_eb));
-    cudaError_t e = moe::launch_fused(a, h->fgrid, s);
+    cudaError_t e = la ? moe::launch_fused_la(a, h->fgrid_la, s) : moe::launch_fused(a, h->fgrid, s);
     ps.done();
     if (e != cudaSuccess) return cuda_fail(h, e, "fused decode step launch");
   }
@@ -807,7 +822,12 @@ moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, in
   MOE_CK(h, cudaEventRecord(h->err_ev, s));
   h->err_pending = true;
   if (l1 == c.n_layers) h->steps_launched++;
-  h->bar_epoch += 3u * (unsigned)(l1 - l0) * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
+  if (la) {
+    h->bar_epoch += (unsigned)h->fgrid_la;  // one grid barrier (after the router phase)
+    h->wbar_epoch += (unsigned)c.n_layers * (unsigned)(h->fgrid_la - 1);  // one worker barrier per layer
+  } else {
+    h->bar_epoch += 3u * (unsigned)(l1 - l0) * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
+  }
   if (a.phase_ts) {
     // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
     static const int cls[4] = {PC_PH_R, PC_PH_S, PC_PH_C, PC_PH_D};
@@ -997,7 +1017,10 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   h->route->seq = 0;
   if (cudaHostGetDevicePointer((void**)&h->route_dev, (void*)h->route, 0) != cudaSuccess)
     return bail(MOE_ERR_CUDA, "mapped routing buffer has no device address");
-  if (cudaMalloc(&h->u, sizeof(float) * cfg->max_batch * cfg->top_k * cfg->d_ff) != cudaSuccess)
+  // u per rank; the device lookahead kernel keeps two layers' u (layer parity)
+  const int64_t u_sets = cfg->lookahead && cfg->schedule == MOE_SCHEDULE_DEVICE ? std::max(2, cfg->max_batch)
+                                                                                  : cfg->max_batch;
+  if (cudaMalloc(&h->u, sizeof(float) * u_sets * cfg->top_k * cfg->d_ff) != cudaSuccess)
     return bail(MOE_ERR_OOM, "u allocation failed");
   const int64_t act = (int64_t)cfg->n_layers * cfg->max_batch * cfg->d * h->asize;
   if (cudaMalloc(&h->hid_dev, act) != cudaSuccess || cudaMalloc(&h->out_dev, act) != cudaSuccess)
@@ -1030,13 +1053,25 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   } else if (h->dev_mode) {
     h->fgrid = moe::fused_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
     if (h->fgrid <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the device-driven schedule");
+    if (cfg->lookahead) {
+      // a victim's old contents may still be read by the kLookaheadDepth + 1 layers in flight
+      const int64_t need_cap = (int64_t)(moe::kLookaheadDepth + 2) * cfg->top_k;
+      if (h->cap < h->n_gid && h->cap < need_cap)
+        return bail(MOE_ERR_INVALID, "lookahead in the device schedule needs at least " + std::to_string(need_cap) +
+                                         " slots (or every expert resident)");
+      h->fgrid_la = moe::fused_la_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
+      if (h->fgrid_la <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the lookahead kernel");
+      h->lookahead_dev = true;
+    }
   }
   if (h->dev_mode) {
     if (cudaHostGetDevicePointer((void**)&h->arena_dev, h->arena, 0) != cudaSuccess)
       return bail(MOE_ERR_CUDA, "host arena has no device address");
     const int k = cfg->top_k;
     const int64_t pairs = (int64_t)cfg->max_batch * k;
-    const int64_t plan_ints = h->batched ? 2 + 5 * (int64_t)cfg->n_experts + pairs : 3 * (int64_t)k;
+    // batch 1: slot, gid, miss per rank, for one layer ([k]) or, with lookahead, for every layer ([L][k])
+    const int64_t plan_ranks = h->lookahead_dev ? (int64_t)k * cfg->n_layers : (int64_t)k;
+    const int64_t plan_ints = h->batched ? 2 + 5 * (int64_t)cfg->n_experts + pairs : 3 * plan_ranks;
     bool ok = cudaMalloc(&h->d_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
               cudaMalloc(&h->d_slot_key, sizeof(unsigned long long) * h->cap) == cudaSuccess &&
               cudaMalloc(&h->d_cand, sizeof(unsigned long long) * (moe::kMaxRanks + 1)) == cudaSuccess &&
@@ -1050,7 +1085,7 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
               cudaMalloc(&h->d_z, sizeof(float) * std::max<int64_t>(256 * (int64_t)cfg->max_batch,
                                                                     h->n_gid * cfg->max_batch)) == cudaSuccess &&
               cudaMalloc(&h->d_plan, sizeof(int32_t) * plan_ints) == cudaSuccess &&
-              cudaMalloc(&h->d_plan_gate, sizeof(float) * pairs) == cudaSuccess &&
+              cudaMalloc(&h->d_plan_gate, sizeof(float) * std::max(pairs, plan_ranks)) == cudaSuccess &&
               (!h->batched || cudaMalloc(&h->d_sel_e, sizeof(int32_t) * pairs) == cudaSuccess) &&
               (!h->batched || cudaMalloc(&h->d_y, sizeof(float) * pairs * cfg->d) == cudaSuccess) &&
               cudaMalloc(&h->d_trace, sizeof(moe::TraceRec) * std::max<int64_t>(1, cfg->trace_capacity)) == cudaSuccess &&

@@ -52,7 +52,8 @@ BAD = [
     (dict(raw_policy=9), "unknown policy"),
     (dict(policy="rotary", max_batch=4, schedule="host_copy_engine"), "max_batch above 1 needs the device schedule"),
     (dict(raw_lookahead=2), "lookahead must be 0 or 1"),
-    (dict(lookahead=True), "lookahead needs the host copy-engine schedule"),
+    (dict(lookahead=True, max_batch=4), "lookahead in the device schedule needs max_batch 1 and the LRU policy"),
+    (dict(lookahead=True, policy="rotary"), "lookahead in the device schedule needs max_batch 1 and the LRU policy"),
 ]
 
 
