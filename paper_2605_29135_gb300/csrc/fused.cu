@@ -1009,9 +1009,10 @@ __device__ bool wait_count(const FusedArgs& a, const unsigned* p, unsigned targe
 //       one grid barrier;
 //   CTA 0: the lookup step of layers 0 .. L-1 in order (the same calls, clocks, trace and table as
 //       the layer-by-layer kernel), layer m's plan going to plan[m][k] and plan_flag = its clock.
-//       Layer m is decided only after the workers have passed their barrier of layer
-//       m - kLookaheadDepth; with cap >= (kLookaheadDepth + 2) k every victim then has a last use
-//       older than any layer whose rows may still be read (checked by the host);
+//       A miss's bytes reach its slot during layer m's gate-up rows, after the workers' barrier of
+//       layer m - 1, while only layer m - 1's down rows may still read; with cap >= 2 k (checked
+//       by the host) LRU never gives a miss of layer m the slot of an expert layer m - 1 used, so
+//       CTA 0 may run any number of layers ahead;
 //   workers (CTAs 1 ..): per layer, wait for its plan, gate-up rows (the last miss_ctas workers
 //       stream the missed experts from the host tier into their slots), a barrier among the
 //       workers, then the down rows + combine. No barrier follows the down rows: the next layer's
@@ -1057,14 +1058,11 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
   if (!grid_sync(a, nbar)) return;
 
   if (blockIdx.x == 0) {
-    // ---- the lookup steps, in layer order, each at most kLookaheadDepth layers ahead
+    // ---- the lookup steps, in layer order
     for (int m = 0; m < a.L; m++) {
       const int clock = (int)(step * a.L + m + 1);
       if (threadIdx.x == 0) {
-        int ok = 1;
-        if (m >= kLookaheadDepth)
-          ok = wait_count(a, a.wbar_count, a.wbar_base + (unsigned)(m - kLookaheadDepth + 1) * (gridDim.x - 1));
-        s_ok = ok;
+        s_ok = (*(volatile int*)a.err & FERR_FATAL) == 0;
         pend.n = 0;
       }
       __syncthreads();

@@ -103,11 +103,10 @@ int fused_grid(int wdtype, int d, int I, int k);
 cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s);
 
 // Exact layer lookahead at batch 1 under LRU (layers' inputs all given with the step): CTA 0 runs
-// the lookup steps of every layer in order while the other CTAs compute, at most
-// kLookaheadDepth layers ahead of them; needs cap >= (kLookaheadDepth + 2) * k (then no slot is
-// re-assigned while a reader of its old contents may still run). Same decisions, trace and
+// the lookup steps of every layer in order while the other CTAs compute. Needs cap >= 2 k (or
+// every expert resident): then no miss takes the slot of an expert the previous layer-step used,
+// whose down rows may still be running when the miss's bytes arrive. Same decisions, trace and
 // outputs as k_fused.
-constexpr int kLookaheadDepth = 2;
 int fused_la_grid(int wdtype, int d, int I, int k);
 cudaError_t launch_fused_la(const FusedArgs& a, int grid, cudaStream_t s);
 

@@ -1054,8 +1054,9 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     h->fgrid = moe::fused_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
     if (h->fgrid <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the device-driven schedule");
     if (cfg->lookahead) {
-      // a victim's old contents may still be read by the kLookaheadDepth + 1 layers in flight
-      const int64_t need_cap = (int64_t)(moe::kLookaheadDepth + 2) * cfg->top_k;
+      // a miss must never take the slot of an expert the previous layer-step used (its down rows
+      // may still be reading): LRU guarantees it from 2 k slots on
+      const int64_t need_cap = 2 * (int64_t)cfg->top_k;
       if (h->cap < h->n_gid && h->cap < need_cap)
         return bail(MOE_ERR_INVALID, "lookahead in the device schedule needs at least " + std::to_string(need_cap) +
                                          " slots (or every expert resident)");

@@ -178,13 +178,14 @@ def test_preload_then_decode_matches_oracle(P, schedule, cap):
 
 
 # The device schedule with exact layer lookahead: one kernel routes every layer, CTA 0 then decides
-# the layers' lookups in order at most two layers ahead of the compute (cap >= 4 * top_k, or every
-# expert resident). Same trace and outputs as the layer-by-layer kernel, bit for bit.
+# the layers' lookups in order ahead of the compute (cap >= 2 * top_k, or every expert resident).
+# Same trace and outputs as the layer-by-layer kernel, bit for bit.
 LOOKAHEAD = {
-    "tiny3_fp32": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=8),
-    "ragged_fp32": RAGGED["fp32"].replace(cap_slots=8),
-    "ragged_bf16": RAGGED["bf16"].replace(cap_slots=20),
-    "ragged_int4": RAGGED["int4"].replace(cap_slots=12),
+    "tiny3_fp32_cap4": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=4),
+    "tiny3_fp32_cap8": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=8),
+    "ragged_fp32": RAGGED["fp32"].replace(cap_slots=4),
+    "ragged_bf16": RAGGED["bf16"].replace(cap_slots=10),
+    "ragged_int4": RAGGED["int4"].replace(cap_slots=6),
     "tiny3_fp32_resident": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=24),
 }
 
@@ -209,7 +210,7 @@ def test_device_lookahead_stack48_2048_tokens(P, name):
 
 
 def test_device_lookahead_preload_and_small_caps(P):
-    wl = LOOKAHEAD["tiny3_fp32"]
+    wl = LOOKAHEAD["tiny3_fp32_cap8"]
     hidden = synth.hidden_all(wl)
     m = _create(wl, 10, "device_lookahead")
     try:
@@ -223,5 +224,5 @@ def test_device_lookahead_preload_and_small_caps(P):
     recs = [orc.decode_step(hidden[t], compute_out=False, forced_idx=idx[t]).records for t in range(wl.tokens)]
     np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate(recs)))
     with pytest.raises(P.MoEError) as ei:
-        _create(wl, 7, "device_lookahead")  # below 4 * top_k = 8 slots
+        _create(wl, 3, "device_lookahead")  # below 2 * top_k = 4 slots
     assert ei.value.status == -1 and "slots" in str(ei.value)
