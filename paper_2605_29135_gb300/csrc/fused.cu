@@ -1015,8 +1015,9 @@ __device__ bool wait_count(const FusedArgs& a, const unsigned* p, unsigned targe
 //       CTA 0 may run any number of layers ahead;
 //   workers (CTAs 1 ..): per layer, wait for its plan, gate-up rows (the last miss_ctas workers
 //       stream the missed experts from the host tier into their slots), a barrier among the
-//       workers, then the down rows + combine. No barrier follows the down rows: the next layer's
-//       gate-up rows start beside them, writing the other half of the layer-parity u buffer.
+//       workers, then the down rows + combine on the workers that computed hits. No barrier
+//       follows the down rows: the next layer's gate-up rows (and the miss CTAs' streaming of its
+//       misses) start beside them, writing the other half of the layer-parity u buffer.
 template <int WD, int CH>
 __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant__ FusedArgs a) {
   extern __shared__ uint4 smem4[];
@@ -1084,7 +1085,6 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
 
   // ---- workers
   const int wgw = ((int)blockIdx.x - 1) * kFWarps + (threadIdx.x >> 5);
-  const int WW = ((int)gridDim.x - 1) * kFWarps;
   for (int l = 0; l < a.L; l++) {
     const int clock = (int)(step * a.L + l + 1);
     float* u = a.u + (int64_t)(l & 1) * k * a.I;
@@ -1159,14 +1159,20 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
       }
     }
     if (!worker_sync(a, nwbar)) return;
+    // Down rows + combine on the hit workers only: the miss CTAs go straight on to the next
+    // layer's misses, so the host link stays busy. Their copies then overlap these down rows,
+    // which is safe because no miss of layer l + 1 takes the slot of an expert of layer l
+    // (cap >= 2 k).
+    if (miss_cta) continue;
+    const int HWW = (workers - mctas) * kFWarps;
     switch (chd_need) {
-      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
-      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
-      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
-      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
+      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
+      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
+      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
       case 5:
-      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
-      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, wgw, WW, u); break;
+      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
+      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
     }
   }
 }
