@@ -435,7 +435,8 @@ def run_decoder(args, dw):
     P.build()
     peak_hbm, _ = load_peaks()
     e2e_steps = args.e2e_steps or max(8, args.steps // 4)
-    n_tok = args.warmup + args.steps + e2e_steps
+    prof_steps = max(2, args.steps // 2)
+    n_tok = args.warmup + args.steps + prof_steps + e2e_steps
     xs = synth.token_inputs(dw, n_tok)
     m, dec = create_decoder_for_workload(dw, max_tokens=n_tok, device=local, trace_capacity=0)
     eb = P.expert_bytes(m.cfg)
@@ -460,12 +461,27 @@ def run_decoder(args, dw):
     clk = clocks.stop()
     ms = e0.elapsed_time(e1)
     s1 = m.get_stats()
+    # a second pass with the MoE launches bracketed by CUDA events: the rest of the step time is the
+    # attention block (its kernels and the launch gaps between them)
+    first = args.warmup + args.steps
+    m.profile_enable(True)
+    m.profile_read()
+    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    p0.record(stream)
+    for i in range(first, first + prof_steps):
+        dec.step(x_dev[i], y_dev, stream=stream)
+    p1.record(stream)
+    torch.cuda.synchronize()
+    prof = m.profile_read()
+    m.profile_enable(False)
+    moe_ms = prof.get("fused_step", {}).get("total_ms", 0.0) / prof_steps
+    attn_ms = p0.elapsed_time(p1) / prof_steps - moe_ms
     # end to end: the token's input from pinned host memory, the output stream read back, per step
     x_host = raw.pin_memory()
     y_host = torch.empty(wl.d, dtype=torch.float32).pin_memory()
     x_buf = torch.empty_like(x_dev[0])
     t0 = time.perf_counter()
-    for i in range(args.warmup + args.steps, n_tok):
+    for i in range(first + prof_steps, n_tok):
         x_buf.copy_(x_host[i].view(tdt) if wl.adtype != "fp32" else x_host[i], non_blocking=True)
         dec.step(x_buf, y_dev, stream=stream)
         y_host.copy_(y_dev, non_blocking=True)
@@ -495,8 +511,17 @@ def run_decoder(args, dw):
             "step_roofline": {"t_star_ms": t_star * 1e3, "frac": t_star * 1e3 / ms_step, "hbm_bytes_per_step": hbm,
                               "miss_bytes_per_step": miss_b, "h2d_peak_gbs": h2d_gbs, "hbm_peak_gbs": peak_hbm,
                               "hit_rate": 1.0 - misses / max(1, hits + misses)},
-            "roofline": None,
-            "gpu_launches": args.steps * (9 * wl.n_layers + 1),
+            "roofline": {"bound": "hbm", "kernel": "attention block: norms, q/k/v and W_o GEMVs, rotary + KV "
+                                                  "append, split attention + merge (k_dec_*, k_attn_*)",
+                         "achieved": wl.n_layers * (attn_w + kv_read) / (attn_ms * 1e-3) / 1e9 if attn_ms > 0 else None,
+                         "peak": peak_hbm, "unit": "GB/s",
+                         "frac": (wl.n_layers * (attn_w + kv_read) / (attn_ms * 1e-3) / 1e9 / peak_hbm)
+                         if attn_ms > 0 else None,
+                         "traffic": None, "bytes_per_step": wl.n_layers * (attn_w + kv_read),
+                         "ms_per_step": attn_ms, "moe_ms_per_step": moe_ms,
+                         "timing": "profiled step time minus the MoE launches' CUDA-event time; includes the "
+                                   "launch gaps between the attention block's kernels"},
+            "gpu_launches": args.steps * (8 * wl.n_layers + 1),  # 7 attention-block launches + 1 MoE per layer, 1 output
             "clocks": clk,
             "e2e": {"value": e2e_steps / e2e_s, "unit": "tok/s", "h2d_bytes_per_step": wl.d * es,
                     "d2h_bytes_per_step": wl.d * 4, "steps": e2e_steps, "api": "Decoder.step with host copies"}}
