@@ -6,7 +6,7 @@
   (relative L2 <= 1e-5 per row; trace bit-exact; the oracle's k-th / (k+1)-th logit gaps on this
   data are all above 5e-3, so no near-tie can flip a selection);
 - full-size bf16 block (d 2048, 32 query / 4 kv heads of 128, 4095 cached positions, E 128, top-8),
-  3 layers, layer by layer: each piece the GPU logs (attention output, MoE input, MoE output) is
+  3 layers, and a small int4-expert block (head_dim 64, four query heads per kv head), layer by layer: each piece the GPU logs (attention output, MoE input, MoE output) is
   compared with the oracle applied to the GPU's own input of that piece (teacher forcing), within
   the bf16 tolerance 1e-2; the trace is checked against the oracle's slot group fed the GPU's
   selections (accepted only where they match the oracle's up to near-ties);
@@ -28,6 +28,11 @@ pytestmark = pytest.mark.gpu
 TINY = synth.DECODERS["tiny_block_fp32"]
 BLOCK3 = synth.DECODERS["block48_bf16"].replace(
     name="block3_bf16", moe=synth.WORKLOADS["stack48_bf16"].replace(n_layers=3, tokens=3, cap_slots=12))
+# int4 experts (bf16 attention), head_dim 64, four query heads per kv head, a short cache
+SMALL_INT4 = synth.DecoderWorkload(
+    "small_int4", synth.Workload("small_int4", d=512, n_experts=16, top_k=4, d_ff=256, n_layers=3, wdtype="int4",
+                                 adtype="bf16", tokens=5, batch=1, rho=0.8, cap_slots=10),
+    n_heads=8, n_kv_heads=2, head_dim=64, ctx=100)
 
 
 @pytest.fixture(scope="module")
@@ -125,6 +130,16 @@ def test_bf16_block_layer_by_layer_matches_the_oracle(P):
     worst, recs = _teacher_forced(dw, log, idx)
     assert worst.max() <= TOL["bf16"], f"attention / MoE input / MoE output rel L2 {worst}"
     assert np.array_equal(trace_tuples(tr), trace_tuples(recs))
+    _check_chain(out, log)
+
+
+def test_int4_block_layer_by_layer_matches_the_oracle(P):
+    dw = SMALL_INT4
+    out, log, idx, tr = _run(P, dw)
+    worst, recs = _teacher_forced(dw, log, idx)
+    assert worst[:2].max() <= TOL["bf16"] and worst[2] <= TOL["int4"], f"rel L2 {worst}"
+    assert np.array_equal(trace_tuples(tr), trace_tuples(recs))
+    assert (tr["evicted"] >= 0).any()
     _check_chain(out, log)
 
 
