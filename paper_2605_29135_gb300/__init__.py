@@ -296,6 +296,31 @@ class Planner:
         self.destroy()
 
 
+def plan_caps(n_layers: int, n_experts: int, caps, idx, policy: str = "lru", ranks=None, prefetch=None,
+              expert_bytes: int | None = None, preload: bool = False) -> list:
+    """Capacity sweep with the residency planner: replay one recorded routing sequence (idx as for
+    Planner.run) at every slot count in caps. Returns one dict per cap, in the given order: cap,
+    hit_rate, misses, evictions, prefetches, misses and evictions per decode step, and, with
+    expert_bytes, the host-link bytes per decode step the misses and prefetches would move."""
+    T = np.asarray(idx).shape[0]
+    rows = []
+    for cap in caps:
+        p = Planner(n_layers, n_experts, int(cap), policy)
+        try:
+            if preload:
+                p.preload()
+            r = p.run(idx, ranks=ranks, prefetch=prefetch)
+        finally:
+            p.destroy()
+        row = {"cap": int(cap), "hit_rate": r["hit_rate"], "misses": r["misses"], "evictions": r["evictions"],
+               "prefetches": r["prefetches"], "misses_per_step": r["misses"] / max(1, T),
+               "evictions_per_step": r["evictions"] / max(1, T)}
+        if expert_bytes is not None:
+            row["link_bytes_per_step"] = (r["misses"] + r["prefetches"]) * expert_bytes / max(1, T)
+        rows.append(row)
+    return rows
+
+
 class Decoder:
     """Chained decoder blocks around a MoE handle's layers (moe_decoder_create ... _destroy).
 

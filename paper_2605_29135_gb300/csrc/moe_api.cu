@@ -909,8 +909,9 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     return fail(nullptr, MOE_ERR_CAPACITY, buf);
   }
   auto bail = [&](moe_status st, const std::string& msg) {
+    const std::string keep = msg;  // msg may be h->err, which free_all destroys
     free_all(h);
-    return fail(nullptr, st, msg);
+    return fail(nullptr, st, keep);
   };
   if (cfg->device_pool) {
     if ((uintptr_t)cfg->device_pool % 256) return bail(MOE_ERR_INVALID, "device_pool must be 256-byte aligned");

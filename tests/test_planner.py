@@ -309,3 +309,30 @@ def test_run_replays_a_recorded_routing_like_the_oracle():
     with Planner(wl.n_layers, wl.n_experts, 6) as p:
         with pytest.raises(ValueError):
             p.run(idx[:, :2])
+
+
+def test_cap_sweep_counts_match_the_oracle_and_the_full_cap_misses_once_per_expert():
+    from paper_2605_29135_gb300 import plan_caps
+
+    rng = np.random.default_rng(7)
+    L, E, k, T = 3, 12, 3, 20
+    idx = np.stack([[rng.permutation(E)[:k] for _ in range(L)] for _ in range(T)])  # [T x L x k]
+    caps = [k, 2 * k, 10, L * E]
+    rows = plan_caps(L, E, caps, idx, expert_bytes=1000)
+    assert [r["cap"] for r in rows] == caps
+    for cap, row in zip(caps, rows):
+        table = oracle.LRUTable(L * E, cap, E)
+        kinds, ev = [], 0
+        for t in range(T):
+            for l in range(L):
+                r = table.step(t * L + l, sorted(l * E + int(e) for e in idx[t, l]), t)
+                kinds += list(r["kind"])
+                ev += int((r["evicted"] >= 0).sum())
+        kinds = np.array(kinds)
+        assert row["misses"] == int((kinds == 1).sum()) and row["evictions"] == ev
+        assert row["hit_rate"] == pytest.approx((kinds == 0).sum() / len(kinds))
+        assert row["link_bytes_per_step"] == pytest.approx(row["misses"] * 1000 / T)
+    full = rows[-1]
+    assert full["evictions"] == 0 and full["misses"] == len({(l, int(e)) for t in range(T) for l in range(L)
+                                                            for e in idx[t, l]})
+    assert plan_caps(L, E, [L * E], idx, preload=True)[0]["misses"] == 0  # every expert resident up front
