@@ -68,9 +68,14 @@ class DecoderStep:
 
 
 class DecoderOracle:
-    """Batch-1 decode through dw's chained stack, starting after dw.ctx cached positions."""
+    """Batch-1 decode through dw's chained stack, starting after dw.ctx cached positions.
 
-    def __init__(self, dw, cap_slots=None, policy="lru", keep_slot_copies=True, max_tokens=None, moe=None):
+    layers: None (every layer), or the layers whose attention weights and KV caches are built;
+    attention() then serves only those, and decode_token() needs them all. This keeps checks of
+    sampled layers of a large stack cheap; the arithmetic is the same."""
+
+    def __init__(self, dw, cap_slots=None, policy="lru", keep_slot_copies=True, max_tokens=None, moe=None,
+                 layers=None):
         import synth
 
         self.dw = dw
@@ -81,20 +86,22 @@ class DecoderOracle:
             wl, cap_slots=cap_slots, keep_slot_copies=keep_slot_copies, policy=policy)
         wdt = "fp32" if wl.wdtype == "fp32" else "bf16"
         qd, kd = self.Hq * self.D, self.Hkv * self.D
-        self.attn_w = []
-        for l in range(self.L):
+        self.layers = list(range(self.L)) if layers is None else sorted(set(int(l) for l in layers))
+        self.attn_w = {}
+        for l in self.layers:
             a = synth.attention_weights(dw, l)
-            self.attn_w.append({
+            self.attn_w[l] = {
                 "wq": widen(wdt, a["wq"], qd, wl.d), "wk": widen(wdt, a["wk"], kd, wl.d),
                 "wv": widen(wdt, a["wv"], kd, wl.d), "wo": widen(wdt, a["wo"], wl.d, qd),
-                **{n: _widen_vec(wdt, a[n]) for n in ("norm_in", "norm_post", "norm_q", "norm_k")}})
+                **{n: _widen_vec(wdt, a[n]) for n in ("norm_in", "norm_post", "norm_q", "norm_k")}}
         self.Tmax = dw.ctx + (wl.tokens if max_tokens is None else max_tokens)
-        self.K = np.zeros((self.L, self.Hkv, self.Tmax, self.D), dtype=np.float64)
-        self.V = np.zeros_like(self.K)
-        for l in range(self.L):
+        self.K, self.V = {}, {}
+        for l in self.layers:
             K, V = synth.kv_prefix(dw, l)
-            self.K[l, :, :dw.ctx] = synth.act_to_f64(K, wl.adtype)
-            self.V[l, :, :dw.ctx] = synth.act_to_f64(V, wl.adtype)
+            self.K[l] = np.zeros((self.Hkv, self.Tmax, self.D), dtype=np.float64)
+            self.V[l] = np.zeros_like(self.K[l])
+            self.K[l][:, :dw.ctx] = synth.act_to_f64(K, wl.adtype)
+            self.V[l][:, :dw.ctx] = synth.act_to_f64(V, wl.adtype)
         self.pos = dw.ctx
 
     def attention(self, l: int, x: np.ndarray) -> np.ndarray:
@@ -106,8 +113,8 @@ class DecoderOracle:
         v = matvec(w["wv"], a).reshape(self.Hkv, D)
         q = np.stack([rope(rmsnorm(q[h], w["norm_q"], dw.eps), self.pos, dw.rope_theta) for h in range(self.Hq)])
         k = np.stack([rope(rmsnorm(k[g], w["norm_k"], dw.eps), self.pos, dw.rope_theta) for g in range(self.Hkv)])
-        self.K[l, :, self.pos] = k
-        self.V[l, :, self.pos] = v
+        self.K[l][:, self.pos] = k
+        self.V[l][:, self.pos] = v
         o = attend(q, self.K[l], self.V[l], self.pos + 1)
         return matvec(w["wo"], o.reshape(-1))
 
@@ -115,6 +122,8 @@ class DecoderOracle:
         """One decode token: x0 [d] (fp64 values) enters layer 0."""
         if self.pos >= self.Tmax:
             raise RuntimeError("KV cache full")
+        if len(self.layers) != self.L:
+            raise RuntimeError("decode_token needs every layer (built with layers=None)")
         L, d, k, E = self.L, self.d, self.moe.k, self.moe.E
         x = np.array(x0, dtype=np.float64)
         attn = np.empty((L, d))

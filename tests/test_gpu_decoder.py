@@ -143,6 +143,36 @@ def test_int4_block_layer_by_layer_matches_the_oracle(P):
     _check_chain(out, log)
 
 
+def test_block48_bf16_full_size_sampled_layers(P):
+    # the bench's workload (48 blocks, 4095 cached positions, 6 GB pool): the trace of every layer
+    # against the oracle's slot group fed the GPU's selections, the pieces of sampled layers against
+    # the oracle on the GPU's own inputs
+    dw = synth.DECODERS["block48_bf16"]
+    T, sampled = 2, (0, 23, 47)
+    out, log, idx, tr = _run(P, dw, tokens=T)
+    moe = oracle.Oracle.for_workload(dw.moe, keep_slot_copies=False)
+    orc = DecoderOracle(dw, layers=sampled, max_tokens=T, moe=moe)
+    worst, recs = np.zeros(3), []
+    for t in range(T):
+        for l in range(dw.moe.n_layers):
+            m_gpu = log[t, l, 2][None, :]
+            oi, _, oz, _ = oracle.router(moe.routers[l], m_gpu[0], moe.k, moe.renorm)
+            check_routing(idx[t, l][None, :], oi[None, :], oz[None, :], moe.k)
+            o, _, _, _, r = moe.layer_step(l, m_gpu, compute_out=l in sampled, forced_idx=[idx[t, l]])
+            recs.append(r)
+            if l in sampled:
+                x = log[t, l, 0]
+                worst[0] = max(worst[0], rel_l2_rows(log[t, l, 1], orc.attention(l, x)))
+                m_ref = rmsnorm(x + log[t, l, 1], orc.attn_w[l]["norm_post"], dw.eps)
+                worst[1] = max(worst[1], rel_l2_rows(log[t, l, 2], m_ref))
+                worst[2] = max(worst[2], rel_l2_rows(log[t, l, 3], o[0]))
+        moe.token_step += 1
+        orc.pos += 1
+    assert worst.max() <= TOL["bf16"], f"attention / MoE input / MoE output rel L2 {worst}"
+    assert np.array_equal(trace_tuples(tr), trace_tuples(np.concatenate(recs)))
+    _check_chain(out, log)
+
+
 def _check_chain(out, log):
     T, L = log.shape[0], log.shape[1]
     for t in range(T):

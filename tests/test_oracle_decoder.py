@@ -200,7 +200,7 @@ def test_zero_output_projections_pass_the_stream_through():
 
     moe = oracle.Oracle.for_workload(wl, experts=zero_down)
     dec = DecoderOracle(DW, moe=moe, max_tokens=3)
-    for a in dec.attn_w:
+    for a in dec.attn_w.values():
         a["wo"][:] = 0.0
     X0 = _inputs(DW, 3)
     for t in range(3):
@@ -234,6 +234,25 @@ def test_the_cache_grows_by_one_position_per_token_and_refuses_overflow():
     dec.decode_token(X0[0])
     dec.decode_token(X0[1])
     assert dec.pos == DW.ctx + 2
-    assert np.abs(dec.K[:, :, DW.ctx:DW.ctx + 2]).sum() > 0
+    assert all(np.abs(dec.K[l][:, DW.ctx:DW.ctx + 2]).sum() > 0 for l in dec.layers)
     with pytest.raises(RuntimeError):
         dec.decode_token(X0[2])
+
+
+def test_a_subset_of_layers_gives_the_same_attention_as_the_whole_stack():
+    # built for layers 0 and 1 only, the oracle's attention of those layers on the same inputs is
+    # bit-identical to the full oracle's; decode_token refuses to run on a subset
+    X0 = _inputs(DW, 2)
+    full = DecoderOracle(DW)
+    part = DecoderOracle(DW, layers=[1, 0])
+    assert part.layers == [0, 1]
+    for t in range(2):
+        r = full.decode_token(X0[t])
+        x = np.array(X0[t], dtype=np.float64)
+        for l in range(DW.moe.n_layers):
+            np.testing.assert_array_equal(part.attention(l, x), r.attn[l])
+            x = x + r.attn[l] + r.moe_out[l]
+        part.pos += 1
+    one = DecoderOracle(DW, layers=[0])
+    with pytest.raises(RuntimeError):
+        one.decode_token(X0[0])

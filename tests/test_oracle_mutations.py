@@ -119,7 +119,7 @@ def _decoder_mutants():
 
     def value_not_cached(self, l, x):
         out = orig_attention(self, l, x)
-        self.V[l, :, self.pos] = 0.0  # the new position's value row is lost for later tokens
+        self.V[l][:, self.pos] = 0.0  # the new position's value row is lost for later tokens
         return out
 
     def wrong_norm_weights(self, l, x):
