@@ -147,15 +147,27 @@ __global__ void __launch_bounds__(kGemvWarps * 32) k_dec_gemv(const T* W, int ro
   constexpr int EPC = 16 / (int)sizeof(T);  // elements per 16-byte chunk
   const int lane = threadIdx.x & 31;
   const int nch = cols / EPC;
+  constexpr int U = 8;  // chunks in flight per lane: the loads of a batch are issued before any is used
   for (int r = blockIdx.x * kGemvWarps + (threadIdx.x >> 5); r < rows; r += gridDim.x * kGemvWarps) {
     const uint4* row = reinterpret_cast<const uint4*>(W + (int64_t)r * cols);
     float s = 0.f;
-    for (int c = lane; c < nch; c += 32) {
-      const uint4 w = __ldg(row + c);
-      if constexpr (sizeof(T) == 4)
-        s = dot16(w, s_act + c * EPC, s);
-      else
-        s = dot16_bf16(w, s_act + c * EPC, s);
+    for (int c0 = lane; c0 < nch; c0 += 32 * U) {
+      uint4 w[U];
+#pragma unroll
+      for (int j = 0; j < U; j++) {
+        const int c = c0 + 32 * j;
+        w[j] = c < nch ? __ldg(row + c) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int j = 0; j < U; j++) {
+        const int c = c0 + 32 * j;
+        if (c < nch) {  // chunks in ascending order per lane, as one at a time would take them
+          if constexpr (sizeof(T) == 4)
+            s = dot16(w[j], s_act + c * EPC, s);
+          else
+            s = dot16_bf16(w[j], s_act + c * EPC, s);
+        }
+      }
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
