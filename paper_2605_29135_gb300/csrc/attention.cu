@@ -89,10 +89,18 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_split(const float* q, 
   const int64_t p1 = p0 + per < T ? p0 + per : T;
   const CT* Kg = K + (int64_t)g * Tmax * D + lane * VPL;
   const CT* Vg = V + (int64_t)g * Tmax * D + lane * VPL;
+  // two-stage pipeline: the next position's K and V rows are requested before this one is used
+  float kf[VPL], vf[VPL], kn[VPL], vn[VPL];
+  if (p0 + warp < p1) {
+    load_row<VPL>(Kg + (p0 + warp) * D, kf);
+    load_row<VPL>(Vg + (p0 + warp) * D, vf);
+  }
   for (int64_t j = p0 + warp; j < p1; j += kAttnWarps) {
-    float kf[VPL], vf[VPL];
-    load_row<VPL>(Kg + j * D, kf);
-    load_row<VPL>(Vg + j * D, vf);
+    const int64_t jn = j + kAttnWarps;
+    if (jn < p1) {
+      load_row<VPL>(Kg + jn * D, kn);
+      load_row<VPL>(Vg + jn * D, vn);
+    }
 #pragma unroll
     for (int h = 0; h < G; h++) {
       float s = 0.f;
@@ -106,6 +114,11 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_split(const float* q, 
 #pragma unroll
       for (int v = 0; v < VPL; v++) acc[h][v] = fmaf(acc[h][v], c, p * vf[v]);
       m[h] = mn;
+    }
+#pragma unroll
+    for (int v = 0; v < VPL; v++) {
+      kf[v] = kn[v];
+      vf[v] = vn[v];
     }
   }
 #pragma unroll
