@@ -658,7 +658,8 @@ __device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad,
 // the CTA stages u, so the HBM latency overlaps the staging.
 template <int WD, int CHD>
 __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, const float* pgate, int l, int gw,
-                           int W, const float* u = nullptr) {
+                           int W, const float* u = nullptr, bool cta_active = true) {
+  if (!cta_active) return;  // the same for every thread of the CTA
   constexpr int E = Tr<WD>::epc;
   constexpr int KR = 24 / CHD > 8 ? 8 : (24 / CHD < 1 ? 1 : 24 / CHD);
   const int lane = threadIdx.x & 31;
@@ -1039,19 +1040,33 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
   const int k = a.k;
   unsigned nbar = 0, nwbar = 0;
 
-  // ---- phase R, every layer: one router row per warp at a time, h_l read through L2
+  // ---- phase R, every layer: one router row per warp at a time, h_l read through L2; RG chunks of
+  // the row and of h_l in flight per lane (the same per-lane order of chunks as k_fused, so the
+  // logits are bit-identical)
   for (int row = gw; row < a.L * a.E; row += W) {
+    constexpr int RG = 8;
     const int l = row / a.E;
     const uint8_t* wr = a.routers + (int64_t)row * xbytes;
     const uint8_t* hl = (const uint8_t*)a.hidden + (int64_t)l * xbytes;
     float acc = 0.f;
-    for (int c = lane; c < nchr; c += 32) {
-      const uint4 w = ld_stream(wr + (int64_t)c * 16);
-      const uint4 h = ld_cg(hl + (int64_t)c * 16);
-      if (WD == WD_FP32)
-        acc = dot_chunk<WD_FP32>(w, reinterpret_cast<const uint8_t*>(&h), acc);
-      else
-        acc = dot_chunk<WD_BF16>(w, reinterpret_cast<const uint8_t*>(&h), acc);
+    for (int c0 = 0; c0 < nchr; c0 += 32 * RG) {
+      uint4 w[RG], h[RG];
+#pragma unroll
+      for (int j = 0; j < RG; j++) {
+        const int c = c0 + j * 32 + lane;
+        w[j] = c < nchr ? ld_stream(wr + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+        h[j] = c < nchr ? ld_cg(hl + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int j = 0; j < RG; j++) {
+        const int c = c0 + j * 32 + lane;
+        if (c < nchr) {
+          if (WD == WD_FP32)
+            acc = dot_chunk<WD_FP32>(w[j], reinterpret_cast<const uint8_t*>(&h[j]), acc);
+          else
+            acc = dot_chunk<WD_BF16>(w[j], reinterpret_cast<const uint8_t*>(&h[j]), acc);
+        }
+      }
     }
     acc = warp_sum(acc);
     if (lane == 0) a.z[row] = acc;
@@ -1163,16 +1178,16 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
     // layer's misses, so the host link stays busy. Their copies then overlap these down rows,
     // which is safe because no miss of layer l + 1 takes the slot of an expert of layer l
     // (cap >= 2 k).
-    if (miss_cta) continue;
     const int HWW = (workers - mctas) * kFWarps;
+    const bool dact = !miss_cta;
     switch (chd_need) {
-      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
-      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
-      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
-      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
+      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
       case 5:
-      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
-      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, wgw, HWW, u); break;
+      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
     }
   }
 }
