@@ -133,3 +133,15 @@ def test_decoder_config_layout_and_argument_checks_without_gpu(lib):
     assert lib.moe_decoder_set_layer(None, 0, *([None] * 8)) == -1
     assert lib.moe_decoder_set_cache(None, 0, None, None, 0) == -1
     lib.moe_decoder_destroy(None)
+
+
+def test_binding_argument_counts_match_the_header(lib):
+    # every prototype in include/moe.h takes as many arguments as the ctypes declaration passes
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    protos = re.findall(r"\b(moe_[a-z_]+)\s*\(([^)]*)\)\s*;", src)
+    assert len(protos) == len(_declared())
+    for name, params in protos:
+        params = " ".join(params.split())
+        n = 0 if params in ("", "void") else params.count(",") + 1
+        assert len(getattr(lib, name).argtypes) == n, name
