@@ -130,7 +130,7 @@ typedef struct {
                              host link while the others compute the hits (0: library default). Batched
                              steps hand work items to all CTAs, missed experts first, and ignore it */
   int32_t batched_path;   /* MOE_BATCHED_AUTO (default) or MOE_BATCHED_CUDA_CORES */
-  int32_t policy;         /* MOE_POLICY_LRU (default) or MOE_POLICY_ROTARY */
+  int32_t policy;         /* MOE_POLICY_LRU (default), MOE_POLICY_ROTARY or MOE_POLICY_GUIDED */
   int32_t lookahead;      /* 1: exact layer lookahead (the layers' inputs are all given with the step, so the
                              decisions, the trace and the outputs are those of 0). MOE_SCHEDULE_HOST_COPY_ENGINE:
                              route layer l + 1 as soon as layer l's routing has reached the host, and issue its
