@@ -239,3 +239,35 @@ def test_full_cache_missing_weights_and_unsupported_handles(P):
         assert "device schedule" in str(ei.value)
     finally:
         m.destroy()
+
+
+def test_a_moe_layer_that_times_out_is_reported_by_the_next_step_and_the_decoder_recovers(P):
+    # an injected barrier fault makes the first MoE launch's waits run out (0.2 s); the device flag
+    # is sticky, so the step's later MoE launches leave at once. The next decoder step reports
+    # MOE_ERR_TIMEOUT before doing any MoE work, leaves the position where it was, and the steps
+    # after it run on an emptied pool
+    import torch
+
+    from paper_2605_29135_gb300.workload import create_decoder_for_workload
+
+    dw = TINY
+    xs = torch.from_numpy(synth.token_inputs(dw, 4).view(np.float32)).cuda()
+    y = torch.empty(dw.moe.d, dtype=torch.float32, device="cuda")
+    m, dec = create_decoder_for_workload(dw, max_tokens=4)
+    try:
+        dec.step(xs[0], y)
+        m.inject_fault("barrier_timeout")
+        dec.step(xs[1], y)
+        torch.cuda.synchronize()
+        pos = dec.position
+        with pytest.raises(P.MoEError) as ei:
+            dec.step(xs[2], y)
+        assert ei.value.status == -6 and dec.position == pos
+        dec.step(xs[2], y)
+        torch.cuda.synchronize()
+        assert np.isfinite(y.cpu().numpy()).all()
+        tr = m.get_residency_trace()
+        assert tr["step"].max() == 0 and (tr["kind"] == 1).all()  # a cold pool again, step 0
+    finally:
+        dec.destroy()
+        m.destroy()
