@@ -240,6 +240,7 @@ def oracle_layer_sample(wl, hidden, budget_s):
 
 KERNEL_SOURCES = {
     "k_fused": ("fused.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh"),
+    "k_fused_la": ("fused.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh"),
     "k_fused_batched": ("fused_batched.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh", "tc.cuh"),
     "k_fused_batched_tc": ("fused_batched.cu", "fused.cuh", "dev.cuh", "grid.cuh", "topk.cuh", "tc.cuh"),
 }
@@ -285,7 +286,7 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
 
     wr = wl.replace(cap_slots=wl.n_gid)
     m = create_for_workload(wr, device=device, trace_capacity=0, schedule=args.schedule,
-                            batched_path=args.batched_path, policy=args.policy)
+                            batched_path=args.batched_path, policy=args.policy, lookahead=args.lookahead)
     try:
         m.preload()
         n_tok = hid_dev.shape[0]
@@ -316,8 +317,9 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
     phases = {k[len("fused_phase_"):]: round(v["total_ms"] * 1e3 / v["launches"], 2)
               for k, v in prof.items() if k.startswith("fused_phase_") and v["launches"]}
     tensor_cores = prof.get("fused_phase_gather", {}).get("launches", 0) > 0
-    kname = (("k_fused_batched_tc" if tensor_cores else "k_fused_batched") if wl.batch > 1 else "k_fused") \
-        if dom == "fused_step" else dom
+    la_dev = args.lookahead and args.schedule == "device" and wl.batch == 1
+    kname = (("k_fused_batched_tc" if tensor_cores else "k_fused_batched") if wl.batch > 1 else
+             ("k_fused_la" if la_dev else "k_fused")) if dom == "fused_step" else dom
     traffic_file = f"{kname}_{wl.name}_resident.md".replace("k_fused_stack48_bf16", "k_fused_stack48")
     return {"bound": "hbm", "kernel": kname,
             "workload": f"{wl.name} with all {wl.n_gid} experts resident (preloaded), batch {wl.batch}",
@@ -366,6 +368,169 @@ def run_reference(args, wl):
     return 0
 
 
+def decoder_oracle_sample(dw, budget_s: float = 15.0, max_layers: int = 4):
+    """Time the fp64 decoder oracle (as it stands) on its first layers: whole tokens through
+    min(max_layers, L) chained blocks with the workload's KV prefix, scaled to tokens/s of the
+    whole stack by the layer count (every layer does the same work). The experts the sampled tokens
+    need are generated before the clock starts."""
+    import synth
+    from oracle.decoder import DecoderOracle
+
+    n = min(max_layers, dw.moe.n_layers)
+    part = dw.replace(moe=dw.moe.replace(n_layers=n))
+    xs = synth.token_inputs(part, 8)
+    cache = {}
+
+    def fetch(l, e):
+        if (l, e) not in cache:
+            cache[(l, e)] = synth.expert_weights(part.moe, l, e)
+        return cache[(l, e)]
+
+    # a first, untimed pass generates the host tier's experts these tokens route to
+    probe = DecoderOracle(part, max_tokens=8)
+    probe.moe.experts = fetch
+    t0 = time.perf_counter()
+    n_tok = 0
+    while n_tok < 8 and time.perf_counter() - t0 < budget_s:
+        probe.decode_token(synth.act_to_f64(xs[n_tok], part.moe.adtype))
+        n_tok += 1
+    del probe
+    orc = DecoderOracle(part, max_tokens=8)
+    orc.moe.experts = fetch
+    t0 = time.perf_counter()
+    for t in range(n_tok):
+        orc.decode_token(synth.act_to_f64(xs[t], part.moe.adtype))
+    dt = time.perf_counter() - t0
+    return {"value": n_tok * n / dw.moe.n_layers / dt, "unit": "tok/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{n_tok} token(s) through the first {n} of {dw.moe.n_layers} chained decoder blocks of "
+                      f"{dw.name} (context {dw.ctx}), fp64, {dt:.1f} s, scaled by {dw.moe.n_layers}/{n} layers"}
+
+
+def run_decoder(args, dw):
+    """Chained decoder blocks (attention over a KV cache, then the MoE layer) at batch 1: one step
+    is one decode token through every block (moe_decoder_step)."""
+    import torch
+
+    import paper_2605_29135_gb300 as P
+    import synth
+    from paper_2605_29135_gb300.workload import create_decoder_for_workload
+
+    wl = dw.moe
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        cb = decoder_oracle_sample(dw)
+        print(json.dumps({"metric": "chained MoE decoder tok/s at batch 1 under 6 GB expert cap",
+                          "value": cb["value"], "unit": "tok/s", "impl": "reference", "n_gpus": args.gpus,
+                          "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / cb["value"],
+                          "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                          "data": "synthetic (seeded)", "config": {"workload": dw.name, "context": dw.ctx},
+                          "cpu_baseline": cb,
+                          "e2e": {"value": cb["value"], "unit": "tok/s", "h2d_bytes_per_step": 0,
+                                  "d2h_bytes_per_step": 0}}))
+        return 0
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    P.build()
+    peak_hbm, _ = load_peaks()
+    e2e_steps = args.e2e_steps or max(8, args.steps // 4)
+    prof_steps = max(2, args.steps // 2)
+    n_tok = args.warmup + args.steps + prof_steps + e2e_steps
+    xs = synth.token_inputs(dw, n_tok)
+    m, dec = create_decoder_for_workload(dw, max_tokens=n_tok, device=local, trace_capacity=0)
+    eb = P.expert_bytes(m.cfg)
+    h2d_gbs = measure_h2d(torch, eb)
+    tdt = torch.float32 if wl.adtype == "fp32" else torch.bfloat16
+    raw = torch.from_numpy(xs.view(np.float32) if wl.adtype == "fp32" else xs.view(np.int16))
+    x_dev = raw.cuda().view(tdt) if wl.adtype != "fp32" else raw.cuda()
+    y_dev = torch.empty(wl.d, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    for i in range(args.warmup):
+        dec.step(x_dev[i], y_dev, stream=stream)
+    torch.cuda.synchronize()
+    s0 = m.get_stats()
+    clocks = ClockSampler(local)
+    clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.warmup, args.warmup + args.steps):
+        dec.step(x_dev[i], y_dev, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    s1 = m.get_stats()
+    # a second pass with the MoE launches bracketed by CUDA events: the rest of the step time is the
+    # attention block (its kernels and the launch gaps between them)
+    first = args.warmup + args.steps
+    m.profile_enable(True)
+    m.profile_read()
+    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    p0.record(stream)
+    for i in range(first, first + prof_steps):
+        dec.step(x_dev[i], y_dev, stream=stream)
+    p1.record(stream)
+    torch.cuda.synchronize()
+    prof = m.profile_read()
+    m.profile_enable(False)
+    moe_ms = prof.get("fused_step", {}).get("total_ms", 0.0) / prof_steps
+    attn_ms = p0.elapsed_time(p1) / prof_steps - moe_ms
+    # end to end: the token's input from pinned host memory, the output stream read back, per step
+    x_host = raw.pin_memory()
+    y_host = torch.empty(wl.d, dtype=torch.float32).pin_memory()
+    x_buf = torch.empty_like(x_dev[0])
+    t0 = time.perf_counter()
+    for i in range(first + prof_steps, n_tok):
+        x_buf.copy_(x_host[i].view(tdt) if wl.adtype != "fp32" else x_host[i], non_blocking=True)
+        dec.step(x_buf, y_dev, stream=stream)
+        y_host.copy_(y_dev, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+    e2e_s = time.perf_counter() - t0
+    dec.destroy()
+    m.destroy()
+    es = 4 if wl.adtype == "fp32" else 2
+    qd, kd = dw.n_heads * dw.head_dim, dw.n_kv_heads * dw.head_dim
+    attn_w = ((qd + 2 * kd) * wl.d + wl.d * qd + 2 * wl.d + 2 * dw.head_dim) * es
+    mean_pos = dw.ctx + args.warmup + (args.steps + 1) / 2  # positions read per layer, averaged over the window
+    kv_read = 2 * kd * mean_pos * es
+    misses, hits = s1["misses"] - s0["misses"], s1["hits"] - s0["hits"]
+    hbm = wl.n_layers * (attn_w + kv_read + wl.router_bytes()) + (hits + misses) / args.steps * eb
+    miss_b = misses * eb / args.steps
+    t_star = max(hbm / (peak_hbm * 1e9), miss_b / (h2d_gbs * 1e9))
+    ms_step = ms / args.steps
+    line = {"metric": "chained MoE decoder tok/s at batch 1 under 6 GB expert cap", "value": args.steps / (ms * 1e-3),
+            "unit": "tok/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if es == 2 else "f32",
+            "data": "synthetic (seeded weights, N(0, 1) KV prefix, AR(1) token inputs)",
+            "config": {"workload": dw.name, "layers": wl.n_layers, "d": wl.d, "heads": dw.n_heads,
+                       "kv_heads": dw.n_kv_heads, "head_dim": dw.head_dim, "context": dw.ctx,
+                       "experts_per_layer": wl.n_experts, "top_k": wl.top_k, "d_ff": wl.d_ff,
+                       "cap_slots": wl.cap_slots, "batch": 1, "parallelism": "single GPU",
+                       "l2": "inputs larger than L2 (2.2 GB of attention weights and KV cache per token)"},
+            "step_roofline": {"t_star_ms": t_star * 1e3, "frac": t_star * 1e3 / ms_step, "hbm_bytes_per_step": hbm,
+                              "miss_bytes_per_step": miss_b, "h2d_peak_gbs": h2d_gbs, "hbm_peak_gbs": peak_hbm,
+                              "hit_rate": 1.0 - misses / max(1, hits + misses)},
+            "roofline": {"bound": "hbm", "kernel": "attention block: norms, q/k/v and W_o GEMVs, rotary + KV "
+                                                  "append, split attention + merge (k_dec_*, k_attn_*)",
+                         "achieved": wl.n_layers * (attn_w + kv_read) / (attn_ms * 1e-3) / 1e9 if attn_ms > 0 else None,
+                         "peak": peak_hbm, "unit": "GB/s",
+                         "frac": (wl.n_layers * (attn_w + kv_read) / (attn_ms * 1e-3) / 1e9 / peak_hbm)
+                         if attn_ms > 0 else None,
+                         "traffic": None, "bytes_per_step": wl.n_layers * (attn_w + kv_read),
+                         "ms_per_step": attn_ms, "moe_ms_per_step": moe_ms,
+                         "timing": "profiled step time minus the MoE launches' CUDA-event time; includes the "
+                                   "launch gaps between the attention block's kernels"},
+            "gpu_launches": args.steps * (8 * wl.n_layers + 1),  # 7 attention-block launches + 1 MoE per layer, 1 output
+            "clocks": clk,
+            "e2e": {"value": e2e_steps / e2e_s, "unit": "tok/s", "h2d_bytes_per_step": wl.d * es,
+                    "d2h_bytes_per_step": wl.d * 4, "steps": e2e_steps, "api": "Decoder.step with host copies"}}
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = decoder_oracle_sample(dw)
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -381,8 +546,12 @@ def main():
     ap.add_argument("--layers", type=int, default=None, help="layer count override (small profiling cases)")
     ap.add_argument("--preload", action="store_true", help="fill the pool (moe_preload) before the warm-up")
     ap.add_argument("--miss-ctas", type=int, default=0, help="CTAs streaming missed experts (0: library default)")
-    ap.add_argument("--policy", default="lru", choices=["lru", "rotary"],
-                    help="slot-group replacement policy (rotary: host copy-engine schedule only)")
+    ap.add_argument("--policy", default="lru", choices=["lru", "rotary", "guided"],
+                    help="slot-group replacement policy (rotary: batch 1; guided: device schedule, batch 1)")
+    ap.add_argument("--lookahead", action="store_true",
+                    help="exact layer lookahead: host copy-engine schedule, route layer l + 1 and issue its copies "
+                         "while layer l computes; device schedule, one kernel routes every layer, then CTA 0 runs "
+                         "the lookups up to two layers ahead of the compute")
     ap.add_argument("--batched-path", default="auto", choices=["auto", "cuda_cores"],
                     help="expert FFN of batched steps: tensor cores where the shape allows, or CUDA cores")
     args = ap.parse_args()
@@ -390,6 +559,8 @@ def main():
         ap.error("--warmup must be >= 3")
     import synth
 
+    if args.workload in synth.DECODERS:
+        return run_decoder(args, synth.DECODERS[args.workload])
     wl = synth.WORKLOADS[args.workload]
     if args.layers is not None:
         wl = wl.replace(n_layers=args.layers)
@@ -430,7 +601,7 @@ def main():
     thp0 = anon_huge_kb()
     t_setup = time.perf_counter()
     m = create_for_workload(wl, device=local, trace_capacity=0, schedule=args.schedule, miss_ctas=args.miss_ctas,
-                            batched_path=args.batched_path, policy=args.policy)
+                            batched_path=args.batched_path, policy=args.policy, lookahead=args.lookahead)
     t_setup = time.perf_counter() - t_setup
     thp_gb = (anon_huge_kb() - thp0) / 1e6
     eb = P.expert_bytes(m.cfg)
@@ -523,6 +694,7 @@ def main():
                    "parallelism": "replicas" if world > 1 else "single GPU", "schedule": args.schedule,
                    "miss_ctas": args.miss_ctas or "default",
                    "batched_path": args.batched_path if wl.batch > 1 else None, "policy": args.policy,
+                   "lookahead": args.lookahead,
                    "l2": f"inputs larger than L2 ({wl.cap_slots * eb / 1e9:.1f} GB pool, "
                          f"{hbm_bytes_step / 1e9:.1f} GB of expert weights read per step)"},
         "step_roofline": {"bound": "h2d" if t_h2d >= t_hbm else "hbm", "t_star_ms": t_star * 1e3,

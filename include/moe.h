@@ -97,13 +97,14 @@ enum { MOE_BATCHED_AUTO = 0, MOE_BATCHED_CUDA_CORES = 1 };
  *     previous occupant. A miss returns to the slot it was last evicted from when that slot holds no
  *     expert of the layer-step (reverse rotation), else takes the first such slot at or after the
  *     hand, which then moves past it (forward rotation). Hits change nothing. Misses in ascending
- *     global id. Both schedules, max_batch 1. */
+ *     global id. Both schedules; a batched step (device schedule) applies it to the union of the
+ *     batch's experts. */
 /*   MOE_POLICY_GUIDED: router-guided replacement, one reading of the paper's residency decisions
  *     that use information produced during execution (Sec. 3). Each layer keeps the rank of every
  *     expert in its most recent routing (0 = highest logit; for a batch, the best rank over its
  *     sequences). A miss takes the lowest free slot, else evicts the resident not needed this
  *     layer-step with the largest rank, ties to the more recent use, then to the lower global id.
- *     Residency planner only for now (moe_create rejects it). */
+ *     Both schedules (device: n_layers * n_experts < 2^23), and the residency planner. */
 enum { MOE_POLICY_LRU = 0, MOE_POLICY_ROTARY = 1, MOE_POLICY_GUIDED = 2 };
 
 typedef struct {
@@ -129,7 +130,17 @@ typedef struct {
                              host link while the others compute the hits (0: library default). Batched
                              steps hand work items to all CTAs, missed experts first, and ignore it */
   int32_t batched_path;   /* MOE_BATCHED_AUTO (default) or MOE_BATCHED_CUDA_CORES */
-  int32_t policy;         /* MOE_POLICY_LRU (default) or MOE_POLICY_ROTARY */
+  int32_t policy;         /* MOE_POLICY_LRU (default), MOE_POLICY_ROTARY or MOE_POLICY_GUIDED */
+  int32_t lookahead;      /* 1: exact layer lookahead (the layers' inputs are all given with the step, so the
+                             decisions, the trace and the outputs are those of 0). MOE_SCHEDULE_HOST_COPY_ENGINE:
+                             route layer l + 1 as soon as layer l's routing has reached the host, and issue its
+                             miss copies while layer l computes; a copy into a slot layer l still reads waits
+                             for layer l's kernels. MOE_SCHEDULE_DEVICE (max_batch 1, MOE_POLICY_LRU): one kernel
+                             routes every layer first, then CTA 0 runs the layers' lookups in order ahead of
+                             the other CTAs, which compute each layer with one barrier among them; needs
+                             cap_slots >= 2 * top_k unless every expert is resident. Steps of a
+                             chained decoder (moe_decoder_step) run layer by layer whatever this says.
+                             0 (default): one layer after another. */
 } moe_config;
 
 /* One residency record: a requested expert's outcome in one layer-step. */
@@ -220,6 +231,13 @@ moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_
 
 moe_status moe_get_stats(moe_handle* h, moe_stats* out);
 
+/* Router logits of the last decode step, fp32 [n_layers x max_batch x n_experts] (z = W_r h as the
+ * device computed it; the router-guided policy ranks experts by them; rows b >= the step's batch
+ * are stale). MOE_SCHEDULE_DEVICE, or MOE_SCHEDULE_HOST_COPY_ENGINE under MOE_POLICY_GUIDED
+ * (MOE_ERR_INVALID otherwise, or if n is below n_layers * max_batch * n_experts). Waits for the
+ * step. */
+moe_status moe_get_last_logits(moe_handle* h, float* z, int64_t n);
+
 /* Empty the slot pool (all experts non-resident), step clock 0, trace and stats cleared. */
 moe_status moe_reset_residency(moe_handle* h);
 
@@ -280,6 +298,78 @@ moe_status moe_inject_fault(moe_handle* h, int32_t kind);
 #define MOE_NOALLOC_MAX_EXPERTS 256
 moe_status moe_route_noalloc(const void* w_r, const void* hidden, int32_t rows, int32_t n_experts, int32_t d,
                              int32_t top_k, int32_t renorm, int32_t wdtype, int32_t* idx, float* gate, void* stream);
+
+/* ---- Attention of the decoder block around the MoE layer ------------------------------------
+ * Grouped-query attention of one decode token over a KV cache (the decoder the paper ran kept a
+ * 4096-token context). No handle; nothing is allocated.
+ *   q        device fp32 [n_heads x head_dim], already normalised, rotated (scale 1/sqrt(head_dim)
+ *            is applied inside)
+ *   k_cache, v_cache  device [n_kv_heads x max_pos x head_dim] of cache_dtype (MOE_DTYPE_BF16 or
+ *            MOE_DTYPE_FP32), 16-byte aligned; positions [0, n_pos) are read
+ *   out      device fp32 [n_heads x head_dim]: query head h reads kv head h / (n_heads / n_kv_heads);
+ *            out_h = sum_j softmax_j(q_h . k_j / sqrt(head_dim)) v_j
+ *   scratch  device fp32 of at least moe_attention_scratch_floats(...) floats (per-split partials)
+ *   stream   cudaStream_t the two kernels are ordered on (NULL = legacy default stream)
+ * head_dim 64 or 128; n_heads / n_kv_heads in {1, 2, 4, 8}; 1 <= n_pos <= max_pos. MOE_ERR_INVALID
+ * for other arguments (moe_attention_scratch_floats returns -1 for them), MOE_ERR_CUDA if a
+ * launch fails. */
+int64_t moe_attention_scratch_floats(int32_t n_heads, int32_t n_kv_heads, int32_t head_dim, int64_t n_pos);
+moe_status moe_attention_decode(const float* q, const void* k_cache, const void* v_cache, int32_t cache_dtype,
+                                int32_t n_heads, int32_t n_kv_heads, int32_t head_dim, int64_t max_pos, int64_t n_pos,
+                                float* out, float* scratch, int64_t scratch_floats, void* stream);
+
+/* ---- Chained decoder blocks around the MoE layer ---------------------------------------------
+ * One decode token at batch 1 through a stack of decoder blocks whose layers feed one another:
+ * the paper's end-to-end setting (a whole MoE decoder at a 4096-token context, Sec.
+ * "Experimental Setup"). The paper prints no architecture; the block is a Qwen3-MoE-class
+ * reading. Per layer l, with the residual stream x (fp32) at position p:
+ *   a = RMSNorm(x) * w_in;  q = W_q a [n_heads x head_dim];  k = W_k a, v = W_v a [n_kv_heads x head_dim]
+ *   q_h = RoPE(RMSNorm(q_h) * w_q, p);  k_g = RoPE(RMSNorm(k_g) * w_k, p);  (k_g, v_g) -> cache row p
+ *   o_h = sum_j softmax_j(q_h . K_j / sqrt(head_dim)) V_j over rows 0..p of kv head h / (n_heads / n_kv_heads)
+ *   x += W_o [o_0 .. o_{n_heads-1}];  m = RMSNorm(x) * w_post;  x += MoE_l(m)
+ * RMSNorm(y) = y / sqrt(mean(y^2) + eps); RoPE rotates element i with element i + head_dim/2 by
+ * the angle p * rope_theta^(-2i/head_dim). MoE_l is layer l of the handle's decode step (routing,
+ * one residency step of its slot group, expert FFN, combine); layer l + 1 routes on what layer l
+ * produced, so every layer's MoE runs after its own attention.
+ *
+ * moe_decoder_create: moe must use MOE_SCHEDULE_DEVICE with max_batch 1, and outlives the
+ *   decoder. Decode steps of the decoder advance the handle's decode steps, trace, statistics and
+ *   slot group like moe_decode_step does (one decode step per token). Weights, KV caches and the
+ *   MoE layers' inputs and outputs use the handle's activation storage: fp32 (MOE_DTYPE_FP32
+ *   experts) or bf16 (bf16 and int4 experts). head_dim 64 or 128; n_heads / n_kv_heads in
+ *   {1, 2, 4, 8}; d a multiple of 16 bytes of activations; d and n_heads * head_dim at most 12288;
+ *   max_pos = KV-cache rows per layer. Allocates every layer's weights and caches on the handle's
+ *   device. MOE_ERR_INVALID / MOE_ERR_OOM with the message in moe_decoder_last_error(NULL).
+ * moe_decoder_set_layer: host pointers, copied: wq [n_heads*head_dim x d], wk and wv
+ *   [n_kv_heads*head_dim x d], wo [d x n_heads*head_dim] (row-major, out x in), norm_in and
+ *   norm_post [d], norm_q and norm_k [head_dim].
+ * moe_decoder_set_cache: host K and V [n_kv_heads x n_pos x head_dim], copied into rows
+ *   [0, n_pos) of the layer's cache, which then holds n_pos positions (n_pos in [0, max_pos]).
+ * moe_decoder_step: x_in device [d] in the activation storage (the stream entering layer 0);
+ *   x_out device fp32 [d] (the stream after the last layer); layer_log NULL or device fp32
+ *   [n_layers x 4 x d]: per layer the stream entering it, W_o o, the MoE input as stored, and the
+ *   MoE output as stored. Every layer's cache must hold the same number p of positions; the step
+ *   writes row p and reads rows 0..p, then every layer holds p + 1. Returns after enqueueing on
+ *   stream. MOE_ERR_NOT_REGISTERED if a layer's weights are missing, MOE_ERR_CAPACITY when p =
+ *   max_pos, the MoE's status (its message copied) if a MoE layer fails, which empties the pool;
+ *   a failed step leaves the positions unchanged. Not thread-safe per decoder.
+ * moe_decoder_position: positions each layer's cache holds (-1 for NULL). */
+typedef struct moe_decoder moe_decoder;
+typedef struct {
+  int32_t n_heads, n_kv_heads, head_dim;
+  int32_t reserved; /* 0 */
+  int64_t max_pos;
+  double eps, rope_theta;
+} moe_decoder_config;
+moe_status moe_decoder_create(moe_handle* moe, const moe_decoder_config* cfg, moe_decoder** out);
+moe_status moe_decoder_set_layer(moe_decoder* dec, int32_t layer, const void* wq, const void* wk, const void* wv,
+                                 const void* wo, const void* norm_in, const void* norm_post, const void* norm_q,
+                                 const void* norm_k);
+moe_status moe_decoder_set_cache(moe_decoder* dec, int32_t layer, const void* k, const void* v, int64_t n_pos);
+moe_status moe_decoder_step(moe_decoder* dec, const void* x_in, float* x_out, float* layer_log, void* stream);
+int64_t moe_decoder_position(const moe_decoder* dec);
+const char* moe_decoder_last_error(const moe_decoder* dec);
+void moe_decoder_destroy(moe_decoder* dec);
 
 /* ---- Residency planner ------------------------------------------------------------------------
  * The library's host slot table (the code the MOE_SCHEDULE_HOST_COPY_ENGINE schedule runs, and

@@ -400,8 +400,11 @@ class Oracle:
             ys[rk], _ = expert_ffn(Wg, Wu, Wd, h)
         return combine(ys, gate), idx, gate
 
-    def decode_step(self, hidden_raw: np.ndarray, compute_out: bool = True, forced_idx=None) -> StepResult:
-        """One decode step over all layers. hidden_raw: raw activation storage [L x B x d]."""
+    def decode_step(self, hidden_raw: np.ndarray, compute_out: bool = True, forced_idx=None,
+                    forced_ranks=None) -> StepResult:
+        """One decode step over all layers. hidden_raw: raw activation storage [L x B x d].
+        forced_idx [L x B x k] / forced_ranks [L x E] replace the routing's choices and the guided
+        policy's ranks (to replay a run whose fp32 logits swapped near-equal experts)."""
         import synth
 
         L, B = hidden_raw.shape[0], hidden_raw.shape[1]
@@ -414,14 +417,15 @@ class Oracle:
         recs = []
         for l in range(L):
             o, idx[l], gate[l], z[l], r = self.layer_step(l, h[l], compute_out,
-                                                          None if forced_idx is None else forced_idx[l])
+                                                          None if forced_idx is None else forced_idx[l],
+                                                          None if forced_ranks is None else forced_ranks[l])
             if compute_out:
                 out[l] = o
             recs.append(r)
         self.token_step += 1
         return StepResult(out, np.concatenate(recs), idx, gate, z)
 
-    def layer_step(self, l: int, h: np.ndarray, compute_out: bool = True, forced_idx=None):
+    def layer_step(self, l: int, h: np.ndarray, compute_out: bool = True, forced_idx=None, forced_ranks=None):
         """Layer l of the current decode step on fp64 inputs h [B x d]: routing, one residency step,
         expert FFNs from the slot copies and the combine. The clock is token_step * L + l; the
         caller advances token_step once per decode step (decode_step does).
@@ -436,7 +440,8 @@ class Oracle:
             idx[b], gate[b], z[b], _ = router(self.routers[l], h[b], self.k, self.renorm, fi)
         needed = sorted(set(int(l * self.E + e) for e in idx.ravel()))
         if self.policy == "guided":
-            self.table.set_layer_ranks(l, np.min([route_ranks(z[b]) for b in range(B)], axis=0))
+            ranks = np.min([route_ranks(z[b]) for b in range(B)], axis=0) if forced_ranks is None else forced_ranks
+            self.table.set_layer_ranks(l, ranks)
         r = self.table.step(clock, needed, self.token_step)
         if self.prefetch:
             admit = set()

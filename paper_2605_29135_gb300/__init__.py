@@ -15,7 +15,8 @@ import ctypes
 import numpy as np
 
 from . import _lib
-from ._lib import BATCHED_PATH, DTYPE, POLICY, SCHEDULE, STATUS, KernelTime, MoeConfig, Stats, TraceRec
+from ._lib import (BATCHED_PATH, DTYPE, POLICY, SCHEDULE, STATUS, DecoderConfig, KernelTime, MoeConfig, Stats,
+                   TraceRec)
 
 TRACE_DTYPE = np.dtype([("step", np.int32), ("layer", np.int32), ("expert", np.int32), ("kind", np.int32),
                         ("slot", np.int32), ("evicted", np.int32)])
@@ -29,12 +30,13 @@ class MoEError(RuntimeError):
 
 def make_config(d, n_experts, top_k, d_ff, n_layers, wdtype, adtype, cap_slots=0, cap_bytes=0, renorm=True,
                 device=0, max_batch=1, trace_capacity=1 << 22, device_pool=None, schedule="device",
-                miss_ctas=0, batched_path="auto", policy="lru") -> MoeConfig:
+                miss_ctas=0, batched_path="auto", policy="lru", lookahead=False) -> MoeConfig:
     return MoeConfig(d=d, n_experts=n_experts, top_k=top_k, d_ff=d_ff, n_layers=n_layers, max_batch=max_batch,
                      wdtype=DTYPE[wdtype], adtype=DTYPE[adtype], cap_slots=cap_slots, cap_bytes=cap_bytes,
                      renorm=1 if renorm else 0, device=device, device_pool=device_pool,
                      trace_capacity=trace_capacity, schedule=SCHEDULE[schedule], miss_ctas=miss_ctas,
-                     batched_path=BATCHED_PATH[batched_path], policy=POLICY[policy])
+                     batched_path=BATCHED_PATH[batched_path], policy=POLICY[policy],
+                     lookahead=1 if lookahead else 0)
 
 
 def expert_bytes(cfg: MoeConfig) -> int:
@@ -159,6 +161,13 @@ class MoE:
         self._check(self.lib.moe_get_last_routing(self.h, _ptr(idx), _ptr(gate), n))
         shape = (self.cfg.n_layers, self.cfg.max_batch, self.cfg.top_k)
         return idx.reshape(shape), gate.reshape(shape)
+
+    def get_last_logits(self) -> np.ndarray:
+        """Router logits of the last step, float32 [n_layers x max_batch x n_experts] (device schedule)."""
+        c = self.cfg
+        z = np.empty(c.n_layers * c.max_batch * c.n_experts, dtype=np.float32)
+        self._check(self.lib.moe_get_last_logits(self.h, _ptr(z), z.size))
+        return z.reshape(c.n_layers, c.max_batch, c.n_experts)
 
     def get_stats(self) -> dict:
         s = Stats()
@@ -318,6 +327,117 @@ def plan_caps(n_layers: int, n_experts: int, caps, idx, policy: str = "lru", ran
             row["link_bytes_per_step"] = (r["misses"] + r["prefetches"]) * expert_bytes / max(1, T)
         rows.append(row)
     return rows
+
+
+class Decoder:
+    """Chained decoder blocks around a MoE handle's layers (moe_decoder_create ... _destroy).
+
+    The MoE handle (device schedule, max_batch 1) must outlive the decoder; decoder steps advance
+    its decode steps, trace and slot group. Weights and caches use the handle's activation storage
+    (float32, or bf16 bits as uint16)."""
+
+    def __init__(self, moe: MoE, n_heads: int, n_kv_heads: int, head_dim: int, max_pos: int, eps: float = 1e-6,
+                 rope_theta: float = 1e6):
+        self.lib = _lib.load()
+        self.moe = moe
+        self.cfg = DecoderConfig(n_heads=n_heads, n_kv_heads=n_kv_heads, head_dim=head_dim, reserved=0,
+                                 max_pos=max_pos, eps=eps, rope_theta=rope_theta)
+        self.es = 4 if moe.cfg.adtype == DTYPE["fp32"] else 2
+        h = ctypes.c_void_p()
+        st = self.lib.moe_decoder_create(moe.h, ctypes.byref(self.cfg), ctypes.byref(h))
+        if st != 0:
+            raise MoEError(st, self.lib.moe_decoder_last_error(None).decode())
+        self.h = h
+
+    def _check(self, st):
+        if st != 0:
+            raise MoEError(st, self.lib.moe_decoder_last_error(self.h).decode())
+
+    def set_layer(self, layer: int, wq, wk, wv, wo, norm_in, norm_post, norm_q, norm_k):
+        """Host arrays in the activation storage: wq [n_heads*head_dim x d], wk and wv
+        [n_kv_heads*head_dim x d], wo [d x n_heads*head_dim], norm_in and norm_post [d], norm_q and
+        norm_k [head_dim]."""
+        c, d = self.cfg, self.moe.cfg.d
+        qd, kd = c.n_heads * c.head_dim, c.n_kv_heads * c.head_dim
+        arrs = [np.ascontiguousarray(a) for a in (wq, wk, wv, wo, norm_in, norm_post, norm_q, norm_k)]
+        sizes = (qd * d, kd * d, kd * d, d * qd, d, d, c.head_dim, c.head_dim)
+        names = ("wq", "wk", "wv", "wo", "norm_in", "norm_post", "norm_q", "norm_k")
+        for name, a, n in zip(names, arrs, sizes):
+            _check_buffer(name, a, n * self.es, "host")
+        self._check(self.lib.moe_decoder_set_layer(self.h, layer, *(_ptr(a) for a in arrs)))
+
+    def set_cache(self, layer: int, K, V):
+        """K, V: host arrays [n_kv_heads x n_pos x head_dim] in the activation storage."""
+        K, V = np.ascontiguousarray(K), np.ascontiguousarray(V)
+        c = self.cfg
+        if K.shape != V.shape or K.ndim != 3 or K.shape[0] != c.n_kv_heads or K.shape[2] != c.head_dim:
+            raise ValueError("K and V must both be [n_kv_heads x n_pos x head_dim]")
+        n = K.shape[1]
+        for name, a in (("K", K), ("V", V)):
+            _check_buffer(name, a, c.n_kv_heads * n * c.head_dim * self.es, "host")
+        self._check(self.lib.moe_decoder_set_cache(self.h, layer, _ptr(K), _ptr(V), n))
+
+    def step(self, x_in, x_out, layer_log=None, stream=None):
+        """x_in: device tensor [d] in the activation dtype; x_out: device float32 [d]; layer_log:
+        None or device float32 [n_layers x 4 x d] (stream entering each layer, W_o o, MoE input,
+        MoE output)."""
+        import torch
+
+        m = self.moe.cfg
+        _check_buffer("x_in", x_in, m.d * self.es, "device", m.device)
+        _check_buffer("x_out", x_out, m.d * 4, "device", m.device)
+        if layer_log is not None:
+            _check_buffer("layer_log", layer_log, m.n_layers * 4 * m.d * 4, "device", m.device)
+        if stream is None:
+            stream = torch.cuda.current_stream(x_in.device)
+        self._check(self.lib.moe_decoder_step(self.h, _ptr(x_in), _ptr(x_out), _ptr(layer_log),
+                                              ctypes.c_void_p(stream.cuda_stream)))
+
+    @property
+    def position(self) -> int:
+        return int(self.lib.moe_decoder_position(self.h))
+
+    def destroy(self):
+        if getattr(self, "h", None):
+            self.lib.moe_decoder_destroy(self.h)
+            self.h = None
+
+    close = destroy
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def attention_decode(q, k_cache, v_cache, n_pos: int, stream=None):
+    """Grouped-query attention of one decode token (moe_attention_decode). q: device float32
+    [n_heads x head_dim]; k_cache, v_cache: device bfloat16 or float32 [n_kv_heads x max_pos x
+    head_dim]. Returns out, device float32 [n_heads x head_dim]."""
+    import torch
+
+    Hq, D = q.shape
+    Hkv, Tmax, D2 = k_cache.shape
+    if D2 != D or tuple(v_cache.shape) != tuple(k_cache.shape):
+        raise ValueError("q, k_cache and v_cache shapes disagree")
+    if q.dtype != torch.float32 or k_cache.dtype != v_cache.dtype or k_cache.dtype not in (torch.bfloat16,
+                                                                                         torch.float32):
+        raise ValueError("q must be float32, the caches both bfloat16 or both float32")
+    cache_dtype = DTYPE["fp32"] if k_cache.dtype == torch.float32 else DTYPE["bf16"]
+    lib = _lib.load()
+    n = lib.moe_attention_scratch_floats(Hq, Hkv, D, n_pos)
+    if n < 0:
+        raise MoEError(-1, "moe_attention_decode does not take this shape")
+    scratch = torch.empty(n, dtype=torch.float32, device=q.device)
+    out = torch.empty((Hq, D), dtype=torch.float32, device=q.device)
+    if stream is None:
+        stream = torch.cuda.current_stream(q.device)
+    st = lib.moe_attention_decode(_ptr(q), _ptr(k_cache), _ptr(v_cache), cache_dtype, Hq, Hkv, D, Tmax, n_pos,
+                                  _ptr(out), _ptr(scratch), n, ctypes.c_void_p(stream.cuda_stream))
+    if st != 0:
+        raise MoEError(st, "moe_attention_decode rejected the arguments" if st == -1 else "launch failed")
+    return out
 
 
 def route_noalloc(w_r, hidden, top_k: int, renorm: bool = True, stream=None):

@@ -26,7 +26,10 @@ EXPORTS = ["moe_expert_bytes", "moe_pool_bytes", "moe_create", "moe_set_router",
            "moe_decode_step", "moe_decode_step_host", "moe_get_residency_trace", "moe_get_last_routing",
            "moe_get_stats", "moe_reset_residency", "moe_profile_enable", "moe_profile_read", "moe_last_error",
            "moe_destroy", "moe_route_noalloc", "moe_preload", "moe_inject_fault", "moe_planner_create",
-           "moe_planner_preload", "moe_planner_step", "moe_planner_last_error", "moe_planner_destroy"]
+           "moe_planner_preload", "moe_planner_step", "moe_planner_last_error", "moe_planner_destroy",
+           "moe_get_last_logits", "moe_attention_scratch_floats", "moe_attention_decode", "moe_decoder_create",
+           "moe_decoder_set_layer", "moe_decoder_set_cache", "moe_decoder_step", "moe_decoder_position",
+           "moe_decoder_last_error", "moe_decoder_destroy"]
 
 
 class MoeConfig(ctypes.Structure):
@@ -35,7 +38,14 @@ class MoeConfig(ctypes.Structure):
                 ("wdtype", ctypes.c_int32), ("adtype", ctypes.c_int32), ("cap_slots", ctypes.c_int64),
                 ("cap_bytes", ctypes.c_int64), ("renorm", ctypes.c_int32), ("device", ctypes.c_int32),
                 ("device_pool", ctypes.c_void_p), ("trace_capacity", ctypes.c_int64), ("schedule", ctypes.c_int32),
-                ("miss_ctas", ctypes.c_int32), ("batched_path", ctypes.c_int32), ("policy", ctypes.c_int32)]
+                ("miss_ctas", ctypes.c_int32), ("batched_path", ctypes.c_int32), ("policy", ctypes.c_int32),
+                ("lookahead", ctypes.c_int32)]
+
+
+class DecoderConfig(ctypes.Structure):
+    _fields_ = [("n_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("reserved", ctypes.c_int32), ("max_pos", ctypes.c_int64), ("eps", ctypes.c_double),
+                ("rope_theta", ctypes.c_double)]
 
 
 class TraceRec(ctypes.Structure):
@@ -114,6 +124,26 @@ def load(path: str | None = None):
         L.moe_planner_step.restype = ctypes.c_int
         L.moe_planner_last_error.argtypes = [vp]
         L.moe_planner_last_error.restype = ctypes.c_char_p
+        L.moe_get_last_logits.argtypes = [vp, vp, i64]
+        L.moe_get_last_logits.restype = ctypes.c_int
+        L.moe_attention_scratch_floats.argtypes = [i32, i32, i32, i64]
+        L.moe_attention_scratch_floats.restype = i64
+        L.moe_attention_decode.argtypes = [vp, vp, vp, i32, i32, i32, i32, i64, i64, vp, vp, i64, vp]
+        L.moe_attention_decode.restype = ctypes.c_int
+        L.moe_decoder_create.argtypes = [vp, ctypes.POINTER(DecoderConfig), ctypes.POINTER(vp)]
+        L.moe_decoder_create.restype = ctypes.c_int
+        L.moe_decoder_set_layer.argtypes = [vp, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+        L.moe_decoder_set_layer.restype = ctypes.c_int
+        L.moe_decoder_set_cache.argtypes = [vp, i32, vp, vp, i64]
+        L.moe_decoder_set_cache.restype = ctypes.c_int
+        L.moe_decoder_step.argtypes = [vp, vp, vp, vp, vp]
+        L.moe_decoder_step.restype = ctypes.c_int
+        L.moe_decoder_position.argtypes = [vp]
+        L.moe_decoder_position.restype = i64
+        L.moe_decoder_last_error.argtypes = [vp]
+        L.moe_decoder_last_error.restype = ctypes.c_char_p
+        L.moe_decoder_destroy.argtypes = [vp]
+        L.moe_decoder_destroy.restype = None
         L.moe_planner_destroy.argtypes = [vp]
         L.moe_planner_destroy.restype = None
         _lib = L

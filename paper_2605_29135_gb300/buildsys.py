@@ -12,7 +12,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(HERE, "libmoe.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["kernels.cu", "fused.cu", "fused_batched.cu", "moe_api.cu", "noalloc.cu", "slot_table.cpp", "planner.cpp"]
+SOURCES = ["kernels.cu", "fused.cu", "fused_batched.cu", "moe_api.cu", "noalloc.cu", "attention.cu", "decoder.cu", "slot_table.cpp",
+           "planner.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]
 

@@ -1,11 +1,18 @@
 // Device-driven decode step (sm_103a): one cooperative persistent kernel per decode step.
 //
-// Per layer, four phases separated by grid barriers:
+// Per layer, phases R, C and D are separated by grid barriers; phase S runs in CTA 0 alongside
+// the start of phase C. Every CTA repeats the layer's top-k and classifies the selected experts
+// as hits or misses from the lookup table as it was before the step (S holds its table writes
+// back until phase D), so the hit rows of phase C start right after R; only the miss CTAs wait
+// (bounded) for CTA 0's published plan, which holds the misses' slots.
 //   R  router logits z = W_r h, one warp per expert row;
 //   S  CTA 0: top-k (ties -> lower id) and gates, then one step of the lookup table: hits keep
 //      their slot, misses (ascending global id) take the lowest free slot, else the unpinned
-//      resident with the smallest (last use, global id); records go to the trace buffer and the
-//      per-rank plan (slot, miss flag, gate) to global memory;
+//      resident with the smallest key: (last use, global id) under LRU; under router-guided
+//      replacement the largest rank in its layer's latest routing first (this layer's ranks are
+//      refreshed from z before the lookup), then the most recent use; the rotary ring otherwise.
+//      Records go to the trace buffer and the per-rank plan (slot, miss flag, gate) to global
+//      memory;
 //   C  gate-up rows of every rank, u_r[i] = silu(W_g[i] . h) * (W_u[i] . h). A few "miss CTAs"
 //      stream every missed expert from the page-locked host tier over NVLink-C2C: its gate/up
 //      rows are stored into the freed slot and used for u in the same pass, and its W_d region
@@ -14,8 +21,9 @@
 //      requests near what saturates it (tens of warps, not thousands);
 //   D  down rows + combine from the slots, out[o] = sum_r g_r (W_d^(r)[o] . u_r) in rank order.
 //
-// All CTAs are co-resident (cooperative launch). Every barrier wait is bounded by a timeout on
-// the global timer; on expiry the kernel sets an error flag and every CTA returns.
+// All CTAs are co-resident (cooperative launch). Every barrier wait, and the miss CTAs' wait for
+// the plan, is bounded by a timeout on the global timer; on expiry the kernel sets an error flag
+// and every CTA returns.
 #include <cuda_bf16.h>
 #include <math.h>
 
@@ -69,6 +77,24 @@ __device__ void find_victim_candidates(const FusedArgs& a) {
   if (threadIdx.x == 0) a.cand[kMaxRanks] = (unsigned long long)a.k;
 }
 
+// Lookup-table writes of a layer-step, held back until phase D: during phase C every CTA classifies
+// the layer's selected experts as hits or misses from the table as it was before the step, while
+// CTA 0 is still deciding the step (thread 0 of CTA 0 records, the same thread applies).
+struct PendingTable {
+  int n;
+  int gid[2 * kMaxRanks];
+  int val[2 * kMaxRanks];
+  __device__ void set(int g, int v) {
+    gid[n] = g;
+    val[n] = v;
+    n++;
+  }
+  __device__ void apply(const FusedArgs& a) {
+    for (int i = 0; i < n; i++) a.slot_of[gid[i]] = val[i];
+    n = 0;
+  }
+};
+
 // Rotary slot-group step for the misses of one layer-step (thread 0 of CTA 0; at most k misses,
 // in ascending id). A miss returns to the slot it was last evicted from when that slot holds no
 // expert of the step (reverse rotation), else takes the first such slot at or after the hand, which
@@ -77,7 +103,7 @@ __device__ void find_victim_candidates(const FusedArgs& a) {
 // at most k pinned slots and takes at most k), updated here as the step places experts.
 __device__ void rotary_place(const FusedArgs& a, int l, int clock, int k, int E, const int* need, const int* miss,
                              int* slot_out, int* evict_out, const int* ps_e, const int* ps_gid, int* win_gid,
-                             int* win_prior, int hand0, int nused0) {
+                             int* win_prior, int hand0, int nused0, PendingTable& pend) {
   const int nw = 2 * k + 1 < a.cap ? 2 * k + 1 : (int)a.cap;
   int placed_slot[kMaxRanks], placed_gid[kMaxRanks];
   int np = 0;
@@ -141,7 +167,7 @@ __device__ void rotary_place(const FusedArgs& a, int l, int clock, int k, int E,
     }
     // evict the occupant; bookkeeping of previous occupants
     if (occ >= 0) {
-      a.slot_of[occ] = -1;
+      pend.set(occ, -1);
       evictions++;
     } else {
       nused++;
@@ -158,7 +184,7 @@ __device__ void rotary_place(const FusedArgs& a, int l, int clock, int k, int E,
     if (wj >= 0) win_prior[wj] = occ;
     if (occ >= 0) a.prior_slot_of[occ] = slot;
     a.prior_slot_of[g] = -1;
-    a.slot_of[g] = slot;
+    pend.set(g, slot);
     placed_slot[np] = slot;
     placed_gid[np] = g;
     np++;
@@ -178,7 +204,8 @@ __device__ void rotary_place(const FusedArgs& a, int l, int clock, int k, int E,
 // Phase S, run by CTA 0 (all its threads). Every global read the phase needs is issued at its
 // start, side by side: the logits (warp 0), the layer's row of the lookup table, the pool's fill
 // count, the trace position and the victim candidates (warps 1-7).
-__device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t step) {
+__device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t step, PendingTable& pend,
+                                  int64_t po = 0) {
   __shared__ int s_idx[kMaxRanks];
   __shared__ float s_gate[kMaxRanks];
   __shared__ int s_need[kMaxRanks];   // needed global ids, ascending
@@ -199,13 +226,20 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   __shared__ int s_hand;
   __shared__ unsigned long long s_ckey[kFWarps][kMaxRanks];  // each warp's smallest candidate keys
   __shared__ int s_cslot[kFWarps][kMaxRanks];
+  // router-guided: the layer's logits and ranks, the refreshed keys of its residents that the step
+  // does not use (~0 otherwise), their nev smallest, and the candidates' keys
+  __shared__ float s_z[256];
+  __shared__ int s_rank[256];
+  __shared__ unsigned long long s_lkey[256];
+  __shared__ unsigned long long s_lsel[kMaxRanks];
+  __shared__ unsigned long long s_cand_key[kMaxRanks];
   const int k = a.k, E = a.E;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (warp == 0) {
     int my_i;
     float my_g;
-    warp_topk(a.z, E, k, a.renorm, lane, my_i, my_g);
+    warp_topk(a.z + (int64_t)l * E, E, k, a.renorm, lane, my_i, my_g);
     if (lane < k && (my_i < 0 || my_i >= E)) {
       atomicOr(a.err, FERR_BAD_ROUTE);
       my_i = lane;  // keep the step well-defined; the host reports the error
@@ -254,11 +288,16 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
       const int nc = (int)__ldcg(a.cand + kMaxRanks);
       if (lane == 0) s_ncand = nc;
       if (lane < nc) {
-        const int g = (int)(uint32_t)(__ldcg(a.cand + lane) & 0xffffffffull);
-        s_cand_gid[lane] = g;
-        s_cand_slot[lane] = a.slot_of[g];
+        const unsigned long long key = __ldcg(a.cand + lane);
+        const int g = slot_key_gid(key, a.policy);
+        const bool ok = g >= 0 && g < a.L * E;  // a free slot's key (~0) names no expert
+        s_cand_key[lane] = ok ? key : ~0ull;
+        s_cand_gid[lane] = ok ? g : -1;
+        s_cand_slot[lane] = ok ? a.slot_of[g] : -1;
       }
     }
+    if (a.policy == 2)
+      for (int e = threadIdx.x - 32; e < E; e += blockDim.x - 32) s_z[e] = __ldcg(a.z + (int64_t)l * E + e);
   }
   __syncthreads();
   if (threadIdx.x < k) {
@@ -270,10 +309,36 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
   __syncthreads();
   if (a.policy == 1) {
     if (threadIdx.x == 0) rotary_place(a, l, clock, k, E, s_need, s_miss, s_slot, s_evict, s_ps_e, s_ps_gid, s_win_gid,
-                                       s_win_prior, s_hand, s_nused);
+                                       s_win_prior, s_hand, s_nused, pend);
     __syncthreads();
   }
-  if (threadIdx.x == 0 && a.policy == 0) {
+  if (a.policy == 2) {
+    // Refresh the layer's ranks from this routing (rank = logits that beat the expert's, ties to the
+    // lower id, in the top-k's order), and the keys of its residents this step does not use; the
+    // used ones get their keys below, with this step's clock.
+    for (int e = threadIdx.x; e < E; e += blockDim.x) {
+      const uint32_t ke = ord_key(s_z[e]);
+      int rank = 0;
+      for (int j = 0; j < E; j++) {
+        const uint32_t kj = ord_key(s_z[j]);
+        rank += (kj > ke || (kj == ke && j < e)) ? 1 : 0;
+      }
+      s_rank[e] = rank;
+      a.rank[l * E + e] = rank;
+      const int g = l * E + e;
+      const int sl = s_slot_e[e];
+      bool used = false;
+      for (int t = 0; t < k; t++) used |= s_need[t] == g;
+      unsigned long long lk = ~0ull;
+      if (sl >= 0 && !used) {
+        lk = guided_key(E, rank, guided_key_last_use(__ldcg(a.slot_key + sl)), g);
+        a.slot_key[sl] = lk;
+      }
+      s_lkey[e] = lk;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && (a.policy == 0 || a.policy == 2)) {
     // misses in ascending id take free slots [n_used, cap) first
     int n_used = s_nused;
     int nev = 0;
@@ -286,25 +351,84 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     }
     if (n_used != s_nused) *a.n_used = n_used;
     s_nev = nev;
+    if (a.policy == 2) s_nev_found = 0;  // the guided merge below decides
     // Victims: the nev smallest slot keys (last use, id) among slots that hold no expert of this
     // step (every slot is occupied when eviction is needed). They are among the k smallest keys
     // of the pool (at most k - nev of those belong to this step's hits), which phase C of the
     // previous layer-step left in a.cand. s_nev_found < nev sends the phase to the full scan.
-    int j = 0;
-    for (int c = 0; c < s_ncand && j < nev; c++) {
-      const int g = s_cand_gid[c];
-      bool needed = false;
-      for (int t = 0; t < k; t++) needed |= (s_need[t] == g);
-      if (needed) continue;
-      s_vgid[j] = g;
-      s_vslot[j] = s_cand_slot[c];
-      j++;
+    if (a.policy == 0) {
+      int j = 0;
+      for (int c = 0; c < s_ncand && j < nev; c++) {
+        const int g = s_cand_gid[c];
+        if (g < 0) break;  // ascending keys: only free slots' keys follow
+        bool needed = false;
+        for (int t = 0; t < k; t++) needed |= (s_need[t] == g);
+        if (needed) continue;
+        s_vgid[j] = g;
+        s_vslot[j] = s_cand_slot[c];
+        j++;
+      }
+      s_nev_found = j;
     }
-    s_nev_found = j;
   }
   __syncthreads();
-  const int nev = a.policy == 0 ? s_nev : 0;
-  if (nev > 0 && s_nev_found < nev) {  // (LRU only: nev is 0 under the rotary policy)
+  const int nev = (a.policy == 0 || a.policy == 2) ? s_nev : 0;
+  if (a.policy == 2 && nev > 0) {
+    // Victims: the nev smallest keys among residents this step does not use. Only this layer's keys
+    // changed since phase C of the previous layer-step left the pool's k smallest keys in a.cand,
+    // so the candidates of other layers, ascending, are still the smallest keys of other layers;
+    // merge them with the nev smallest refreshed keys of this layer. Running out of candidates
+    // before nev victims sends the phase to the full scan.
+    if (warp == 0) {
+      unsigned long long lk[8];
+#pragma unroll
+      for (int q = 0; q < 8; q++) {
+        const int e = q * 32 + lane;
+        lk[q] = e < E ? s_lkey[e] : ~0ull;
+      }
+      for (int j = 0; j < nev; j++) {
+        unsigned long long best = ~0ull;
+        int bq = 0;
+#pragma unroll
+        for (int q = 0; q < 8; q++)
+          if (lk[q] < best) {
+            best = lk[q];
+            bq = q;
+          }
+        const unsigned long long wmin = shfl_min_u64(best);
+        const unsigned win = __ballot_sync(kFull, best == wmin && wmin != ~0ull);
+        if (win && lane == __ffs(win) - 1) {
+#pragma unroll
+          for (int q = 0; q < 8; q++)
+            if (q == bq) lk[q] = ~0ull;
+        }
+        if (lane == 0) s_lsel[j] = wmin;
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int c = 0, li = 0, j = 0;
+      for (; j < nev; j++) {
+        while (c < s_ncand && s_cand_gid[c] >= 0 && s_cand_gid[c] / E == l) c++;  // this layer's are stale
+        if (c >= s_ncand || s_cand_gid[c] < 0) break;  // other layers' next key unknown: full scan
+        const unsigned long long ck = s_cand_key[c];
+        const unsigned long long lk = s_lsel[li];
+        if (lk < ck) {
+          const int g = slot_key_gid(lk, 2);
+          s_vgid[j] = g;
+          s_vslot[j] = s_slot_e[g - l * E];
+          li++;
+        } else {
+          s_vgid[j] = s_cand_gid[c];
+          s_vslot[j] = s_cand_slot[c];
+          c++;
+        }
+      }
+      s_nev_found = j;
+    }
+    __syncthreads();
+  }
+  if (nev > 0 && s_nev_found < nev) {  // (LRU and router-guided: nev is 0 under the rotary policy)
     // Full scan: each warp finds the nev smallest of its slots, warp 0 takes the nev smallest of
     // those candidates.
     for (int j = 0; j < nev; j++) {
@@ -367,13 +491,13 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
         if (lane == 0) {
           if (!win) atomicOr(a.err, FERR_NO_VICTIM);
           s_vslot[j] = win ? vslot : -1;
-          s_vgid[j] = win ? (int)(uint32_t)(wmin & 0xffffffffull) : -1;
+          s_vgid[j] = win ? slot_key_gid(wmin, a.policy) : -1;
         }
       }
     }
     __syncthreads();
   }
-  if (threadIdx.x == 0 && a.policy == 0) {
+  if (threadIdx.x == 0 && (a.policy == 0 || a.policy == 2)) {
     int j = 0;
     unsigned long long hits = 0, misses = 0, evictions = 0;
     for (int t = 0; t < k; t++) {
@@ -388,16 +512,20 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
         const int v = s_vgid[j];
         j++;
         if (vs >= 0) {
-          a.slot_of[v] = -1;
+          pend.set(v, -1);
           s_slot[t] = vs;
           s_evict[t] = v;
           evictions++;
         }
       }
-      if (s_slot[t] >= 0) a.slot_of[g] = s_slot[t];
+      if (s_slot[t] >= 0) pend.set(g, s_slot[t]);
     }
-    for (int t = 0; t < k; t++)
-      if (s_slot[t] >= 0) a.slot_key[s_slot[t]] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)s_need[t];
+    for (int t = 0; t < k; t++) {
+      if (s_slot[t] < 0) continue;
+      a.slot_key[s_slot[t]] = a.policy == 2
+                                  ? guided_key(E, s_rank[s_need[t] - l * E], (uint32_t)clock, s_need[t])
+                                  : ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)s_need[t];
+    }
     atomicAdd(a.stats + STAT_HITS, hits);
     atomicAdd(a.stats + STAT_MISSES, misses);
     atomicAdd(a.stats + STAT_EVICTIONS, evictions);
@@ -422,10 +550,10 @@ __device__ void select_and_lookup(const FusedArgs& a, int l, int clock, int64_t 
     const int g = l * E + s_idx[t];
     int q = 0;
     while (s_need[q] != g) q++;
-    a.plan_slot[t] = s_slot[q] < 0 ? 0 : s_slot[q];
-    a.plan_gid[t] = g;
-    a.plan_miss[t] = s_miss[q];
-    a.plan_gate[t] = s_gate[t];
+    a.plan_slot[po + t] = s_slot[q] < 0 ? 0 : s_slot[q];
+    a.plan_gid[po + t] = g;
+    a.plan_miss[po + t] = s_miss[q];
+    a.plan_gate[po + t] = s_gate[t];
     a.route_idx[l * k + t] = s_idx[t];
     a.route_gate[l * k + t] = s_gate[t];
   }
@@ -448,7 +576,7 @@ __device__ __forceinline__ float scale_at(const uint16_t* p, bool from_host) {
 // u_r[i] = silu(W_g[i] . x) * (W_u[i] . x) with x staged in shared memory.
 template <int WD, int CH>
 __device__ __forceinline__ void gateup_row(const FusedArgs& a, const uint8_t* src, uint8_t* slot, bool from_host,
-                                           const uint8_t* xs, int r, int i, int lane) {
+                                           const uint8_t* xs, int r, int i, int lane, float* u = nullptr) {
   const int64_t rb = a.lay.row_bytes_gu;
   const int nch = (int)(rb / 16);
   const int G = a.d / 128;
@@ -508,13 +636,13 @@ __device__ __forceinline__ void gateup_row(const FusedArgs& a, const uint8_t* sr
   }
   ag = warp_sum(ag);
   au = warp_sum(au);
-  if (lane == 0) a.u[(int64_t)r * a.I + i] = ag / (1.0f + expf(-ag)) * au;
+  if (lane == 0) (u ? u : a.u)[(int64_t)r * a.I + i] = ag / (1.0f + expf(-ag)) * au;
 }
 
 // Stage the k u vectors ([k x I] fp32, rank-major) into shared memory, padded by 4 floats per
 // 32 so the 16-byte reads of a warp spread over all banks.
-__device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad) {
-  const float4* u4 = reinterpret_cast<const float4*>(a.u);
+__device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad, const float* u = nullptr) {
+  const float4* u4 = reinterpret_cast<const float4*>(u ? u : a.u);
   const int n4 = a.k * a.I / 4;
 #pragma unroll 4
   for (int q = threadIdx.x; q < n4; q += blockDim.x) {
@@ -530,7 +658,8 @@ __device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad)
 // the CTA stages u, so the HBM latency overlaps the staging.
 template <int WD, int CHD>
 __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, const float* pgate, int l, int gw,
-                           int W) {
+                           int W, const float* u = nullptr, bool cta_active = true) {
+  if (!cta_active) return;  // the same for every thread of the CTA
   constexpr int E = Tr<WD>::epc;
   constexpr int KR = 24 / CHD > 8 ? 8 : (24 / CHD < 1 ? 1 : 24 / CHD);
   const int lane = threadIdx.x & 31;
@@ -564,7 +693,7 @@ __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, cons
     }
   };
   issue(gw, 0);
-  stage_u(a, us, ipad);
+  stage_u(a, us, ipad, u);
   __syncthreads();
   for (int o = gw; o < a.d; o += W) {
     float acc = 0.f;
@@ -605,6 +734,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
   __shared__ int p_slot[kMaxRanks], p_gid[kMaxRanks], p_miss[kMaxRanks];
   __shared__ float p_gate[kMaxRanks];
   __shared__ int p_mr[kMaxRanks], p_hr[kMaxRanks], p_nm, p_nh;  // miss / hit ranks of this layer-step
+  __shared__ PendingTable pend;                                    // CTA 0: the step's held-back table writes
   const int asize = WD == WD_FP32 ? 4 : 2;
   const int xbytes = a.d * asize;
   uint8_t* xs = reinterpret_cast<uint8_t*>(smem4);
@@ -619,7 +749,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
   unsigned nbar = 0;  // grid barriers passed in this launch
   if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[a.L * 4] = gtimer();
 
-  for (int l = 0; l < a.L; l++) {
+  for (int l = a.l_begin; l < a.l_end; l++) {
     const int clock = (int)(step * a.L + l + 1);  // 0 is older than every step (preloaded experts)
     // ---- phase R: router logits. A warp's row loads (8 chunks per lane at a time) are issued
     // before the CTA stages h, so their latency overlaps the staging.
@@ -658,20 +788,38 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
           }
         }
         acc = warp_sum(acc);
-        if (lane == 0) a.z[gw] = acc;
+        if (lane == 0) a.z[(int64_t)l * a.E + gw] = acc;
       }
     }
     if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 0] = gtimer();
-    // ---- phase S: selection and lookup table (CTA 0)
-    if (blockIdx.x == 0) select_and_lookup(a, l, clock, step);
-    if (!grid_sync(a, nbar)) return;
-    if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 1] = gtimer();
-    if (threadIdx.x < a.k) {
-      p_slot[threadIdx.x] = __ldcg(a.plan_slot + threadIdx.x);
-      p_gid[threadIdx.x] = __ldcg(a.plan_gid + threadIdx.x);
-      p_miss[threadIdx.x] = __ldcg(a.plan_miss + threadIdx.x);
-      p_gate[threadIdx.x] = __ldcg(a.plan_gate + threadIdx.x);
+    // ---- selection, in every CTA: the same top-k as phase S computes, and hit or miss from the
+    // lookup table as it was before this step (phase S holds its table writes back until phase D,
+    // and a selected expert that is resident keeps its slot). Hits need nothing else from S.
+    if (threadIdx.x < 32) {
+      int my_i;
+      float my_g;
+      warp_topk(a.z + (int64_t)l * a.E, a.E, a.k, a.renorm, lane, my_i, my_g);
+      if (lane < a.k) {
+        if (my_i < 0 || my_i >= a.E) my_i = lane;  // as phase S does (it reports the error)
+        const int gid = l * a.E + my_i;
+        const int sl = __ldcg(a.slot_of + gid);
+        p_gid[lane] = gid;
+        p_gate[lane] = my_g;
+        p_miss[lane] = sl < 0;
+        p_slot[lane] = sl < 0 ? 0 : sl;  // a miss's slot comes with CTA 0's plan
+      }
+    }
+    // ---- phase S: the lookup-table step (CTA 0), then its plan is published to the miss CTAs
+    if (blockIdx.x == 0) {
+      if (threadIdx.x == 0) pend.n = 0;
+      select_and_lookup(a, l, clock, step, pend);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        __threadfence();
+        asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(a.plan_flag), "r"((unsigned)clock) : "memory");
+        if (a.phase_ts) a.phase_ts[l * 4 + 1] = gtimer();
+      }
     }
     __syncthreads();
     // ---- phase C: gate-up rows; miss CTAs stream the missed experts into their slots
@@ -702,13 +850,40 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
         asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
       }
     }
-    // With a full pool that can evict, CTA 0 finds the next layer-step's victim candidates
-    // instead of computing hit rows.
-    const bool cand_cta0 = a.may_evict && __ldcg(a.n_used) >= a.cap;
-    if (blockIdx.x == 0 && cand_cta0) find_victim_candidates(a);
+    // CTA 0 leads phase S and computes no hit rows; with a full pool that can evict it then finds
+    // the next layer-step's victim candidates.
+    if (blockIdx.x == 0 && a.may_evict && __ldcg(a.n_used) >= a.cap) find_victim_candidates(a);
     const int mctas = nm > 0 ? (a.miss_ctas < (int)gridDim.x - 2 ? a.miss_ctas : (int)gridDim.x - 2) : 0;
-    const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;  // the last CTAs (CTA 0 leads phase S)
+    const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;  // the last CTAs
+    bool plan_ok = true;
     if (miss_cta) {
+      // the misses' slots: wait (bounded) for CTA 0's plan of this layer-step
+      __shared__ int s_plan_ok;
+      if (threadIdx.x == 0) {
+        int ok = 1;
+        if ((int)(ld_acquire_u32(a.plan_flag) - (unsigned)clock) < 0) {
+          const uint64_t t0 = gtimer();
+          while ((int)(ld_acquire_u32(a.plan_flag) - (unsigned)clock) < 0) {
+            if (*(volatile int*)a.err & FERR_FATAL) {
+              ok = 0;
+              break;
+            }
+            if (gtimer() - t0 > a.barrier_timeout_ns) {
+              atomicOr(a.err, FERR_BARRIER_TIMEOUT);
+              ok = 0;
+              break;
+            }
+            __nanosleep(20);
+          }
+        }
+        s_plan_ok = ok;
+      }
+      __syncthreads();
+      plan_ok = s_plan_ok != 0;
+      if (plan_ok && threadIdx.x < a.k && p_miss[threadIdx.x]) p_slot[threadIdx.x] = __ldcg(a.plan_slot + threadIdx.x);
+      __syncthreads();
+    }
+    if (miss_cta && plan_ok) {
       const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
       const int MW = mctas * kFWarps;
       // gate/up rows of every missed expert: host -> slot, and u from the same registers
@@ -741,10 +916,9 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
         }
         for (; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
       }
-    } else if (!(cand_cta0 && blockIdx.x == 0)) {
-      const int c0 = cand_cta0 ? 1 : 0;
-      const int hw = ((int)blockIdx.x - c0) * kFWarps + (threadIdx.x >> 5);
-      const int HW = ((int)gridDim.x - mctas - c0) * kFWarps;
+    } else if (!miss_cta && blockIdx.x != 0) {
+      const int hw = ((int)blockIdx.x - 1) * kFWarps + (threadIdx.x >> 5);
+      const int HW = ((int)gridDim.x - mctas - 1) * kFWarps;
       // When this layer-step also streams misses over the host link, phase C leaves HBM mostly
       // idle: bring the hit experts' W_d regions into L2 meanwhile, so phase D reads them from L2.
       // (With every expert a hit the prefetches would compete with the gate/up rows instead.)
@@ -768,6 +942,11 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
     }
     if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 2] = gtimer();
+    // CTA 0's plan is visible to every CTA now: the misses' slots; CTA 0 applies the step's table
+    // writes (the next reader is the next layer-step, after two more barriers)
+    if (threadIdx.x < a.k && p_miss[threadIdx.x]) p_slot[threadIdx.x] = __ldcg(a.plan_slot + threadIdx.x);
+    if (blockIdx.x == 0 && threadIdx.x == 0) pend.apply(a);
+    __syncthreads();
     // ---- phase D: down rows + combine, every expert read from its slot
     switch (chd_need) {
       case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, gw, W); break;
@@ -781,7 +960,236 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
     if (!grid_sync(a, nbar)) return;
     if (a.phase_ts && blockIdx.x == 0 && threadIdx.x == 0) a.phase_ts[l * 4 + 3] = gtimer();
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
+  if (a.l_end == a.L && blockIdx.x == 0 && threadIdx.x == 0) *a.step = step + 1;
+}
+
+// Barrier among the worker CTAs (1 .. gridDim.x - 1) of the lookahead kernel, bounded like grid_sync.
+__device__ bool worker_sync(const FusedArgs& a, unsigned& nbar) {
+  __shared__ int s_abort;
+  __syncthreads();
+  nbar++;
+  if (threadIdx.x == 0) {
+    const unsigned target = a.wbar_base + nbar * (gridDim.x - 1);
+    __threadfence();
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a.wbar_count), "r"(1u) : "memory");
+    if ((int)(ld_acquire_u32(a.wbar_count) - target) < 0) {
+      const uint64_t t0 = gtimer();
+      while ((int)(ld_acquire_u32(a.wbar_count) - target) < 0) {
+        if (*(volatile int*)a.err & FERR_FATAL) break;
+        if (gtimer() - t0 > a.barrier_timeout_ns) {
+          atomicOr(a.err, FERR_BARRIER_TIMEOUT);
+          break;
+        }
+        __nanosleep(20);
+      }
+    }
+    s_abort = *(volatile int*)a.err & FERR_FATAL;
+  }
+  __syncthreads();
+  return s_abort == 0;
+}
+
+// Thread 0 waits (bounded) until the counter p has reached target (wrapping compare); false on a
+// timeout (sets FERR_BARRIER_TIMEOUT) or when another CTA has flagged a fatal error.
+__device__ bool wait_count(const FusedArgs& a, const unsigned* p, unsigned target) {
+  if ((int)(ld_acquire_u32(p) - target) >= 0) return true;
+  const uint64_t t0 = gtimer();
+  while ((int)(ld_acquire_u32(p) - target) < 0) {
+    if (*(volatile int*)a.err & FERR_FATAL) return false;
+    if (gtimer() - t0 > a.barrier_timeout_ns) {
+      atomicOr(a.err, FERR_BARRIER_TIMEOUT);
+      return false;
+    }
+    __nanosleep(20);
+  }
+  return true;
+}
+
+// Exact layer lookahead, batch 1, LRU. One launch per decode step:
+//   R   router logits of every layer (row l * E + e per warp, hidden read from global memory), then
+//       one grid barrier;
+//   CTA 0: the lookup step of layers 0 .. L-1 in order (the same calls, clocks, trace and table as
+//       the layer-by-layer kernel), layer m's plan going to plan[m][k] and plan_flag = its clock.
+//       A miss's bytes reach its slot during layer m's gate-up rows, after the workers' barrier of
+//       layer m - 1, while only layer m - 1's down rows may still read; with cap >= 2 k (checked
+//       by the host) LRU never gives a miss of layer m the slot of an expert layer m - 1 used, so
+//       CTA 0 may run any number of layers ahead;
+//   workers (CTAs 1 ..): per layer, wait for its plan, gate-up rows (the last miss_ctas workers
+//       stream the missed experts from the host tier into their slots), a barrier among the
+//       workers, then the down rows + combine on the workers that computed hits. No barrier
+//       follows the down rows: the next layer's gate-up rows (and the miss CTAs' streaming of its
+//       misses) start beside them, writing the other half of the layer-parity u buffer.
+template <int WD, int CH>
+__global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant__ FusedArgs a) {
+  extern __shared__ uint4 smem4[];
+  __shared__ int p_slot[kMaxRanks], p_gid[kMaxRanks], p_miss[kMaxRanks];
+  __shared__ float p_gate[kMaxRanks];
+  __shared__ int p_mr[kMaxRanks], p_hr[kMaxRanks], p_nm, p_nh;
+  __shared__ PendingTable pend;
+  __shared__ int s_ok;
+  const int asize = WD == WD_FP32 ? 4 : 2;
+  const int xbytes = a.d * asize;
+  uint8_t* xs = reinterpret_cast<uint8_t*>(smem4);
+  float* us = reinterpret_cast<float*>(xs + ((xbytes + 15) & ~15));
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * kFWarps + (threadIdx.x >> 5);
+  const int W = gridDim.x * kFWarps;
+  const int64_t step = *(volatile int64_t*)a.step;
+  const int nchr = xbytes / 16;
+  const int chd_need = (int)((a.lay.row_bytes_d / 16 + 31) / 32);
+  const int k = a.k;
+  unsigned nbar = 0, nwbar = 0;
+
+  // ---- phase R, every layer: one router row per warp at a time, h_l read through L2; RG chunks of
+  // the row and of h_l in flight per lane (the same per-lane order of chunks as k_fused, so the
+  // logits are bit-identical)
+  for (int row = gw; row < a.L * a.E; row += W) {
+    constexpr int RG = 8;
+    const int l = row / a.E;
+    const uint8_t* wr = a.routers + (int64_t)row * xbytes;
+    const uint8_t* hl = (const uint8_t*)a.hidden + (int64_t)l * xbytes;
+    float acc = 0.f;
+    for (int c0 = 0; c0 < nchr; c0 += 32 * RG) {
+      uint4 w[RG], h[RG];
+#pragma unroll
+      for (int j = 0; j < RG; j++) {
+        const int c = c0 + j * 32 + lane;
+        w[j] = c < nchr ? ld_stream(wr + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+        h[j] = c < nchr ? ld_cg(hl + (int64_t)c * 16) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int j = 0; j < RG; j++) {
+        const int c = c0 + j * 32 + lane;
+        if (c < nchr) {
+          if (WD == WD_FP32)
+            acc = dot_chunk<WD_FP32>(w[j], reinterpret_cast<const uint8_t*>(&h[j]), acc);
+          else
+            acc = dot_chunk<WD_BF16>(w[j], reinterpret_cast<const uint8_t*>(&h[j]), acc);
+        }
+      }
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) a.z[row] = acc;
+  }
+  if (!grid_sync(a, nbar)) return;
+
+  if (blockIdx.x == 0) {
+    // ---- the lookup steps, in layer order
+    for (int m = 0; m < a.L; m++) {
+      const int clock = (int)(step * a.L + m + 1);
+      if (threadIdx.x == 0) {
+        s_ok = (*(volatile int*)a.err & FERR_FATAL) == 0;
+        pend.n = 0;
+      }
+      __syncthreads();
+      if (!s_ok) return;
+      select_and_lookup(a, m, clock, step, pend, (int64_t)m * k);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        pend.apply(a);  // nothing else reads the table in this kernel
+        __threadfence();
+        asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(a.plan_flag), "r"((unsigned)clock) : "memory");
+      }
+      __syncthreads();
+      if (a.may_evict && __ldcg(a.n_used) >= a.cap) find_victim_candidates(a);
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) *a.step = step + 1;
+    return;
+  }
+
+  // ---- workers
+  const int wgw = ((int)blockIdx.x - 1) * kFWarps + (threadIdx.x >> 5);
+  for (int l = 0; l < a.L; l++) {
+    const int clock = (int)(step * a.L + l + 1);
+    float* u = a.u + (int64_t)(l & 1) * k * a.I;
+    __syncthreads();  // the previous layer's down rows are done with p_slot / p_gate in this CTA
+    if (threadIdx.x == 0) s_ok = wait_count(a, a.plan_flag, (unsigned)clock);
+    __syncthreads();
+    if (!s_ok) return;
+    if (threadIdx.x < k) {
+      const int64_t q = (int64_t)l * k + threadIdx.x;
+      p_slot[threadIdx.x] = __ldcg(a.plan_slot + q);
+      p_gid[threadIdx.x] = __ldcg(a.plan_gid + q);
+      p_miss[threadIdx.x] = __ldcg(a.plan_miss + q);
+      p_gate[threadIdx.x] = __ldcg(a.plan_gate + q);
+    }
+    stage16(reinterpret_cast<uint4*>(xs), (const uint8_t*)a.hidden + (int64_t)l * xbytes, xbytes, threadIdx.x,
+            blockDim.x);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int nm = 0, nh = 0;
+      for (int r = 0; r < k; r++) {
+        if (p_miss[r])
+          p_mr[nm++] = r;
+        else
+          p_hr[nh++] = r;
+      }
+      p_nm = nm;
+      p_nh = nh;
+    }
+    __syncthreads();
+    const int nm = p_nm, nh = p_nh;
+    const int workers = (int)gridDim.x - 1;
+    const int mctas = nm > 0 ? (a.miss_ctas < workers - 1 ? a.miss_ctas : workers - 1) : 0;
+    const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;
+    if (nm > 0 && a.touch_shift > 0) {
+      const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
+      const int64_t gt0 = ((int64_t)blockIdx.x - 1) * kFThreads + threadIdx.x;
+      const int64_t GT = (int64_t)workers * kFThreads;
+      for (int64_t q = gt0; q < (int64_t)nm * pages; q += GT) {
+        const int mi = (int)(q / pages);
+        const uint8_t* pa = a.arena + (int64_t)p_gid[p_mr[mi]] * a.slot_stride + ((q - (int64_t)mi * pages) << a.touch_shift);
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+      }
+    }
+    if (miss_cta) {
+      const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
+      const int MW = mctas * kFWarps;
+      for (int p = mw; p < nm * a.I; p += MW) {
+        const int r = p_mr[p / a.I];
+        const int i = p - (p / a.I) * a.I;
+        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
+        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride;
+        gateup_row<WD, CH>(a, src, slot, true, xs, r, i, lane, u);
+      }
+      const int64_t dbytes = a.lay.total - a.lay.d_off;
+      const int64_t nq = dbytes / 16;
+      const int mt = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFThreads + threadIdx.x;
+      const int MT = mctas * kFThreads;
+      for (int mi = 0; mi < nm; mi++) {
+        const int r = p_mr[mi];
+        uint8_t* dst = a.pool + (int64_t)p_slot[r] * a.slot_stride + a.lay.d_off;
+        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride + a.lay.d_off;
+        for (int64_t q = mt; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
+      }
+    } else {
+      const int hw = wgw;
+      const int HW = (workers - mctas) * kFWarps;
+      for (int p = hw; p < nh * a.I; p += HW) {
+        const int r = p_hr[p / a.I];
+        const int i = p - (p / a.I) * a.I;
+        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
+        gateup_row<WD, CH>(a, slot, slot, false, xs, r, i, lane, u);
+      }
+    }
+    if (!worker_sync(a, nwbar)) return;
+    // Down rows + combine on the hit workers only: the miss CTAs go straight on to the next
+    // layer's misses, so the host link stays busy. Their copies then overlap these down rows,
+    // which is safe because no miss of layer l + 1 takes the slot of an expert of layer l
+    // (cap >= 2 k).
+    const int HWW = (workers - mctas) * kFWarps;
+    const bool dact = !miss_cta;
+    switch (chd_need) {
+      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 5:
+      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+    }
+  }
 }
 
 size_t fused_smem(int wdtype, int d, int I, int k) {
@@ -864,6 +1272,39 @@ int pick_ch_f(int64_t rb) {
     }                                                              \
   } while (0)
 
+template <int WD, int CH>
+int grid_of_la(size_t smem) {
+  static int occ = -1;
+  static size_t occ_smem = 0;
+  if (occ < 0 || occ_smem != smem) {
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(k_fused_la<WD, CH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    int o = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, k_fused_la<WD, CH>, kFThreads, smem) != cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    occ = o;
+    occ_smem = smem;
+  }
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = sms * (occ < 2 ? occ : 2);
+  return grid >= 3 ? grid : 0;  // CTA 0 and at least two workers
+}
+
+template <int WD, int CH>
+cudaError_t run_fused_la(const FusedArgs& a, int grid, cudaStream_t s) {
+  const size_t smem = fused_smem(a.wdtype, a.d, a.I, a.k);
+  void* params[] = {(void*)&a};
+  return cudaLaunchCooperativeKernel((const void*)k_fused_la<WD, CH>, dim3(grid), dim3(kFThreads), params, smem, s);
+}
+
 int fused_grid(int wdtype, int d, int I, int k) {
   const BlobLayout lay = make_layout(wdtype, d, I);
   const int ch = pick_ch_f(lay.row_bytes_gu);
@@ -876,6 +1317,21 @@ int fused_grid(int wdtype, int d, int I, int k) {
 cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s) {
   const int ch = pick_ch_f(a.lay.row_bytes_gu);
   MOE_F_DISPATCH(run_fused, a.wdtype, ch, a, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+int fused_la_grid(int wdtype, int d, int I, int k) {
+  const BlobLayout lay = make_layout(wdtype, d, I);
+  const int ch = pick_ch_f(lay.row_bytes_gu);
+  const size_t smem = fused_smem(wdtype, d, I, k);
+  if (smem > 200 * 1024) return 0;
+  MOE_F_DISPATCH(grid_of_la, wdtype, ch, smem);
+  return 0;
+}
+
+cudaError_t launch_fused_la(const FusedArgs& a, int grid, cudaStream_t s) {
+  const int ch = pick_ch_f(a.lay.row_bytes_gu);
+  MOE_F_DISPATCH(run_fused_la, a.wdtype, ch, a, grid, s);
   return cudaErrorInvalidValue;
 }
 

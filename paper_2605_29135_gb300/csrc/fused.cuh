@@ -22,6 +22,9 @@ constexpr int FERR_FATAL = FERR_BARRIER_TIMEOUT | FERR_PIPE_TIMEOUT;
 
 struct FusedArgs {
   int L, E, k, d, I, renorm, wdtype;
+  int l_begin, l_end;          // layers [l_begin, l_end) run in this launch; the launch that ends at
+                               // layer L completes the decode step (a chained decoder launches one
+                               // layer at a time, each after the attention that produces its input)
   BlobLayout lay;
   int64_t slot_stride;
   int64_t cap;
@@ -32,11 +35,13 @@ struct FusedArgs {
   const uint8_t* arena;        // host tier (device-accessible address of page-locked host memory)
   // residency state (device): lookup table and recency
   int32_t* slot_of;            // [L*E], -1 if not resident
-  unsigned long long* slot_key;// [cap]: (last use << 32) | global id of the resident expert; ~0 if free
+  unsigned long long* slot_key;// [cap]: replacement key of the resident expert (smallest = first victim),
+                               // ~0 if free. LRU and rotary: (last use << 32) | global id. Router-guided:
+                               // guided_key(E, rank, last use, global id)
   int32_t* n_used;             // slots handed out so far; [n_used, cap) are free
   int64_t* step;               // decode steps completed (clock = step * L + layer)
   // per-layer scratch (device)
-  float* z;                    // [E] router logits
+  float* z;                    // [L][E] router logits of the current decode step
   int32_t* plan_slot;          // [k] slot of rank r
   int32_t* plan_gid;           // [k] global expert id of rank r
   int32_t* plan_miss;          // [k] 1 if rank r was a miss this layer-step
@@ -61,17 +66,49 @@ struct FusedArgs {
   // phase C (off the critical path) for the next layer-step's phase S; cand[kMaxRanks] holds how
   // many are valid (0: phase S scans every slot).
   unsigned long long* cand;    // [kMaxRanks + 1]
-  int may_evict;               // LRU with cap < experts in the stack (else no victim search is needed)
+  int may_evict;               // LRU or router-guided with cap < experts in the stack (else no victim
+                               // search is needed)
   // Rotary slot-group policy (policy == 1): each slot's previous occupant, its inverse, the hand.
-  int policy;                  // 0 LRU, 1 rotary
+  int policy;                  // 0 LRU, 1 rotary, 2 router-guided
   int32_t* prior;              // [cap]: global id last evicted from the slot, -1 none
   int32_t* prior_slot_of;      // [L*E]: the slot whose previous occupant is the id, -1 none
   int32_t* hand;               // [1]
+  // Router-guided policy (policy == 2): every expert's rank in its layer's latest routing
+  // (0 = highest logit, ties to the lower id; E before the layer's first routing).
+  int32_t* rank;               // [L*E]
+  unsigned* plan_flag;         // clock of the last layer-step whose plan CTA 0 has published (0: none)
+  // Exact layer lookahead (k_fused_la): the worker CTAs' barrier counter and its value at launch.
+  // The plan arrays then hold every layer's plan, [L][k].
+  unsigned* wbar_count;
+  unsigned wbar_base;
 };
+
+// Router-guided replacement key: the victim is the smallest key, i.e. the largest rank, then the
+// most recent use, then the lowest global id. Fields: E - rank (9 bits), ~last use (32 bits),
+// global id (23 bits; the host checks L * E < 2^23).
+constexpr int kGuidedGidBits = 23;
+__host__ __device__ __forceinline__ unsigned long long guided_key(int E, int rank, uint32_t last_use, int gid) {
+  return ((unsigned long long)(uint32_t)(E - rank) << 55) | ((unsigned long long)(0xffffffffu - last_use) << 23) |
+         (unsigned long long)(uint32_t)gid;
+}
+__host__ __device__ __forceinline__ uint32_t guided_key_last_use(unsigned long long key) {
+  return 0xffffffffu - (uint32_t)((key >> 23) & 0xffffffffull);
+}
+__host__ __device__ __forceinline__ int slot_key_gid(unsigned long long key, int policy) {
+  return policy == 2 ? (int)(key & ((1ull << kGuidedGidBits) - 1)) : (int)(uint32_t)(key & 0xffffffffull);
+}
 
 // Maximum co-resident CTAs for the fused kernel of this shape (0 if it cannot launch).
 int fused_grid(int wdtype, int d, int I, int k);
 cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s);
+
+// Exact layer lookahead at batch 1 under LRU (layers' inputs all given with the step): CTA 0 runs
+// the lookup steps of every layer in order while the other CTAs compute. Needs cap >= 2 k (or
+// every expert resident): then no miss takes the slot of an expert the previous layer-step used,
+// whose down rows may still be running when the miss's bytes arrive. Same decisions, trace and
+// outputs as k_fused.
+int fused_la_grid(int wdtype, int d, int I, int k);
+cudaError_t launch_fused_la(const FusedArgs& a, int grid, cudaStream_t s);
 
 // Batched decode step: B sequences per step, one cooperative kernel over all layers. Per layer
 // the needed experts are the union of every sequence's top k; each needed expert is read once
@@ -107,7 +144,7 @@ struct BatchArgs {
   int32_t* n_used;
   int64_t* step;
   // per-layer scratch
-  float* z;                    // [B][E]
+  float* z;                    // [L][Bmax][E] router logits of the current decode step
   int32_t* sel_e;              // [B*k] expert of pair p = b*k + r
   float* sel_g;                // [B*k] its gate
   int32_t* plan_n;             // [2] distinct experts needed this layer-step, and how many missed
@@ -134,6 +171,13 @@ struct BatchArgs {
   int touch_shift;             // log2 of the translation-warming touch stride (0: no touches)
   int tg_max;                  // pairs staged in shared memory at a time (batched_tg)
   int router_tb;               // sequences per router work item (batched_router_tb)
+  int policy;                  // 0 LRU, 1 rotary, 2 router-guided
+  int32_t* rank;               // [L*E] router-guided: rank in the layer's latest routing (best over the batch)
+  int32_t* rank_best;          // [E] router-guided scratch: this layer-step's best rank over the batch
+  // Rotary slot-group policy (policy == 1), as in FusedArgs
+  int32_t* prior;              // [cap]
+  int32_t* prior_slot_of;      // [n_gid]
+  int32_t* hand;               // [1]
 };
 
 // Pairs staged per group for this shape, and the co-resident grid (0: shape or cap unsupported).

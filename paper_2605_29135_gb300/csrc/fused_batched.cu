@@ -120,7 +120,7 @@ __device__ __forceinline__ void router_block(const BatchArgs& a, int l, int tb, 
       }
     }
     acc = warp_sum(acc);
-    if (lane == 0) a.z[(int64_t)(b0 + t) * a.E + e] = acc;
+    if (lane == 0) a.z[((int64_t)l * a.Bmax + b0 + t) * a.E + e] = acc;
     if (nchr > 32 * RG && t + 1 < nt) {  // back to the row's first part for the next vector
 #pragma unroll
       for (int j = 0; j < RG; j++) {
@@ -132,6 +132,81 @@ __device__ __forceinline__ void router_block(const BatchArgs& a, int l, int tb, 
 }
 
 // ---- phase S: union of the pairs' experts, one lookup-table step, trace and plan (CTA 0)
+// Rotary slot-group step for the misses of a batched layer-step (thread 0 of CTA 0): the rule of
+// the batch-1 kernel applied to the union of the batch's experts, misses in ascending id. A miss
+// returns to the slot it was last evicted from when that slot holds no expert of the step
+// (reverse rotation), else takes the first such slot at or after the hand, which moves past it
+// (forward rotation); the occupant is evicted and remembered as the slot's previous occupant, and
+// the placed expert stops being anyone's previous occupant. Up to E misses per step, so the slot
+// state is read and written in global memory as it goes rather than staged: the occupant of a slot
+// is the low half of its key (all ones: empty), and each placement writes its key at once.
+// needed(o): o belongs to layer l and has pairs this step (tot[o - l * E] > 0).
+__device__ void batched_rotary_place(const BatchArgs& a, int l, int clock, int n, const int* need_e,
+                                     const int* miss, const int* tot, int* slot_out, int* evict_out,
+                                     int* n_evicted) {
+  const int E = a.E;
+  const int64_t cap = a.cap;
+  auto occupant = [&](int64_t sl) {
+    const unsigned long long key = __ldcg(a.slot_key + sl);
+    return key == ~0ull ? -1 : (int)(uint32_t)(key & 0xffffffffull);
+  };
+  auto needed = [&](int o) { return o >= l * E && o < (l + 1) * E && tot[o - l * E] > 0; };
+  int hand = *(volatile int32_t*)a.hand;
+  int nused = *(volatile int32_t*)a.n_used;
+  int evicted = 0;
+  for (int q = 0; q < n; q++) {
+    if (!miss[q]) continue;
+    const int g = l * E + need_e[q];
+    int slot = -1, occ = -1;
+    int ps = __ldcg(a.prior_slot_of + g);
+    if (ps >= 0 && __ldcg(a.prior + ps) != g) ps = -1;  // the inverse entry is stale
+    if (ps >= 0) {
+      const int o = occupant(ps);
+      if (o < 0 || !needed(o)) {
+        slot = ps;
+        occ = o;
+      }
+    }
+    if (slot < 0) {
+      for (int64_t j = 0; j < cap; j++) {
+        const int64_t sl = (hand + j) % cap;
+        const int o = occupant(sl);
+        if (o < 0 || !needed(o)) {
+          slot = (int)sl;
+          occ = o;
+          break;
+        }
+      }
+      if (slot < 0) {
+        atomicOr(a.err, FERR_NO_VICTIM);
+        slot_out[q] = -1;
+        continue;
+      }
+      hand = (int)((slot + 1) % cap);
+    }
+    if (occ >= 0) {
+      a.slot_of[occ] = -1;
+      evicted++;
+    } else {
+      nused++;
+    }
+    if (ps >= 0) a.prior[ps] = -1;  // g is placed: no longer a previous occupant
+    const int u = __ldcg(a.prior + slot);  // the slot's previous occupant loses its return slot
+    if (u >= 0) a.prior_slot_of[u] = -1;
+    a.prior[slot] = occ;
+    if (occ >= 0) a.prior_slot_of[occ] = slot;
+    a.prior_slot_of[g] = -1;
+    a.slot_of[g] = slot;
+    a.slot_key[slot] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)g;
+    __threadfence_block();
+    slot_out[q] = slot;
+    evict_out[q] = occ;
+  }
+  *a.hand = hand;
+  *a.n_used = nused;
+  *n_evicted = evicted;
+}
+
 __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t step, unsigned long long* keys) {
   constexpr int kChunks = kMaxPairs / 32;
   __shared__ int s_sel[kMaxPairs];       // expert of pair p
@@ -150,13 +225,18 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   __shared__ int s_off[256];
   __shared__ int s_n, s_nm, s_nused0, s_nfree, s_nev, s_nevicted;
   __shared__ unsigned long long s_trace_base;
+  __shared__ int s_grank[256];           // router-guided: each expert's best rank over the batch
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int E = a.E, P = a.B * a.k;
   const int nchunks = (P + 31) / 32;
+  const bool guided = a.policy == 2;
 
   // every global read this step needs, issued together
   for (int p = tid; p < P; p += blockDim.x) s_sel[p] = __ldcg(a.sel_e + p);
-  for (int e = tid; e < E; e += blockDim.x) s_slot_e[e] = a.slot_of[l * E + e];
+  for (int e = tid; e < E; e += blockDim.x) {
+    s_slot_e[e] = a.slot_of[l * E + e];
+    if (guided) s_grank[e] = __ldcg(a.rank_best + e);
+  }
   if (tid == 0) {
     s_nused0 = *a.n_used;
     s_trace_base = *(volatile unsigned long long*)a.trace_n;
@@ -186,6 +266,16 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
     s_tot[e] = run;
   }
   __syncthreads();
+  if (guided) {
+    // the layer's ranks from this step's routing; its residents this step does not use get their
+    // refreshed keys before the victims are sorted below (the used ones get theirs with this clock)
+    for (int e = tid; e < E; e += blockDim.x) {
+      a.rank[l * E + e] = s_grank[e];
+      const int sl = s_slot_e[e];
+      if (sl >= 0 && s_tot[e] == 0)
+        a.slot_key[sl] = guided_key(E, s_grank[e], guided_key_last_use(__ldcg(a.slot_key + sl)), l * E + e);
+    }
+  }
   if (warp == 0) {
     // needed experts (at least one pair) ascending, with their slots; then the misses' ranks
     int base = 0;
@@ -218,7 +308,7 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
     if (lane == 0) {
       const int nfree = (int)(a.cap - s_nused0);
       const int take = nm < nfree ? nm : nfree;
-      *a.n_used = s_nused0 + take;
+      if (a.policy != 1) *a.n_used = s_nused0 + take;
       s_n = n;
       s_nm = nm;
       s_nfree = nfree;
@@ -227,7 +317,10 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   }
   __syncthreads();
   const int n = s_n, nm = s_nm, nfree = s_nfree, nev = s_nev;
-  if (nev > 0) {
+  if (a.policy == 1) {
+    if (tid == 0 && nm > 0) batched_rotary_place(a, l, clock, n, s_need, s_miss, s_tot, s_slot, s_evict, &s_nevicted);
+    __syncthreads();
+  } else if (nev > 0) {
     // Every slot is occupied. Sort the slot keys (last use << 32 | id) ascending, with the slots
     // of this step's hits pinned at the maximum: the first nev keys are the victims.
     int N2 = 1;
@@ -256,7 +349,7 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
   // place the misses: free slots first, then the victims in ascending key order
   for (int q = tid; q < n; q += blockDim.x) {
     s_pos[q] = s_miss[q] ? s_mbefore[q] : nm + (q - s_mbefore[q]);
-    if (!s_miss[q]) continue;
+    if (!s_miss[q] || a.policy == 1) continue;
     const int m = s_mbefore[q];
     int slot = -1;
     if (m < nfree) {
@@ -266,7 +359,7 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
       if (key == ~0ull) {
         atomicOr(a.err, FERR_NO_VICTIM);
       } else {
-        const int v = (int)(uint32_t)(key & 0xffffffffull);
+        const int v = slot_key_gid(key, a.policy);
         slot = a.slot_of[v];
         s_evict[q] = v;
         atomicAdd(&s_nevicted, 1);
@@ -312,7 +405,9 @@ __device__ void batched_select(const BatchArgs& a, int l, int clock, int64_t ste
       const int gid = l * E + s_need[q];
       const int sl = s_slot[q];
       if (s_miss[q] && sl >= 0) a.slot_of[gid] = sl;
-      if (sl >= 0) a.slot_key[sl] = ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)gid;
+      if (sl >= 0)
+        a.slot_key[sl] = guided ? guided_key(E, s_grank[s_need[q]], (uint32_t)clock, gid)
+                                : ((unsigned long long)(uint32_t)clock << 32) | (uint32_t)gid;
       if (base_rec + q < (unsigned long long)a.trace_cap) {
         TraceRec rec;
         rec.step = (int32_t)step;
@@ -576,6 +671,10 @@ __device__ void down_item(const BatchArgs& a, int pos, int oblk, float* us, int*
 
 // ---- phase R for all CTAs: items (block of a.router_tb sequences, block of 8 router rows)
 __device__ __forceinline__ void phase_router(const BatchArgs& a, int l, uint8_t* xs) {
+  // router-guided: phase T folds every sequence's ranks into rank_best (the previous layer-step's
+  // phase S has read it)
+  if (a.policy == 2 && blockIdx.x == 0)
+    for (int e = threadIdx.x; e < a.E; e += blockDim.x) a.rank_best[e] = a.E;
   const int rtb = a.router_tb;
   const int ntb = (a.B + rtb - 1) / rtb;
   const int neb = (a.E + kBWarps - 1) / kBWarps;
@@ -588,12 +687,49 @@ __device__ __forceinline__ void phase_router(const BatchArgs& a, int l, uint8_t*
   }
 }
 
+// Router-guided policy: every expert's rank in one sequence's routing (the logits that beat its own,
+// ties to the lower id, in the top-k's order), folded into the layer-step's best rank over the
+// batch. One warp; lane holds experts lane, lane + 32, ... (E <= 256).
+__device__ __forceinline__ void fold_ranks(const BatchArgs& a, const float* z, int lane) {
+  constexpr int PER = 8;
+  uint32_t key[PER];
+  int rank[PER];
+#pragma unroll
+  for (int q = 0; q < PER; q++) {
+    const int e = q * 32 + lane;
+    key[q] = e < a.E ? ord_key(__ldcg(z + e)) : 0u;
+    rank[q] = 0;
+  }
+#pragma unroll
+  for (int qj = 0; qj < PER; qj++) {
+    if (qj * 32 >= a.E) break;
+    for (int src = 0; src < 32; src++) {
+      const int j = qj * 32 + src;
+      const uint32_t kj = __shfl_sync(kFull, key[qj], src);
+      if (j < a.E) {
+#pragma unroll
+        for (int q = 0; q < PER; q++) {
+          const int e = q * 32 + lane;
+          rank[q] += (kj > key[q] || (kj == key[q] && j < e)) ? 1 : 0;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < PER; q++) {
+    const int e = q * 32 + lane;
+    if (e < a.E) atomicMin(a.rank_best + e, rank[q]);
+  }
+}
+
 // ---- phase T: one warp per sequence
 __device__ __forceinline__ void phase_topk(const BatchArgs& a, int l, int gw, int W, int lane) {
   for (int b = gw; b < a.B; b += W) {
     int my_i;
     float my_g;
-    warp_topk(a.z + (int64_t)b * a.E, a.E, a.k, a.renorm, lane, my_i, my_g);
+    const float* zb = a.z + ((int64_t)l * a.Bmax + b) * a.E;
+    warp_topk(zb, a.E, a.k, a.renorm, lane, my_i, my_g);
+    if (a.policy == 2) fold_ranks(a, zb, lane);
     if (lane < a.k) {
       if (my_i < 0 || my_i >= a.E) {
         atomicOr(a.err, FERR_BAD_ROUTE);

@@ -145,6 +145,8 @@ __global__ void __launch_bounds__(kRouterWarps * 32) k_router(const __grid_const
     a.out->idx[lane] = my_i;
     a.out->gate[lane] = ex / denom;
   }
+  if (a.want_z)
+    for (int e = lane; e < a.E; e += 32) a.out->z[e] = zs[e];
   __syncwarp();
   __threadfence_system();
   if (lane == 0) a.out->seq = a.seq;

@@ -54,6 +54,7 @@ struct DownArgs {
 struct RouteOut {
   int32_t idx[kMaxRanks];
   float gate[kMaxRanks];
+  float z[256];          // the logits, when RouterArgs::want_z (router-guided policy)
   volatile int64_t seq;  // written last, after a system-scope fence
 };
 
@@ -64,6 +65,7 @@ struct RouterArgs {
   int wdtype;         // WD_FP32 or WD_BF16
   RouteOut* out;      // device address of host-mapped memory
   int64_t seq;
+  int want_z;         // also publish the E logits
 };
 
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);

@@ -31,6 +31,7 @@
 #include "fused.cuh"
 #include "kernels.cuh"
 #include "moe.h"
+#include "moe_internal.h"
 #include "slot_table.h"
 
 namespace {
@@ -103,6 +104,7 @@ struct moe_handle {
   cudaStream_t copy_stream = nullptr;
   cudaStream_t host_stream = nullptr;
   std::vector<cudaEvent_t> copy_ev;
+  cudaEvent_t layer_ev[2] = {nullptr, nullptr};  // host schedule with lookahead: layer l's last kernel done
   void* hid_dev = nullptr;
   void* out_dev = nullptr;
   // residency state of the host-driven schedule
@@ -116,6 +118,8 @@ struct moe_handle {
   moe_stats stats{};
   std::vector<int32_t> last_idx;
   std::vector<float> last_gate;
+  std::vector<float> last_z;      // host schedule, router-guided: [L][E] logits of the last step
+  std::vector<int32_t> ranks;     // host schedule, router-guided: scratch [E]
   // profiling
   bool prof = false;
   std::vector<PendingTime> pending;
@@ -136,12 +140,17 @@ struct moe_handle {
   int tg_max = 0;
   int touch_shift = 12;
   unsigned bar_epoch = 0;  // grid-barrier counter value at the start of the next fused launch
+  bool lookahead_dev = false;  // device schedule with exact layer lookahead (k_fused_la) for whole steps
+  int fgrid_la = 0;
+  unsigned wbar_epoch = 0;     // its worker-barrier counter value at the start of the next launch
   const uint8_t* arena_dev = nullptr;
   int32_t* d_slot_of = nullptr;
   unsigned long long* d_slot_key = nullptr;
   unsigned long long* d_cand = nullptr;  // batch-1 kernel: victim candidates [kMaxRanks + 1]
   int32_t* d_prior = nullptr;            // rotary policy: previous occupant per slot [cap]
   int32_t* d_prior_slot_of = nullptr;    // rotary policy: its inverse [n_gid]
+  int32_t* d_rank = nullptr;             // router-guided policy: rank in the layer's latest routing [n_gid]
+  int32_t* d_rank_best = nullptr;        // router-guided, batched: the layer-step's best rank [256]
   int32_t* d_hand = nullptr;             // rotary policy: the hand [1]
   int32_t* d_n_used = nullptr;
   int64_t* d_step = nullptr;
@@ -223,9 +232,13 @@ std::string check_config(const moe_config* c) {
   if (c->schedule != MOE_SCHEDULE_DEVICE && c->schedule != MOE_SCHEDULE_HOST_COPY_ENGINE) return "unknown schedule";
   if (c->miss_ctas < 0) return "miss_ctas must be >= 0";
   if (c->batched_path != MOE_BATCHED_AUTO && c->batched_path != MOE_BATCHED_CUDA_CORES) return "unknown batched_path";
-  if (c->policy == MOE_POLICY_GUIDED) return "the router-guided policy is available in the residency planner only";
-  if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY) return "unknown policy";
-  if (c->policy == MOE_POLICY_ROTARY && c->max_batch != 1) return "the rotary policy runs at batch 1";
+  if (c->policy != MOE_POLICY_LRU && c->policy != MOE_POLICY_ROTARY && c->policy != MOE_POLICY_GUIDED)
+    return "unknown policy";
+  if (c->policy == MOE_POLICY_GUIDED && (int64_t)c->n_layers * c->n_experts >= (1LL << moe::kGuidedGidBits))
+    return "the router-guided policy needs n_layers * n_experts < 2^23";
+  if (c->lookahead != 0 && c->lookahead != 1) return "lookahead must be 0 or 1";
+  if (c->lookahead && c->schedule == MOE_SCHEDULE_DEVICE && (c->max_batch != 1 || c->policy != MOE_POLICY_LRU))
+    return "lookahead in the device schedule needs max_batch 1 and the LRU policy";
   return "";
 }
 
@@ -242,6 +255,10 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_cand, 0, sizeof(unsigned long long) * (moe::kMaxRanks + 1));
   cudaMemset(h->d_prior, 0xff, sizeof(int32_t) * h->cap);
   cudaMemset(h->d_prior_slot_of, 0xff, sizeof(int32_t) * h->n_gid);
+  {
+    const std::vector<int32_t> unrouted((size_t)h->n_gid, h->cfg.n_experts);  // rank E: not routed yet
+    cudaMemcpy(h->d_rank, unrouted.data(), sizeof(int32_t) * h->n_gid, cudaMemcpyHostToDevice);
+  }
   cudaMemset(h->d_hand, 0, sizeof(int32_t));
   cudaMemset(h->d_n_used, 0, sizeof(int32_t));
   cudaMemset(h->d_step, 0, sizeof(int64_t));
@@ -249,6 +266,7 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_stats, 0, sizeof(unsigned long long) * moe::STAT_N);
   cudaMemset(h->d_bar, 0, sizeof(unsigned) * 4);
   h->bar_epoch = 0;
+  h->wbar_epoch = 0;
   cudaMemset(h->d_err, 0, sizeof(int));
   cudaDeviceSynchronize();
   *h->h_err = 0;
@@ -348,6 +366,7 @@ moe_status launch_router(moe_handle* h, int32_t layer, const void* hidden_l, cud
   a.wdtype = h->cfg.wdtype == MOE_DTYPE_FP32 ? moe::WD_FP32 : moe::WD_BF16;
   a.out = h->route_dev;
   a.seq = ++h->route_seq;
+  a.want_z = h->cfg.policy == MOE_POLICY_GUIDED;
   ProfScope ps(h, s, PC_ROUTER, (int64_t)a.E * a.d * h->router_eb + (int64_t)a.d * h->asize);
   cudaError_t e = moe::launch_router(a, s);
   ps.done();
@@ -359,6 +378,7 @@ struct Need {
   int32_t gid;
   int32_t slot;
   bool miss;
+  int32_t evicted;  // global id the miss evicted, -1 if none
 };
 
 // One layer-step of the lookup table (rules in slot_table.h; needs in ascending gid). Fills each
@@ -374,6 +394,7 @@ moe_status residency_step(moe_handle* h, int32_t layer, std::vector<Need>& needs
     Need& n = needs[i];
     n.slot = d.slot;
     n.miss = d.kind == moe::SLOT_MISS;
+    n.evicted = d.evicted;
     if (n.miss) {
       h->stats.misses++;
       h->stats.miss_bytes += h->lay.total;
@@ -401,10 +422,12 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
   if (h->prof) harvest(h, false);
   h->last_idx.assign((size_t)L * k, -1);
   h->last_gate.assign((size_t)L * k, 0.f);
+  if (c.policy == MOE_POLICY_GUIDED) h->last_z.assign((size_t)L * E, 0.f);
   moe_status st = launch_router(h, 0, hidden, s);
   if (st != MOE_OK) return st;
   std::vector<Need> needs;
   std::vector<int32_t> rank_gid(k);
+  std::vector<int32_t> prev_needed;  // lookahead: the global ids layer l - 1 reads
   for (int32_t l = 0; l < L; l++) {
     const void* hid_l = (const uint8_t*)hidden + (int64_t)l * act_row;
     NvtxRange layer_range("layer", l);
@@ -424,11 +447,32 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       h->last_idx[(size_t)l * k + r] = e;
       h->last_gate[(size_t)l * k + r] = rgate[r];
       rank_gid[r] = l * E + e;
-      needs.push_back(Need{l * E + e, -1, false});
+      needs.push_back(Need{l * E + e, -1, false, -1});
     }
     std::sort(needs.begin(), needs.end(), [](const Need& a, const Need& b) { return a.gid < b.gid; });
+    if (c.policy == MOE_POLICY_GUIDED) {
+      // the layer's ranks from this routing: the logits that beat each expert's, ties to the
+      // lower id (the router's own order)
+      float* zl = h->last_z.data() + (size_t)l * E;
+      const volatile float* rz = h->route->z;
+      for (int32_t e = 0; e < E; e++) zl[e] = rz[e];
+      h->ranks.resize(E);
+      for (int32_t e = 0; e < E; e++) {
+        int32_t r = 0;
+        for (int32_t j = 0; j < E; j++) r += (zl[j] > zl[e] || (zl[j] == zl[e] && j < e)) ? 1 : 0;
+        h->ranks[e] = r;
+      }
+      h->table.set_ranks(l, h->ranks.data());
+    }
     for (size_t i = 1; i < needs.size(); i++)
       if (needs[i].gid == needs[i - 1].gid) return fail(h, MOE_ERR_INVALID, "router produced duplicate expert ids");
+    // Lookahead: layer l's routing is in host arrays now, so layer l + 1's router may overwrite the
+    // routing buffer. Launched here, it runs on the GPU before layer l's kernels enqueued below,
+    // and the next iteration issues layer l + 1's miss copies while layer l computes.
+    if (c.lookahead && l + 1 < L) {
+      st = launch_router(h, l + 1, (const uint8_t*)hidden + (int64_t)(l + 1) * act_row, s);
+      if (st != MOE_OK) return st;
+    }
     const int64_t clock = h->token_step * L + l + 1;  // 0 is older than every step (preloaded experts)
     {
       NvtxRange r("slot lookup", l);
@@ -438,8 +482,17 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
     h->stats.layer_steps++;
     // selective loads: misses in ascending gid on the copy stream
     int n_miss = 0;
+    bool waited_prev = false;
     for (auto& n : needs) {
       if (!n.miss) continue;
+      // Lookahead: layer l - 1's kernels may still be running. A victim they read is overwritten
+      // only after its last kernel (every layer before it has finished: layer l's router ran
+      // after it). With cap >= 2 x a layer-step's experts an LRU victim is never such an expert.
+      if (c.lookahead && !waited_prev && n.evicted >= 0 &&
+          std::find(prev_needed.begin(), prev_needed.end(), n.evicted) != prev_needed.end()) {
+        MOE_CK(h, cudaStreamWaitEvent(h->copy_stream, h->layer_ev[(l - 1) & 1], 0));
+        waited_prev = true;
+      }
       ProfScope ps(h, h->copy_stream, PC_COPY, h->lay.total);
       if (h->fault == MOE_FAULT_COPY_ERROR) {  // an armed copy fault: this copy "fails"
         h->fault = MOE_FAULT_NONE;
@@ -510,7 +563,11 @@ moe_status decode_impl(moe_handle* h, const void* hidden, void* out, cudaStream_
       ps.done();
       if (e != cudaSuccess) return cuda_fail(h, e, "down/combine launch");
     }
-    if (l + 1 < L) {
+    if (c.lookahead) {
+      MOE_CK(h, cudaEventRecord(h->layer_ev[l & 1], s));
+      prev_needed.clear();
+      for (auto& n : needs) prev_needed.push_back(n.gid);
+    } else if (l + 1 < L) {
       st = launch_router(h, l + 1, (const uint8_t*)hidden + (int64_t)(l + 1) * act_row, s);
       if (st != MOE_OK) return st;
     }
@@ -654,6 +711,12 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   a.touch_shift = h->touch_shift;
   a.tg_max = h->tg_max;
   a.router_tb = moe::batched_router_tb(c.wdtype, c.d, c.d_ff, h->batched_tc);
+  a.policy = c.policy;
+  a.rank = h->d_rank;
+  a.rank_best = h->d_rank_best;
+  a.prior = h->d_prior;
+  a.prior_slot_of = h->d_prior_slot_of;
+  a.hand = h->d_hand;
   a.map_gu = h->map_gu;
   a.map_d = h->map_d;
   a.map_x = h->map_x;
@@ -681,14 +744,17 @@ moe_status decode_batched(moe_handle* h, const void* hidden, void* out, int32_t 
   return MOE_OK;
 }
 
-moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
-  moe_status st = check_device_error(h, false);
-  if (st != MOE_OK) return st;
-  if (h->batched) return decode_batched(h, hidden, out, batch, s);
+// Layers [l0, l1) of a batch-1 decode step in one launch of the fused kernel; the launch that
+// reaches the last layer completes the step. Per-phase profiling covers whole-step launches only.
+moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, int32_t l0, int32_t l1,
+                                cudaStream_t s) {
   const moe_config& c = h->cfg;
   const int k = c.top_k;
+  const bool whole = l0 == 0 && l1 == c.n_layers;
   moe::FusedArgs a{};
   a.L = c.n_layers;
+  a.l_begin = l0;
+  a.l_end = l1;
   a.E = c.n_experts;
   a.k = k;
   a.d = c.d;
@@ -707,10 +773,12 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   a.slot_key = h->d_slot_key;
   a.cand = h->d_cand;
   a.policy = c.policy;
-  a.may_evict = h->cap < h->n_gid && c.policy == MOE_POLICY_LRU;
+  a.may_evict = h->cap < h->n_gid && c.policy != MOE_POLICY_ROTARY;
+  a.rank = h->d_rank;
   a.prior = h->d_prior;
   a.prior_slot_of = h->d_prior_slot_of;
   a.hand = h->d_hand;
+  a.plan_flag = h->d_bar + 1;  // cleared with the barrier counter
   a.n_used = h->d_n_used;
   a.step = h->d_step;
   a.z = h->d_z;
@@ -732,25 +800,69 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   arm_barrier_fault(h, a.bar_base, a.barrier_timeout_ns);
   a.miss_ctas = c.miss_ctas > 0 ? c.miss_ctas : kDefaultMissCtas;
   a.touch_shift = h->touch_shift;
-  a.phase_ts = phase_buffer(h);
+  // whole steps of a lookahead handle: every layer's plan at plan[l][k], one grid barrier per launch
+  const bool la = whole && h->lookahead_dev;
+  if (la) {
+    const int64_t Lk = (int64_t)c.n_layers * k;
+    a.plan_gid = h->d_plan + Lk;
+    a.plan_miss = h->d_plan + 2 * Lk;
+    a.wbar_count = h->d_bar + 2;
+    a.wbar_base = h->wbar_epoch;
+    a.may_evict = a.may_evict && c.policy == MOE_POLICY_LRU;
+  }
+  a.phase_ts = whole && !la ? phase_buffer(h) : nullptr;
   {
     ProfScope ps(h, s, PC_FUSED,
-                 (int64_t)c.n_layers * (k * h->lay.total + (int64_t)c.n_experts * c.d * h->router_eb));
-    cudaError_t e = moe::launch_fused(a, h->fgrid, s);
+                 (int64_t)(l1 - l0) * (k * h->lay.total + (int64_t)c.n_experts * c.d * h->router_eb));
+    cudaError_t e = la ? moe::launch_fused_la(a, h->fgrid_la, s) : moe::launch_fused(a, h->fgrid, s);
     ps.done();
     if (e != cudaSuccess) return cuda_fail(h, e, "fused decode step launch");
   }
   MOE_CK(h, cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, s));
   MOE_CK(h, cudaEventRecord(h->err_ev, s));
   h->err_pending = true;
-  h->steps_launched++;
-  h->bar_epoch += 4u * (unsigned)c.n_layers * (unsigned)h->fgrid;  // every CTA arrives at 4 barriers per layer
+  if (l1 == c.n_layers) h->steps_launched++;
+  if (la) {
+    h->bar_epoch += (unsigned)h->fgrid_la;  // one grid barrier (after the router phase)
+    h->wbar_epoch += (unsigned)c.n_layers * (unsigned)(h->fgrid_la - 1);  // one worker barrier per layer
+  } else {
+    h->bar_epoch += 3u * (unsigned)(l1 - l0) * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
+  }
   if (a.phase_ts) {
     // phase durations of this step (the copy waits for the step; profiling runs are not timed for overlap)
     static const int cls[4] = {PC_PH_R, PC_PH_S, PC_PH_C, PC_PH_D};
     return harvest_phases(h, a.phase_ts, 4, cls, s);
   }
   return MOE_OK;
+}
+
+moe_status check_registered(moe_handle* h) {
+  if (h->all_registered) return MOE_OK;
+  for (int32_t l = 0; l < h->cfg.n_layers; l++)
+    if (!h->router_set[l]) return fail(h, MOE_ERR_NOT_REGISTERED, "router of layer " + std::to_string(l) + " not set");
+  for (int64_t g = 0; g < h->n_gid; g++)
+    if (!h->registered[g])
+      return fail(h, MOE_ERR_NOT_REGISTERED, "expert " + std::to_string(g % h->cfg.n_experts) + " of layer " +
+                                                 std::to_string(g / h->cfg.n_experts) + " not registered");
+  h->all_registered = true;
+  return MOE_OK;
+}
+
+// The pool contents are unknown after a failed step: wait for the streams, empty the pool.
+void recover_after_failure(moe_handle* h, cudaStream_t s) {
+  std::string keep = h->err;
+  cudaStreamSynchronize(s);
+  cudaStreamSynchronize(h->copy_stream);
+  cudaGetLastError();
+  reset_state(h);
+  h->err = keep;
+}
+
+moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
+  moe_status st = check_device_error(h, false);
+  if (st != MOE_OK) return st;
+  if (h->batched) return decode_batched(h, hidden, out, batch, s);
+  return decode_device_layers(h, hidden, out, 0, h->cfg.n_layers, s);
 }
 
 // The driver's tensor-map encoder, looked up once per process (thread-safe static initialisation).
@@ -811,6 +923,8 @@ void free_all(moe_handle* h) {
   harvest(h, true);
   for (auto e : h->ev_pool) cudaEventDestroy(e);
   for (auto e : h->copy_ev) cudaEventDestroy(e);
+  for (auto e : h->layer_ev)
+    if (e) cudaEventDestroy(e);
   if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   if (h->host_stream) cudaStreamDestroy(h->host_stream);
   if (h->own_pool && h->pool) cudaFree(h->pool);
@@ -819,7 +933,8 @@ void free_all(moe_handle* h) {
   if (h->route) cudaFreeHost(h->route);
   if (h->u) cudaFree(h->u);
   for (void* p : {(void*)h->d_slot_of, (void*)h->d_slot_key, (void*)h->d_cand, (void*)h->d_prior,
-                  (void*)h->d_prior_slot_of, (void*)h->d_hand, (void*)h->d_n_used,
+                  (void*)h->d_prior_slot_of, (void*)h->d_rank, (void*)h->d_rank_best, (void*)h->d_hand,
+                  (void*)h->d_n_used,
                   (void*)h->d_step, (void*)h->d_z, (void*)h->d_plan, (void*)h->d_plan_gate, (void*)h->d_trace,
                   (void*)h->d_trace_n, (void*)h->d_route_idx, (void*)h->d_route_gate, (void*)h->d_stats,
                   (void*)h->d_bar, (void*)h->d_err, (void*)h->d_phase_ts, (void*)h->d_sel_e, (void*)h->d_y,
@@ -902,7 +1017,10 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   h->route->seq = 0;
   if (cudaHostGetDevicePointer((void**)&h->route_dev, (void*)h->route, 0) != cudaSuccess)
     return bail(MOE_ERR_CUDA, "mapped routing buffer has no device address");
-  if (cudaMalloc(&h->u, sizeof(float) * cfg->max_batch * cfg->top_k * cfg->d_ff) != cudaSuccess)
+  // u per rank; the device lookahead kernel keeps two layers' u (layer parity)
+  const int64_t u_sets = cfg->lookahead && cfg->schedule == MOE_SCHEDULE_DEVICE ? std::max(2, cfg->max_batch)
+                                                                                  : cfg->max_batch;
+  if (cudaMalloc(&h->u, sizeof(float) * u_sets * cfg->top_k * cfg->d_ff) != cudaSuccess)
     return bail(MOE_ERR_OOM, "u allocation failed");
   const int64_t act = (int64_t)cfg->n_layers * cfg->max_batch * cfg->d * h->asize;
   if (cudaMalloc(&h->hid_dev, act) != cudaSuccess || cudaMalloc(&h->out_dev, act) != cudaSuccess)
@@ -912,6 +1030,8 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
     return bail(MOE_ERR_CUDA, "stream creation failed");
   h->copy_ev.resize((size_t)cfg->top_k * cfg->max_batch, nullptr);
   for (auto& e : h->copy_ev)
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
+  for (auto& e : h->layer_ev)
     if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return bail(MOE_ERR_CUDA, "event creation failed");
   h->dev_mode = cfg->schedule == MOE_SCHEDULE_DEVICE;
   h->batched = h->dev_mode && cfg->max_batch > 1;
@@ -933,24 +1053,40 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   } else if (h->dev_mode) {
     h->fgrid = moe::fused_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
     if (h->fgrid <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the device-driven schedule");
+    if (cfg->lookahead) {
+      // a miss must never take the slot of an expert the previous layer-step used (its down rows
+      // may still be reading): LRU guarantees it from 2 k slots on
+      const int64_t need_cap = 2 * (int64_t)cfg->top_k;
+      if (h->cap < h->n_gid && h->cap < need_cap)
+        return bail(MOE_ERR_INVALID, "lookahead in the device schedule needs at least " + std::to_string(need_cap) +
+                                         " slots (or every expert resident)");
+      h->fgrid_la = moe::fused_la_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
+      if (h->fgrid_la <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the lookahead kernel");
+      h->lookahead_dev = true;
+    }
   }
   if (h->dev_mode) {
     if (cudaHostGetDevicePointer((void**)&h->arena_dev, h->arena, 0) != cudaSuccess)
       return bail(MOE_ERR_CUDA, "host arena has no device address");
     const int k = cfg->top_k;
     const int64_t pairs = (int64_t)cfg->max_batch * k;
-    const int64_t plan_ints = h->batched ? 2 + 5 * (int64_t)cfg->n_experts + pairs : 3 * (int64_t)k;
+    // batch 1: slot, gid, miss per rank, for one layer ([k]) or, with lookahead, for every layer ([L][k])
+    const int64_t plan_ranks = h->lookahead_dev ? (int64_t)k * cfg->n_layers : (int64_t)k;
+    const int64_t plan_ints = h->batched ? 2 + 5 * (int64_t)cfg->n_experts + pairs : 3 * plan_ranks;
     bool ok = cudaMalloc(&h->d_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
               cudaMalloc(&h->d_slot_key, sizeof(unsigned long long) * h->cap) == cudaSuccess &&
               cudaMalloc(&h->d_cand, sizeof(unsigned long long) * (moe::kMaxRanks + 1)) == cudaSuccess &&
               cudaMalloc(&h->d_prior, sizeof(int32_t) * h->cap) == cudaSuccess &&
               cudaMalloc(&h->d_prior_slot_of, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
+              cudaMalloc(&h->d_rank, sizeof(int32_t) * h->n_gid) == cudaSuccess &&
+              cudaMalloc(&h->d_rank_best, sizeof(int32_t) * 256) == cudaSuccess &&
               cudaMalloc(&h->d_hand, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_n_used, sizeof(int32_t)) == cudaSuccess &&
               cudaMalloc(&h->d_step, sizeof(int64_t)) == cudaSuccess &&
-              cudaMalloc(&h->d_z, sizeof(float) * 256 * cfg->max_batch) == cudaSuccess &&
+              cudaMalloc(&h->d_z, sizeof(float) * std::max<int64_t>(256 * (int64_t)cfg->max_batch,
+                                                                    h->n_gid * cfg->max_batch)) == cudaSuccess &&
               cudaMalloc(&h->d_plan, sizeof(int32_t) * plan_ints) == cudaSuccess &&
-              cudaMalloc(&h->d_plan_gate, sizeof(float) * pairs) == cudaSuccess &&
+              cudaMalloc(&h->d_plan_gate, sizeof(float) * std::max(pairs, plan_ranks)) == cudaSuccess &&
               (!h->batched || cudaMalloc(&h->d_sel_e, sizeof(int32_t) * pairs) == cudaSuccess) &&
               (!h->batched || cudaMalloc(&h->d_y, sizeof(float) * pairs * cfg->d) == cudaSuccess) &&
               cudaMalloc(&h->d_trace, sizeof(moe::TraceRec) * std::max<int64_t>(1, cfg->trace_capacity)) == cudaSuccess &&
@@ -1024,27 +1160,12 @@ moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t
   if (!hidden || !out) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
   if (batch < 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be in [1, max_batch]");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
-  if (!h->all_registered) {
-    for (int32_t l = 0; l < h->cfg.n_layers; l++)
-      if (!h->router_set[l]) return fail(h, MOE_ERR_NOT_REGISTERED, "router of layer " + std::to_string(l) + " not set");
-    for (int64_t g = 0; g < h->n_gid; g++)
-      if (!h->registered[g])
-        return fail(h, MOE_ERR_NOT_REGISTERED, "expert " + std::to_string(g % h->cfg.n_experts) + " of layer " +
-                                                   std::to_string(g / h->cfg.n_experts) + " not registered");
-    h->all_registered = true;
-  }
+  moe_status st = check_registered(h);
+  if (st != MOE_OK) return st;
   NvtxRange range(h->dev_mode ? "moe_decode_step (device schedule)" : "moe_decode_step (host schedule)");
-  moe_status st = h->dev_mode ? decode_device(h, hidden, out, batch, (cudaStream_t)stream)
-                              : decode_impl(h, hidden, out, (cudaStream_t)stream);
-  if (st != MOE_OK) {
-    // The pool contents are unknown after a failed step: wait for the streams, empty the pool.
-    std::string keep = h->err;
-    cudaStreamSynchronize((cudaStream_t)stream);
-    cudaStreamSynchronize(h->copy_stream);
-    cudaGetLastError();
-    reset_state(h);
-    h->err = keep;
-  }
+  st = h->dev_mode ? decode_device(h, hidden, out, batch, (cudaStream_t)stream)
+                   : decode_impl(h, hidden, out, (cudaStream_t)stream);
+  if (st != MOE_OK) recover_after_failure(h, (cudaStream_t)stream);
   return st;
 }
 
@@ -1106,6 +1227,24 @@ moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_
   if (n < (int64_t)h->last_idx.size()) return fail(h, MOE_ERR_INVALID, "routing buffer too small");
   if (idx) memcpy(idx, h->last_idx.data(), h->last_idx.size() * sizeof(int32_t));
   if (gate) memcpy(gate, h->last_gate.data(), h->last_gate.size() * sizeof(float));
+  return MOE_OK;
+}
+
+moe_status moe_get_last_logits(moe_handle* h, float* z, int64_t n) {
+  if (!h || !z) return MOE_ERR_INVALID;
+  const int64_t need = h->n_gid * h->cfg.max_batch;
+  if (n < need) return fail(h, MOE_ERR_INVALID, "buffer below n_layers * max_batch * n_experts");
+  if (!h->dev_mode) {
+    if (h->cfg.policy != MOE_POLICY_GUIDED)
+      return fail(h, MOE_ERR_INVALID, "the host schedule keeps router logits under the router-guided policy only");
+    std::fill(z, z + need, 0.f);
+    std::copy(h->last_z.begin(), h->last_z.end(), z);
+    return MOE_OK;
+  }
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  moe_status st = check_device_error(h, true);
+  if (st != MOE_OK) return st;
+  MOE_CK(h, cudaMemcpy(z, h->d_z, sizeof(float) * need, cudaMemcpyDeviceToHost));
   return MOE_OK;
 }
 
@@ -1173,6 +1312,12 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
   int32_t n_used = 0;
   MOE_CK(h, cudaMemcpy(slot_of.data(), h->d_slot_of, sizeof(int32_t) * h->n_gid, cudaMemcpyDeviceToHost));
   MOE_CK(h, cudaMemcpy(&n_used, h->d_n_used, sizeof n_used, cudaMemcpyDeviceToHost));
+  const bool guided = h->cfg.policy == MOE_POLICY_GUIDED;
+  std::vector<int32_t> rank;
+  if (guided) {
+    rank.resize(h->n_gid);
+    MOE_CK(h, cudaMemcpy(rank.data(), h->d_rank, sizeof(int32_t) * h->n_gid, cudaMemcpyDeviceToHost));
+  }
   int64_t loaded = 0;
   std::vector<unsigned long long> keys;
   std::vector<int32_t> kslots;
@@ -1182,7 +1327,8 @@ moe_status moe_preload(moe_handle* h, int64_t* n_loaded) {
     MOE_CK(h, cudaMemcpyAsync(h->pool + (int64_t)slot * h->slot_stride, h->arena + g * h->slot_stride, h->lay.total,
                               cudaMemcpyHostToDevice, h->copy_stream));
     slot_of[g] = slot;
-    keys.push_back((unsigned long long)(uint32_t)g);  // last use 0: older than every decode step
+    // last use 0: older than every decode step
+    keys.push_back(guided ? moe::guided_key(h->cfg.n_experts, rank[g], 0u, (int32_t)g) : (unsigned long long)(uint32_t)g);
     kslots.push_back(slot);
     loaded++;
   }
@@ -1245,3 +1391,40 @@ void moe_destroy(moe_handle* h) {
 }
 
 }  // extern "C"
+
+namespace moe {
+
+bool moe_shape(const moe_handle* h, MoeShape* out) {
+  if (!h || !out) return false;
+  const moe_config& c = h->cfg;
+  out->d = c.d;
+  out->n_layers = c.n_layers;
+  out->top_k = c.top_k;
+  out->n_experts = c.n_experts;
+  out->wdtype = c.wdtype;
+  out->adtype = c.adtype;
+  out->device = c.device;
+  out->device_batch1 = h->dev_mode && !h->batched && c.max_batch == 1;
+  return true;
+}
+
+moe_status moe_run_layer(moe_handle* h, const void* hidden, void* out, int32_t layer, cudaStream_t s) {
+  if (!h) return MOE_ERR_INVALID;
+  if (!h->dev_mode || h->batched) return fail(h, MOE_ERR_INVALID, "a chained decoder needs the batch-1 device schedule");
+  if (layer < 0 || layer >= h->cfg.n_layers) return fail(h, MOE_ERR_INVALID, "layer out of range");
+  MOE_CK(h, cudaSetDevice(h->cfg.device));
+  moe_status st = MOE_OK;
+  if (layer == 0) {
+    st = check_registered(h);
+    if (st != MOE_OK) return st;
+    st = check_device_error(h, false);
+    if (st != MOE_OK) return st;
+  }
+  st = decode_device_layers(h, hidden, out, layer, layer + 1, s);
+  if (st != MOE_OK) recover_after_failure(h, s);
+  return st;
+}
+
+const char* moe_error_text(const moe_handle* h) { return h ? h->err.c_str() : ""; }
+
+}  // namespace moe

@@ -99,3 +99,20 @@ def test_sample_units_walk_sequences_then_layers_then_tokens():
     assert u[0] == (0, 0, 0) and u[63] == (0, 0, 63) and u[64] == (0, 1, 0) and u[129] == (0, 2, 1)
     wl1 = synth.WORKLOADS["stack48_bf16"]
     assert bench.sample_units(wl1, 50)[-1] == (1, 1, 0)
+
+
+def test_decoder_reference_arm_prints_one_line_on_rank_zero(monkeypatch, capsys):
+    import argparse
+    import json
+
+    import synth
+
+    args = argparse.Namespace(warmup=3, steps=4, gpus=1, impl="reference")
+    monkeypatch.setenv("RANK", "1")
+    assert bench.run_decoder(args, synth.DECODERS["tiny_block_fp32"]) == 0
+    assert capsys.readouterr().out == ""
+    monkeypatch.setenv("RANK", "0")
+    assert bench.run_decoder(args, synth.DECODERS["tiny_block_fp32"]) == 0
+    line = json.loads(capsys.readouterr().out)
+    assert line["impl"] == "reference" and line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle"
+    assert line["config"]["workload"] == "tiny_block_fp32"

@@ -50,7 +50,10 @@ BAD = [
     (dict(miss_ctas=-1), "miss_ctas must be >= 0"),
     (dict(raw_batched_path=3), "unknown batched_path"),
     (dict(raw_policy=9), "unknown policy"),
-    (dict(policy="rotary", max_batch=4), "rotary policy runs at batch 1"),
+    (dict(policy="rotary", max_batch=4, schedule="host_copy_engine"), "max_batch above 1 needs the device schedule"),
+    (dict(raw_lookahead=2), "lookahead must be 0 or 1"),
+    (dict(lookahead=True, max_batch=4), "lookahead in the device schedule needs max_batch 1 and the LRU policy"),
+    (dict(lookahead=True, policy="rotary"), "lookahead in the device schedule needs max_batch 1 and the LRU policy"),
 ]
 
 

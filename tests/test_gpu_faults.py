@@ -41,15 +41,17 @@ def _expect_recovery(m, wl, hidden, cap):
     assert rel_l2_rows(out, np.stack([r.out for r in res])).max() <= TOL[wl.wdtype]
 
 
-@pytest.mark.parametrize("batch", [1, 4])
-def test_device_wait_that_runs_out_reports_timeout_and_recovers(P, batch):
+@pytest.mark.parametrize("batch,lookahead", [(1, False), (4, False), (1, True)])
+def test_device_wait_that_runs_out_reports_timeout_and_recovers(P, batch, lookahead):
+    # lookahead: the device schedule's lookahead kernel, whose router-phase barrier is the one
+    # that runs out; every CTA leaves it, so no worker waits for a plan that never comes
     import torch
 
     from paper_2605_29135_gb300.workload import create_for_workload
 
     wl = synth.WORKLOADS["tiny_fp32"].replace(n_layers=2, tokens=8, batch=batch)
     hidden = synth.hidden_all(wl)
-    m = create_for_workload(wl, cap_slots=8)
+    m = create_for_workload(wl, cap_slots=8, lookahead=lookahead)
     try:
         h = torch.from_numpy(hidden[0].view(np.float32)).cuda()
         o = torch.empty_like(h)

@@ -27,13 +27,19 @@ def P():
     return P
 
 
-SCHEDULES = ["device", "host_copy_engine"]
+# "host_lookahead": the host copy-engine schedule routing layer l + 1 while layer l computes; it
+# must give the same trace and outputs as the others
+SCHEDULES = ["device", "host_copy_engine", "host_lookahead"]
 _ORACLE_CACHE = {}
 
 
 def _create(wl, cap, schedule="device"):
     from paper_2605_29135_gb300.workload import create_for_workload
 
+    if schedule == "host_lookahead":
+        return create_for_workload(wl, cap_slots=cap, schedule="host_copy_engine", lookahead=True)
+    if schedule == "device_lookahead":
+        return create_for_workload(wl, cap_slots=cap, schedule="device", lookahead=True)
     return create_for_workload(wl, cap_slots=cap, schedule=schedule)
 
 
@@ -99,7 +105,8 @@ def test_cap_invariance_bit_exact_across_schedules(P, name):
     tokens = min(wl.tokens, 96)
     hidden = synth.hidden_all(wl, tokens)
     outs = []
-    for cap, schedule in ((wl.cap_slots, "device"), (wl.n_gid, "device"), (wl.cap_slots, "host_copy_engine")):
+    for cap, schedule in ((wl.cap_slots, "device"), (wl.n_gid, "device"), (wl.cap_slots, "host_copy_engine"),
+                          (wl.cap_slots, "host_lookahead")):
         m = _create(wl, cap, schedule)
         try:
             outs.append(run_gpu(m, hidden, wl.adtype)[0])
@@ -107,6 +114,7 @@ def test_cap_invariance_bit_exact_across_schedules(P, name):
             m.destroy()
     np.testing.assert_array_equal(outs[0], outs[1])
     np.testing.assert_array_equal(outs[0], outs[2])
+    np.testing.assert_array_equal(outs[0], outs[3])
 
 
 RAGGED = {
@@ -167,3 +175,54 @@ def test_preload_then_decode_matches_oracle(P, schedule, cap):
     assert rel_l2_rows(out, np.stack(ref)).max() <= TOL["fp32"]
     if cap >= wl.n_gid:
         assert (tr["kind"] == 0).all()
+
+
+# The device schedule with exact layer lookahead: one kernel routes every layer, CTA 0 then decides
+# the layers' lookups in order ahead of the compute (cap >= 2 * top_k, or every expert resident).
+# Same trace and outputs as the layer-by-layer kernel, bit for bit.
+LOOKAHEAD = {
+    "tiny3_fp32_cap4": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=4),
+    "tiny3_fp32_cap8": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=8),
+    "ragged_fp32": RAGGED["fp32"].replace(cap_slots=4),
+    "ragged_bf16": RAGGED["bf16"].replace(cap_slots=10),
+    "ragged_int4": RAGGED["int4"].replace(cap_slots=6),
+    "tiny3_fp32_resident": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=24),
+}
+
+
+@pytest.mark.parametrize("name", list(LOOKAHEAD))
+def test_device_lookahead_matches_oracle_and_the_layer_by_layer_kernel(P, name):
+    wl = LOOKAHEAD[name]
+    out, tr, _, _ = _parity(P, wl, wl.cap_slots, wl.tokens, schedule="device_lookahead")
+    if wl.cap_slots < wl.n_gid:
+        assert (tr["evicted"] >= 0).sum() > 0
+    out2, tr2, _, _ = _parity(P, wl, wl.cap_slots, wl.tokens, schedule="device")
+    np.testing.assert_array_equal(out, out2)
+    np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(tr2))
+
+
+@pytest.mark.parametrize("name", ["stack48_int4", "stack48_bf16"])
+def test_device_lookahead_stack48_2048_tokens(P, name):
+    wl = synth.WORKLOADS[name]
+    samples = [(t, l) for t in (0, 1023, 2047) for l in range(0, 48, 6)]
+    _, tr, _, _ = _parity(P, wl, wl.cap_slots, wl.tokens, samples=samples, threads=16, schedule="device_lookahead")
+    assert len(tr) == wl.tokens * wl.n_layers * wl.top_k
+
+
+def test_device_lookahead_preload_and_small_caps(P):
+    wl = LOOKAHEAD["tiny3_fp32_cap8"]
+    hidden = synth.hidden_all(wl)
+    m = _create(wl, 10, "device_lookahead")
+    try:
+        assert m.preload() == 10
+        out, idx, _ = run_gpu(m, hidden, wl.adtype)
+        tr = m.get_residency_trace()
+    finally:
+        m.destroy()
+    orc = oracle.Oracle.for_workload(wl, cap_slots=10)
+    orc.preload()
+    recs = [orc.decode_step(hidden[t], compute_out=False, forced_idx=idx[t]).records for t in range(wl.tokens)]
+    np.testing.assert_array_equal(trace_tuples(tr), trace_tuples(np.concatenate(recs)))
+    with pytest.raises(P.MoEError) as ei:
+        _create(wl, 3, "device_lookahead")  # below 2 * top_k = 4 slots
+    assert ei.value.status == -1 and "slots" in str(ei.value)

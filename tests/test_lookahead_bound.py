@@ -1,0 +1,70 @@
+"""The bound the device schedule's exact layer lookahead rests on, checked on the oracle's LRU.
+
+In that kernel CTA 0 decides the lookup of layer-step m ahead of the other CTAs, and the missed
+experts' bytes go into their slots during layer-step m's gate-up rows. At that moment every row of
+layer-steps before m - 1 has been read (a barrier separates them), but the down rows of m - 1 may
+still be reading. So the slot a miss takes must not hold an expert of layer-step m - 1. Under LRU
+with lower-id ties that holds whenever the pool has at least 2 k slots: the experts of m - 1 carry
+the newest timestamp apart from m's own, and at least k older residents remain for the at most k
+misses. Here the oracle's LRU checks the claim at the tightest cap on random routings (single
+sequence and batched unions, cold and preloaded pools), and shows that one slot fewer breaks it.
+"""
+import random
+
+import oracle
+
+
+def _victims_avoid_previous_step(L, E, k, cap, steps, seed, batch=1, preload=False):
+    """Run random layer-steps through the oracle's LRU; True if no miss evicted an expert that the
+    layer-step just before it used."""
+    rng = random.Random(seed)
+    tbl = oracle.LRUTable(L * E, cap, E)
+    if preload:
+        tbl.preload()
+    clock = 0
+    prev = set()
+    for t in range(steps):
+        for l in range(L):
+            needed = set()
+            for _ in range(batch):
+                needed.update(l * E + e for e in rng.sample(range(E), k))
+            for r in tbl.step(clock, sorted(needed), t):
+                if r["evicted"] >= 0 and int(r["evicted"]) in prev:
+                    return False
+            prev = needed
+            clock += 1
+    return True
+
+
+def test_no_victim_from_the_previous_layer_step_at_the_tightest_cap():
+    checked = 0
+    for seed in range(80):
+        rng = random.Random(1000 + seed)
+        L, E = rng.randint(1, 6), rng.randint(4, 24)
+        k = rng.randint(1, min(8, E // 2))
+        cap = 2 * k
+        if cap >= L * E:
+            continue
+        checked += 1
+        assert _victims_avoid_previous_step(L, E, k, cap, steps=12, seed=seed, preload=seed % 2 == 0), seed
+    assert checked > 50
+
+
+def test_batched_unions_need_the_bound_on_distinct_experts():
+    # with a batch, k is replaced by the most distinct experts one layer-step can need
+    for seed in range(30):
+        rng = random.Random(2000 + seed)
+        L, E, k, B = rng.randint(1, 4), rng.randint(8, 20), rng.randint(1, 3), rng.randint(2, 3)
+        cap = 2 * min(E, k * B)
+        if cap >= L * E:
+            continue
+        assert _victims_avoid_previous_step(L, E, k, cap, steps=10, seed=seed, batch=B), seed
+
+
+def test_one_slot_fewer_can_evict_from_the_previous_layer_step():
+    broken = 0
+    for seed in range(100):
+        rng = random.Random(3000 + seed)
+        k = rng.randint(2, 4)
+        broken += not _victims_avoid_previous_step(3, 16, k, 2 * k - 1, steps=10, seed=seed)
+    assert broken > 0
