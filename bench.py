@@ -29,6 +29,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 2**20  # GB300 L2
 SMI_FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
               "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
               "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
@@ -151,42 +152,49 @@ def host_tier_fits(need_bytes_per_replica: float, replicas_per_host: int, availa
     return not available_bytes or need_bytes_per_replica * replicas_per_host <= 0.9 * available_bytes
 
 
-def oracle_cpu_baseline(wl, hidden, budget_s: float = 15.0):
-    """Time the fp64 oracle (as it stands) decoding whole tokens of the workload on the host cores.
-
-    The host tier of the oracle is the seeded generator; experts needed by the sampled tokens are
-    generated before the clock starts, so only the oracle's own work (routing, residency, slot
-    copies, expert FFN, combine) is timed. A batch of several sequences is sampled per (layer,
-    sequence) instead (one decode step of the batch would take minutes)."""
+def oracle_token_times(wl, hidden, n_tokens, budget_s=None):
+    """Seconds the fp64 oracle (as it stands) takes for each of the first n_tokens decode tokens of
+    a batch-1 workload, from a cold pool: every layer's routing, residency step with its slot
+    copies, expert FFN and combine, on the host cores. The oracle's host tier is the seeded
+    generator; the experts a token routes to are generated before that token's clock starts (an
+    untimed routing pass finds them), so only the oracle's own work is timed. Stops early once the
+    timed seconds pass budget_s."""
     import oracle
     import synth
     from concurrent.futures import ThreadPoolExecutor
 
-    if wl.batch > 1:
-        return oracle_layer_sample(wl, hidden, budget_s)
-
     routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
     probe = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers)
-    max_tok = 12  # ~1 s per token on 16 cores: a sample of ~10 s
-    need = set()
-    for t in range(max_tok):
-        r = probe.decode_step(hidden[t], compute_out=False)
-        for l in range(wl.n_layers):
-            need.update((l, int(e)) for e in r.idx[l, 0])
-    with ThreadPoolExecutor(max_workers=os.cpu_count()) as ex:
-        cache = dict(zip(sorted(need), ex.map(lambda le: synth.expert_weights(wl, *le), sorted(need))))
+    cache = {}
     orc = oracle.Oracle.for_workload(wl, routers=routers, experts=lambda l, e: cache[(l, e)])
-    t0 = time.perf_counter()
-    done = 0
-    while done < max_tok:
-        orc.decode_step(hidden[done])
-        done += 1
-        if time.perf_counter() - t0 > budget_s:
-            break
-    dt = time.perf_counter() - t0
-    return {"value": done / dt, "unit": "tok/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{done} whole decode token(s) of {wl.name} ({wl.n_layers} layers, cap {wl.cap_slots}), "
-                      f"cold pool, fp64, {dt:.1f} s"}
+    times = []
+    with ThreadPoolExecutor(max_workers=os.cpu_count()) as ex:
+        for t in range(n_tokens):
+            r = probe.decode_step(hidden[t], compute_out=False)
+            need = sorted({(l, int(e)) for l in range(wl.n_layers) for e in r.idx[l].ravel()})
+            for key in [key for key in cache if key not in set(need)]:
+                del cache[key]
+            new = [le for le in need if le not in cache]
+            cache.update(zip(new, ex.map(lambda le: synth.expert_weights(wl, *le), new)))
+            t0 = time.perf_counter()
+            orc.decode_step(hidden[t])
+            times.append(time.perf_counter() - t0)
+            if budget_s is not None and sum(times) > budget_s:
+                break
+    return times
+
+
+def oracle_cpu_baseline(wl, hidden, budget_s: float = 15.0):
+    """The fp64 oracle timed on a bounded sample of the workload (see oracle_token_times). A batch
+    of several sequences is sampled per (layer, sequence) instead (one decode step of the batch
+    would take minutes)."""
+    if wl.batch > 1:
+        return oracle_layer_sample(wl, hidden, budget_s)
+    times = oracle_token_times(wl, hidden, 32, budget_s)
+    dt = sum(times)
+    return {"value": len(times) / dt, "unit": "tok/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"the first {len(times)} whole decode tokens of {wl.name} ({wl.n_layers} layers, cap "
+                      f"{wl.cap_slots}), cold pool, fp64, {dt:.1f} s timed"}
 
 
 def sample_units(wl, n_units):
@@ -331,38 +339,65 @@ def resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, de
             "misses_in_window": s1["misses"] - s0["misses"], "phase_us_per_layer": phases}
 
 
-def run_reference(args, wl):
-    """The reference arm: the fp64 oracle on the host cores, one step = one layer of one token."""
-    import oracle
+def workload_config(wl, args, world: int) -> dict:
+    """The line's config object, built from the workload and the options only (never from a
+    measurement), so that both arms print the same dict."""
     import synth
-    from concurrent.futures import ThreadPoolExecutor
 
+    eb = synth.expert_bytes(wl.d, wl.d_ff, wl.wdtype)
+    return {"workload": wl.name, "layers": wl.n_layers, "d": wl.d, "experts_per_layer": wl.n_experts,
+            "top_k": wl.top_k, "d_ff": wl.d_ff, "weights": wl.wdtype, "cap_slots": wl.cap_slots,
+            "cap_bytes": wl.cap_slots * eb, "host_tier_bytes": wl.n_gid * eb, "batch": wl.batch,
+            "parallelism": "replicas" if world > 1 else "single GPU", "schedule": args.schedule,
+            "miss_ctas": args.miss_ctas or "default",
+            "batched_path": args.batched_path if wl.batch > 1 else None, "policy": args.policy,
+            "lookahead": args.lookahead,
+            "l2": (f"inputs larger than L2 ({wl.cap_slots * eb / 1e9:.1f} GB pool; every step reads at least "
+                   f"{wl.n_layers * wl.top_k * eb / 1e9:.1f} GB of expert weights)")
+                  if wl.n_layers * wl.top_k * eb > L2_BYTES else "inputs fit in L2 (a correctness-sized case)"}
+
+
+def run_reference(args, wl):
+    """The reference arm: the fp64 oracle on the host cores, on the GPU arm's workload, metric and
+    config. At batch 1 one step is one decode token through every layer, from a cold pool, as on
+    the GPU; a batch of several sequences is timed per (layer, sequence) unit and scaled."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    L = wl.n_layers
-    n_ls = args.warmup + args.steps
-    units = sample_units(wl, n_ls)
-    hidden = synth.hidden_all(wl, units[-1][0] + 1)
-    run = layer_oracle(wl, hidden, units)
-    for u in units[:args.warmup]:
-        run(u)
-    t0 = time.perf_counter()
-    for u in units[args.warmup:]:
-        run(u)
-    dt = time.perf_counter() - t0
-    tok_s = args.steps / L / dt
+    import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if wl.batch == 1:
+        hidden = synth.hidden_all(wl, args.warmup + args.steps)
+        times = oracle_token_times(wl, hidden, args.warmup + args.steps)[args.warmup:]
+        dt = sum(times)
+        tok_s = args.steps / dt
+        sample = (f"decode tokens {args.warmup}..{args.warmup + args.steps - 1} of {wl.name} after {args.warmup} "
+                  f"untimed ones, all {wl.n_layers} layers each, from a cold pool (slot copies kept), fp64; "
+                  f"each token's experts generated before its clock starts")
+        step = "one decode token through every layer, as on the GPU arm"
+    else:
+        n_ls = args.warmup + args.steps
+        units = sample_units(wl, n_ls)
+        hidden = synth.hidden_all(wl, units[-1][0] + 1)
+        run = layer_oracle(wl, hidden, units)
+        for u in units[:args.warmup]:
+            run(u)
+        t0 = time.perf_counter()
+        for u in units[args.warmup:]:
+            run(u)
+        dt = time.perf_counter() - t0
+        tok_s = args.steps / wl.n_layers / dt
+        sample = (f"{args.steps} (layer, sequence) units of {wl.name} in decode order, each layer's expert FFN read "
+                  f"from the host tier (residency does not change outputs); tok/s = units / layers / s")
+        step = "one layer of one sequence's token (a whole batch-64 step takes minutes on the host)"
     line = {"metric": "MoE decode tok/s at batch 1 under 6 GB expert cap; expert-path HBM GB/s vs peak", "value": tok_s,
             "unit": "tok/s", "impl": "reference", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f64", "data": "synthetic (seeded)",
-            "config": {"workload": wl.name, "layers": L, "d": wl.d, "experts": wl.n_experts, "top_k": wl.top_k,
-                       "d_ff": wl.d_ff, "cap_slots": wl.cap_slots, "batch": wl.batch,
-                       "step": "one layer of one sequence's token (router, top-k expert FFN, combine)"},
+            "dtype": "f64", "data": "synthetic (seeded: N(0, 1/sqrt(fan_in)) weights, AR(1) hidden streams)",
+            "config": workload_config(wl, args, world), "step": step,
             "cpu_baseline": {"value": tok_s, "unit": "tok/s", "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": f"{args.steps} (layer, sequence) units (= {args.steps / L:.2f} tokens) of "
-                                       f"{wl.name} in decode order, each layer's expert FFN read from the host tier "
-                                       "(residency does not change outputs)"},
+                             "sample": sample},
             "e2e": {"value": tok_s, "unit": "tok/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -688,15 +723,7 @@ def main():
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": {"fp32": "f32", "bf16": "bf16", "int4": "int4 weights, bf16 activations, f32 accumulation"}[wl.wdtype],
         "data": "synthetic (seeded: N(0, 1/sqrt(fan_in)) weights, AR(1) hidden streams)",
-        "config": {"workload": wl.name, "layers": wl.n_layers, "d": wl.d, "experts_per_layer": wl.n_experts,
-                   "top_k": wl.top_k, "d_ff": wl.d_ff, "weights": wl.wdtype, "cap_slots": wl.cap_slots,
-                   "cap_bytes": wl.cap_slots * eb, "host_tier_bytes": wl.n_gid * eb, "batch": wl.batch,
-                   "parallelism": "replicas" if world > 1 else "single GPU", "schedule": args.schedule,
-                   "miss_ctas": args.miss_ctas or "default",
-                   "batched_path": args.batched_path if wl.batch > 1 else None, "policy": args.policy,
-                   "lookahead": args.lookahead,
-                   "l2": f"inputs larger than L2 ({wl.cap_slots * eb / 1e9:.1f} GB pool, "
-                         f"{hbm_bytes_step / 1e9:.1f} GB of expert weights read per step)"},
+        "config": workload_config(wl, args, world),
         "step_roofline": {"bound": "h2d" if t_h2d >= t_hbm else "hbm", "t_star_ms": t_star * 1e3,
                           "frac": t_star * 1e3 / ms_step, "hbm_bytes_per_step": hbm_bytes_step,
                           "miss_bytes_per_step": miss_bytes_step, "h2d_peak_gbs": h2d_gbs,

@@ -176,18 +176,23 @@ int64_t moe_expert_bytes(const moe_config* cfg);
 /* Bytes the device expert pool needs for cfg (slots * 256-B aligned slot stride), or < 0 if cfg is invalid. */
 int64_t moe_pool_bytes(const moe_config* cfg);
 
-/* Validate cfg, allocate the device pool (unless cfg->device_pool is given), the pinned host
+/* Paper: the fixed slot group and its capacity (Sec. "Rotary GPU Concept", Fig. 1 "Rotary Slot
+ * Group"); the capacity error is the clean form of the start-up failure of Sec. "Failure Analysis".
+ * Validate cfg, allocate the device pool (unless cfg->device_pool is given), the pinned host
  * arena for all n_layers * n_experts experts, router storage and work buffers.
  * MOE_ERR_CAPACITY if the slot count is below min(E, k * max_batch), the most distinct experts
  * one layer-step can need (a clean failure instead of a start-up that cannot run).
  * On failure *out is NULL and nothing stays allocated. */
 moe_status moe_create(const moe_config* cfg, moe_handle** out);
 
-/* Router weights of one layer: W_r [E x d] row-major, host memory, fp32 when wdtype is FP32,
+/* Paper: the router whose output is Fig. 1's "Routing Result" (Sec. "Rotary GPU Concept").
+ * Router weights of one layer: W_r [E x d] row-major, host memory, fp32 when wdtype is FP32,
  * else bf16. Copied to device memory (routers are always resident, outside the slot cap). */
 moe_status moe_set_router(moe_handle* h, int32_t layer, const void* w_r);
 
-/* One expert's weights into the pinned host tier (the paper's host memory tier). Row-major,
+/* Paper: Fig. 1 "Host Memory / Storage Tier", the full weights kept outside the accelerator
+ * (Sec. "Rotary GPU Concept").
+ * One expert's weights into the pinned host tier (the paper's host memory tier). Row-major,
  * out x in: w_gate [I x d], w_up [I x d], w_down [d x I].
  *   FP32/BF16: elements of that type.
  *   INT4_G128: packed nibbles, byte j of a row = element 2j (low nibble) and 2j+1 (high),
@@ -198,9 +203,12 @@ moe_status moe_set_router(moe_handle* h, int32_t layer, const void* w_r);
 moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t expert, const void* w_gate,
                                      const void* w_up, const void* w_down, const void* scales);
 
-/* One decode step over all layers for `batch` sequences (1 <= batch <= max_batch; MOE_ERR_INVALID
+/* Paper: Fig. 1's cycle, routing result -> lookup table -> selective load into slots / evict
+ * (Sec. "Rotary GPU Concept"), run once per layer of a decode step.
+ * One decode step over all layers for `batch` sequences (1 <= batch <= max_batch; MOE_ERR_INVALID
  * otherwise). hidden: device [n_layers x batch x d] (adtype), the input of every layer; out:
- * device [n_layers x batch x d] (adtype). Work is ordered on `stream`
+ * device [n_layers x batch x d] (adtype); both 16-byte aligned (MOE_ERR_INVALID otherwise, before
+ * any launch). Work is ordered on `stream`
  * (a cudaStream_t; NULL = legacy default stream). hidden must stay valid and out must not be
  * read until `stream` reaches the end of the step. Calls on one handle must use one stream or
  * be serialised by the caller.
@@ -215,20 +223,27 @@ moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t exper
  * returned. */
 moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t batch, void* stream);
 
-/* moe_decode_step on host buffers (pinned or pageable): copies hidden to the device, runs the
+/* Paper: as moe_decode_step (Fig. 1), with the step's activations in host memory.
+ * moe_decode_step on host buffers (pinned or pageable): copies hidden to the device, runs the
  * step on an internal stream, copies out back and waits for completion. */
 moe_status moe_decode_step_host(moe_handle* h, const void* hidden_host, void* out_host, int32_t batch);
 
-/* Copy residency records [start, start + cap) of the trace into buf. *n_copied = records copied,
+/* Paper: the history of Fig. 1's "Lookup Table" (sub-module id -> slot position) and of the
+ * selective loads and evictions behind it (Sec. "Rotary GPU Concept").
+ * Copy residency records [start, start + cap) of the trace into buf. *n_copied = records copied,
  * *n_total = records kept. MOE_ERR_TRACE_OVERFLOW (after copying) if records were dropped. */
 moe_status moe_get_residency_trace(moe_handle* h, int64_t start, moe_trace_rec* buf, int64_t cap,
                                    int64_t* n_copied, int64_t* n_total);
 
-/* Routing of the last decode step: idx int32 [n_layers x max_batch x k], gate fp32 [same]; n is
+/* Paper: Fig. 1 "Routing Result" (routing vector r) of the last step.
+ * Routing of the last decode step: idx int32 [n_layers x max_batch x k], gate fp32 [same]; n is
  * the entries buf can hold (MOE_ERR_INVALID if below n_layers * max_batch * k). Rows b >= the last
  * step's batch are stale. */
 moe_status moe_get_last_routing(moe_handle* h, int32_t* idx, float* gate, int64_t n);
 
+/* Paper: the counts of Fig. 1's selective loads and evictions (Sec. "Rotary GPU Concept"); the
+ * transfer cost the Discussion names is miss_bytes. MOE_SCHEDULE_DEVICE: waits for the handle's
+ * outstanding steps. */
 moe_status moe_get_stats(moe_handle* h, moe_stats* out);
 
 /* Router logits of the last decode step, fp32 [n_layers x max_batch x n_experts] (z = W_r h as the
@@ -238,10 +253,12 @@ moe_status moe_get_stats(moe_handle* h, moe_stats* out);
  * step. */
 moe_status moe_get_last_logits(moe_handle* h, float* z, int64_t n);
 
-/* Empty the slot pool (all experts non-resident), step clock 0, trace and stats cleared. */
+/* Paper: the slot group of Fig. 1 emptied (every sub-module back in the host tier only).
+ * Empty the slot pool (all experts non-resident), step clock 0, trace and stats cleared. */
 moe_status moe_reset_residency(moe_handle* h);
 
-/* Warm start: copy experts into free slots in ascending global id order until the pool is full
+/* Paper: Fig. 1 "selective load" ahead of the first step (a warm slot group).
+ * Warm start: copy experts into free slots in ascending global id order until the pool is full
  * (with cap_slots >= n_layers * n_experts every expert becomes resident). Preloaded experts count
  * as used before every decode step, so they are the first victims; the copies are not residency
  * records and do not change the stats. Synchronous; *n_loaded (optional) = experts copied. */
@@ -413,10 +430,12 @@ const char* moe_planner_last_error(const moe_planner* p);
 /* NULL is a no-op. */
 void moe_planner_destroy(moe_planner* p);
 
-/* Message of the last failure on h (or of the last failed moe_create if h is NULL). */
+/* Paper: no counterpart (error reporting of this ABI).
+ * Message of the last failure on h (or of the last failed moe_create if h is NULL). */
 const char* moe_last_error(const moe_handle* h);
 
-/* Wait for outstanding work, free everything. NULL is a no-op. */
+/* Paper: no counterpart (releases the slot group, the host tier and the work buffers).
+ * Wait for outstanding work, free everything. NULL is a no-op. */
 void moe_destroy(moe_handle* h);
 
 #ifdef __cplusplus

@@ -1158,6 +1158,10 @@ moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t exper
 moe_status moe_decode_step(moe_handle* h, const void* hidden, void* out, int32_t batch, void* stream) {
   if (!h) return MOE_ERR_INVALID;
   if (!hidden || !out) return fail(h, MOE_ERR_INVALID, "NULL hidden or out");
+  // the kernels move activation rows as 16-byte vectors: refuse a misaligned buffer here instead
+  // of faulting the launch
+  if ((((uintptr_t)hidden | (uintptr_t)out) & 15) != 0)
+    return fail(h, MOE_ERR_INVALID, "hidden and out must be 16-byte aligned");
   if (batch < 1 || batch > h->cfg.max_batch) return fail(h, MOE_ERR_INVALID, "batch must be in [1, max_batch]");
   MOE_CK(h, cudaSetDevice(h->cfg.device));
   moe_status st = check_registered(h);

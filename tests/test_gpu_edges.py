@@ -147,6 +147,9 @@ def test_boundary_rejects_bad_requests(P):
         assert m.lib.moe_decode_step(m.h, ptr(h.data_ptr()), ptr(o.data_ptr()), 0, None) == -1  # batch 0
         assert m.lib.moe_decode_step(m.h, None, ptr(o.data_ptr()), 1, None) == -1  # NULL hidden
         assert m.lib.moe_decode_step(m.h, ptr(h.data_ptr()), None, 1, None) == -1  # NULL out
+        # misaligned activation buffers are refused before any launch (one fp32 element off)
+        assert m.lib.moe_decode_step(m.h, ptr(h.data_ptr() + 4), ptr(o.data_ptr()), 1, None) == -1
+        assert m.lib.moe_decode_step(m.h, ptr(h.data_ptr()), ptr(o.data_ptr() + 4), 1, None) == -1
         assert m.get_stats()["layer_steps"] == 0  # nothing ran
         m.decode_step(h, o, batch=4)  # the handle still works
         torch.cuda.synchronize()
