@@ -91,7 +91,8 @@ def _replay(wl, cap, hidden, idx, ranks, preload=False, compute_out=True):
 
 
 def _oracle_z(wl, hidden):
-    orc = oracle.Oracle.for_workload(wl, keep_slot_copies=False, policy="guided")
+    # logits only: a pool holding every expert, so any batch's needed set fits
+    orc = oracle.Oracle.for_workload(wl, cap_slots=wl.n_gid, keep_slot_copies=False, policy="guided")
     return np.stack([orc.decode_step(hidden[t], compute_out=False).z for t in range(hidden.shape[0])])
 
 
