@@ -86,14 +86,23 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
-def measure_h2d(torch, nbytes_chunk: int, total: int = 2 << 30) -> float:
-    """Pinned host -> device copy-engine bandwidth for expert-sized chunks (GB/s)."""
+def measure_h2d(torch, nbytes_chunk: int, seconds: float = 2.0, total: int = 2 << 30) -> float:
+    """Pinned host -> device copy-engine bandwidth for expert-sized chunks (GB/s): back-to-back
+    passes over a 2 GB page-locked buffer for `seconds`, best pass.
+
+    The host link's rate depends on its recent load: after ~20 s without traffic the first second
+    of streaming runs 2-3x slower (measured on GB300: a decode replaying the same tokens after a
+    20 s pause took 27 ms for its first tokens against 10 ms after a 0-2 s pause). A sustained
+    measurement therefore reports the loaded link, and run right before a decode's warm-up steps it
+    leaves the link in the state a running decode keeps it in."""
     n = max(1, total // nbytes_chunk)
     src = torch.empty(n * nbytes_chunk, dtype=torch.uint8, pin_memory=True)
     dst = torch.empty(n * nbytes_chunk, dtype=torch.uint8, device="cuda")
     s = torch.cuda.Stream()
     best = 0.0
-    for _ in range(3):
+    t_end = time.perf_counter() + seconds
+    reps = 0
+    while reps < 3 or time.perf_counter() < t_end:
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(s):
@@ -104,6 +113,7 @@ def measure_h2d(torch, nbytes_chunk: int, total: int = 2 << 30) -> float:
             e1.record(s)
         e1.synchronize()
         best = max(best, n * nbytes_chunk / (e0.elapsed_time(e1) * 1e-3) / 1e9)
+        reps += 1
     del src, dst
     return best
 
@@ -361,10 +371,11 @@ def workload_config(wl, args, world: int) -> dict:
                   if wl.n_layers * wl.top_k * eb > L2_BYTES else "inputs fit in L2 (a correctness-sized case)"}
 
 
-def lookahead_variant(args, wl, hid_dev, out_dev, stream, link_gbs, peak_hbm, peak_src, device, eb, world):
-    """The same workload, tokens and step count under exact layer lookahead (the device kernel that
-    routes every layer first and decides the lookups ahead of the compute): identical trace and
-    outputs, reported beside the layer-by-layer headline, with its own all-resident roofline."""
+def layer_variant(args, wl, hid_dev, out_dev, stream, link_gbs, peak_hbm, peak_src, device, eb, world):
+    """The same workload, tokens and step count on the layer-by-layer kernel (k_fused: each layer
+    routed, looked up and computed before the next layer's input is read, as a chained model needs):
+    identical trace and outputs, reported beside the exact-lookahead headline with its own
+    all-resident roofline."""
     import torch
     from argparse import Namespace
 
@@ -372,8 +383,9 @@ def lookahead_variant(args, wl, hid_dev, out_dev, stream, link_gbs, peak_hbm, pe
 
     n_tok = hid_dev.shape[0]
     m = create_for_workload(wl, device=device, trace_capacity=0, schedule="device", miss_ctas=args.miss_ctas,
-                            policy=args.policy, lookahead=True)
+                            policy=args.policy, lookahead=False)
     try:
+        measure_h2d(torch, eb)  # the link loaded as before the headline's warm-up
         if args.preload:
             m.preload()
         for i in range(args.warmup):
@@ -396,12 +408,12 @@ def lookahead_variant(args, wl, hid_dev, out_dev, stream, link_gbs, peak_hbm, pe
     miss_b = misses * eb / args.steps
     hbm_b = (hits + misses) / args.steps * eb + wl.n_layers * wl.router_bytes()
     t_star = max(hbm_b / (peak_hbm * 1e9), miss_b / (link_gbs * 1e9))
-    out = {"kernel": "k_fused_la", "value": whole_job_rate(args.steps, world, ms * args.steps * 1e-3),
+    out = {"kernel": "k_fused", "value": whole_job_rate(args.steps, world, ms * args.steps * 1e-3),
            "unit": "tok/s", "ms_per_step": ms, "step_roofline_frac": t_star * 1e3 / ms,
            "achieved_h2d_gbs": miss_b / (ms * 1e-3) / 1e9, "hit_rate": 1.0 - misses / max(1, hits + misses)}
     if not args.no_resident:
-        la = Namespace(**{**vars(args), "lookahead": True})
-        out["roofline"] = resident_roofline(la, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, device, eb)
+        lb = Namespace(**{**vars(args), "lookahead": False})
+        out["roofline"] = resident_roofline(lb, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, device, eb)
     return out
 
 
@@ -631,12 +643,13 @@ def main():
     ap.add_argument("--miss-ctas", type=int, default=0, help="CTAs streaming missed experts (0: library default)")
     ap.add_argument("--policy", default="lru", choices=["lru", "rotary", "guided"],
                     help="slot-group replacement policy (rotary: batch 1; guided: device schedule, batch 1)")
-    ap.add_argument("--lookahead", action="store_true",
-                    help="exact layer lookahead: host copy-engine schedule, route layer l + 1 and issue its copies "
-                         "while layer l computes; device schedule, one kernel routes every layer, then CTA 0 runs "
-                         "the lookups up to two layers ahead of the compute")
-    ap.add_argument("--no-lookahead-compare", action="store_true",
-                    help="skip the exact-lookahead measurement reported beside a batch-1 device-schedule headline")
+    ap.add_argument("--lookahead", default="auto", choices=["auto", "on", "off"],
+                    help="exact layer lookahead (the layers' inputs all come with the step): host copy-engine "
+                         "schedule, route layer l + 1 and issue its copies while layer l computes; device schedule, "
+                         "one kernel routes every layer, then CTA 0 runs the lookups ahead of the compute. auto: on "
+                         "for batch-1 LRU steps of the device schedule, off otherwise")
+    ap.add_argument("--no-compare", action="store_true",
+                    help="skip the layer-by-layer kernel measured beside a lookahead headline")
     ap.add_argument("--batched-path", default="auto", choices=["auto", "cuda_cores"],
                     help="expert FFN of batched steps: tensor cores where the shape allows, or CUDA cores")
     args = ap.parse_args()
@@ -651,6 +664,8 @@ def main():
         wl = wl.replace(n_layers=args.layers)
     if args.cap is not None:
         wl = wl.replace(cap_slots=args.cap)
+    args.lookahead = args.lookahead == "on" or (
+        args.lookahead == "auto" and args.schedule == "device" and wl.batch == 1 and args.policy == "lru")
     if args.impl == "reference":
         return run_reference(args, wl)
 
@@ -690,13 +705,14 @@ def main():
     t_setup = time.perf_counter() - t_setup
     thp_gb = (anon_huge_kb() - thp0) / 1e6
     eb = P.expert_bytes(m.cfg)
-    h2d_gbs = measure_h2d(torch, eb)
 
     tdt = torch.float32 if wl.adtype == "fp32" else torch.bfloat16
     raw = torch.from_numpy(hidden.view(np.float32) if wl.adtype == "fp32" else hidden.view(np.int16))
     hid_dev = raw.cuda().view(tdt) if wl.adtype != "fp32" else raw.cuda()
     out_dev = torch.empty_like(hid_dev[0])
     stream = torch.cuda.current_stream()
+    # the link ceiling, sustained, right before the warm-up steps (see measure_h2d)
+    h2d_gbs = measure_h2d(torch, eb)
 
     def step(i):
         m.decode_step(hid_dev[i % n_tok], out_dev, batch=wl.batch, stream=stream)
@@ -799,9 +815,9 @@ def main():
                 "steps": e2e_steps, "api": "moe_decode_step_host"},
     }
     m.destroy()
-    if wl.batch == 1 and args.schedule == "device" and not args.lookahead and not args.no_lookahead_compare:
-        line["lookahead"] = lookahead_variant(args, wl, hid_dev, out_dev, stream, link_gbs, peak_hbm, peak_src,
-                                              local, eb, world)
+    if wl.batch == 1 and args.schedule == "device" and args.lookahead and not args.no_compare:
+        line["layer_by_layer"] = layer_variant(args, wl, hid_dev, out_dev, stream, link_gbs, peak_hbm, peak_src,
+                                               local, eb, world)
     if not args.no_resident:
         line["roofline"] = resident_roofline(args, wl, hid_dev, out_dev, stream, peak_hbm, peak_src, local, eb)
     del hid_dev, out_dev

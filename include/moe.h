@@ -199,10 +199,7 @@ moe_status moe_set_router(moe_handle* h, int32_t layer, const void* w_r);
  *              two's complement; `scales` = bf16 [I x d/128] (gate) ++ [I x d/128] (up)
  *              ++ [d x I/128] (down). NULL otherwise.
  * The weights are repacked into the slot layout. If the expert is resident its slot copy is
- * NOT refreshed; call moe_reset_residency after re-registering resident experts.
- * MOE_SCHEDULE_DEVICE: the call also enqueues, on an internal stream, one GPU read per 4 KB page
- * of the expert's image in the host tier, so that the GPU's address translations of the tier are
- * resolved while it is built rather than during the first decode steps that stream it. */
+ * NOT refreshed; call moe_reset_residency after re-registering resident experts. */
 moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t expert, const void* w_gate,
                                      const void* w_up, const void* w_down, const void* scales);
 

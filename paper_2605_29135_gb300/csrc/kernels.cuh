@@ -69,10 +69,6 @@ struct RouterArgs {
 };
 
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
-// One 4-byte read from the GPU of every (1 << shift)-byte page of [base, base + bytes) (base is a
-// device address of page-locked host memory): resolves the GPU's address translations of those
-// pages ahead of the decode steps that stream them.
-cudaError_t launch_touch_pages(const uint8_t* base, int64_t bytes, int shift, cudaStream_t s);
 cudaError_t launch_gateup(const GateUpArgs& a, int wdtype, cudaStream_t s);
 cudaError_t launch_down_combine(const DownArgs& a, int wdtype, cudaStream_t s);
 

@@ -103,7 +103,6 @@ struct moe_handle {
   float* u = nullptr;  // device [k][I]
   cudaStream_t copy_stream = nullptr;
   cudaStream_t host_stream = nullptr;
-  cudaStream_t warm_stream = nullptr;  // device schedule: the host tier's page-translation warm-up
   std::vector<cudaEvent_t> copy_ev;
   cudaEvent_t layer_ev[2] = {nullptr, nullptr};  // host schedule with lookahead: layer l's last kernel done
   void* hid_dev = nullptr;
@@ -928,7 +927,6 @@ void free_all(moe_handle* h) {
     if (e) cudaEventDestroy(e);
   if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   if (h->host_stream) cudaStreamDestroy(h->host_stream);
-  if (h->warm_stream) cudaStreamDestroy(h->warm_stream);
   if (h->own_pool && h->pool) cudaFree(h->pool);
   if (h->arena) cudaFreeHost(h->arena);
   if (h->routers) cudaFree(h->routers);
@@ -1070,8 +1068,6 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   if (h->dev_mode) {
     if (cudaHostGetDevicePointer((void**)&h->arena_dev, h->arena, 0) != cudaSuccess)
       return bail(MOE_ERR_CUDA, "host arena has no device address");
-    if (cudaStreamCreateWithFlags(&h->warm_stream, cudaStreamNonBlocking) != cudaSuccess)
-      return bail(MOE_ERR_CUDA, "stream creation failed");
     const int k = cfg->top_k;
     const int64_t pairs = (int64_t)cfg->max_batch * k;
     // batch 1: slot, gid, miss per rank, for one layer ([k]) or, with lookahead, for every layer ([L][k])
@@ -1155,14 +1151,6 @@ moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t exper
     memcpy(dst + L.d_scale_off, s + 2 * c.d_ff * G, (size_t)(c.d * (c.d_ff / 128) * 2));
   }
   if (h->slot_stride > L.total) memset(dst + L.total, 0, h->slot_stride - L.total);
-  if (h->warm_stream) {
-    // The device schedule's kernels read this image over the host link. The GPU's first read of
-    // each 4 KB page of the host tier is slow (its address translation), which made the first
-    // ~100 decode tokens of the 48-layer stack up to 2.7x slower than later ones. Reading one word
-    // per page here, while the tier is built, moves that cost to set-up.
-    MOE_CK(h, cudaSetDevice(c.device));
-    MOE_CK(h, moe::launch_touch_pages(h->arena_dev + gid * h->slot_stride, h->slot_stride, 12, h->warm_stream));
-  }
   h->registered[gid] = 1;
   return MOE_OK;
 }

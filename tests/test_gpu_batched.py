@@ -11,6 +11,7 @@ a 6 GB pool cap (635 slots) for a few steps. bf16 shapes whose d is a multiple o
 of 64 run both expert-FFN paths: tensor cores (tcgen05 grouped GEMM, pairs per expert padded
 to 16, 32, 48 or 64 columns) and CUDA cores.
 """
+import functools
 from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
@@ -39,7 +40,11 @@ def _create(wl, cap, **kw):
 
 def _check_outputs(wl, hidden, idx, gate, out, samples, threads=8):
     routers = [synth.router_weights(wl, l) for l in range(wl.n_layers)]
-    orc = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers)
+    # rows in layer order, so that the rows of one layer share the generated experts they route to
+    orc = oracle.Oracle.for_workload(wl, keep_slot_copies=False, routers=routers,
+                                     experts=functools.lru_cache(maxsize=512)(
+                                         lambda l, e: synth.expert_weights(wl, l, e)))
+    samples = sorted(samples, key=lambda tlb: (tlb[1], tlb[0], tlb[2]))
 
     def one(tlb):
         t, l, b = tlb
@@ -203,6 +208,15 @@ def test_layer_bf16_batch64(P, path):
     samples = [(t, l, int(b)) for t in range(wl.tokens) for l in range(wl.n_layers)
                for b in rng.choice(64, size=4, replace=False)]
     _parity(wl, wl.cap_slots, samples=samples, threads=16, path=path)
+
+
+def test_stack48_batch64_all_resident(P):
+    # the benchmarked uncapped batch-64 configuration: all 6144 experts preloaded into a 58 GB pool,
+    # 48 layers, 64 sequences, tensor-core expert FFN; every request hits
+    wl = synth.WORKLOADS["stack48_batch64"].replace(tokens=3, cap_slots=6144)
+    samples = [(t, l, b) for t in (0, 2) for l in range(wl.n_layers) for b in (0, 31, 63)]
+    _, tr = _parity(wl, wl.cap_slots, samples=samples, threads=16, preload=True)
+    assert (tr["kind"] == 0).all() and len(tr) > 0
 
 
 def test_stack48_batch64_capped_steps(P):
