@@ -212,7 +212,12 @@ moe_status moe_register_host_experts(moe_handle* h, int32_t layer, int32_t exper
  * (a cudaStream_t; NULL = legacy default stream). hidden must stay valid and out must not be
  * read until `stream` reaches the end of the step. Calls on one handle must use one stream or
  * be serialised by the caller.
- *   MOE_SCHEDULE_DEVICE: enqueues one kernel and returns. A failure detected on the device
+ *   MOE_SCHEDULE_DEVICE: enqueues one kernel and returns. The first step after creation, a reset
+ *     or a gap of 2 s or more since the previous step's launch (with a pool smaller than the
+ *     stack) first enqueues one read per 4 KB page of the host tier from all SMs: after an idle
+ *     gap the host link's first reads run 2-3x slower for ~1 s of streaming, and this pass pays
+ *     that cost once (about 0.5-0.7 s for a 58 GB tier) instead of over the next ~100 steps.
+ *     A failure detected on the device
  *     (a grid barrier that timed out, an invalid routing result) is reported by the next call
  *     on the handle that synchronises (decode_step, get_stats, get_residency_trace, ...), as
  *     MOE_ERR_TIMEOUT or MOE_ERR_CUDA, and empties the pool.

@@ -8,6 +8,8 @@
 // expert occupies or on the grid size, so results are bit-identical between capped and
 // uncapped pools.
 #include <cooperative_groups.h>
+
+#include <algorithm>
 #include <cuda_bf16.h>
 #include <math.h>
 
@@ -416,6 +418,24 @@ cudaError_t launch_gateup(const GateUpArgs& a, int wdtype, cudaStream_t s) {
     MOE_G(WD_INT4)
   }
 #undef MOE_G
+}
+
+namespace {
+
+__global__ void __launch_bounds__(256) k_touch_pages(const uint8_t* base, int64_t bytes, int shift) {
+  const int64_t pages = (bytes + (1ll << shift) - 1) >> shift;
+  for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < pages; p += (int64_t)gridDim.x * blockDim.x)
+    asm volatile("{ .reg .u32 t; ld.volatile.global.u32 t, [%0]; }" ::"l"(base + (p << shift)) : "memory");
+}
+
+}  // namespace
+
+cudaError_t launch_touch_pages(const uint8_t* base, int64_t bytes, int shift, cudaStream_t s) {
+  if (bytes <= 0) return cudaSuccess;
+  const int64_t pages = (bytes + (1ll << shift) - 1) >> shift;
+  const int blocks = (int)std::min<int64_t>((pages + 255) / 256, 1024);
+  k_touch_pages<<<blocks, 256, 0, s>>>(base, bytes, shift);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_down_combine(const DownArgs& a, int wdtype, cudaStream_t s) {

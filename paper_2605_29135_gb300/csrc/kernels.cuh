@@ -69,6 +69,9 @@ struct RouterArgs {
 };
 
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
+// One 4-byte read from the SMs of every (1 << shift)-byte page of [base, base + bytes), base a
+// device address of page-locked host memory (the host tier).
+cudaError_t launch_touch_pages(const uint8_t* base, int64_t bytes, int shift, cudaStream_t s);
 cudaError_t launch_gateup(const GateUpArgs& a, int wdtype, cudaStream_t s);
 cudaError_t launch_down_combine(const DownArgs& a, int wdtype, cudaStream_t s);
 

@@ -144,6 +144,10 @@ struct moe_handle {
   int fgrid_la = 0;
   unsigned wbar_epoch = 0;     // its worker-barrier counter value at the start of the next launch
   const uint8_t* arena_dev = nullptr;
+  // host time of the last decode-step launch (device schedule): after an idle gap the first step
+  // re-reads one word per page of the host tier first (see decode_device)
+  std::chrono::steady_clock::time_point last_launch{};
+  bool launched = false;
   int32_t* d_slot_of = nullptr;
   unsigned long long* d_slot_key = nullptr;
   unsigned long long* d_cand = nullptr;  // batch-1 kernel: victim candidates [kMaxRanks + 1]
@@ -272,6 +276,7 @@ void reset_device_state(moe_handle* h) {
   *h->h_err = 0;
   h->err_pending = false;
   h->steps_launched = 0;
+  h->launched = false;  // the next step re-reads the host tier's pages first
 }
 
 void reset_state(moe_handle* h) {
@@ -858,9 +863,26 @@ void recover_after_failure(moe_handle* h, cudaStream_t s) {
   h->err = keep;
 }
 
+// After the host link has been idle for a while the SMs' reads of the host tier run 2-3x slower
+// and recover only over ~1 s of streaming. Measured on GB300 with the 48-layer bf16 stack (58 GB
+// tier): after 20 s idle (or right after the tier is built) the first 10 tokens took 23-28 ms each
+// against 8.5-9 ms back to back, recovering over ~100 tokens (~0.7 s lost in all); after a 2 s gap
+// the loss was ~20 ms; copy-engine traffic in the gap made no difference. One read per 4 KB page
+// of the whole tier from all SMs at once before the first step after a gap of kIdleRewarm or more
+// pays about the same once (0.5-0.7 s cold for 58 GB) and leaves the following steps at the loaded
+// rate. Shorter gaps are left to recover by themselves (the pass costs ~50 ms even when warm).
+constexpr std::chrono::milliseconds kIdleRewarm{2000};
+
 moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
   moe_status st = check_device_error(h, false);
   if (st != MOE_OK) return st;
+  const auto now = std::chrono::steady_clock::now();
+  if (h->cap < h->n_gid && (!h->launched || now - h->last_launch >= kIdleRewarm)) {
+    NvtxRange range("re-read the host tier's pages after an idle gap");
+    MOE_CK(h, moe::launch_touch_pages(h->arena_dev, (int64_t)h->arena_bytes, 12, s));
+  }
+  h->last_launch = now;
+  h->launched = true;
   if (h->batched) return decode_batched(h, hidden, out, batch, s);
   return decode_device_layers(h, hidden, out, 0, h->cfg.n_layers, s);
 }
