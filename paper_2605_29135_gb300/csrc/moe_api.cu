@@ -618,9 +618,10 @@ moe_status check_device_error(moe_handle* h, bool sync) {
   if (e & moe::FERR_BARRIER_TIMEOUT) msg += " a grid barrier timed out;";
   if (e & moe::FERR_BAD_ROUTE) msg += " the router produced an invalid expert id (non-finite logits?);";
   if (e & moe::FERR_NO_VICTIM) msg += " no evictable slot;";
+  if (e & moe::FERR_PIPE_TIMEOUT) msg += " a wait for copies into shared memory timed out;";
   msg += " the pool was emptied";
   reset_state(h);
-  return fail(h, (e & moe::FERR_BARRIER_TIMEOUT) ? MOE_ERR_TIMEOUT : MOE_ERR_CUDA, msg);
+  return fail(h, (e & moe::FERR_FATAL) ? MOE_ERR_TIMEOUT : MOE_ERR_CUDA, msg);
 }
 
 // Per-phase durations of the last profiled step from the kernel's global-timer stamps.
@@ -873,9 +874,8 @@ void recover_after_failure(moe_handle* h, cudaStream_t s) {
 // rate. Shorter gaps are left to recover by themselves (the pass costs ~50 ms even when warm).
 constexpr std::chrono::milliseconds kIdleRewarm{2000};
 
-moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
-  moe_status st = check_device_error(h, false);
-  if (st != MOE_OK) return st;
+// Enqueues the re-read pass on s before a step that follows an idle gap (device schedule).
+moe_status rewarm_if_idle(moe_handle* h, cudaStream_t s) {
   const auto now = std::chrono::steady_clock::now();
   if (h->cap < h->n_gid && (!h->launched || now - h->last_launch >= kIdleRewarm)) {
     NvtxRange range("re-read the host tier's pages after an idle gap");
@@ -883,6 +883,14 @@ moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t b
   }
   h->last_launch = now;
   h->launched = true;
+  return MOE_OK;
+}
+
+moe_status decode_device(moe_handle* h, const void* hidden, void* out, int32_t batch, cudaStream_t s) {
+  moe_status st = check_device_error(h, false);
+  if (st != MOE_OK) return st;
+  st = rewarm_if_idle(h, s);
+  if (st != MOE_OK) return st;
   if (h->batched) return decode_batched(h, hidden, out, batch, s);
   return decode_device_layers(h, hidden, out, 0, h->cfg.n_layers, s);
 }
@@ -1444,6 +1452,8 @@ moe_status moe_run_layer(moe_handle* h, const void* hidden, void* out, int32_t l
     st = check_registered(h);
     if (st != MOE_OK) return st;
     st = check_device_error(h, false);
+    if (st != MOE_OK) return st;
+    st = rewarm_if_idle(h, s);  // once per decoder token, before its first MoE layer
     if (st != MOE_OK) return st;
   }
   st = decode_device_layers(h, hidden, out, layer, layer + 1, s);

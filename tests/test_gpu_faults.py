@@ -41,19 +41,26 @@ def _expect_recovery(m, wl, hidden, cap):
     assert rel_l2_rows(out, np.stack([r.out for r in res])).max() <= TOL[wl.wdtype]
 
 
-@pytest.mark.parametrize("batch,lookahead", [(1, False), (4, False), (1, True)])
-def test_device_wait_that_runs_out_reports_timeout_and_recovers(P, batch, lookahead):
+@pytest.mark.parametrize("batch,lookahead,dtype", [(1, False, "fp32"), (4, False, "fp32"), (1, True, "fp32"),
+                                                   (1, True, "bf16")])
+def test_device_wait_that_runs_out_reports_timeout_and_recovers(P, batch, lookahead, dtype):
     # lookahead: the device schedule's lookahead kernel, whose router-phase barrier is the one
-    # that runs out; every CTA leaves it, so no worker waits for a plan that never comes
+    # that runs out; every CTA leaves it, so no worker waits for a plan that never comes (bf16:
+    # its bulk-copy variant, whose warps have issued no copies yet when they leave)
     import torch
 
     from paper_2605_29135_gb300.workload import create_for_workload
 
     wl = synth.WORKLOADS["tiny_fp32"].replace(n_layers=2, tokens=8, batch=batch)
+    if dtype == "bf16":
+        wl = wl.replace(wdtype="bf16", adtype="bf16")
     hidden = synth.hidden_all(wl)
     m = create_for_workload(wl, cap_slots=8, lookahead=lookahead)
     try:
-        h = torch.from_numpy(hidden[0].view(np.float32)).cuda()
+        if dtype == "bf16":
+            h = torch.from_numpy(hidden[0].view(np.int16)).cuda().view(torch.bfloat16)
+        else:
+            h = torch.from_numpy(hidden[0].view(np.float32)).cuda()
         o = torch.empty_like(h)
         m.decode_step(h, o, batch=batch)  # a normal step first
         m.inject_fault("barrier_timeout")
