@@ -88,13 +88,8 @@ class ClockSampler:
 
 def measure_h2d(torch, nbytes_chunk: int, seconds: float = 2.0, total: int = 2 << 30) -> float:
     """Pinned host -> device copy-engine bandwidth for expert-sized chunks (GB/s): back-to-back
-    passes over a 2 GB page-locked buffer for `seconds`, best pass.
-
-    The host link's rate depends on its recent load: after ~20 s without traffic the first second
-    of streaming runs 2-3x slower (measured on GB300: a decode replaying the same tokens after a
-    20 s pause took 27 ms for its first tokens against 10 ms after a 0-2 s pause). A sustained
-    measurement therefore reports the loaded link, and run right before a decode's warm-up steps it
-    leaves the link in the state a running decode keeps it in."""
+    passes over a 2 GB page-locked buffer for `seconds`, best pass (a sustained figure: an idle
+    link starts slower)."""
     n = max(1, total // nbytes_chunk)
     src = torch.empty(n * nbytes_chunk, dtype=torch.uint8, pin_memory=True)
     dst = torch.empty(n * nbytes_chunk, dtype=torch.uint8, device="cuda")
@@ -385,7 +380,6 @@ def layer_variant(args, wl, hid_dev, out_dev, stream, link_gbs, peak_hbm, peak_s
     m = create_for_workload(wl, device=device, trace_capacity=0, schedule="device", miss_ctas=args.miss_ctas,
                             policy=args.policy, lookahead=False)
     try:
-        measure_h2d(torch, eb)  # the link loaded as before the headline's warm-up
         if args.preload:
             m.preload()
         for i in range(args.warmup):
@@ -711,7 +705,7 @@ def main():
     hid_dev = raw.cuda().view(tdt) if wl.adtype != "fp32" else raw.cuda()
     out_dev = torch.empty_like(hid_dev[0])
     stream = torch.cuda.current_stream()
-    # the link ceiling, sustained, right before the warm-up steps (see measure_h2d)
+    # the copy-engine ceiling of the host link, sustained (see measure_h2d)
     h2d_gbs = measure_h2d(torch, eb)
 
     def step(i):

@@ -153,22 +153,42 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_split(const float* q, 
 }
 
 // out[h] = sum_s acc_s exp(m_s - M) / sum_s l_s exp(m_s - M) over the splits of h's kv head; one CTA
-// per query head, one thread per dim.
+// per query head, one thread per dim. The splits' maxima and sums are first staged in shared
+// memory by all threads at once and the weights exp(m_s - M) formed once per split; each sum still
+// runs over the splits in ascending order.
 __global__ void k_attn_merge(const float* part, int D, int G, int nsplit, float* out) {
+  extern __shared__ float s_ml[];  // [2][nsplit]: the splits' maxima, then their weights; their sums
+  __shared__ float s_M, s_L;
+  float* s_c = s_ml;
+  float* s_l = s_ml + nsplit;
   const int h = blockIdx.x, dd = threadIdx.x;
   const int g = h / G, hh = h - g * G;
   const float* base = part + ((int64_t)g * nsplit * G + hh) * (D + 2);
   const int64_t stride = (int64_t)G * (D + 2);
-  float M = -INFINITY;
-  for (int s = 0; s < nsplit; s++) M = fmaxf(M, base[s * stride + D]);
-  float L = 0.f, A = 0.f;
-  for (int s = 0; s < nsplit; s++) {
-    const float* ps = base + s * stride;
-    const float c = expf(ps[D] - M);
-    L = fmaf(ps[D + 1], c, L);
-    A = fmaf(ps[dd], c, A);
+  for (int sp = threadIdx.x; sp < nsplit; sp += blockDim.x) {
+    s_c[sp] = base[sp * stride + D];
+    s_l[sp] = base[sp * stride + D + 1];
   }
-  out[(int64_t)h * D + dd] = A / L;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float M = -INFINITY;
+    for (int sp = 0; sp < nsplit; sp++) M = fmaxf(M, s_c[sp]);
+    s_M = M;
+  }
+  __syncthreads();
+  const float M = s_M;
+  for (int sp = threadIdx.x; sp < nsplit; sp += blockDim.x) s_c[sp] = expf(s_c[sp] - M);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float L = 0.f;
+    for (int sp = 0; sp < nsplit; sp++) L = fmaf(s_l[sp], s_c[sp], L);
+    s_L = L;
+  }
+  float A = 0.f;
+#pragma unroll 16
+  for (int sp = 0; sp < nsplit; sp++) A = fmaf(base[sp * stride + dd], s_c[sp], A);
+  __syncthreads();
+  out[(int64_t)h * D + dd] = A / s_L;
 }
 
 // Splits per kv head: about two CTAs per SM over all kv heads, at least 16 positions each, and no
@@ -211,7 +231,7 @@ cudaError_t launch_attention(const float* q, const void* k_cache, const void* v_
   cudaError_t e = head_dim == 128 ? launch_split<CT, 4>(G, q, K, V, n_kv_heads, max_pos, n_pos, per, nsplit, scratch, s)
                                   : launch_split<CT, 2>(G, q, K, V, n_kv_heads, max_pos, n_pos, per, nsplit, scratch, s);
   if (e != cudaSuccess) return e;
-  k_attn_merge<<<n_heads, head_dim, 0, s>>>(scratch, head_dim, G, nsplit, out);
+  k_attn_merge<<<n_heads, head_dim, 2 * nsplit * sizeof(float), s>>>(scratch, head_dim, G, nsplit, out);
   return cudaGetLastError();
 }
 
