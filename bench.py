@@ -181,7 +181,8 @@ def oracle_token_times(wl, hidden, n_tokens, budget_s=None):
         for t in range(n_tokens):
             r = probe.decode_step(hidden[t], compute_out=False)
             need = sorted({(l, int(e)) for l in range(wl.n_layers) for e in r.idx[l].ravel()})
-            for key in [key for key in cache if key not in set(need)]:
+            need_set = set(need)
+            for key in [key for key in cache if key not in need_set]:
                 del cache[key]
             new = [le for le in need if le not in cache]
             cache.update(zip(new, ex.map(lambda le: synth.expert_weights(wl, *le), new)))

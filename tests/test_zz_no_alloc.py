@@ -23,7 +23,7 @@ import pytest
 
 import oracle
 import synth
-from tests.gpu_harness import NEAR_TIE, check_routing
+from tests.gpu_harness import check_routing
 
 # (workload, tokens, renorm): tokens are also the row count of the batched call
 CASES = {
@@ -60,7 +60,7 @@ def _noalloc_all(P, wl, hid, routers, renorm):
     twice = [np.empty_like(single[0]), np.empty_like(single[1])]
     for t in range(T):
         for l in range(L):
-            for rep, dst in ((0, single), (1, twice)):
+            for dst in (single, twice):
                 idx, gate = P.route_noalloc(routers[l], hid[t, l].contiguous(), wl.top_k, renorm=renorm)
                 torch.cuda.synchronize()
                 dst[0][t, l], dst[1][t, l] = idx.cpu().numpy()[0], gate.cpu().numpy()[0]
