@@ -116,3 +116,24 @@ def test_decoder_reference_arm_prints_one_line_on_rank_zero(monkeypatch, capsys)
     line = json.loads(capsys.readouterr().out)
     assert line["impl"] == "reference" and line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle"
     assert line["config"]["workload"] == "tiny_block_fp32"
+
+
+def test_reference_arm_prints_the_gpu_arms_config(capsys):
+    # both arms build `config` from the workload and the options alone, so the driver can compare
+    # them key for key; the reference arm's step is one decode token at batch 1
+    import json
+    from argparse import Namespace
+
+    import synth
+
+    wl = synth.WORKLOADS["tiny_fp32"]
+    args = Namespace(gpus=1, steps=2, warmup=3, schedule="device", miss_ctas=0, batched_path="auto", policy="lru",
+                     lookahead=True)
+    assert bench.run_reference(args, wl) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference"
+    assert line["config"] == bench.workload_config(wl, args, 1)
+    assert line["config"] == json.loads(json.dumps(bench.workload_config(wl, args, 1)))
+    assert line["step"].startswith("one decode token")
+    assert line["metric"].startswith("MoE decode tok/s")
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["value"] > 0
