@@ -656,9 +656,13 @@ __device__ __forceinline__ void stage_u(const FusedArgs& a, float* us, int ipad,
 // Phase D (all experts in their slots) for one value of the chunks-per-lane count of a W_d row:
 // stages u, then out[o] = sum_r g_r (W_d^(r)[o] . u_r). A warp's first rows are requested before
 // the CTA stages u, so the HBM latency overlaps the staging.
+// With np > 1 (the lookahead kernel's layer groups) the phase covers layers l .. l + np - 1 at once:
+// pslot / pgate hold np plans of kMaxRanks entries, u the np layers' k x I vectors one after the
+// other, us room for np staged copies; rows q = m * d + o (layer l + m, output row o) are spread
+// over the warps, each computed exactly as with np = 1.
 template <int WD, int CHD>
 __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, const float* pgate, int l, int gw,
-                           int W, const float* u = nullptr, bool cta_active = true) {
+                           int W, const float* u = nullptr, bool cta_active = true, int np = 1) {
   if (!cta_active) return;  // the same for every thread of the CTA
   constexpr int E = Tr<WD>::epc;
   constexpr int KR = 24 / CHD > 8 ? 8 : (24 / CHD < 1 ? 1 : 24 / CHD);
@@ -667,15 +671,18 @@ __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, cons
   const int nch = (int)(rb / 16);
   const int G = a.I / 128;
   const int ipad = ipad_of(a.I);
+  const int rows = np * a.d;
   uint4 w[KR][CHD];
   float sc[KR][CHD];
-  // loads of ranks [r0, r0 + KR) of row o into w / sc (predicated, no break: keeps them in registers)
-  auto issue = [&](int o, int r0) {
+  // loads of ranks [r0, r0 + KR) of row q into w / sc (predicated, no break: keeps them in registers)
+  auto issue = [&](int q, int r0) {
+    const int m = q < rows ? q / a.d : 0;
+    const int o = q < rows ? q - m * a.d : a.d;
 #pragma unroll
     for (int rr = 0; rr < KR; rr++) {
       const int r = r0 + rr;
       const bool rok = r < a.k && o < a.d;
-      const uint8_t* slot = a.pool + (int64_t)pslot[r < a.k ? r : 0] * a.slot_stride;
+      const uint8_t* slot = a.pool + (int64_t)pslot[m * kMaxRanks + (r < a.k ? r : 0)] * a.slot_stride;
       const int64_t roff = a.lay.d_off + (int64_t)(o < a.d ? o : 0) * rb;
 #pragma unroll
       for (int j = 0; j < CHD; j++) {
@@ -693,17 +700,20 @@ __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, cons
     }
   };
   issue(gw, 0);
-  stage_u(a, us, ipad, u);
+  for (int m = 0; m < np; m++)
+    stage_u(a, us + (int64_t)m * a.k * ipad, ipad, (u ? u : a.u) + (int64_t)m * a.k * a.I);
   __syncthreads();
-  for (int o = gw; o < a.d; o += W) {
+  for (int q = gw; q < rows; q += W) {
+    const int m = q / a.d;
+    const int o = q - m * a.d;
     float acc = 0.f;
     for (int r0 = 0; r0 < a.k; r0 += KR) {
-      if (o != gw || r0 != 0) issue(o, r0);
+      if (q != gw || r0 != 0) issue(q, r0);
 #pragma unroll
       for (int rr = 0; rr < KR; rr++) {
         const int r = r0 + rr;
         if (r >= a.k) continue;
-        const float* ur = us + r * ipad;
+        const float* ur = us + (int64_t)m * a.k * ipad + r * ipad;
         float part = 0.f;
 #pragma unroll
         for (int j = 0; j < CHD; j++) {
@@ -715,15 +725,15 @@ __device__ void down_phase(const FusedArgs& a, float* us, const int* pslot, cons
               part = dot_chunk_u<WD>(w[rr][j], ur + upad(c * E), part);
           }
         }
-        acc = fmaf(pgate[r], part, acc);
+        acc = fmaf(pgate[m * kMaxRanks + r], part, acc);
       }
     }
     acc = warp_sum(acc);
     if (lane == 0) {
       if (WD == WD_FP32)
-        reinterpret_cast<float*>(a.out)[(int64_t)l * a.d + o] = acc;
+        reinterpret_cast<float*>(a.out)[(int64_t)(l + m) * a.d + o] = acc;
       else
-        reinterpret_cast<__nv_bfloat16*>(a.out)[(int64_t)l * a.d + o] = __float2bfloat16_rn(acc);
+        reinterpret_cast<__nv_bfloat16*>(a.out)[(int64_t)(l + m) * a.d + o] = __float2bfloat16_rn(acc);
     }
   }
 }
@@ -1086,15 +1096,17 @@ __device__ void la_lookups(const FusedArgs& a, int64_t step, PendingTable& pend,
 template <int WD, int CH>
 __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant__ FusedArgs a) {
   extern __shared__ uint4 smem4[];
-  __shared__ int p_slot[kMaxRanks], p_gid[kMaxRanks], p_miss[kMaxRanks];
-  __shared__ float p_gate[kMaxRanks];
-  __shared__ int p_mr[kMaxRanks], p_hr[kMaxRanks], p_nm, p_nh;
+  // the plans and inputs of the layers of one group (a.la_group layers, 1 or kLaGroupMax)
+  __shared__ int p_slot[kLaGroupMax][kMaxRanks], p_gid[kLaGroupMax][kMaxRanks], p_miss[kLaGroupMax][kMaxRanks];
+  __shared__ float p_gate[kLaGroupMax][kMaxRanks];
+  __shared__ int p_mr[kLaGroupMax][kMaxRanks], p_hr[kLaGroupMax][kMaxRanks], p_nm[kLaGroupMax], p_nh[kLaGroupMax];
   __shared__ PendingTable pend;
   __shared__ int s_ok;
   const int asize = WD == WD_FP32 ? 4 : 2;
   const int xbytes = a.d * asize;
-  uint8_t* xs = reinterpret_cast<uint8_t*>(smem4);
-  float* us = reinterpret_cast<float*>(xs + ((xbytes + 15) & ~15));
+  const int xpad = (xbytes + 15) & ~15;
+  uint8_t* xs0 = reinterpret_cast<uint8_t*>(smem4);               // [la_group][xpad]
+  float* us = reinterpret_cast<float*>(xs0 + a.la_group * xpad);  // [la_group][k x ipad]
   const int lane = threadIdx.x & 31;
   const int gw = blockIdx.x * kFWarps + (threadIdx.x >> 5);
   const int W = gridDim.x * kFWarps;
@@ -1110,112 +1122,134 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
     return;
   }
 
-  // ---- workers
+  // ---- workers: the layers in groups of P = a.la_group, one worker barrier per group
   const int wgw = ((int)blockIdx.x - 1) * kFWarps + (threadIdx.x >> 5);
-  for (int l = 0; l < a.L; l++) {
-    const int clock = (int)(step * a.L + l + 1);
-    float* u = a.u + (int64_t)(l & 1) * k * a.I;
-    __syncthreads();  // the previous layer's down rows are done with p_slot / p_gate in this CTA
-    if (threadIdx.x == 0) s_ok = wait_count(a, a.plan_flag, (unsigned)clock);
+  const int P = a.la_group;
+  const int workers = (int)gridDim.x - 1;
+  for (int l0 = 0; l0 < a.L; l0 += P) {
+    const int np = a.L - l0 < P ? a.L - l0 : P;
+    // u of this group: groups alternate between two sets of P layers' vectors
+    float* ug = a.u + (int64_t)(((l0 / P) & 1) * P) * k * a.I;
+    __syncthreads();  // the previous group's down rows are done with the plans and u in this CTA
+    if (threadIdx.x == 0) s_ok = wait_count(a, a.plan_flag, (unsigned)(step * a.L + l0 + np));
     __syncthreads();
     if (!s_ok) return;
-    if (threadIdx.x < k) {
-      const int64_t q = (int64_t)l * k + threadIdx.x;
-      p_slot[threadIdx.x] = __ldcg(a.plan_slot + q);
-      p_gid[threadIdx.x] = __ldcg(a.plan_gid + q);
-      p_miss[threadIdx.x] = __ldcg(a.plan_miss + q);
-      p_gate[threadIdx.x] = __ldcg(a.plan_gate + q);
+    if (threadIdx.x < np * k) {
+      const int m = threadIdx.x / k, r = threadIdx.x - m * k;
+      const int64_t q = (int64_t)(l0 + m) * k + r;
+      p_slot[m][r] = __ldcg(a.plan_slot + q);
+      p_gid[m][r] = __ldcg(a.plan_gid + q);
+      p_miss[m][r] = __ldcg(a.plan_miss + q);
+      p_gate[m][r] = __ldcg(a.plan_gate + q);
     }
-    stage16(reinterpret_cast<uint4*>(xs), (const uint8_t*)a.hidden + (int64_t)l * xbytes, xbytes, threadIdx.x,
-            blockDim.x);
+    for (int m = 0; m < np; m++)
+      stage16(reinterpret_cast<uint4*>(xs0 + m * xpad), (const uint8_t*)a.hidden + (int64_t)(l0 + m) * xbytes, xbytes,
+              threadIdx.x, blockDim.x);
     __syncthreads();
     if (threadIdx.x == 0) {
-      int nm = 0, nh = 0;
-      for (int r = 0; r < k; r++) {
-        if (p_miss[r])
-          p_mr[nm++] = r;
-        else
-          p_hr[nh++] = r;
+      for (int m = 0; m < np; m++) {
+        int nm = 0, nh = 0;
+        for (int r = 0; r < k; r++) {
+          if (p_miss[m][r])
+            p_mr[m][nm++] = r;
+          else
+            p_hr[m][nh++] = r;
+        }
+        p_nm[m] = nm;
+        p_nh[m] = nh;
       }
-      p_nm = nm;
-      p_nh = nh;
     }
     __syncthreads();
-    const int nm = p_nm, nh = p_nh;
-    const int workers = (int)gridDim.x - 1;
-    const int mctas = nm > 0 ? (a.miss_ctas < workers - 1 ? a.miss_ctas : workers - 1) : 0;
+    int nm_all = 0, nh_all = 0;
+    for (int m = 0; m < np; m++) {
+      nm_all += p_nm[m];
+      nh_all += p_nh[m];
+    }
+    const int mctas = nm_all > 0 ? (a.miss_ctas < workers - 1 ? a.miss_ctas : workers - 1) : 0;
     const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;
-    if (nm > 0 && a.touch_shift > 0) {
+    if (nm_all > 0 && a.touch_shift > 0) {
       const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
       const int64_t gt0 = ((int64_t)blockIdx.x - 1) * kFThreads + threadIdx.x;
       const int64_t GT = (int64_t)workers * kFThreads;
-      for (int64_t q = gt0; q < (int64_t)nm * pages; q += GT) {
-        const int mi = (int)(q / pages);
-        const uint8_t* pa = a.arena + (int64_t)p_gid[p_mr[mi]] * a.slot_stride + ((q - (int64_t)mi * pages) << a.touch_shift);
+      for (int64_t q = gt0; q < (int64_t)nm_all * pages; q += GT) {
+        int mi = (int)(q / pages), m = 0;
+        while (mi >= p_nm[m]) mi -= p_nm[m++];  // the group's misses in layer order
+        const uint8_t* pa =
+            a.arena + (int64_t)p_gid[m][p_mr[m][mi]] * a.slot_stride + ((q - (q / pages) * pages) << a.touch_shift);
         asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
       }
     }
     if (miss_cta) {
       const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
       const int MW = mctas * kFWarps;
-      for (int p = mw; p < nm * a.I; p += MW) {
-        const int r = p_mr[p / a.I];
+      // gate/up rows of every missed expert of the group, layer by layer: host -> slot, and u
+      for (int p = mw; p < nm_all * a.I; p += MW) {
+        int mi = p / a.I, m = 0;
+        while (mi >= p_nm[m]) mi -= p_nm[m++];
+        const int r = p_mr[m][mi];
         const int i = p - (p / a.I) * a.I;
-        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
-        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride;
-        gateup_row<WD, CH>(a, src, slot, true, xs, r, i, lane, u);
+        uint8_t* slot = a.pool + (int64_t)p_slot[m][r] * a.slot_stride;
+        const uint8_t* src = a.arena + (int64_t)p_gid[m][r] * a.slot_stride;
+        gateup_row<WD, CH>(a, src, slot, true, xs0 + m * xpad, r, i, lane, ug + (int64_t)m * k * a.I);
       }
       const int64_t dbytes = a.lay.total - a.lay.d_off;
       const int64_t nq = dbytes / 16;
       const int mt = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFThreads + threadIdx.x;
       const int MT = mctas * kFThreads;
-      for (int mi = 0; mi < nm; mi++) {
-        const int r = p_mr[mi];
-        uint8_t* dst = a.pool + (int64_t)p_slot[r] * a.slot_stride + a.lay.d_off;
-        const uint8_t* src = a.arena + (int64_t)p_gid[r] * a.slot_stride + a.lay.d_off;
-        for (int64_t q = mt; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
-      }
+      for (int m = 0; m < np; m++)
+        for (int mi = 0; mi < p_nm[m]; mi++) {
+          const int r = p_mr[m][mi];
+          uint8_t* dst = a.pool + (int64_t)p_slot[m][r] * a.slot_stride + a.lay.d_off;
+          const uint8_t* src = a.arena + (int64_t)p_gid[m][r] * a.slot_stride + a.lay.d_off;
+          for (int64_t q = mt; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
+        }
     } else {
       const int hw = wgw;
       const int HW = (workers - mctas) * kFWarps;
-      for (int p = hw; p < nh * a.I; p += HW) {
-        const int r = p_hr[p / a.I];
+      for (int p = hw; p < nh_all * a.I; p += HW) {
+        int hi = p / a.I, m = 0;
+        while (hi >= p_nh[m]) hi -= p_nh[m++];
+        const int r = p_hr[m][hi];
         const int i = p - (p / a.I) * a.I;
-        uint8_t* slot = a.pool + (int64_t)p_slot[r] * a.slot_stride;
-        gateup_row<WD, CH>(a, slot, slot, false, xs, r, i, lane, u);
+        uint8_t* slot = a.pool + (int64_t)p_slot[m][r] * a.slot_stride;
+        gateup_row<WD, CH>(a, slot, slot, false, xs0 + m * xpad, r, i, lane, ug + (int64_t)m * k * a.I);
       }
-      // In a layer-step that streams misses the hit workers wait at the barrier for the miss CTAs:
+      // In a group that streams misses the hit workers wait at the barrier for the miss CTAs:
       // done with its gate/up rows, a warp requests into L2 the W_d rows of the hit experts that
       // its down rows will read after the barrier, and the down rows then start from L2. (With
-      // every expert a hit the requests would only compete with the layer's last gate/up rows:
-      // measured 0.59 -> 0.57 of HBM peak resident, while the capped int4 stack gained 18%.)
-      if (nm > 0) {
+      // every expert a hit the requests would only compete with the last gate/up rows: measured
+      // 0.59 -> 0.57 of HBM peak resident, while the capped int4 stack gained 18%.)
+      if (nm_all > 0) {
         const int64_t rbd = a.lay.row_bytes_d;
         const int nl = (int)((rbd + 127) >> 7);
-        for (int o = wgw; o < a.d; o += HW)
-          for (int q = lane; q < nh * nl; q += 32) {
-            const int r = p_hr[q / nl];
-            const uint8_t* pa =
-                a.pool + (int64_t)p_slot[r] * a.slot_stride + a.lay.d_off + (int64_t)o * rbd + ((int64_t)(q % nl) << 7);
+        for (int q = wgw; q < np * a.d; q += HW) {
+          const int m = q / a.d, o = q - m * a.d;
+          for (int t = lane; t < p_nh[m] * nl; t += 32) {
+            const int r = p_hr[m][t / nl];
+            const uint8_t* pa = a.pool + (int64_t)p_slot[m][r] * a.slot_stride + a.lay.d_off + (int64_t)o * rbd +
+                                ((int64_t)(t % nl) << 7);
             asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
           }
+        }
       }
     }
     if (!worker_sync(a, nwbar)) return;
-    // Down rows + combine on the hit workers only: the miss CTAs go straight on to the next
-    // layer's misses, so the host link stays busy. Their copies then overlap these down rows,
-    // which is safe because no miss of layer l + 1 takes the slot of an expert of layer l
-    // (cap >= 2 k).
+    // Down rows + combine of the group's layers on the hit workers only: the miss CTAs go
+    // straight on to the next group's misses, so the host link stays busy. Their copies then
+    // overlap these down rows, which is safe because no miss of a layer takes the slot of an
+    // expert of any of the 2 P - 1 layers before it (cap >= 2 P k, checked by the host).
     const int HWW = (workers - mctas) * kFWarps;
     const bool dact = !miss_cta;
+    const int* ps = &p_slot[0][0];
+    const float* pg = &p_gate[0][0];
     switch (chd_need) {
-      case 1: down_phase<WD, 1>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
-      case 2: down_phase<WD, 2>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
-      case 3: down_phase<WD, 3>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
-      case 4: down_phase<WD, 4>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 1: down_phase<WD, 1>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
+      case 2: down_phase<WD, 2>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
+      case 3: down_phase<WD, 3>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
+      case 4: down_phase<WD, 4>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
       case 5:
-      case 6: down_phase<WD, 6>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
-      default: down_phase<WD, 8>(a, us, p_slot, p_gate, l, wgw, HWW, u, dact); break;
+      case 6: down_phase<WD, 6>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
+      default: down_phase<WD, 8>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
     }
   }
 }
@@ -1326,9 +1360,14 @@ int grid_of_la(size_t smem) {
   return grid >= 3 ? grid : 0;  // CTA 0 and at least two workers
 }
 
+// The lookahead kernel stages the inputs and u vectors of a whole layer group.
+size_t fused_la_smem(int wdtype, int d, int I, int k, int group) {
+  return (size_t)group * fused_smem(wdtype, d, I, k);
+}
+
 template <int WD, int CH>
 cudaError_t run_fused_la(const FusedArgs& a, int grid, cudaStream_t s) {
-  const size_t smem = fused_smem(a.wdtype, a.d, a.I, a.k);
+  const size_t smem = fused_la_smem(a.wdtype, a.d, a.I, a.k, a.la_group);
   void* params[] = {(void*)&a};
   return cudaLaunchCooperativeKernel((const void*)k_fused_la<WD, CH>, dim3(grid), dim3(kFThreads), params, smem, s);
 }
@@ -1348,10 +1387,10 @@ cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s) {
   return cudaErrorInvalidValue;
 }
 
-int fused_la_grid(int wdtype, int d, int I, int k) {
+int fused_la_grid(int wdtype, int d, int I, int k, int group) {
   const BlobLayout lay = make_layout(wdtype, d, I);
   const int ch = pick_ch_f(lay.row_bytes_gu);
-  const size_t smem = fused_smem(wdtype, d, I, k);
+  const size_t smem = fused_la_smem(wdtype, d, I, k, group);
   if (smem > 200 * 1024) return 0;
   MOE_F_DISPATCH(grid_of_la, wdtype, ch, smem);
   return 0;

@@ -16,6 +16,9 @@ struct TraceRec {
 };
 
 enum { STAT_HITS = 0, STAT_MISSES = 1, STAT_EVICTIONS = 2, STAT_LAYER_STEPS = 3, STAT_N = 4 };
+// Layers per worker barrier of the lookahead kernel when the pool allows it (cap >= 2 x this x k).
+constexpr int kLaGroupMax = 2;
+
 enum { FERR_BARRIER_TIMEOUT = 1, FERR_BAD_ROUTE = 2, FERR_NO_VICTIM = 4, FERR_PIPE_TIMEOUT = 8 };
 // Flags after which every CTA leaves the kernel at its next grid barrier.
 constexpr int FERR_FATAL = FERR_BARRIER_TIMEOUT | FERR_PIPE_TIMEOUT;
@@ -81,6 +84,7 @@ struct FusedArgs {
   // The plan arrays then hold every layer's plan, [L][k].
   unsigned* wbar_count;
   unsigned wbar_base;
+  int la_group;                // layers per worker barrier (1 or kLaGroupMax; needs cap >= 2 la_group k)
 };
 
 // Router-guided replacement key: the victim is the smallest key, i.e. the largest rank, then the
@@ -107,7 +111,7 @@ cudaError_t launch_fused(const FusedArgs& a, int grid, cudaStream_t s);
 // every expert resident): then no miss takes the slot of an expert the previous layer-step used,
 // whose down rows may still be running when the miss's bytes arrive. Same decisions, trace and
 // outputs as k_fused.
-int fused_la_grid(int wdtype, int d, int I, int k);
+int fused_la_grid(int wdtype, int d, int I, int k, int group);
 cudaError_t launch_fused_la(const FusedArgs& a, int grid, cudaStream_t s);
 
 // Batched decode step: B sequences per step, one cooperative kernel over all layers. Per layer

@@ -146,6 +146,7 @@ struct moe_handle {
   unsigned bar_epoch = 0;  // grid-barrier counter value at the start of the next fused launch
   bool lookahead_dev = false;  // device schedule with exact layer lookahead (k_fused_la) for whole steps
   int fgrid_la = 0;
+  int la_group = 1;            // layers per worker barrier of the lookahead kernel
   unsigned wbar_epoch = 0;     // its worker-barrier counter value at the start of the next launch
   const uint8_t* arena_dev = nullptr;
   // host time of the last decode-step launch (device schedule): after an idle gap the first step
@@ -819,6 +820,7 @@ moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, in
     a.plan_miss = h->d_plan + 2 * Lk;
     a.wbar_count = h->d_bar + 2;
     a.wbar_base = h->wbar_epoch;
+    a.la_group = h->la_group;
     a.may_evict = a.may_evict && c.policy == MOE_POLICY_LRU;
   }
   a.phase_ts = whole && !la ? phase_buffer(h) : nullptr;
@@ -835,7 +837,8 @@ moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, in
   if (l1 == c.n_layers) h->steps_launched++;
   if (la) {
     h->bar_epoch += (unsigned)h->fgrid_la;  // one grid barrier (after the router phase)
-    h->wbar_epoch += (unsigned)c.n_layers * (unsigned)(h->fgrid_la - 1);  // one worker barrier per layer
+    const unsigned groups = (unsigned)((c.n_layers + h->la_group - 1) / h->la_group);
+    h->wbar_epoch += groups * (unsigned)(h->fgrid_la - 1);  // one worker barrier per layer group
   } else {
     h->bar_epoch += 3u * (unsigned)(l1 - l0) * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
   }
@@ -1053,8 +1056,9 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   if (cudaHostGetDevicePointer((void**)&h->route_dev, (void*)h->route, 0) != cudaSuccess)
     return bail(MOE_ERR_CUDA, "mapped routing buffer has no device address");
   // u per rank; the device lookahead kernel keeps two layers' u (layer parity)
-  const int64_t u_sets = cfg->lookahead && cfg->schedule == MOE_SCHEDULE_DEVICE ? std::max(2, cfg->max_batch)
-                                                                                  : cfg->max_batch;
+  const int64_t u_sets = cfg->lookahead && cfg->schedule == MOE_SCHEDULE_DEVICE
+                             ? std::max(2 * moe::kLaGroupMax, cfg->max_batch)
+                             : cfg->max_batch;
   if (cudaMalloc(&h->u, sizeof(float) * u_sets * cfg->top_k * cfg->d_ff) != cudaSuccess)
     return bail(MOE_ERR_OOM, "u allocation failed");
   const int64_t act = (int64_t)cfg->n_layers * cfg->max_batch * cfg->d * h->asize;
@@ -1095,7 +1099,16 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
       if (h->cap < h->n_gid && h->cap < need_cap)
         return bail(MOE_ERR_INVALID, "lookahead in the device schedule needs at least " + std::to_string(need_cap) +
                                          " slots (or every expert resident)");
-      h->fgrid_la = moe::fused_la_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k);
+      // layers per worker barrier: a group of P layers needs a miss never to take the slot of an
+      // expert of the 2 P - 1 layer-steps before it, which LRU guarantees from 2 P k slots on
+      h->la_group = cfg->n_layers >= 2 && (h->cap >= h->n_gid || h->cap >= 2 * moe::kLaGroupMax * (int64_t)cfg->top_k)
+                        ? moe::kLaGroupMax
+                        : 1;
+      h->fgrid_la = moe::fused_la_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k, h->la_group);
+      if (h->fgrid_la <= 0 && h->la_group > 1) {
+        h->la_group = 1;
+        h->fgrid_la = moe::fused_la_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k, 1);
+      }
       if (h->fgrid_la <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the lookahead kernel");
       h->lookahead_dev = true;
     }

@@ -68,3 +68,43 @@ def test_one_slot_fewer_can_evict_from_the_previous_layer_step():
         k = rng.randint(2, 4)
         broken += not _victims_avoid_previous_step(3, 16, k, 2 * k - 1, steps=10, seed=seed)
     assert broken > 0
+
+
+def _victims_avoid_recent_steps(L, E, k, cap, steps, seed, depth):
+    """Like _victims_avoid_previous_step for the `depth` layer-steps before each one."""
+    rng = random.Random(seed)
+    tbl = oracle.LRUTable(L * E, cap, E)
+    clock = 0
+    recent = []
+    for t in range(steps):
+        for l in range(L):
+            needed = set(l * E + e for e in rng.sample(range(E), k))
+            used = set().union(*recent) if recent else set()
+            for r in tbl.step(clock, sorted(needed), t):
+                if r["evicted"] >= 0 and int(r["evicted"]) in used:
+                    return False
+            recent = (recent + [needed])[-depth:]
+            clock += 1
+    return True
+
+
+def test_layer_groups_need_2_p_k_slots():
+    # The lookahead kernel with groups of P layers per worker barrier writes a miss of a layer while
+    # the down rows of the previous group and the gate/up rows of its own group may still read: the
+    # 2 P - 1 layer-steps before it. LRU keeps their experts from (2 P - 1 + 1) k = 2 P k slots on.
+    for P in (2, 3):
+        depth = 2 * P - 1
+        checked = 0
+        for seed in range(60):
+            rng = random.Random(4000 + 100 * P + seed)
+            L, E = rng.randint(2, 6), rng.randint(8, 32)
+            k = rng.randint(1, min(4, E // (2 * P)))
+            cap = 2 * P * k
+            if cap >= L * E:
+                continue
+            checked += 1
+            assert _victims_avoid_recent_steps(L, E, k, cap, steps=10, seed=seed, depth=depth), (P, seed)
+        assert checked > 30
+        broken = sum(not _victims_avoid_recent_steps(4, 24, 3, 2 * P * 3 - 1, steps=10, seed=s, depth=depth)
+                     for s in range(60))
+        assert broken > 0
