@@ -137,8 +137,9 @@ typedef struct {
                              miss copies while layer l computes; a copy into a slot layer l still reads waits
                              for layer l's kernels. MOE_SCHEDULE_DEVICE (max_batch 1, MOE_POLICY_LRU): one kernel
                              routes every layer first, then CTA 0 runs the layers' lookups in order ahead of
-                             the other CTAs, which compute each layer with one barrier among them; needs
-                             cap_slots >= 2 * top_k unless every expert is resident. Steps of a
+                             the other CTAs, which compute each layer with one barrier among them (two
+                             layers per barrier from 4 * top_k slots on); needs cap_slots >= 2 * top_k
+                             unless every expert is resident. Steps of a
                              chained decoder (moe_decoder_step) run layer by layer whatever this says.
                              0 (default): one layer after another. */
 } moe_config;
