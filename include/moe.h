@@ -137,9 +137,11 @@ typedef struct {
                              miss copies while layer l computes; a copy into a slot layer l still reads waits
                              for layer l's kernels. MOE_SCHEDULE_DEVICE (max_batch 1, MOE_POLICY_LRU): one kernel
                              routes every layer first, then CTA 0 runs the layers' lookups in order ahead of
-                             the other CTAs, which compute each layer with one barrier among them (two
-                             layers per barrier from 4 * top_k slots on); needs cap_slots >= 2 * top_k
-                             unless every expert is resident. Steps of a
+                             the other CTAs, which compute the layers in groups (two layers per group from
+                             4 * top_k slots on), arriving on a counter after each group's gate/up rows;
+                             from 3 * top_k slots per layer of a group, or with every expert resident, a
+                             group's down rows run after the next group's gate/up rows. Needs cap_slots >=
+                             2 * top_k unless every expert is resident. Steps of a
                              chained decoder (moe_decoder_step) run layer by layer whatever this says.
                              0 (default): one layer after another. */
 } moe_config;

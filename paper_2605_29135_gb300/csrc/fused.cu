@@ -974,17 +974,29 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused(const __grid_constant__ 
 }
 
 // Barrier among the worker CTAs (1 .. gridDim.x - 1) of the lookahead kernel, bounded like grid_sync.
-__device__ bool worker_sync(const FusedArgs& a, unsigned& nbar) {
-  __shared__ int s_abort;
+// The worker CTAs' arrival counters of the lookahead kernel (every CTA but CTA 0 arrives once per
+// layer group, on the counter of the group's parity). worker_arrive: this CTA's threads are done
+// with group g's writes (u, slots), then one release-add. worker_wait: thread 0 waits (bounded,
+// like grid_sync) until every worker has arrived for group g; false in every thread of the CTA
+// once a fatal error flag is set. A CTA arrives for g + 2 only after every worker arrived for g,
+// so the parity counter reaches its target for g exactly when all of g's arrivals are in, even
+// with CTAs one group apart (a single counter would count g + 1's early arrivals as g's).
+__device__ void worker_arrive(const FusedArgs& a, int g) {
   __syncthreads();
-  nbar++;
   if (threadIdx.x == 0) {
-    const unsigned target = a.wbar_base + nbar * (gridDim.x - 1);
     __threadfence();
-    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a.wbar_count), "r"(1u) : "memory");
-    if ((int)(ld_acquire_u32(a.wbar_count) - target) < 0) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a.wbar_count + (g & 1)), "r"(1u) : "memory");
+  }
+}
+
+__device__ bool worker_wait(const FusedArgs& a, int g) {
+  __shared__ int s_abort;
+  if (threadIdx.x == 0) {
+    const unsigned* cnt = a.wbar_count + (g & 1);
+    const unsigned target = a.wbar_base[g & 1] + (unsigned)(g / 2 + 1) * (gridDim.x - 1);
+    if ((int)(ld_acquire_u32(cnt) - target) < 0) {
       const uint64_t t0 = gtimer();
-      while ((int)(ld_acquire_u32(a.wbar_count) - target) < 0) {
+      while ((int)(ld_acquire_u32(cnt) - target) < 0) {
         if (*(volatile int*)a.err & FERR_FATAL) break;
         if (gtimer() - t0 > a.barrier_timeout_ns) {
           atomicOr(a.err, FERR_BARRIER_TIMEOUT);
@@ -1084,22 +1096,26 @@ __device__ void la_lookups(const FusedArgs& a, int64_t step, PendingTable& pend,
 //       one grid barrier;
 //   CTA 0: the lookup step of layers 0 .. L-1 in order (the same calls, clocks, trace and table as
 //       the layer-by-layer kernel), layer m's plan going to plan[m][k] and plan_flag = its clock.
-//       A miss's bytes reach its slot during layer m's gate-up rows, after the workers' barrier of
-//       layer m - 1, while only layer m - 1's down rows may still read; with cap >= 2 k (checked
-//       by the host) LRU never gives a miss of layer m the slot of an expert layer m - 1 used, so
-//       CTA 0 may run any number of layers ahead;
-//   workers (CTAs 1 ..): per layer, wait for its plan, gate-up rows (the last miss_ctas workers
-//       stream the missed experts from the host tier into their slots), a barrier among the
-//       workers, then the down rows + combine on the workers that computed hits. No barrier
-//       follows the down rows: the next layer's gate-up rows (and the miss CTAs' streaming of its
-//       misses) start beside them, writing the other half of the layer-parity u buffer.
+//       Table writes change no slot's bytes: those change only when the miss CTAs stream a miss,
+//       so CTA 0 may run any number of layers ahead;
+//   workers (CTAs 1 ..): the layers in groups of a.la_group. Per group: wait for its plans, the
+//       gate-up rows (the last miss_ctas workers stream the missed experts from the host tier into
+//       their slots), an arrival on the workers' counter, then the down rows + combine of a group
+//       whose arrivals are all in, on the workers that computed its hits: the same group
+//       (unskewed) or the one before (skewed). No barrier follows the down rows: the next group's
+//       gate-up rows (and the miss CTAs' streaming of its misses) start beside them. A miss lands
+//       while the down rows of the groups before may still read; the host picks the group size
+//       and the skew so that LRU never hands a miss the slot of an expert they use.
 template <int WD, int CH>
 __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant__ FusedArgs a) {
   extern __shared__ uint4 smem4[];
-  // the plans and inputs of the layers of one group (a.la_group layers, 1 or kLaGroupMax)
-  __shared__ int p_slot[kLaGroupMax][kMaxRanks], p_gid[kLaGroupMax][kMaxRanks], p_miss[kLaGroupMax][kMaxRanks];
-  __shared__ float p_gate[kLaGroupMax][kMaxRanks];
-  __shared__ int p_mr[kLaGroupMax][kMaxRanks], p_hr[kLaGroupMax][kMaxRanks], p_nm[kLaGroupMax], p_nh[kLaGroupMax];
+  // The plans of two groups' layers (a.la_group layers each, 1 or kLaGroupMax), by group parity:
+  // group g's down rows may run after group g + 1's gate/up rows have loaded their plan.
+  __shared__ int p_slot[2][kLaGroupMax][kMaxRanks], p_gid[2][kLaGroupMax][kMaxRanks];
+  __shared__ int p_miss[2][kLaGroupMax][kMaxRanks];
+  __shared__ float p_gate[2][kLaGroupMax][kMaxRanks];
+  __shared__ int p_mr[2][kLaGroupMax][kMaxRanks], p_hr[2][kLaGroupMax][kMaxRanks];
+  __shared__ int p_nm[2][kLaGroupMax], p_nh[2][kLaGroupMax], p_mctas[2];
   __shared__ PendingTable pend;
   __shared__ int s_ok;
   const int asize = WD == WD_FP32 ? 4 : 2;
@@ -1113,7 +1129,7 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
   const int64_t step = *(volatile int64_t*)a.step;
   const int chd_need = (int)((a.lay.row_bytes_d / 16 + 31) / 32);
   const int k = a.k;
-  unsigned nbar = 0, nwbar = 0;
+  unsigned nbar = 0;
 
   la_router_all<WD>(a, gw, W, lane);
   if (!grid_sync(a, nbar)) return;
@@ -1122,134 +1138,161 @@ __global__ void __launch_bounds__(kFThreads, 2) k_fused_la(const __grid_constant
     return;
   }
 
-  // ---- workers: the layers in groups of P = a.la_group, one worker barrier per group
+  // ---- workers: the layers in groups of P = a.la_group. Each worker CTA arrives once per group
+  // on the worker counter after its gate/up rows; the down rows of group g start once every
+  // worker has arrived for g. Unskewed (a.la_skew = 0) a CTA runs gate/up(g), arrive, wait for g,
+  // down(g); skewed (1) it runs gate/up(g), arrive, wait for g - 1, down(g - 1), so the wait
+  // almost never stalls and the CTAs' down rows and gate/up rows interleave in HBM.
   const int wgw = ((int)blockIdx.x - 1) * kFWarps + (threadIdx.x >> 5);
   const int P = a.la_group;
+  const int G = (a.L + P - 1) / P;
   const int workers = (int)gridDim.x - 1;
-  for (int l0 = 0; l0 < a.L; l0 += P) {
-    const int np = a.L - l0 < P ? a.L - l0 : P;
-    // u of this group: groups alternate between two sets of P layers' vectors
-    float* ug = a.u + (int64_t)(((l0 / P) & 1) * P) * k * a.I;
-    __syncthreads();  // the previous group's down rows are done with the plans and u in this CTA
-    if (threadIdx.x == 0) s_ok = wait_count(a, a.plan_flag, (unsigned)(step * a.L + l0 + np));
-    __syncthreads();
-    if (!s_ok) return;
-    if (threadIdx.x < np * k) {
-      const int m = threadIdx.x / k, r = threadIdx.x - m * k;
-      const int64_t q = (int64_t)(l0 + m) * k + r;
-      p_slot[m][r] = __ldcg(a.plan_slot + q);
-      p_gid[m][r] = __ldcg(a.plan_gid + q);
-      p_miss[m][r] = __ldcg(a.plan_miss + q);
-      p_gate[m][r] = __ldcg(a.plan_gate + q);
-    }
-    for (int m = 0; m < np; m++)
-      stage16(reinterpret_cast<uint4*>(xs0 + m * xpad), (const uint8_t*)a.hidden + (int64_t)(l0 + m) * xbytes, xbytes,
-              threadIdx.x, blockDim.x);
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      for (int m = 0; m < np; m++) {
-        int nm = 0, nh = 0;
-        for (int r = 0; r < k; r++) {
-          if (p_miss[m][r])
-            p_mr[m][nm++] = r;
-          else
-            p_hr[m][nh++] = r;
-        }
-        p_nm[m] = nm;
-        p_nh[m] = nh;
+  const int skew = a.la_skew;
+  // u of group g: 2 (unskewed) or 4 (skewed) sets of P layers' vectors, in turn. Skewed, a CTA
+  // writes u of group g after every worker arrived for g - 2, when a CTA may not yet have staged
+  // u of g - 3 for its down rows, hence four.
+  const int nu = skew ? 4 : 2;
+  for (int g = 0; g < G + skew; g++) {
+    if (g < G) {
+      const int l0 = g * P;
+      const int np = a.L - l0 < P ? a.L - l0 : P;
+      const int b = g & 1;
+      float* ug = a.u + (int64_t)((g % nu) * P) * k * a.I;
+      __syncthreads();  // this CTA's down rows of group g - 2 (plan buffer b) and its gate/up rows of g - 1 (x) are done
+      if (threadIdx.x == 0) s_ok = wait_count(a, a.plan_flag, (unsigned)(step * a.L + l0 + np));
+      __syncthreads();
+      if (!s_ok) return;
+      if (threadIdx.x < np * k) {
+        const int m = threadIdx.x / k, r = threadIdx.x - m * k;
+        const int64_t q = (int64_t)(l0 + m) * k + r;
+        p_slot[b][m][r] = __ldcg(a.plan_slot + q);
+        p_gid[b][m][r] = __ldcg(a.plan_gid + q);
+        p_miss[b][m][r] = __ldcg(a.plan_miss + q);
+        p_gate[b][m][r] = __ldcg(a.plan_gate + q);
       }
-    }
-    __syncthreads();
-    int nm_all = 0, nh_all = 0;
-    for (int m = 0; m < np; m++) {
-      nm_all += p_nm[m];
-      nh_all += p_nh[m];
-    }
-    const int mctas = nm_all > 0 ? (a.miss_ctas < workers - 1 ? a.miss_ctas : workers - 1) : 0;
-    const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;
-    if (nm_all > 0 && a.touch_shift > 0) {
-      const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
-      const int64_t gt0 = ((int64_t)blockIdx.x - 1) * kFThreads + threadIdx.x;
-      const int64_t GT = (int64_t)workers * kFThreads;
-      for (int64_t q = gt0; q < (int64_t)nm_all * pages; q += GT) {
-        int mi = (int)(q / pages), m = 0;
-        while (mi >= p_nm[m]) mi -= p_nm[m++];  // the group's misses in layer order
-        const uint8_t* pa =
-            a.arena + (int64_t)p_gid[m][p_mr[m][mi]] * a.slot_stride + ((q - (q / pages) * pages) << a.touch_shift);
-        asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
-      }
-    }
-    if (miss_cta) {
-      const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
-      const int MW = mctas * kFWarps;
-      // gate/up rows of every missed expert of the group, layer by layer: host -> slot, and u
-      for (int p = mw; p < nm_all * a.I; p += MW) {
-        int mi = p / a.I, m = 0;
-        while (mi >= p_nm[m]) mi -= p_nm[m++];
-        const int r = p_mr[m][mi];
-        const int i = p - (p / a.I) * a.I;
-        uint8_t* slot = a.pool + (int64_t)p_slot[m][r] * a.slot_stride;
-        const uint8_t* src = a.arena + (int64_t)p_gid[m][r] * a.slot_stride;
-        gateup_row<WD, CH>(a, src, slot, true, xs0 + m * xpad, r, i, lane, ug + (int64_t)m * k * a.I);
-      }
-      const int64_t dbytes = a.lay.total - a.lay.d_off;
-      const int64_t nq = dbytes / 16;
-      const int mt = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFThreads + threadIdx.x;
-      const int MT = mctas * kFThreads;
       for (int m = 0; m < np; m++)
-        for (int mi = 0; mi < p_nm[m]; mi++) {
-          const int r = p_mr[m][mi];
-          uint8_t* dst = a.pool + (int64_t)p_slot[m][r] * a.slot_stride + a.lay.d_off;
-          const uint8_t* src = a.arena + (int64_t)p_gid[m][r] * a.slot_stride + a.lay.d_off;
-          for (int64_t q = mt; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
+        stage16(reinterpret_cast<uint4*>(xs0 + m * xpad), (const uint8_t*)a.hidden + (int64_t)(l0 + m) * xbytes, xbytes,
+                threadIdx.x, blockDim.x);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        int nm_all = 0;
+        for (int m = 0; m < np; m++) {
+          int nm = 0, nh = 0;
+          for (int r = 0; r < k; r++) {
+            if (p_miss[b][m][r])
+              p_mr[b][m][nm++] = r;
+            else
+              p_hr[b][m][nh++] = r;
+          }
+          p_nm[b][m] = nm;
+          p_nh[b][m] = nh;
+          nm_all += nm;
         }
-    } else {
-      const int hw = wgw;
-      const int HW = (workers - mctas) * kFWarps;
-      for (int p = hw; p < nh_all * a.I; p += HW) {
-        int hi = p / a.I, m = 0;
-        while (hi >= p_nh[m]) hi -= p_nh[m++];
-        const int r = p_hr[m][hi];
-        const int i = p - (p / a.I) * a.I;
-        uint8_t* slot = a.pool + (int64_t)p_slot[m][r] * a.slot_stride;
-        gateup_row<WD, CH>(a, slot, slot, false, xs0 + m * xpad, r, i, lane, ug + (int64_t)m * k * a.I);
+        p_mctas[b] = nm_all > 0 ? (a.miss_ctas < workers - 1 ? a.miss_ctas : workers - 1) : 0;
       }
-      // In a group that streams misses the hit workers wait at the barrier for the miss CTAs:
-      // done with its gate/up rows, a warp requests into L2 the W_d rows of the hit experts that
-      // its down rows will read after the barrier, and the down rows then start from L2. (With
-      // every expert a hit the requests would only compete with the last gate/up rows: measured
-      // 0.59 -> 0.57 of HBM peak resident, while the capped int4 stack gained 18%.)
-      if (nm_all > 0) {
-        const int64_t rbd = a.lay.row_bytes_d;
-        const int nl = (int)((rbd + 127) >> 7);
-        for (int q = wgw; q < np * a.d; q += HW) {
-          const int m = q / a.d, o = q - m * a.d;
-          for (int t = lane; t < p_nh[m] * nl; t += 32) {
-            const int r = p_hr[m][t / nl];
-            const uint8_t* pa = a.pool + (int64_t)p_slot[m][r] * a.slot_stride + a.lay.d_off + (int64_t)o * rbd +
-                                ((int64_t)(t % nl) << 7);
-            asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+      __syncthreads();
+      int nm_all = 0, nh_all = 0;
+      for (int m = 0; m < np; m++) {
+        nm_all += p_nm[b][m];
+        nh_all += p_nh[b][m];
+      }
+      const int mctas = p_mctas[b];
+      const bool miss_cta = (int)blockIdx.x >= (int)gridDim.x - mctas;
+      if (nm_all > 0 && a.touch_shift > 0) {
+        const int64_t pages = (a.lay.total + (1 << a.touch_shift) - 1) >> a.touch_shift;
+        const int64_t gt0 = ((int64_t)blockIdx.x - 1) * kFThreads + threadIdx.x;
+        const int64_t GT = (int64_t)workers * kFThreads;
+        for (int64_t q = gt0; q < (int64_t)nm_all * pages; q += GT) {
+          int mi = (int)(q / pages), m = 0;
+          while (mi >= p_nm[b][m]) mi -= p_nm[b][m++];  // the group's misses in layer order
+          const uint8_t* pa = a.arena + (int64_t)p_gid[b][m][p_mr[b][m][mi]] * a.slot_stride +
+                              ((q - (q / pages) * pages) << a.touch_shift);
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+        }
+      }
+      if (miss_cta) {
+        // A miss's bytes go into a slot whose previous expert no reader may still need: every
+        // worker must have arrived for g - 1 (unskewed that wait passed before the down rows of
+        // g - 1). The readers left are then the down rows of g - 2 (skewed only) and g - 1 and
+        // the gate/up rows of g, i.e. at most 3 P - 1 layer-steps before the miss's own, which
+        // LRU keeps from 3 P k slots on (2 P k unskewed); the host checks the cap.
+        if (g > 0 && !worker_wait(a, g - 1)) return;
+        const int mw = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFWarps + (threadIdx.x >> 5);
+        const int MW = mctas * kFWarps;
+        // gate/up rows of every missed expert of the group, layer by layer: host -> slot, and u
+        for (int p = mw; p < nm_all * a.I; p += MW) {
+          int mi = p / a.I, m = 0;
+          while (mi >= p_nm[b][m]) mi -= p_nm[b][m++];
+          const int r = p_mr[b][m][mi];
+          const int i = p - (p / a.I) * a.I;
+          uint8_t* slot = a.pool + (int64_t)p_slot[b][m][r] * a.slot_stride;
+          const uint8_t* src = a.arena + (int64_t)p_gid[b][m][r] * a.slot_stride;
+          gateup_row<WD, CH>(a, src, slot, true, xs0 + m * xpad, r, i, lane, ug + (int64_t)m * k * a.I);
+        }
+        const int64_t dbytes = a.lay.total - a.lay.d_off;
+        const int64_t nq = dbytes / 16;
+        const int mt = ((int)blockIdx.x - ((int)gridDim.x - mctas)) * kFThreads + threadIdx.x;
+        const int MT = mctas * kFThreads;
+        for (int m = 0; m < np; m++)
+          for (int mi = 0; mi < p_nm[b][m]; mi++) {
+            const int r = p_mr[b][m][mi];
+            uint8_t* dst = a.pool + (int64_t)p_slot[b][m][r] * a.slot_stride + a.lay.d_off;
+            const uint8_t* src = a.arena + (int64_t)p_gid[b][m][r] * a.slot_stride + a.lay.d_off;
+            for (int64_t q = mt; q < nq; q += MT) st_v4(dst + q * 16, ld_stream(src + q * 16));
+          }
+      } else {
+        const int hw = wgw;
+        const int HW = (workers - mctas) * kFWarps;
+        for (int p = hw; p < nh_all * a.I; p += HW) {
+          int hi = p / a.I, m = 0;
+          while (hi >= p_nh[b][m]) hi -= p_nh[b][m++];
+          const int r = p_hr[b][m][hi];
+          const int i = p - (p / a.I) * a.I;
+          uint8_t* slot = a.pool + (int64_t)p_slot[b][m][r] * a.slot_stride;
+          gateup_row<WD, CH>(a, slot, slot, false, xs0 + m * xpad, r, i, lane, ug + (int64_t)m * k * a.I);
+        }
+        // In a group that streams misses the hit workers wait for the miss CTAs before the
+        // group's down rows: done with its gate/up rows, a warp requests into L2 the W_d rows of
+        // the hit experts that its down rows will read, and those rows then start from L2. (With
+        // every expert a hit the requests would only compete with the last gate/up rows: measured
+        // 0.59 -> 0.57 of HBM peak resident, while the capped int4 stack gained 18%.)
+        if (nm_all > 0) {
+          const int64_t rbd = a.lay.row_bytes_d;
+          const int nl = (int)((rbd + 127) >> 7);
+          for (int q = wgw; q < np * a.d; q += HW) {
+            const int m = q / a.d, o = q - m * a.d;
+            for (int t = lane; t < p_nh[b][m] * nl; t += 32) {
+              const int r = p_hr[b][m][t / nl];
+              const uint8_t* pa = a.pool + (int64_t)p_slot[b][m][r] * a.slot_stride + a.lay.d_off +
+                                  (int64_t)o * rbd + ((int64_t)(t % nl) << 7);
+              asm volatile("prefetch.global.L2 [%0];" ::"l"(pa));
+            }
           }
         }
       }
+      worker_arrive(a, g);
     }
-    if (!worker_sync(a, nwbar)) return;
-    // Down rows + combine of the group's layers on the hit workers only: the miss CTAs go
-    // straight on to the next group's misses, so the host link stays busy. Their copies then
-    // overlap these down rows, which is safe because no miss of a layer takes the slot of an
-    // expert of any of the 2 P - 1 layers before it (cap >= 2 P k, checked by the host).
-    const int HWW = (workers - mctas) * kFWarps;
-    const bool dact = !miss_cta;
-    const int* ps = &p_slot[0][0];
-    const float* pg = &p_gate[0][0];
+    // Down rows + combine of group dg on the CTAs that computed its hits: its miss CTAs go
+    // straight on to the next group's misses, so the host link stays busy.
+    const int dg = g - skew;
+    if (dg < 0) continue;
+    if (!worker_wait(a, dg)) return;
+    const int db = dg & 1;
+    const int dl0 = dg * P;
+    const int dnp = a.L - dl0 < P ? a.L - dl0 : P;
+    const int HWW = (workers - p_mctas[db]) * kFWarps;
+    const bool dact = (int)blockIdx.x < (int)gridDim.x - p_mctas[db];
+    const int* ps = &p_slot[db][0][0];
+    const float* pg = &p_gate[db][0][0];
+    const float* ud = a.u + (int64_t)((dg % nu) * P) * k * a.I;
     switch (chd_need) {
-      case 1: down_phase<WD, 1>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
-      case 2: down_phase<WD, 2>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
-      case 3: down_phase<WD, 3>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
-      case 4: down_phase<WD, 4>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
+      case 1: down_phase<WD, 1>(a, us, ps, pg, dl0, wgw, HWW, ud, dact, dnp); break;
+      case 2: down_phase<WD, 2>(a, us, ps, pg, dl0, wgw, HWW, ud, dact, dnp); break;
+      case 3: down_phase<WD, 3>(a, us, ps, pg, dl0, wgw, HWW, ud, dact, dnp); break;
+      case 4: down_phase<WD, 4>(a, us, ps, pg, dl0, wgw, HWW, ud, dact, dnp); break;
       case 5:
-      case 6: down_phase<WD, 6>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
-      default: down_phase<WD, 8>(a, us, ps, pg, l0, wgw, HWW, ug, dact, np); break;
+      case 6: down_phase<WD, 6>(a, us, ps, pg, dl0, wgw, HWW, ud, dact, dnp); break;
+      default: down_phase<WD, 8>(a, us, ps, pg, dl0, wgw, HWW, ud, dact, dnp); break;
     }
   }
 }

@@ -80,11 +80,13 @@ struct FusedArgs {
   // (0 = highest logit, ties to the lower id; E before the layer's first routing).
   int32_t* rank;               // [L*E]
   unsigned* plan_flag;         // clock of the last layer-step whose plan CTA 0 has published (0: none)
-  // Exact layer lookahead (k_fused_la): the worker CTAs' barrier counter and its value at launch.
-  // The plan arrays then hold every layer's plan, [L][k].
-  unsigned* wbar_count;
-  unsigned wbar_base;
+  // Exact layer lookahead (k_fused_la): the worker CTAs' arrival counters, one per parity of the
+  // layer group, and their values at launch. The plan arrays then hold every layer's plan, [L][k].
+  unsigned* wbar_count;        // [2]
+  unsigned wbar_base[2];
   int la_group;                // layers per worker barrier (1 or kLaGroupMax; needs cap >= 2 la_group k)
+  int la_skew;                 // 1: a group's down rows run after the next group's gate/up rows (needs
+                               // cap >= 3 la_group k, or every expert resident, and u for 4 groups)
 };
 
 // Router-guided replacement key: the victim is the smallest key, i.e. the largest rank, then the

@@ -147,7 +147,8 @@ struct moe_handle {
   bool lookahead_dev = false;  // device schedule with exact layer lookahead (k_fused_la) for whole steps
   int fgrid_la = 0;
   int la_group = 1;            // layers per worker barrier of the lookahead kernel
-  unsigned wbar_epoch = 0;     // its worker-barrier counter value at the start of the next launch
+  int la_skew = 0;             // lookahead kernel: down rows of a group after the next group's gate/up rows
+  unsigned wbar_epoch[2] = {0, 0};  // its worker arrival counters (by group parity) at the next launch
   const uint8_t* arena_dev = nullptr;
   // host time of the last decode-step launch (device schedule): after an idle gap the first step
   // re-reads one word per page of the host tier first (see decode_device)
@@ -173,7 +174,8 @@ struct moe_handle {
   int32_t* d_route_idx = nullptr;
   float* d_route_gate = nullptr;
   unsigned long long* d_stats = nullptr;
-  unsigned* d_bar = nullptr;  // barrier count, (unused), batched work-item counters [2]
+  unsigned* d_bar = nullptr;  // barrier count, plan flag, then [2]: batched work-item counters or the
+                              // lookahead kernel's worker arrival counters
   int* d_err = nullptr;
   int* h_err = nullptr;       // pinned copy of d_err after each step
   cudaEvent_t err_ev = nullptr;
@@ -275,7 +277,7 @@ void reset_device_state(moe_handle* h) {
   cudaMemset(h->d_stats, 0, sizeof(unsigned long long) * moe::STAT_N);
   cudaMemset(h->d_bar, 0, sizeof(unsigned) * 4);
   h->bar_epoch = 0;
-  h->wbar_epoch = 0;
+  h->wbar_epoch[0] = h->wbar_epoch[1] = 0;
   cudaMemset(h->d_err, 0, sizeof(int));
   cudaDeviceSynchronize();
   *h->h_err = 0;
@@ -818,9 +820,11 @@ moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, in
     const int64_t Lk = (int64_t)c.n_layers * k;
     a.plan_gid = h->d_plan + Lk;
     a.plan_miss = h->d_plan + 2 * Lk;
-    a.wbar_count = h->d_bar + 2;
-    a.wbar_base = h->wbar_epoch;
+    a.wbar_count = h->d_bar + 2;  // [2], free at batch 1
+    a.wbar_base[0] = h->wbar_epoch[0];
+    a.wbar_base[1] = h->wbar_epoch[1];
     a.la_group = h->la_group;
+    a.la_skew = h->la_skew;
     a.may_evict = a.may_evict && c.policy == MOE_POLICY_LRU;
   }
   a.phase_ts = whole && !la ? phase_buffer(h) : nullptr;
@@ -838,7 +842,9 @@ moe_status decode_device_layers(moe_handle* h, const void* hidden, void* out, in
   if (la) {
     h->bar_epoch += (unsigned)h->fgrid_la;  // one grid barrier (after the router phase)
     const unsigned groups = (unsigned)((c.n_layers + h->la_group - 1) / h->la_group);
-    h->wbar_epoch += groups * (unsigned)(h->fgrid_la - 1);  // one worker barrier per layer group
+    // every worker arrives once per layer group, on the counter of the group's parity
+    h->wbar_epoch[0] += ((groups + 1) / 2) * (unsigned)(h->fgrid_la - 1);
+    h->wbar_epoch[1] += (groups / 2) * (unsigned)(h->fgrid_la - 1);
   } else {
     h->bar_epoch += 3u * (unsigned)(l1 - l0) * (unsigned)h->fgrid;  // every CTA arrives at 3 barriers per layer
   }
@@ -1055,9 +1061,9 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
   h->route->seq = 0;
   if (cudaHostGetDevicePointer((void**)&h->route_dev, (void*)h->route, 0) != cudaSuccess)
     return bail(MOE_ERR_CUDA, "mapped routing buffer has no device address");
-  // u per rank; the device lookahead kernel keeps two layers' u (layer parity)
+  // u per rank; the device lookahead kernel keeps the u of up to four groups of layers
   const int64_t u_sets = cfg->lookahead && cfg->schedule == MOE_SCHEDULE_DEVICE
-                             ? std::max(2 * moe::kLaGroupMax, cfg->max_batch)
+                             ? std::max(4 * moe::kLaGroupMax, cfg->max_batch)
                              : cfg->max_batch;
   if (cudaMalloc(&h->u, sizeof(float) * u_sets * cfg->top_k * cfg->d_ff) != cudaSuccess)
     return bail(MOE_ERR_OOM, "u allocation failed");
@@ -1110,6 +1116,10 @@ moe_status moe_create(const moe_config* cfg, moe_handle** out) {
         h->fgrid_la = moe::fused_la_grid(cfg->wdtype, cfg->d, cfg->d_ff, cfg->top_k, 1);
       }
       if (h->fgrid_la <= 0) return bail(MOE_ERR_INVALID, "shape not supported by the lookahead kernel");
+      // Skewed workers (a group's down rows after the next group's gate/up rows) leave the down
+      // rows of one more group reading while misses land: 3 P - 1 layer-steps before a miss's
+      // own, kept by LRU from 3 P k slots on; with every expert resident nothing is evicted.
+      h->la_skew = h->cap >= h->n_gid || h->cap >= 3 * (int64_t)h->la_group * cfg->top_k ? 1 : 0;
       h->lookahead_dev = true;
     }
   }

@@ -190,10 +190,18 @@ def test_preload_then_decode_matches_oracle(P, schedule, cap):
 
 # The device schedule with exact layer lookahead: one kernel routes every layer, CTA 0 then decides
 # the layers' lookups in order ahead of the compute (cap >= 2 * top_k, or every expert resident).
-# Same trace and outputs as the layer-by-layer kernel, bit for bit.
+# Same trace and outputs as the layer-by-layer kernel, bit for bit. The workers take layers in
+# groups of P = 2 from 4 * top_k slots (else 1) and run skewed (a group's down rows after the next
+# group's gate/up rows) from 3 * P * top_k slots or with every expert resident. tiny_fp32 has
+# top_k = 2: 8 layers at cap 6 run P = 1 skewed, cap 11 P = 2 unskewed, cap 12 P = 2 skewed.
 LOOKAHEAD = {
     "tiny3_fp32_cap4": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=4),
     "tiny3_fp32_cap8": synth.WORKLOADS["tiny_fp32"].replace(n_layers=3, cap_slots=8),
+    "tiny8_fp32_cap6_p1_skewed": synth.WORKLOADS["tiny_fp32"].replace(n_layers=8, tokens=32, cap_slots=6),
+    "tiny8_fp32_cap11_p2": synth.WORKLOADS["tiny_fp32"].replace(n_layers=8, tokens=32, cap_slots=11),
+    "tiny8_fp32_cap12_p2_skewed": synth.WORKLOADS["tiny_fp32"].replace(n_layers=8, tokens=32, cap_slots=12),
+    "tiny8_bf16_cap12_p2_skewed": synth.WORKLOADS["tiny_fp32"].replace(n_layers=8, tokens=32, cap_slots=12,
+                                                                       wdtype="bf16", adtype="bf16"),
     "ragged_fp32": RAGGED["fp32"].replace(cap_slots=4),
     "ragged_bf16": RAGGED["bf16"].replace(cap_slots=10),
     "ragged_int4": RAGGED["int4"].replace(cap_slots=6),

@@ -108,3 +108,27 @@ def test_layer_groups_need_2_p_k_slots():
         broken = sum(not _victims_avoid_recent_steps(4, 24, 3, 2 * P * 3 - 1, steps=10, seed=s, depth=depth)
                      for s in range(60))
         assert broken > 0
+
+
+def test_skewed_workers_need_3_p_k_slots():
+    # Skewed, a worker CTA runs the down rows of group g - 1 after the gate/up rows of group g, and
+    # the miss CTAs of a group start once every worker has arrived for the group before. A miss of a
+    # layer then lands while the down rows of the two groups before its own and the gate/up rows of
+    # its own group may still read: the 3 P - 1 layer-steps before it, which LRU keeps from
+    # (3 P - 1 + 1) k = 3 P k slots on.
+    for P in (1, 2, 3):
+        depth = 3 * P - 1
+        checked = 0
+        for seed in range(60):
+            rng = random.Random(5000 + 100 * P + seed)
+            L, E = rng.randint(2, 6), rng.randint(6 * P, 40)
+            k = rng.randint(1, min(4, E // (3 * P)))
+            cap = 3 * P * k
+            if cap >= L * E:
+                continue
+            checked += 1
+            assert _victims_avoid_recent_steps(L, E, k, cap, steps=10, seed=seed, depth=depth), (P, seed)
+        assert checked > 30
+        broken = sum(not _victims_avoid_recent_steps(4, 30, 3, 3 * P * 3 - 1, steps=10, seed=s, depth=depth)
+                     for s in range(60))
+        assert broken > 0
