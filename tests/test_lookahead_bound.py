@@ -8,6 +8,9 @@ with lower-id ties that holds whenever the pool has at least 2 k slots: the expe
 the newest timestamp apart from m's own, and at least k older residents remain for the at most k
 misses. Here the oracle's LRU checks the claim at the tightest cap on random routings (single
 sequence and batched unions, cold and preloaded pools), and shows that one slot fewer breaks it.
+The kernel's two refinements widen the window of layer-steps that may still read when a miss
+lands, and the same check covers them: layers in groups of P per arrival (2 P - 1 layer-steps,
+2 P k slots) and workers skewed by one group (3 P - 1 layer-steps, 3 P k slots).
 """
 import random
 
